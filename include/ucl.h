@@ -1,0 +1,213 @@
+/*
+ * ucl.h -- C ABI of the GB300 executor for upper-case-lower-case (UCL) EinSum
+ * over tensor-relations.
+ *
+ * A tensor-relation (paper Sec. 4.2) is a set of tuples (key, tile): the key is
+ * the vector of values of the operand's upper-case (promoted) labels, the tile
+ * is the dense sub-tensor over its lower-case (demoted) labels.  One binary
+ * UCL EinSum is evaluated as the TR-SQL template of Sec. 5 (Eq. eqn-TRA):
+ *
+ *     SELECT up(W), SUM(K(valU, valV)) FROM U NATURAL JOIN V GROUP BY up(W)
+ *
+ * where K is the lower-case EinSum applied to the two joined tiles.  The
+ * executor runs every step on the GPU: key packing, radix sort and merge-join
+ * of the keys, a batched tile contraction (tcgen05 tensor cores for bf16
+ * GEMM-shaped kernels, FFMA otherwise) whose epilogue performs the segmented
+ * group-by sum, and compaction of the output relation.
+ *
+ * Conventions shared by every call:
+ *   - Every call returns a ucl_status and never aborts.  On error an output
+ *     handle is set to NULL and inputs are left untouched; ucl_last_error()
+ *     gives a one-line reason.
+ *   - Device pointers are CUDA device addresses on the context's device.
+ *   - All GPU work is asynchronous on the context's stream, except where a
+ *     call documents a host synchronisation.
+ *   - Not thread-safe: one context is used by one host thread at a time.
+ */
+#ifndef UCL_H
+#define UCL_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    UCL_OK = 0,
+    UCL_ERR_ARG = 1,         /* NULL handle, bad pointer, n < 0, unknown enum */
+    UCL_ERR_SPEC = 2,        /* malformed spec string (grammar below) */
+    UCL_ERR_SHAPE = 3,       /* arity or extents disagree with the spec */
+    UCL_ERR_DUP_KEY = 4,     /* two tuples of one relation share a key (Sec. 4.2: one tuple per key) */
+    UCL_ERR_KEY_RANGE = 5,   /* a key value outside [0, bound) */
+    UCL_ERR_OOM = 6,         /* the allocator returned NULL */
+    UCL_ERR_CUDA = 7,        /* a CUDA runtime call failed */
+    UCL_ERR_UNSUPPORTED = 8, /* valid but outside this build (e.g. > 64 key bits, > 3 inputs) */
+    UCL_ERR_TIMEOUT = 9      /* a device-side wait ran out; the context stays usable */
+} ucl_status;
+
+typedef enum { UCL_BF16 = 0, UCL_F32 = 1 } ucl_dtype;
+
+typedef enum { UCL_EPI_NONE = 0, UCL_EPI_RELU = 1 } ucl_epilogue;
+
+/* Where ucl_relation_create reads keys and tiles from. */
+typedef enum {
+    UCL_MEM_DEVICE_BORROW = 0, /* device memory the caller keeps alive and unchanged while the relation lives */
+    UCL_MEM_DEVICE_COPY = 1,   /* device memory copied into library-owned buffers */
+    UCL_MEM_HOST_COPY = 2      /* host memory (pinned or pageable) copied to the device */
+} ucl_mem;
+
+/* Contraction kernel choice; AUTO picks tcgen05 when the tile kernel is a
+ * bf16 GEMM that fits it, FFMA otherwise. */
+typedef enum { UCL_PATH_AUTO = 0, UCL_PATH_SIMT = 1, UCL_PATH_TC = 2 } ucl_path;
+
+typedef struct ucl_ctx ucl_ctx;
+typedef struct ucl_rel ucl_rel;
+
+/* Allocator hooks.  alloc returns device memory of at least `bytes` bytes
+ * (256-byte aligned) or NULL; free releases it.  Both must be ordered on the
+ * context's stream (a caching allocator bound to that stream, or
+ * cudaMallocAsync/cudaFreeAsync on it).  NULL hooks select
+ * cudaMallocAsync/cudaFreeAsync on the context's stream. */
+typedef void *(*ucl_alloc_fn)(size_t bytes, void *user);
+typedef void (*ucl_free_fn)(void *ptr, size_t bytes, void *user);
+
+typedef struct {
+    ucl_dtype out_dtype;  /* dtype of the output tiles */
+    ucl_epilogue epi;     /* applied after the full group-by sum */
+    float scale;          /* out = epi(scale * sum); 1.0f for a plain sum */
+    int path;             /* ucl_path */
+} ucl_einsum_opts;
+
+#define UCL_NSTAGES 4
+
+/* Counters and stage timings of the last ucl_einsum on a context. */
+typedef struct {
+    int64_t n_pairs;       /* joined tuple pairs (one kernel invocation each) */
+    int64_t n_segments;    /* output tuples = distinct output keys */
+    double flops;          /* 2 * n_pairs * prod(all lower extents of the kernel) */
+    double bytes_contract; /* algorithmic bytes of the contraction stage */
+    int path;              /* ucl_path actually used (SIMT or TC) */
+    int launches;          /* GPU kernels launched by the call */
+    int timed;             /* 1 if stage_ms is valid (timing enabled) */
+    /* stage_ms: [0] key pack/sort/join count, [1] pair expansion, pair sort,
+     * segments, [2] tile contraction + fused group-by, [3] split-segment fixup
+     * and output key compaction.  CUDA-event times on the context stream. */
+    float stage_ms[UCL_NSTAGES];
+} ucl_stats;
+
+/* --------------------------------------------------------------- context */
+
+/* Create a context on `device` that issues work on `stream` (a cudaStream_t,
+ * NULL = the legacy default stream).  Allocates a small device status word
+ * and pinned host scratch; device workspace grows on demand through the
+ * allocator hooks and is reused across calls. */
+ucl_status ucl_ctx_create(int device, void *stream, ucl_alloc_fn alloc, ucl_free_fn free_fn, void *user,
+                          ucl_ctx **out);
+
+/* Synchronises the stream, then frees the workspace.  Relations created on
+ * the context must be destroyed first. */
+ucl_status ucl_ctx_destroy(ucl_ctx *ctx);
+
+/* Drain the context's stream and report device-side failures (a bounded wait
+ * that ran out: UCL_ERR_TIMEOUT; a failed bounds check: UCL_ERR_CUDA) raised
+ * by kernels of earlier calls.  Such failures are sticky: if not collected
+ * here they surface at the next synchronising call of the context. */
+ucl_status ucl_ctx_synchronize(ucl_ctx *ctx);
+
+/* Enable (1) or disable (0) CUDA-event stage timing for later calls. */
+ucl_status ucl_ctx_set_timing(ucl_ctx *ctx, int enable);
+
+/* Statistics of the last ucl_einsum; synchronises on its last event when
+ * timing is enabled. */
+ucl_status ucl_get_last_stats(ucl_ctx *ctx, ucl_stats *out);
+
+/* Stage times of every ucl_einsum made with timing enabled since the last
+ * reset, so that a caller can time many calls without synchronising between
+ * them: ms[c * UCL_NSTAGES + s] receives stage s of call c (the stages of
+ * ucl_stats.stage_ms) for c < max_calls; *n_calls (if not NULL) the number of
+ * calls recorded.  Synchronises on the last recorded event.  reset != 0
+ * forgets the recorded calls and recycles their events. */
+ucl_status ucl_ctx_timings(ucl_ctx *ctx, float *ms, int max_calls, int *n_calls, int reset);
+
+/* ------------------------------------------------------------- relations */
+
+/* Create a tensor-relation (Sec. 4.2, schema (INT up[1], ..., TENSOR val)).
+ *   n          number of tuples (>= 0)
+ *   u          number of key columns = promoted labels (0..15)
+ *   keys       int32 [n, u] row-major; column c holds values in [0, key_bounds[c])
+ *   key_bounds int64 [u], each >= 1 (host memory)
+ *   r          number of tile dimensions = demoted labels (0..15; 0 = scalar tiles)
+ *   tile_shape int64 [r], each >= 1 (host memory)
+ *   dtype      element type of the tiles
+ *   tiles      [n, prod(tile_shape)] row-major tiles, last dimension fastest
+ *   mem        where keys and tiles live (ucl_mem); with BORROW the tiles
+ *              must be 16-byte aligned for the tensor-core path to apply
+ * Validates on the GPU that every key is in range (UCL_ERR_KEY_RANGE) and that
+ * no key repeats (UCL_ERR_DUP_KEY), and records whether the keys are already
+ * in ascending order; synchronises the stream once (twice if unsorted).
+ * Returns UCL_ERR_UNSUPPORTED if the key bit widths, ceil(log2(bound)) per
+ * column, sum to more than 64. */
+ucl_status ucl_relation_create(ucl_ctx *ctx, int64_t n, int u, const int32_t *keys, const int64_t *key_bounds,
+                               int r, const int64_t *tile_shape, ucl_dtype dtype, const void *tiles, ucl_mem mem,
+                               ucl_rel **out);
+
+/* Frees library-owned buffers (stream-ordered).  Borrowed memory is untouched. */
+ucl_status ucl_relation_destroy(ucl_rel *rel);
+
+/* Shape of a relation.  key_bounds / tile_shape may be NULL; otherwise they
+ * receive u / r entries. */
+ucl_status ucl_relation_info(const ucl_rel *rel, int64_t *n, int *u, int *r, int64_t *key_bounds,
+                             int64_t *tile_shape, ucl_dtype *dtype);
+
+/* Device addresses of the key array [n, u] and tile array [n, tile]. */
+ucl_status ucl_relation_data(const ucl_rel *rel, const int32_t **keys, const void **tiles);
+
+/* Copy keys (int32 [n, u]) and tiles ([n, tile] in the relation's dtype) to
+ * host memory; either destination may be NULL.  Synchronises the stream. */
+ucl_status ucl_relation_download(const ucl_rel *rel, int32_t *keys_host, void *tiles_host);
+
+/* ----------------------------------------------------------------- einsum */
+
+/* Evaluate one UCL EinSum (Sec. 4.3 notation, Sec. 5 Eq. eqn-TRA).
+ *
+ * Spec grammar: "<op>,<op>->" "<out>" with 1 or 2 input operands (n_in).
+ * Each operand is a string of letters, one letter per label; an upper-case
+ * letter is a promoted label (a key column, in the order the upper-case
+ * letters appear), a lower-case letter a demoted label (a tile dimension, in
+ * the order the lower-case letters appear).  Letters are case-sensitive
+ * labels: 'J' and 'j' are two labels, as in a tile index J and an offset j of
+ * one reshaped dense index.  A label appears at most once per operand; every
+ * output label appears in some input; a label has one extent everywhere.
+ * Labels absent from the output are summed: upper ones by the group-by, lower
+ * ones inside the tile kernel.  Shared upper labels are the join attributes;
+ * with none the join is a cross product (Sec. 6.2).  n_in = 1 is a unary
+ * EinSum (a group-by sum over one relation, e.g. with the relu epilogue).
+ *
+ * Output: a new relation owned by the library (destroy it with
+ * ucl_relation_destroy), one tuple per distinct output key produced by at
+ * least one joined pair -- also when its sum is zero -- in ascending
+ * lexicographic key order; tiles row-major over the output's lower labels.
+ *
+ * Synchronises the stream twice (after the join count and after the segment
+ * count: both sizes depend on the data).  The contraction is deterministic:
+ * pairs of one output key are summed in a fixed order.
+ * Errors: UCL_ERR_SPEC / SHAPE for spec-relation mismatches, UCL_ERR_OOM,
+ * UCL_ERR_UNSUPPORTED (more than 2^31-1 joined pairs, > 64 key bits),
+ * UCL_ERR_TIMEOUT / UCL_ERR_CUDA for device failures. */
+ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec, int n_in, ucl_rel *const *in, const ucl_einsum_opts *opts,
+                      ucl_rel **out);
+
+/* ------------------------------------------------------------ diagnostics */
+
+const char *ucl_status_str(ucl_status st);
+
+/* One-line description of the last error on this context ("" if none). */
+const char *ucl_last_error(const ucl_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* UCL_H */

@@ -1,0 +1,866 @@
+// api.cu -- the C ABI (include/ucl.h): spec parsing and validation, plan
+// building, relation management and the stage schedule of one UCL EinSum.
+//
+// Stage schedule of ucl_einsum (paper Sec. 5, Eq. eqn-TRA):
+//   0  pack keys -> radix sort both inputs by join key (skipped for inputs
+//      already sorted by it) -> per-U-tuple matching range in V -> scan;
+//      host sync #1 reads the pair count
+//   1  expand pairs (u, v, packed output key) -> stable radix sort by output
+//      key -> segment heads -> scan; host sync #2 reads the segment count
+//   2  allocate the output relation; segment starts + output keys; tile
+//      contraction with the group-by sum fused into its epilogue
+//   3  fixup of segments split across work units
+#include <algorithm>
+#include <cstdio>
+#include <new>
+
+#include "internal.cuh"
+
+using namespace ucl;
+
+namespace {
+
+struct Oom {};
+
+// ------------------------------------------------------------------ spec
+
+struct Label {
+    char c;
+    bool upper;
+    int64_t ext = 0;
+    int pos[4] = {-1, -1, -1, -1};   // key column / tile dim in input k (k < 3), output at [3]
+};
+
+struct Spec {
+    int n_in = 0;
+    std::string op[3];
+    std::string out;
+    std::vector<Label> labs;
+    int find(char c) const {
+        for (size_t i = 0; i < labs.size(); ++i)
+            if (labs[i].c == c) return (int)i;
+        return -1;
+    }
+    const std::string &operand(int k) const { return k == 3 ? out : op[k]; }
+};
+
+bool is_alpha(char c) { return (c >= 'a' && c <= 'z') || (c >= 'A' && c <= 'Z'); }
+bool is_upper(char c) { return c >= 'A' && c <= 'Z'; }
+
+ucl_status parse_spec(ucl_ctx *ctx, const char *text, int n_in, Spec &s) {
+    if (!text) return fail(ctx, UCL_ERR_ARG, "spec is NULL");
+    if (n_in < 1 || n_in > 2) return fail(ctx, n_in == 3 ? UCL_ERR_UNSUPPORTED : UCL_ERR_ARG, "n_in must be 1 or 2");
+    std::string t(text);
+    size_t arrow = t.find("->");
+    if (arrow == std::string::npos) return fail(ctx, UCL_ERR_SPEC, "spec has no '->'");
+    std::string lhs = t.substr(0, arrow);
+    s.out = t.substr(arrow + 2);
+    int k = 0;
+    for (char c : lhs) {
+        if (c == ',') {
+            if (++k >= 3) return fail(ctx, UCL_ERR_SPEC, "too many operands");
+        } else if (is_alpha(c)) {
+            s.op[k] += c;
+        } else {
+            return fail(ctx, UCL_ERR_SPEC, std::string("bad character in spec: ") + c);
+        }
+    }
+    if (k + 1 != n_in) return fail(ctx, UCL_ERR_SPEC, "operand count does not match n_in");
+    s.n_in = n_in;
+    for (char c : s.out)
+        if (!is_alpha(c)) return fail(ctx, UCL_ERR_SPEC, std::string("bad character in output: ") + c);
+    for (int i = 0; i <= n_in; ++i) {
+        const std::string &o = i < n_in ? s.op[i] : s.out;
+        if ((int)o.size() > kMaxCols) return fail(ctx, UCL_ERR_UNSUPPORTED, "operand has more than 15 labels");
+        for (size_t a = 0; a < o.size(); ++a)
+            for (size_t b = a + 1; b < o.size(); ++b)
+                if (o[a] == o[b]) return fail(ctx, UCL_ERR_SPEC, std::string("label repeated in one operand: ") + o[a]);
+    }
+    for (int i = 0; i < n_in; ++i)
+        for (char c : s.op[i])
+            if (s.find(c) < 0) {
+                Label L;
+                L.c = c;
+                L.upper = is_upper(c);
+                s.labs.push_back(L);
+            }
+    for (char c : s.out)
+        if (s.find(c) < 0) return fail(ctx, UCL_ERR_SPEC, std::string("output label not in any input: ") + c);
+    for (int i = 0; i <= n_in; ++i) {
+        const std::string &o = i < n_in ? s.op[i] : s.out;
+        int cu = 0, cl = 0;
+        for (char c : o) {
+            Label &L = s.labs[s.find(c)];
+            L.pos[i < n_in ? i : 3] = L.upper ? cu++ : cl++;
+        }
+    }
+    if ((int)s.labs.size() > kMaxLow + kMaxCols) return fail(ctx, UCL_ERR_UNSUPPORTED, "too many labels");
+    return UCL_OK;
+}
+
+// Arity and extents of the inputs against the spec (Sec. 3: one bound per label).
+ucl_status bind_extents(ucl_ctx *ctx, Spec &s, ucl_rel *const *in) {
+    for (int k = 0; k < s.n_in; ++k) {
+        const ucl_rel *R = in[k];
+        if (!R) return fail(ctx, UCL_ERR_ARG, "input relation is NULL");
+        if (R->ctx != ctx) return fail(ctx, UCL_ERR_ARG, "input relation belongs to another context");
+        int nu = 0, nl = 0;
+        for (char c : s.op[k]) (is_upper(c) ? nu : nl)++;
+        if (R->u != nu || R->r != nl)
+            return fail(ctx, UCL_ERR_SHAPE, "operand " + std::to_string(k) + " '" + s.op[k] +
+                                                "' does not match the relation's key/tile arity");
+        for (Label &L : s.labs) {
+            int p = L.pos[k];
+            if (p < 0) continue;
+            int64_t e = L.upper ? R->bounds[p] : R->shape[p];
+            if (L.ext == 0) L.ext = e;
+            else if (L.ext != e)
+                return fail(ctx, UCL_ERR_SHAPE, std::string("label '") + L.c + "' has two different extents");
+        }
+    }
+    return UCL_OK;
+}
+
+// Row-major stride of lower label L inside operand k's tile (0 if absent).
+int64_t tile_stride(const Spec &s, int k, const Label &L) {
+    int p = L.pos[k];
+    if (p < 0) return 0;
+    int64_t st = 1;
+    const std::string &o = s.operand(k);
+    for (int a = (int)o.size() - 1; a >= 0; --a) {
+        const Label &M = s.labs[s.find(o[a])];
+        if (M.upper) continue;
+        if (M.pos[k] == p) break;
+        st *= M.ext;
+    }
+    return st;
+}
+
+struct KeyPlan {
+    std::vector<int> join;   // label ids of the join attributes, U's order
+    int join_bits = 0;
+    KeyPack join_u{}, join_v{};
+    KeyPack out_u{}, out_v{};
+    int out_bits = 0;
+    KeyUnpack unpack{};
+    int64_t out_bounds[kMaxCols] = {};
+    int uw = 0;
+    bool ident_u = false, ident_v = false;   // input already ordered by its join key
+};
+
+ucl_status plan_keys(ucl_ctx *ctx, const Spec &s, ucl_rel *const *in, KeyPlan &kp) {
+    const int n = s.n_in;
+    // output key: W's upper labels, first most significant
+    std::vector<int> wl;
+    for (char c : s.out) {
+        int L = s.find(c);
+        if (s.labs[L].upper) wl.push_back(L);
+    }
+    kp.uw = (int)wl.size();
+    int total = 0;
+    for (int L : wl) total += bit_width(s.labs[L].ext);
+    if (total > 64) return fail(ctx, UCL_ERR_UNSUPPORTED, "output key needs more than 64 bits");
+    kp.out_bits = total;
+    kp.unpack.uw = kp.uw;
+    int shift = total;
+    for (int q = 0; q < kp.uw; ++q) {
+        const Label &L = s.labs[wl[q]];
+        int b = bit_width(L.ext);
+        shift -= b;
+        kp.unpack.shift[q] = shift;
+        kp.unpack.bits[q] = b;
+        kp.out_bounds[q] = L.ext;
+        // supplier: U if it has the label, else V
+        if (L.pos[0] >= 0)
+            kp.out_u.f[kp.out_u.nf++] = KeyField{L.pos[0], shift, b};
+        else
+            kp.out_v.f[kp.out_v.nf++] = KeyField{L.pos[1], shift, b};
+    }
+    if (n < 2) return UCL_OK;
+    // join attributes: upper labels of both inputs, in U's order
+    for (char c : s.op[0]) {
+        int L = s.find(c);
+        if (s.labs[L].upper && s.labs[L].pos[1] >= 0) kp.join.push_back(L);
+    }
+    total = 0;
+    for (int L : kp.join) total += bit_width(s.labs[L].ext);
+    if (total > 64) return fail(ctx, UCL_ERR_UNSUPPORTED, "join key needs more than 64 bits");
+    kp.join_bits = total;
+    shift = total;
+    for (int L : kp.join) {
+        int b = bit_width(s.labs[L].ext);
+        shift -= b;
+        kp.join_u.f[kp.join_u.nf++] = KeyField{s.labs[L].pos[0], shift, b};
+        kp.join_v.f[kp.join_v.nf++] = KeyField{s.labs[L].pos[1], shift, b};
+    }
+    // an input whose keys are sorted and whose leading key columns are the
+    // join attributes in the same order is already grouped by join key
+    for (int k = 0; k < 2; ++k) {
+        bool ok = in[k]->sorted != 0;
+        for (size_t q = 0; q < kp.join.size() && ok; ++q) ok = s.labs[kp.join[q]].pos[k] == (int)q;
+        (k == 0 ? kp.ident_u : kp.ident_v) = ok || kp.join.empty();
+    }
+    return UCL_OK;
+}
+
+ucl_status plan_lower(ucl_ctx *ctx, const Spec &s, ucl_rel *const *in, LowerPlan &lp) {
+    memset(&lp, 0, sizeof(lp));
+    lp.tile_u = in[0]->tile;
+    lp.tile_v = s.n_in > 1 ? in[1]->tile : 1;
+    lp.tile_w = 1;
+    for (char c : s.out) {
+        const Label &L = s.labs[s.find(c)];
+        if (L.upper) continue;
+        lp.w_ext[lp.nw] = (int)L.ext;
+        lp.w_su[lp.nw] = (int)tile_stride(s, 0, L);
+        lp.w_sv[lp.nw] = s.n_in > 1 ? (int)tile_stride(s, 1, L) : 0;
+        lp.tile_w *= L.ext;
+        lp.nw++;
+    }
+    lp.n_c = 1;
+    for (const Label &L : s.labs) {
+        if (L.upper || L.pos[3] >= 0) continue;
+        if (lp.nc >= kMaxLow) return fail(ctx, UCL_ERR_UNSUPPORTED, "too many contracted labels");
+        lp.c_ext[lp.nc] = (int)L.ext;
+        lp.c_su[lp.nc] = (int)tile_stride(s, 0, L);
+        lp.c_sv[lp.nc] = s.n_in > 1 ? (int)tile_stride(s, 1, L) : 0;
+        lp.n_c *= L.ext;
+        lp.nc++;
+    }
+    if (lp.tile_w >= (1ll << 31) || lp.tile_u >= (1ll << 31) || lp.tile_v >= (1ll << 31))
+        return fail(ctx, UCL_ERR_UNSUPPORTED, "tile has 2^31 or more elements");
+    return UCL_OK;
+}
+
+// tcgen05 shape: exactly one M label (lower, in A and W), one N label (lower,
+// in B and W) and one K label (lower, in A and B), nothing else lower; both
+// operands bf16.  The operand giving the larger M-side extent becomes A.
+bool plan_tc(const Spec &s, ucl_rel *const *in, TcPlan &tp, std::string *why) {
+    memset(&tp, 0, sizeof(tp));
+    if (s.n_in != 2) { *why = "unary"; return false; }
+    if (in[0]->dtype != UCL_BF16 || in[1]->dtype != UCL_BF16) { *why = "operands are not bf16"; return false; }
+    int mu = -1, nv = -1, kk = -1;
+    for (size_t i = 0; i < s.labs.size(); ++i) {
+        const Label &L = s.labs[i];
+        if (L.upper) continue;
+        bool a = L.pos[0] >= 0, b = L.pos[1] >= 0, w = L.pos[3] >= 0;
+        if (a && !b && w) { if (mu >= 0) { *why = "several labels of U's output side"; return false; } mu = (int)i; }
+        else if (!a && b && w) { if (nv >= 0) { *why = "several labels of V's output side"; return false; } nv = (int)i; }
+        else if (a && b && !w) { if (kk >= 0) { *why = "several contracted labels"; return false; } kk = (int)i; }
+        else { *why = "batch or single-operand lower labels"; return false; }
+    }
+    if (mu < 0 || nv < 0 || kk < 0) { *why = "tile kernel is not a GEMM"; return false; }
+    const Label &Lu = s.labs[mu], &Lv = s.labs[nv], &Lk = s.labs[kk];
+    // A gets the side with an extent of 128 or 256; prefer U on ties
+    auto m_ok = [](int64_t e) { return e == 128 || e == 256; };
+    auto n_ok = [](int64_t e) { return e >= 16 && e <= 256 && e % 16 == 0; };
+    if (m_ok(Lu.ext) && n_ok(Lv.ext)) tp.a_is_u = 1;
+    else if (m_ok(Lv.ext) && n_ok(Lu.ext)) tp.a_is_u = 0;
+    else { *why = "M/N extents do not fit tcgen05 (M 128|256, N 16..256 step 16)"; return false; }
+    if (Lk.ext % 16 != 0 || Lk.ext > 256) { *why = "K extent not a multiple of 16 up to 256"; return false; }
+    const int ka = tp.a_is_u ? 0 : 1, kb = 1 - ka;
+    const Label &LM = tp.a_is_u ? Lu : Lv, &LN = tp.a_is_u ? Lv : Lu;
+    tp.M = (int)LM.ext;
+    tp.N = (int)LN.ext;
+    tp.K = (int)Lk.ext;
+    tp.m_blocks = tp.M / 128;
+    // K-major when K is the fastest tile dim of the operand
+    tp.a_kmajor = Lk.pos[ka] > LM.pos[ka];
+    tp.b_kmajor = Lk.pos[kb] > LN.pos[kb];
+    tp.sWm = tile_stride(s, 3, LM);
+    tp.sWn = tile_stride(s, 3, LN);
+    return true;
+}
+
+// --------------------------------------------------------------- helpers
+
+size_t dsize(ucl_dtype d) { return d == UCL_BF16 ? 2 : 4; }
+
+void arena_reset(ucl_ctx *ctx) {
+    Arena &A = ctx->arena;
+    if (A.blocks.size() > 1) {
+        size_t total = A.total();
+        for (auto &b : A.blocks) ctx_free(ctx, b.ptr, b.size);
+        A.blocks.clear();
+        char *p = (char *)ctx_alloc(ctx, total);
+        if (p) A.blocks.push_back({p, total});
+    }
+    A.used = 0;
+}
+
+void record(ucl_ctx *ctx, int i) {
+    if (ctx->cur_ev) cudaEventRecord(ctx->cur_ev[i], ctx->stream);
+}
+
+// Claim the events of one timed call (grows the pool on demand).
+ucl_status begin_timed_call(ucl_ctx *ctx) {
+    ctx->cur_ev = nullptr;
+    if (!ctx->timing) return UCL_OK;
+    const size_t per = UCL_NSTAGES + 1, need = per * (ctx->ev_calls + 1);
+    while (ctx->ev_pool.size() < need) {
+        cudaEvent_t e;
+        ucl_status st = cuda_check(ctx, cudaEventCreate(&e), "cudaEventCreate");
+        if (st) return st;
+        ctx->ev_pool.push_back(e);
+    }
+    ctx->cur_ev = &ctx->ev_pool[per * ctx->ev_calls];
+    ctx->ev_calls++;
+    return UCL_OK;
+}
+
+// Read n int64 device scalars after draining the stream.  Word 0 of the
+// device status holds error bits raised by any earlier kernel of this context
+// (sticky until reported here); word 1 holds validation flags (returned in
+// *flags, cleared).
+ucl_status sync_read(ucl_ctx *ctx, const int64_t *dev, int n, int64_t *host, uint32_t *flags = nullptr) {
+    cudaError_t e = cudaSuccess;
+    if (n > 0) e = cudaMemcpyAsync(ctx->h_pinned, dev, sizeof(int64_t) * n, cudaMemcpyDeviceToHost, ctx->stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(ctx->h_pinned + 7, ctx->d_status, 2 * sizeof(uint32_t), cudaMemcpyDeviceToHost,
+                            ctx->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(ctx->stream);
+    if (e != cudaSuccess) return cuda_check(ctx, e, "stream sync");
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_check(ctx, e, "kernel launch");
+    for (int i = 0; i < n; ++i) host[i] = ctx->h_pinned[i];
+    uint32_t words[2];
+    memcpy(words, ctx->h_pinned + 7, sizeof(words));
+    if (flags) *flags = words[1];
+    if (words[0] | words[1]) cudaMemsetAsync(ctx->d_status, 0, 2 * sizeof(uint32_t), ctx->stream);
+    if (words[0] & kStTimeout) return fail(ctx, UCL_ERR_TIMEOUT, "a device-side wait timed out");
+    if (words[0] & kStBadIndex) return fail(ctx, UCL_ERR_CUDA, "a device-side bounds check failed");
+    return UCL_OK;
+}
+
+struct Fail {
+    ucl_status st;
+};
+
+// Throw on error so that the stage schedule can bail out from any depth.
+void check(ucl_status st) {
+    if (st != UCL_OK) throw Fail{st};
+}
+
+ucl_rel *new_rel(ucl_ctx *ctx) {
+    ucl_rel *r = new (std::nothrow) ucl_rel();
+    if (r) {
+        r->ctx = ctx;
+        ctx->live_rels++;
+    }
+    return r;
+}
+
+KeyPack full_pack(const ucl_rel *R, int *bits) {
+    KeyPack kp{};
+    int total = 0;
+    for (int c = 0; c < R->u; ++c) total += bit_width(R->bounds[c]);
+    *bits = total;
+    int shift = total;
+    for (int c = 0; c < R->u; ++c) {
+        int b = bit_width(R->bounds[c]);
+        shift -= b;
+        kp.f[kp.nf++] = KeyField{c, shift, b};
+    }
+    return kp;
+}
+
+}  // namespace
+
+// =================================================================== ucl::
+
+namespace ucl {
+
+int bit_width(int64_t bound) {
+    int b = 0;
+    while (b < 63 && ((int64_t)1 << b) < bound) ++b;
+    return b;
+}
+
+ucl_status fail(ucl_ctx *ctx, ucl_status st, const std::string &msg) {
+    if (ctx) ctx->err = msg;
+    return st;
+}
+
+ucl_status cuda_check(ucl_ctx *ctx, cudaError_t e, const char *what) {
+    if (e == cudaSuccess) return UCL_OK;
+    cudaGetLastError();
+    return fail(ctx, UCL_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+void *ctx_alloc(ucl_ctx *ctx, size_t bytes) {
+    if (bytes == 0) bytes = 256;
+    bytes = (bytes + 255) & ~(size_t)255;
+    if (ctx->alloc) return ctx->alloc(bytes, ctx->user);
+    void *p = nullptr;
+    if (cudaMallocAsync(&p, bytes, ctx->stream) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    return p;
+}
+
+void ctx_free(ucl_ctx *ctx, void *p, size_t bytes) {
+    if (!p) return;
+    bytes = (bytes + 255) & ~(size_t)255;
+    if (ctx->free_fn) ctx->free_fn(p, bytes, ctx->user);
+    else cudaFreeAsync(p, ctx->stream);
+}
+
+void *ws_get(ucl_ctx *ctx, size_t bytes) {
+    Arena &A = ctx->arena;
+    bytes = (bytes + 255) & ~(size_t)255;
+    if (bytes == 0) bytes = 256;
+    if (A.blocks.empty() || A.used + bytes > A.blocks.back().size) {
+        size_t want = std::max(bytes, std::max((size_t)(1 << 22), A.total()));
+        char *p = (char *)ctx_alloc(ctx, want);
+        if (!p) throw Oom();
+        A.blocks.push_back({p, want});
+        A.used = 0;
+    }
+    char *p = A.blocks.back().ptr + A.used;
+    A.used += bytes;
+    return p;
+}
+
+}  // namespace ucl
+
+// ===================================================================== ABI
+
+extern "C" {
+
+const char *ucl_status_str(ucl_status st) {
+    switch (st) {
+        case UCL_OK: return "UCL_OK";
+        case UCL_ERR_ARG: return "UCL_ERR_ARG";
+        case UCL_ERR_SPEC: return "UCL_ERR_SPEC";
+        case UCL_ERR_SHAPE: return "UCL_ERR_SHAPE";
+        case UCL_ERR_DUP_KEY: return "UCL_ERR_DUP_KEY";
+        case UCL_ERR_KEY_RANGE: return "UCL_ERR_KEY_RANGE";
+        case UCL_ERR_OOM: return "UCL_ERR_OOM";
+        case UCL_ERR_CUDA: return "UCL_ERR_CUDA";
+        case UCL_ERR_UNSUPPORTED: return "UCL_ERR_UNSUPPORTED";
+        case UCL_ERR_TIMEOUT: return "UCL_ERR_TIMEOUT";
+    }
+    return "UCL_ERR_UNKNOWN";
+}
+
+const char *ucl_last_error(const ucl_ctx *ctx) { return ctx ? ctx->err.c_str() : "NULL context"; }
+
+ucl_status ucl_ctx_create(int device, void *stream, ucl_alloc_fn alloc, ucl_free_fn free_fn, void *user,
+                          ucl_ctx **out) {
+    if (!out) return UCL_ERR_ARG;
+    *out = nullptr;
+    if ((alloc == nullptr) != (free_fn == nullptr)) return UCL_ERR_ARG;
+    ucl_ctx *ctx = new (std::nothrow) ucl_ctx();
+    if (!ctx) return UCL_ERR_OOM;
+    ctx->device = device;
+    ctx->stream = (cudaStream_t)stream;
+    ctx->alloc = alloc;
+    ctx->free_fn = free_fn;
+    ctx->user = user;
+    ucl_status st = cuda_check(ctx, cudaSetDevice(device), "cudaSetDevice");
+    if (!st) st = cuda_check(ctx, cudaDeviceGetAttribute(&ctx->sm_count, cudaDevAttrMultiProcessorCount, device),
+                             "device attribute");
+    if (!st) st = cuda_check(ctx, cudaMalloc(&ctx->d_status, 256), "cudaMalloc status");
+    if (!st) st = cuda_check(ctx, cudaMemset(ctx->d_status, 0, 256), "cudaMemset status");
+    if (!st) st = cuda_check(ctx, cudaMallocHost(&ctx->h_pinned, 8 * sizeof(int64_t)), "cudaMallocHost");
+    if (st) {
+        if (ctx->d_status) cudaFree(ctx->d_status);
+        if (ctx->h_pinned) cudaFreeHost(ctx->h_pinned);
+        delete ctx;
+        return st;
+    }
+    *out = ctx;
+    return UCL_OK;
+}
+
+ucl_status ucl_ctx_destroy(ucl_ctx *ctx) {
+    if (!ctx) return UCL_ERR_ARG;
+    if (ctx->live_rels) return fail(ctx, UCL_ERR_ARG, "relations still alive on this context");
+    cudaStreamSynchronize(ctx->stream);
+    for (auto &b : ctx->arena.blocks) ctx_free(ctx, b.ptr, b.size);
+    cudaStreamSynchronize(ctx->stream);
+    cudaFree(ctx->d_status);
+    cudaFreeHost(ctx->h_pinned);
+    for (cudaEvent_t e : ctx->ev_pool) cudaEventDestroy(e);
+    delete ctx;
+    return UCL_OK;
+}
+
+ucl_status ucl_ctx_set_timing(ucl_ctx *ctx, int enable) {
+    if (!ctx) return UCL_ERR_ARG;
+    ctx->timing = enable ? 1 : 0;
+    return UCL_OK;
+}
+
+ucl_status ucl_ctx_synchronize(ucl_ctx *ctx) {
+    if (!ctx) return UCL_ERR_ARG;
+    cudaSetDevice(ctx->device);
+    return sync_read(ctx, nullptr, 0, nullptr);
+}
+
+ucl_status ucl_get_last_stats(ucl_ctx *ctx, ucl_stats *out) {
+    if (!ctx || !out) return UCL_ERR_ARG;
+    if (ctx->last.timed && ctx->cur_ev) {
+        cudaError_t e = cudaEventSynchronize(ctx->cur_ev[UCL_NSTAGES]);
+        if (e != cudaSuccess) return cuda_check(ctx, e, "event sync");
+        for (int i = 0; i < UCL_NSTAGES; ++i)
+            cudaEventElapsedTime(&ctx->last.stage_ms[i], ctx->cur_ev[i], ctx->cur_ev[i + 1]);
+    }
+    *out = ctx->last;
+    return UCL_OK;
+}
+
+ucl_status ucl_ctx_timings(ucl_ctx *ctx, float *ms, int max_calls, int *n_calls, int reset) {
+    if (!ctx || (max_calls > 0 && !ms)) return UCL_ERR_ARG;
+    const int per = UCL_NSTAGES + 1;
+    if (n_calls) *n_calls = ctx->ev_calls;
+    if (ctx->ev_calls > 0 && max_calls > 0) {
+        cudaError_t e = cudaEventSynchronize(ctx->ev_pool[(size_t)per * ctx->ev_calls - 1]);
+        if (e != cudaSuccess) return cuda_check(ctx, e, "event sync");
+        for (int c = 0; c < ctx->ev_calls && c < max_calls; ++c)
+            for (int i = 0; i < UCL_NSTAGES; ++i)
+                cudaEventElapsedTime(&ms[c * UCL_NSTAGES + i], ctx->ev_pool[(size_t)per * c + i],
+                                     ctx->ev_pool[(size_t)per * c + i + 1]);
+    }
+    if (reset) {
+        ctx->ev_calls = 0;
+        ctx->cur_ev = nullptr;
+        ctx->last.timed = 0;
+    }
+    return UCL_OK;
+}
+
+ucl_status ucl_relation_create(ucl_ctx *ctx, int64_t n, int u, const int32_t *keys, const int64_t *key_bounds,
+                               int r, const int64_t *tile_shape, ucl_dtype dtype, const void *tiles, ucl_mem mem,
+                               ucl_rel **out) {
+    if (!out) return fail(ctx, UCL_ERR_ARG, "out is NULL");
+    *out = nullptr;
+    if (!ctx) return UCL_ERR_ARG;
+    if (n < 0 || u < 0 || u > kMaxCols || r < 0 || r > kMaxCols) return fail(ctx, UCL_ERR_ARG, "bad n, u or r");
+    if (dtype != UCL_BF16 && dtype != UCL_F32) return fail(ctx, UCL_ERR_ARG, "bad dtype");
+    if (mem != UCL_MEM_DEVICE_BORROW && mem != UCL_MEM_DEVICE_COPY && mem != UCL_MEM_HOST_COPY)
+        return fail(ctx, UCL_ERR_ARG, "bad mem");
+    if ((u > 0 && !key_bounds) || (r > 0 && !tile_shape)) return fail(ctx, UCL_ERR_ARG, "bounds/shape is NULL");
+    if (n > 0 && ((u > 0 && !keys) || !tiles)) return fail(ctx, UCL_ERR_ARG, "keys/tiles is NULL");
+    if (n >= (1ll << 32) - 1) return fail(ctx, UCL_ERR_UNSUPPORTED, "2^32 or more tuples");
+    cudaSetDevice(ctx->device);
+    ucl_rel tmp;
+    tmp.ctx = ctx;
+    tmp.n = n;
+    tmp.u = u;
+    tmp.r = r;
+    tmp.dtype = dtype;
+    for (int c = 0; c < u; ++c) {
+        if (key_bounds[c] < 1 || key_bounds[c] > (1ll << 31)) return fail(ctx, UCL_ERR_ARG, "key bound out of [1, 2^31]");
+        tmp.bounds[c] = key_bounds[c];
+    }
+    tmp.tile = 1;
+    for (int q = 0; q < r; ++q) {
+        if (tile_shape[q] < 1) return fail(ctx, UCL_ERR_SHAPE, "tile extent < 1");
+        tmp.shape[q] = tile_shape[q];
+        tmp.tile *= tile_shape[q];
+        if (tmp.tile >= (1ll << 31)) return fail(ctx, UCL_ERR_UNSUPPORTED, "tile has 2^31 or more elements");
+    }
+    KeyPack fp = full_pack(&tmp, &tmp.key_bits);
+    if (tmp.key_bits > 64) return fail(ctx, UCL_ERR_UNSUPPORTED, "key columns need more than 64 bits");
+    if (u == 0 && n > 1) return fail(ctx, UCL_ERR_DUP_KEY, "more than one tuple in a key-less relation");
+
+    size_t kbytes = (size_t)n * u * sizeof(int32_t), tbytes = (size_t)n * tmp.tile * dsize(dtype);
+    size_t koff = (tbytes + 255) & ~(size_t)255;
+    if (mem == UCL_MEM_DEVICE_BORROW) {
+        tmp.keys = const_cast<int32_t *>(keys);
+        tmp.tiles = const_cast<void *>(tiles);
+    } else if (n > 0) {
+        tmp.own_bytes = koff + kbytes;
+        tmp.own_block = ctx_alloc(ctx, tmp.own_bytes);
+        if (!tmp.own_block) return fail(ctx, UCL_ERR_OOM, "allocation of relation storage failed");
+        tmp.tiles = tmp.own_block;
+        tmp.keys = (int32_t *)((char *)tmp.own_block + koff);
+        cudaMemcpyKind kind = mem == UCL_MEM_HOST_COPY ? cudaMemcpyHostToDevice : cudaMemcpyDeviceToDevice;
+        cudaError_t e = cudaMemcpyAsync(tmp.tiles, tiles, tbytes, kind, ctx->stream);
+        if (e == cudaSuccess && kbytes) e = cudaMemcpyAsync(tmp.keys, keys, kbytes, kind, ctx->stream);
+        if (e != cudaSuccess) {
+            ctx_free(ctx, tmp.own_block, tmp.own_bytes);
+            return cuda_check(ctx, e, "copy of relation storage");
+        }
+    }
+    tmp.sorted = 1;
+    ucl_status st = UCL_OK;
+    if (n > 0 && u > 0) {
+        try {
+            arena_reset(ctx);
+            uint64_t *packed = (uint64_t *)ws_get(ctx, sizeof(uint64_t) * n);
+            launch_check_keys(ctx, tmp.keys, u, n, tmp.bounds, fp, packed);
+            uint32_t flags = 0;
+            st = sync_read(ctx, nullptr, 0, nullptr, &flags);
+            if (!st && (flags & kStKeyRange)) st = fail(ctx, UCL_ERR_KEY_RANGE, "key outside [0, bound)");
+            if (!st && (flags & kStUnsorted)) {
+                tmp.sorted = 0;
+                uint64_t *alt = (uint64_t *)ws_get(ctx, sizeof(uint64_t) * n);
+                int which = radix_sort(ctx, packed, nullptr, alt, nullptr, n, tmp.key_bits);
+                launch_check_dups(ctx, which ? alt : packed, n);
+                st = sync_read(ctx, nullptr, 0, nullptr, &flags);
+                if (!st && (flags & kStDupKey)) st = fail(ctx, UCL_ERR_DUP_KEY, "duplicate key");
+            }
+        } catch (Oom &) {
+            st = fail(ctx, UCL_ERR_OOM, "workspace allocation failed");
+        }
+    }
+    if (st) {
+        if (tmp.own_block) ctx_free(ctx, tmp.own_block, tmp.own_bytes);
+        return st;
+    }
+    ucl_rel *R = new_rel(ctx);
+    if (!R) {
+        if (tmp.own_block) ctx_free(ctx, tmp.own_block, tmp.own_bytes);
+        return fail(ctx, UCL_ERR_OOM, "host allocation failed");
+    }
+    *R = tmp;
+    *out = R;
+    ctx->err.clear();
+    return UCL_OK;
+}
+
+ucl_status ucl_relation_destroy(ucl_rel *rel) {
+    if (!rel) return UCL_ERR_ARG;
+    ucl_ctx *ctx = rel->ctx;
+    if (rel->own_block) ctx_free(ctx, rel->own_block, rel->own_bytes);
+    ctx->live_rels--;
+    delete rel;
+    return UCL_OK;
+}
+
+ucl_status ucl_relation_info(const ucl_rel *rel, int64_t *n, int *u, int *r, int64_t *key_bounds,
+                             int64_t *tile_shape, ucl_dtype *dtype) {
+    if (!rel) return UCL_ERR_ARG;
+    if (n) *n = rel->n;
+    if (u) *u = rel->u;
+    if (r) *r = rel->r;
+    if (key_bounds) for (int c = 0; c < rel->u; ++c) key_bounds[c] = rel->bounds[c];
+    if (tile_shape) for (int q = 0; q < rel->r; ++q) tile_shape[q] = rel->shape[q];
+    if (dtype) *dtype = rel->dtype;
+    return UCL_OK;
+}
+
+ucl_status ucl_relation_data(const ucl_rel *rel, const int32_t **keys, const void **tiles) {
+    if (!rel) return UCL_ERR_ARG;
+    if (keys) *keys = rel->keys;
+    if (tiles) *tiles = rel->tiles;
+    return UCL_OK;
+}
+
+ucl_status ucl_relation_download(const ucl_rel *rel, int32_t *keys_host, void *tiles_host) {
+    if (!rel) return UCL_ERR_ARG;
+    ucl_ctx *ctx = rel->ctx;
+    cudaSetDevice(ctx->device);
+    cudaError_t e = cudaSuccess;
+    if (keys_host && rel->n * rel->u > 0)
+        e = cudaMemcpyAsync(keys_host, rel->keys, sizeof(int32_t) * rel->n * rel->u, cudaMemcpyDeviceToHost,
+                            ctx->stream);
+    if (e == cudaSuccess && tiles_host && rel->n > 0)
+        e = cudaMemcpyAsync(tiles_host, rel->tiles, dsize(rel->dtype) * rel->n * rel->tile, cudaMemcpyDeviceToHost,
+                            ctx->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(ctx->stream);
+    return cuda_check(ctx, e, "download");
+}
+
+ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *const *in, const ucl_einsum_opts *opts,
+                      ucl_rel **out) {
+    if (!out) return fail(ctx, UCL_ERR_ARG, "out is NULL");
+    *out = nullptr;
+    if (!ctx || !in) return fail(ctx, UCL_ERR_ARG, "NULL context or inputs");
+    ucl_einsum_opts o{UCL_F32, UCL_EPI_NONE, 1.0f, UCL_PATH_AUTO};
+    if (opts) o = *opts;
+    if ((o.out_dtype != UCL_BF16 && o.out_dtype != UCL_F32) || (o.epi != UCL_EPI_NONE && o.epi != UCL_EPI_RELU) ||
+        o.path < UCL_PATH_AUTO || o.path > UCL_PATH_TC)
+        return fail(ctx, UCL_ERR_ARG, "bad options");
+    Spec s;
+    ucl_status st = parse_spec(ctx, spec_text, n_in, s);
+    if (st) return st;
+    if ((st = bind_extents(ctx, s, in))) return st;
+    KeyPlan kp;
+    if ((st = plan_keys(ctx, s, in, kp))) return st;
+    LowerPlan lp;
+    if ((st = plan_lower(ctx, s, in, lp))) return st;
+    TcPlan tp;
+    std::string why;
+    bool tc_ok = plan_tc(s, in, tp, &why);
+    if (o.path == UCL_PATH_TC && !tc_ok) return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why);
+    cudaSetDevice(ctx->device);
+
+    const ucl_rel *U = in[0];
+    const ucl_rel *V = n_in > 1 ? in[1] : nullptr;
+    const int64_t nU = U->n, nV = V ? V->n : 1;
+    ucl_stats stats{};
+    ctx->launches = 0;
+    ucl_rel *R = nullptr;
+    if ((st = begin_timed_call(ctx))) return st;
+    try {
+        arena_reset(ctx);
+        record(ctx, 0);
+        int64_t *d_scal = (int64_t *)ws_get(ctx, 8 * sizeof(int64_t));
+        // ---------------------------------------------------------- stage 0
+        int64_t P = 0;
+        uint64_t *koU = nullptr, *koV = nullptr, *permU = nullptr, *permV = nullptr;
+        int64_t *off = nullptr;
+        uint32_t *lo = nullptr;
+        if (nU > 0 && nV > 0) {
+            koU = (uint64_t *)ws_get(ctx, 8 * nU);
+            uint64_t *jkU = V ? (uint64_t *)ws_get(ctx, 8 * nU) : nullptr;
+            launch_pack(ctx, U->keys, U->u, nU, kp.join_u, jkU, kp.out_u, koU);
+            if (V) {
+                koV = (uint64_t *)ws_get(ctx, 8 * nV);
+                uint64_t *jkV = (uint64_t *)ws_get(ctx, 8 * nV);
+                launch_pack(ctx, V->keys, V->u, nV, kp.join_v, jkV, kp.out_v, koV);
+                const bool join = !kp.join.empty();
+                if (join && !kp.ident_u) {
+                    uint64_t *vals = (uint64_t *)ws_get(ctx, 8 * nU), *ka = (uint64_t *)ws_get(ctx, 8 * nU),
+                             *va = (uint64_t *)ws_get(ctx, 8 * nU);
+                    launch_iota(ctx, vals, nU);
+                    int w = radix_sort(ctx, jkU, vals, ka, va, nU, kp.join_bits);
+                    if (w) { jkU = ka; permU = va; } else permU = vals;
+                }
+                if (join && !kp.ident_v) {
+                    uint64_t *vals = (uint64_t *)ws_get(ctx, 8 * nV), *ka = (uint64_t *)ws_get(ctx, 8 * nV),
+                             *va = (uint64_t *)ws_get(ctx, 8 * nV);
+                    launch_iota(ctx, vals, nV);
+                    int w = radix_sort(ctx, jkV, vals, ka, va, nV, kp.join_bits);
+                    if (w) { jkV = ka; permV = va; } else permV = vals;
+                }
+                int64_t *cnt = (int64_t *)ws_get(ctx, 8 * nU);
+                lo = (uint32_t *)ws_get(ctx, 4 * nU);
+                off = (int64_t *)ws_get(ctx, 8 * nU);
+                launch_join_count(ctx, join ? jkU : nullptr, nU, join ? jkV : nullptr, nV, cnt, lo);
+                scan_i64(ctx, cnt, off, nU, d_scal);
+                record(ctx, 1);
+                int64_t h;
+                check(sync_read(ctx, d_scal, 1, &h));
+                P = h;
+            } else {
+                record(ctx, 1);
+                P = nU;
+            }
+        } else {
+            record(ctx, 1);
+        }
+        if (P >= (1ll << 31)) check(fail(ctx, UCL_ERR_UNSUPPORTED, "more than 2^31-1 joined pairs"));
+
+        // ---------------------------------------------------------- stage 1
+        int64_t S = 0;
+        uint64_t *pk = nullptr, *pv = nullptr;
+        int64_t *seg_excl = nullptr;
+        if (P > 0) {
+            pk = (uint64_t *)ws_get(ctx, 8 * P);
+            pv = (uint64_t *)ws_get(ctx, 8 * P);
+            uint64_t *pk2 = (uint64_t *)ws_get(ctx, 8 * P), *pv2 = (uint64_t *)ws_get(ctx, 8 * P);
+            if (V)
+                launch_expand(ctx, off, nU, lo, permU, permV, koU, koV, P, pk, pv);
+            else
+                launch_unary_pairs(ctx, koU, P, pk, pv);
+            if (radix_sort(ctx, pk, pv, pk2, pv2, P, kp.out_bits)) { pk = pk2; pv = pv2; }
+            int64_t *flag = (int64_t *)ws_get(ctx, 8 * P);
+            seg_excl = (int64_t *)ws_get(ctx, 8 * P);
+            launch_heads(ctx, pk, P, flag);
+            scan_i64(ctx, flag, seg_excl, P, d_scal + 1);
+            int64_t h;
+            check(sync_read(ctx, d_scal + 1, 1, &h));
+            S = h;
+        }
+
+        // output relation: keys ascending by construction
+        R = new_rel(ctx);
+        if (!R) check(fail(ctx, UCL_ERR_OOM, "host allocation failed"));
+        R->n = S;
+        R->u = kp.uw;
+        R->r = lp.nw;
+        for (int q = 0; q < kp.uw; ++q) R->bounds[q] = kp.out_bounds[q];
+        for (int q = 0; q < lp.nw; ++q) R->shape[q] = lp.w_ext[q];
+        R->dtype = o.out_dtype;
+        R->tile = lp.tile_w;
+        R->sorted = 1;
+        R->key_bits = kp.out_bits;
+        if (S > 0) {
+            size_t tbytes = (size_t)S * lp.tile_w * dsize(o.out_dtype);
+            size_t koff = (tbytes + 255) & ~(size_t)255;
+            R->own_bytes = koff + (size_t)S * kp.uw * 4;
+            R->own_block = ctx_alloc(ctx, R->own_bytes);
+            if (!R->own_block) throw Oom();
+            R->tiles = R->own_block;
+            R->keys = (int32_t *)((char *)R->own_block + koff);
+        }
+
+        // ------------------------------------------------------ stage 2, 3
+        int path = UCL_PATH_SIMT;
+        if (P > 0) {
+            int64_t *seg_start = (int64_t *)ws_get(ctx, 8 * (S + 1));
+            uint32_t *pu = (uint32_t *)ws_get(ctx, 4 * P), *pvi = (uint32_t *)ws_get(ctx, 4 * P);
+            launch_segments(ctx, pk, pv, seg_excl, P, S, kp.unpack, R->keys, seg_start, pu, pvi);
+            record(ctx, 2);
+            ContractArgs a{};
+            a.U = U->tiles;
+            a.V = V ? V->tiles : nullptr;
+            a.du = U->dtype;
+            a.dv = V ? V->dtype : U->dtype;
+            a.nU = nU;
+            a.nV = V ? nV : 0;
+            a.pu = pu;
+            a.pv = pvi;
+            a.seg_start = seg_start;
+            a.S = S;
+            a.out = R->tiles;
+            a.dout = o.out_dtype;
+            a.epi = o.epi;
+            a.scale = o.scale;
+            a.tile_w = lp.tile_w;
+            bool use_tc = tc_ok && o.path != UCL_PATH_SIMT;
+            if (use_tc) {
+                std::string why2;
+                if (!tc_supported(tp, a, &why2)) {
+                    if (o.path == UCL_PATH_TC) check(fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why2));
+                    use_tc = false;
+                }
+            }
+            int G = use_tc ? tc_units(ctx, tp, P) : (int)std::min<int64_t>(P, (int64_t)ctx->sm_count * 4);
+            a.units.P = P;
+            a.units.G = G;
+            a.partials = (float *)ws_get(ctx, sizeof(float) * 2 * (size_t)G * lp.tile_w);
+            if (use_tc) {
+                const ucl_rel *ra = tp.a_is_u ? U : V, *rb = tp.a_is_u ? V : U;
+                check(launch_contract_tc(ctx, a, tp, ra, rb));
+                path = UCL_PATH_TC;
+            } else {
+                launch_contract_simt(ctx, a, lp);
+            }
+            record(ctx, 3);
+            launch_fixup(ctx, a);
+            record(ctx, 4);
+        } else {
+            record(ctx, 2);
+            record(ctx, 3);
+            record(ctx, 4);
+        }
+        check(cuda_check(ctx, cudaGetLastError(), "kernel launch"));
+
+        stats.n_pairs = P;
+        stats.n_segments = S;
+        stats.flops = 2.0 * (double)P * (double)lp.tile_w * (double)lp.n_c;
+        stats.bytes_contract = (double)nU * U->tile * dsize(U->dtype) + (V ? (double)nV * V->tile * dsize(V->dtype) : 0.0) +
+                               (double)S * lp.tile_w * dsize(o.out_dtype) + 8.0 * (double)P;
+        stats.path = path;
+        stats.launches = ctx->launches;
+        stats.timed = ctx->cur_ev != nullptr;
+        ctx->last = stats;
+        *out = R;
+        R = nullptr;
+        ctx->err.clear();
+    } catch (Oom &) {
+        st = fail(ctx, UCL_ERR_OOM, "device allocation failed");
+    } catch (Fail &f) {
+        st = f.st;
+    }
+    if (R) ucl_relation_destroy(R);
+    return st;
+}
+
+}  // extern "C"

@@ -1,0 +1,206 @@
+// internal.cuh -- declarations shared by the executor's translation units.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "ucl.h"
+
+namespace ucl {
+
+constexpr int kMaxCols = 15;     // key columns or tile dims of one operand
+constexpr int kMaxLow = 30;      // lower labels of one binary EinSum
+
+// Device status bits written by kernels (atomicOr into ctx->d_status).
+enum : uint32_t {
+    kStTimeout = 1u,     // a bounded wait ran out
+    kStBadIndex = 2u,    // an index failed its bounds check; the access was skipped
+    kStKeyRange = 4u,    // key outside [0, bound)
+    kStUnsorted = 8u,    // keys not strictly ascending
+    kStDupKey = 16u,     // two equal keys
+};
+
+// One key column copied into a bit field of a packed 64-bit key.
+struct KeyField {
+    int col;
+    int shift;
+    int bits;
+};
+
+// How to build one packed key from a relation's key row.
+struct KeyPack {
+    int nf;
+    KeyField f[kMaxCols];
+};
+
+// Unpacking of the packed output key into the output relation's columns.
+struct KeyUnpack {
+    int uw;
+    int shift[kMaxCols];
+    int bits[kMaxCols];
+};
+
+// Generic lower-label contraction of one pair (FFMA path):
+//   W[w] += sum_c U[offU(w) + cU(c)] * V[offV(w) + cV(c)]
+// w runs over W's lower labels (row-major, W's order), c over the lower
+// labels absent from W.
+struct LowerPlan {
+    int nw;
+    int w_ext[kMaxCols];
+    int w_su[kMaxCols];
+    int w_sv[kMaxCols];
+    int nc;
+    int c_ext[kMaxLow];
+    int c_su[kMaxLow];
+    int c_sv[kMaxLow];
+    int64_t tile_u, tile_v, tile_w, n_c;
+};
+
+// tcgen05 contraction shape: D[M x N] += A[M x K] * B[K x N] per pair, with
+// D = the output tile up to a transpose.
+struct TcPlan {
+    int a_is_u;          // A operand tiles come from U (else from V)
+    int M, N, K;         // M = 128 * m_blocks
+    int m_blocks;
+    int a_kmajor;        // A tile rows run over M (K contiguous) if 1, rows over K if 0
+    int b_kmajor;        // B tile rows run over N (K contiguous) if 1, rows over K if 0
+    int64_t sWm, sWn;    // output tile strides of the M and N indices
+};
+
+// Partition of the pair list into G contiguous units (one CTA each).
+struct Units {
+    int64_t P;
+    int G;
+    __host__ __device__ int64_t begin(int u) const { return P * u / G; }
+};
+
+// Stream-ordered bump allocator over blocks obtained from the context hooks.
+struct Arena {
+    struct Block {
+        char *ptr;
+        size_t size;
+    };
+    std::vector<Block> blocks;
+    size_t used = 0;   // bytes used in the last block
+    size_t total() const {
+        size_t t = 0;
+        for (auto &b : blocks) t += b.size;
+        return t;
+    }
+};
+
+}  // namespace ucl
+
+struct ucl_ctx {
+    int device = 0;
+    cudaStream_t stream = nullptr;
+    ucl_alloc_fn alloc = nullptr;
+    ucl_free_fn free_fn = nullptr;
+    void *user = nullptr;
+    int sm_count = 0;
+    ucl::Arena arena;
+    uint32_t *d_status = nullptr;   // [0] sticky error bits, [1] validation flags
+    int64_t *h_pinned = nullptr;    // pinned host scratch for sizing syncs (8 words)
+    int timing = 0;
+    // CUDA events of timed calls: UCL_NSTAGES + 1 per ucl_einsum, reused
+    // after ucl_ctx_timings(..., reset = 1)
+    std::vector<cudaEvent_t> ev_pool;
+    int ev_calls = 0;      // calls recorded since the last reset
+    cudaEvent_t *cur_ev = nullptr;
+    int launches = 0;
+    ucl_stats last{};
+    std::string err;
+    int live_rels = 0;
+};
+
+struct ucl_rel {
+    ucl_ctx *ctx = nullptr;
+    int64_t n = 0;
+    int u = 0, r = 0;
+    int64_t bounds[ucl::kMaxCols] = {};
+    int64_t shape[ucl::kMaxCols] = {};
+    ucl_dtype dtype = UCL_F32;
+    int64_t tile = 1;            // elements per tile
+    int32_t *keys = nullptr;     // device [n, u]
+    void *tiles = nullptr;       // device [n, tile]
+    void *own_block = nullptr;   // library-owned allocation (keys + tiles), or NULL
+    size_t own_bytes = 0;
+    int sorted = 0;              // keys strictly ascending lexicographically
+    int key_bits = 0;            // sum of column bit widths
+};
+
+namespace ucl {
+
+// ---- context helpers (api.cu)
+void *ctx_alloc(ucl_ctx *ctx, size_t bytes);
+void ctx_free(ucl_ctx *ctx, void *p, size_t bytes);
+void *ws_get(ucl_ctx *ctx, size_t bytes);   // arena workspace, valid until the next arena reset
+ucl_status fail(ucl_ctx *ctx, ucl_status st, const std::string &msg);
+ucl_status cuda_check(ucl_ctx *ctx, cudaError_t e, const char *what);
+int bit_width(int64_t bound);   // bits to store values in [0, bound)
+
+// ---- key stage (keys.cu)
+// Pack each row of keys[n, u] into a 64-bit key; optional second packing.
+void launch_pack(ucl_ctx *ctx, const int32_t *keys, int u, int64_t n, KeyPack a, uint64_t *out_a, KeyPack b,
+                 uint64_t *out_b);
+// Validate keys of a relation: range check against bounds and strict ascending
+// order of the packed full key (sets kStKeyRange / kStUnsorted).
+void launch_check_keys(ucl_ctx *ctx, const int32_t *keys, int u, int64_t n, const int64_t *bounds, KeyPack full,
+                       uint64_t *packed_out);
+// Adjacent-equal check on a sorted array (sets kStDupKey).
+void launch_check_dups(ucl_ctx *ctx, const uint64_t *sorted_keys, int64_t n);
+// Stable LSD radix sort of (key, value) by the low `bits` bits of key.
+// kin/vin and kalt/valt are ping-pong buffers; returns which holds the result
+// (0: kin/vin, 1: kalt/valt).  vin may be NULL (keys only).
+int radix_sort(ucl_ctx *ctx, uint64_t *kin, uint64_t *vin, uint64_t *kalt, uint64_t *valt, int64_t n, int bits);
+// Exclusive scan of n int64 values; writes total to *total_dev if non-NULL.
+void scan_i64(ucl_ctx *ctx, const int64_t *in, int64_t *out, int64_t n, int64_t *total_dev);
+// iota into u64
+void launch_iota(ucl_ctx *ctx, uint64_t *out, int64_t n);
+// Join count: for each U row i (sorted join keys jku), the matching range of V.
+void launch_join_count(ucl_ctx *ctx, const uint64_t *jku, int64_t nu, const uint64_t *jkv, int64_t nv,
+                       int64_t *cnt, uint32_t *lo);
+// Expand pairs: pk = koU[u] | koV[v], pv = (u << 32) | v.
+void launch_expand(ucl_ctx *ctx, const int64_t *off, int64_t nu, const uint32_t *lo, const uint64_t *perm_u,
+                   const uint64_t *perm_v, const uint64_t *ko_u, const uint64_t *ko_v, int64_t P, uint64_t *pk,
+                   uint64_t *pv);
+// Unary: pairs = tuples of U.
+void launch_unary_pairs(ucl_ctx *ctx, const uint64_t *ko_u, int64_t n, uint64_t *pk, uint64_t *pv);
+// Segment heads (flag[p] = 1 where the key changes), as int64 for the scan.
+void launch_heads(ucl_ctx *ctx, const uint64_t *pk, int64_t P, int64_t *flag);
+// Segment starts, output keys, pair index arrays.
+void launch_segments(ucl_ctx *ctx, const uint64_t *pk, const uint64_t *pv, const int64_t *seg_excl, int64_t P,
+                     int64_t S, KeyUnpack un, int32_t *out_keys, int64_t *seg_start, uint32_t *pu, uint32_t *pvi);
+
+// ---- contraction (contract_simt.cu / contract_tc.cu)
+struct ContractArgs {
+    const void *U;
+    const void *V;         // NULL for a unary EinSum
+    ucl_dtype du, dv;
+    int64_t nU, nV;
+    const uint32_t *pu;    // [P] U tuple of each pair
+    const uint32_t *pv;    // [P] V tuple of each pair
+    const int64_t *seg_start;  // [S + 1]
+    int64_t S;
+    Units units;
+    void *out;             // [S, tile_w]
+    ucl_dtype dout;
+    int epi;
+    float scale;
+    float *partials;       // [G, 2, tile_w]
+    int64_t tile_w;
+};
+void launch_contract_simt(ucl_ctx *ctx, const ContractArgs &a, const LowerPlan &lp);
+void launch_fixup(ucl_ctx *ctx, const ContractArgs &a);
+// tcgen05 path; returns false (nothing launched) if the shapes do not fit.
+bool tc_supported(const TcPlan &tp, const ContractArgs &a, std::string *why);
+ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan &tp, const ucl_rel *ra,
+                              const ucl_rel *rb);
+int tc_units(ucl_ctx *ctx, const TcPlan &tp, int64_t P);
+
+}  // namespace ucl

@@ -1,0 +1,406 @@
+// keys.cu -- the relational half of one UCL EinSum on the GPU: key packing,
+// key validation, LSD radix sort, the merge-join (count + expand) and the
+// group-by segmentation of the pair list (paper Sec. 5, the NATURAL JOIN and
+// GROUP BY of the TR-SQL template).
+//
+// Every kernel is a plain grid-stride or reduce-then-scan kernel: no kernel
+// waits on another CTA, so nothing here can spin.
+#include "internal.cuh"
+
+namespace ucl {
+
+namespace {
+
+constexpr int kThreads = 256;
+
+int grid_for(ucl_ctx *ctx, int64_t n, int per_thread = 1) {
+    int64_t want = (n + (int64_t)kThreads * per_thread - 1) / ((int64_t)kThreads * per_thread);
+    int64_t cap = (int64_t)ctx->sm_count * 8;
+    if (want < 1) want = 1;
+    return (int)(want < cap ? want : cap);
+}
+
+__device__ __forceinline__ uint64_t pack_row(const int32_t *row, const KeyPack &kp) {
+    uint64_t k = 0;
+    for (int i = 0; i < kp.nf; ++i) {
+        uint64_t v = (uint32_t)row[kp.f[i].col];
+        k |= v << kp.f[i].shift;
+    }
+    return k;
+}
+
+__global__ void pack_kernel(const int32_t *__restrict__ keys, int u, int64_t n, KeyPack a, uint64_t *out_a,
+                            KeyPack b, uint64_t *out_b) {
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const int32_t *row = keys + i * u;
+        if (out_a) out_a[i] = pack_row(row, a);
+        if (out_b) out_b[i] = pack_row(row, b);
+    }
+}
+
+struct Bounds {
+    int64_t b[kMaxCols];
+};
+
+__global__ void check_keys_kernel(const int32_t *__restrict__ keys, int u, int64_t n, Bounds bd, KeyPack full,
+                                  uint64_t *packed, uint32_t *status) {
+    uint32_t st = 0;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const int32_t *row = keys + i * u;
+        for (int c = 0; c < u; ++c) {
+            int32_t v = row[c];
+            if (v < 0 || (int64_t)v >= bd.b[c]) st |= kStKeyRange;
+        }
+        uint64_t k = pack_row(row, full);
+        if (i > 0 && pack_row(row - u, full) >= k) st |= kStUnsorted;
+        if (packed) packed[i] = k;
+    }
+    if (st) atomicOr(status, st);
+}
+
+__global__ void check_dups_kernel(const uint64_t *__restrict__ k, int64_t n, uint32_t *status) {
+    for (int64_t i = 1 + blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        if (k[i] == k[i - 1]) {
+            atomicOr(status, kStDupKey);
+            return;
+        }
+}
+
+__global__ void iota_kernel(uint64_t *out, int64_t n) {
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        out[i] = (uint64_t)i;
+}
+
+// ------------------------------------------------------------------ scan
+
+constexpr int kScanThreads = 512;
+constexpr int kScanItems = 8;
+constexpr int kScanTile = kScanThreads * kScanItems;
+
+template <typename T>
+__device__ T block_excl_scan(T v, T *total) {
+    __shared__ T warp_sums[kScanThreads / 32];
+    int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    T x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        T y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) warp_sums[w] = x;
+    __syncthreads();
+    if (w == 0) {
+        T s = lane < kScanThreads / 32 ? warp_sums[lane] : T(0);
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            T y = __shfl_up_sync(0xffffffffu, s, o);
+            if (lane >= o) s += y;
+        }
+        if (lane < kScanThreads / 32) warp_sums[lane] = s;
+    }
+    __syncthreads();
+    T before = (w > 0 ? warp_sums[w - 1] : T(0)) + x - v;
+    *total = warp_sums[kScanThreads / 32 - 1];
+    __syncthreads();
+    return before;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kScanThreads) scan_reduce_kernel(const T *__restrict__ in, int64_t n, T *sums) {
+    int64_t base = (int64_t)blockIdx.x * kScanTile + (int64_t)threadIdx.x * kScanItems;
+    T s = 0;
+#pragma unroll
+    for (int j = 0; j < kScanItems; ++j)
+        if (base + j < n) s += in[base + j];
+    T tot;
+    block_excl_scan<T>(s, &tot);
+    if (threadIdx.x == 0) sums[blockIdx.x] = tot;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kScanThreads) scan_tile_kernel(const T *in, T *out, int64_t n, const T *offsets,
+                                                                 T *total_dev) {
+    int64_t base = (int64_t)blockIdx.x * kScanTile + (int64_t)threadIdx.x * kScanItems;
+    T v[kScanItems];
+    T s = 0;
+#pragma unroll
+    for (int j = 0; j < kScanItems; ++j) {
+        v[j] = base + j < n ? in[base + j] : T(0);
+        s += v[j];
+    }
+    T tot;
+    T run = block_excl_scan<T>(s, &tot) + (offsets ? offsets[blockIdx.x] : T(0));
+#pragma unroll
+    for (int j = 0; j < kScanItems; ++j) {
+        if (base + j < n) out[base + j] = run;
+        run += v[j];
+    }
+    if (total_dev && blockIdx.x == gridDim.x - 1 && threadIdx.x == kScanThreads - 1) *total_dev = run;
+}
+
+template <typename T>
+void scan_excl(ucl_ctx *ctx, const T *in, T *out, int64_t n, T *total_dev) {
+    if (n <= 0) {
+        if (total_dev) cudaMemsetAsync(total_dev, 0, sizeof(T), ctx->stream);
+        return;
+    }
+    int64_t nb = (n + kScanTile - 1) / kScanTile;
+    T *sums = nullptr;
+    if (nb > 1) {
+        sums = (T *)ws_get(ctx, sizeof(T) * nb);
+        scan_reduce_kernel<T><<<(unsigned)nb, kScanThreads, 0, ctx->stream>>>(in, n, sums);
+        ctx->launches++;
+        scan_excl<T>(ctx, sums, sums, nb, nullptr);
+    }
+    scan_tile_kernel<T><<<(unsigned)nb, kScanThreads, 0, ctx->stream>>>(in, out, n, sums, total_dev);
+    ctx->launches++;
+}
+
+// ------------------------------------------------------------ radix sort
+
+constexpr int kRadixBits = 8;
+constexpr int kBuckets = 1 << kRadixBits;
+constexpr int kSortThreads = 256;
+constexpr int kSortItems = 16;
+constexpr int kSortTile = kSortThreads * kSortItems;
+
+__global__ void __launch_bounds__(kSortThreads) radix_hist_kernel(const uint64_t *__restrict__ k, int64_t n,
+                                                                  int shift, uint32_t *hist, int nblocks) {
+    __shared__ uint32_t h[kBuckets];
+    h[threadIdx.x] = 0;
+    __syncthreads();
+    int64_t start = (int64_t)blockIdx.x * kSortTile;
+    int64_t end = start + kSortTile < n ? start + kSortTile : n;
+    for (int64_t i = start + threadIdx.x; i < end; i += kSortThreads)
+        atomicAdd(&h[(uint32_t)(k[i] >> shift) & (kBuckets - 1)], 1u);
+    __syncthreads();
+    hist[(int64_t)threadIdx.x * nblocks + blockIdx.x] = h[threadIdx.x];
+}
+
+// Stable scatter: items of the block are ranked in index order, one round of
+// 256 at a time; within a warp equal digits are ranked by __match_any_sync,
+// across warps by a per-digit prefix over the warps' counts.
+__global__ void __launch_bounds__(kSortThreads) radix_scatter_kernel(const uint64_t *__restrict__ kin,
+                                                                     const uint64_t *__restrict__ vin,
+                                                                     uint64_t *__restrict__ kout,
+                                                                     uint64_t *__restrict__ vout, int64_t n,
+                                                                     int shift, const uint32_t *__restrict__ offs,
+                                                                     int nblocks) {
+    constexpr int kWarps = kSortThreads / 32;
+    __shared__ uint32_t base[kBuckets];
+    __shared__ uint32_t wcnt[kWarps][kBuckets];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    base[tid] = offs[(int64_t)tid * nblocks + blockIdx.x];
+    int64_t start = (int64_t)blockIdx.x * kSortTile;
+    int64_t end = start + kSortTile < n ? start + kSortTile : n;
+    for (int64_t r = start; r < end; r += kSortThreads) {
+        for (int i = tid; i < kWarps * kBuckets; i += kSortThreads) (&wcnt[0][0])[i] = 0;
+        __syncthreads();
+        int64_t i = r + tid;
+        bool valid = i < end;
+        uint64_t key = valid ? kin[i] : 0;
+        uint64_t val = (valid && vin) ? vin[i] : 0;
+        uint32_t d = valid ? (uint32_t)(key >> shift) & (kBuckets - 1) : (uint32_t)kBuckets;
+        uint32_t peers = __match_any_sync(0xffffffffu, d);
+        uint32_t below = peers & ((1u << lane) - 1u);
+        if (valid && below == 0) wcnt[warp][d] = __popc(peers);
+        __syncthreads();
+        {
+            uint32_t run = base[tid];
+#pragma unroll
+            for (int w = 0; w < kWarps; ++w) {
+                uint32_t c = wcnt[w][tid];
+                wcnt[w][tid] = run;
+                run += c;
+            }
+            base[tid] = run;
+        }
+        __syncthreads();
+        if (valid) {
+            uint32_t dst = wcnt[warp][d] + __popc(below);
+            kout[dst] = key;
+            if (vin) vout[dst] = val;
+        }
+        __syncthreads();
+    }
+}
+
+// ------------------------------------------------------------------ join
+
+__device__ __forceinline__ int64_t lower_bound_u64(const uint64_t *a, int64_t n, uint64_t k) {
+    int64_t lo = 0, hi = n;
+    while (lo < hi) {
+        int64_t mid = (lo + hi) >> 1;
+        if (a[mid] < k) lo = mid + 1; else hi = mid;
+    }
+    return lo;
+}
+
+__device__ __forceinline__ int64_t upper_bound_u64(const uint64_t *a, int64_t n, uint64_t k) {
+    int64_t lo = 0, hi = n;
+    while (lo < hi) {
+        int64_t mid = (lo + hi) >> 1;
+        if (a[mid] <= k) lo = mid + 1; else hi = mid;
+    }
+    return lo;
+}
+
+__global__ void join_count_kernel(const uint64_t *__restrict__ jku, int64_t nu, const uint64_t *__restrict__ jkv,
+                                  int64_t nv, int64_t *cnt, uint32_t *lo) {
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < nu; i += (int64_t)gridDim.x * blockDim.x) {
+        int64_t l = 0, h = nv;
+        if (jkv) {
+            uint64_t k = jku[i];
+            l = lower_bound_u64(jkv, nv, k);
+            h = upper_bound_u64(jkv + l, nv - l, k) + l;
+        }
+        cnt[i] = h - l;
+        lo[i] = (uint32_t)l;
+    }
+}
+
+__global__ void expand_kernel(const int64_t *__restrict__ off, int64_t nu, const uint32_t *__restrict__ lo,
+                              const uint64_t *__restrict__ perm_u, const uint64_t *__restrict__ perm_v,
+                              const uint64_t *__restrict__ ko_u, const uint64_t *__restrict__ ko_v, int64_t P,
+                              uint64_t *pk, uint64_t *pv) {
+    for (int64_t p = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; p < P; p += (int64_t)gridDim.x * blockDim.x) {
+        // last row i with off[i] <= p
+        int64_t a = 0, b = nu;
+        while (a < b) {
+            int64_t mid = (a + b) >> 1;
+            if (off[mid] <= p) a = mid + 1; else b = mid;
+        }
+        int64_t i = a - 1;
+        int64_t vpos = (int64_t)lo[i] + (p - off[i]);
+        uint64_t u = perm_u ? perm_u[i] : (uint64_t)i;
+        uint64_t v = perm_v ? perm_v[vpos] : (uint64_t)vpos;
+        pk[p] = ko_u[u] | (ko_v ? ko_v[v] : 0ull);
+        pv[p] = (u << 32) | v;
+    }
+}
+
+__global__ void unary_pairs_kernel(const uint64_t *__restrict__ ko_u, int64_t n, uint64_t *pk, uint64_t *pv) {
+    for (int64_t p = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; p < n; p += (int64_t)gridDim.x * blockDim.x) {
+        pk[p] = ko_u[p];
+        pv[p] = (uint64_t)p << 32;
+    }
+}
+
+__global__ void heads_kernel(const uint64_t *__restrict__ pk, int64_t P, int64_t *flag) {
+    for (int64_t p = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; p < P; p += (int64_t)gridDim.x * blockDim.x)
+        flag[p] = (p == 0 || pk[p] != pk[p - 1]) ? 1 : 0;
+}
+
+__global__ void segments_kernel(const uint64_t *__restrict__ pk, const uint64_t *__restrict__ pv,
+                                const int64_t *__restrict__ seg_excl, int64_t P, int64_t S, KeyUnpack un,
+                                int32_t *out_keys, int64_t *seg_start, uint32_t *pu, uint32_t *pvi) {
+    for (int64_t p = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; p < P; p += (int64_t)gridDim.x * blockDim.x) {
+        uint64_t v = pv[p];
+        pu[p] = (uint32_t)(v >> 32);
+        pvi[p] = (uint32_t)v;
+        uint64_t k = pk[p];
+        if (p == 0 || k != pk[p - 1]) {
+            int64_t s = seg_excl[p];
+            seg_start[s] = p;
+            for (int c = 0; c < un.uw; ++c) {
+                uint64_t mask = un.bits[c] ? ((~0ull) >> (64 - un.bits[c])) : 0ull;
+                out_keys[s * un.uw + c] = (int32_t)((k >> un.shift[c]) & mask);
+            }
+        }
+        if (p == 0) seg_start[S] = P;
+    }
+}
+
+}  // namespace
+
+// ------------------------------------------------------------ launchers
+
+void launch_pack(ucl_ctx *ctx, const int32_t *keys, int u, int64_t n, KeyPack a, uint64_t *out_a, KeyPack b,
+                 uint64_t *out_b) {
+    if (n <= 0) return;
+    pack_kernel<<<grid_for(ctx, n), kThreads, 0, ctx->stream>>>(keys, u, n, a, out_a, b, out_b);
+    ctx->launches++;
+}
+
+void launch_check_keys(ucl_ctx *ctx, const int32_t *keys, int u, int64_t n, const int64_t *bounds, KeyPack full,
+                       uint64_t *packed_out) {
+    if (n <= 0) return;
+    Bounds bd{};
+    for (int c = 0; c < u; ++c) bd.b[c] = bounds[c];
+    check_keys_kernel<<<grid_for(ctx, n), kThreads, 0, ctx->stream>>>(keys, u, n, bd, full, packed_out,
+                                                                      ctx->d_status + 1);
+    ctx->launches++;
+}
+
+void launch_check_dups(ucl_ctx *ctx, const uint64_t *sorted_keys, int64_t n) {
+    if (n <= 1) return;
+    check_dups_kernel<<<grid_for(ctx, n), kThreads, 0, ctx->stream>>>(sorted_keys, n, ctx->d_status + 1);
+    ctx->launches++;
+}
+
+void launch_iota(ucl_ctx *ctx, uint64_t *out, int64_t n) {
+    if (n <= 0) return;
+    iota_kernel<<<grid_for(ctx, n), kThreads, 0, ctx->stream>>>(out, n);
+    ctx->launches++;
+}
+
+void scan_i64(ucl_ctx *ctx, const int64_t *in, int64_t *out, int64_t n, int64_t *total_dev) {
+    scan_excl<int64_t>(ctx, in, out, n, total_dev);
+}
+
+int radix_sort(ucl_ctx *ctx, uint64_t *kin, uint64_t *vin, uint64_t *kalt, uint64_t *valt, int64_t n, int bits) {
+    if (bits <= 0 || n <= 1) return 0;
+    int nblocks = (int)((n + kSortTile - 1) / kSortTile);
+    uint32_t *hist = (uint32_t *)ws_get(ctx, sizeof(uint32_t) * (size_t)kBuckets * nblocks);
+    uint64_t *ks = kin, *vs = vin, *kd = kalt, *vd = valt;
+    int which = 0;
+    for (int shift = 0; shift < bits; shift += kRadixBits) {
+        radix_hist_kernel<<<nblocks, kSortThreads, 0, ctx->stream>>>(ks, n, shift, hist, nblocks);
+        ctx->launches++;
+        scan_excl<uint32_t>(ctx, hist, hist, (int64_t)kBuckets * nblocks, nullptr);
+        radix_scatter_kernel<<<nblocks, kSortThreads, 0, ctx->stream>>>(ks, vs, kd, vd, n, shift, hist, nblocks);
+        ctx->launches++;
+        uint64_t *t = ks; ks = kd; kd = t;
+        t = vs; vs = vd; vd = t;
+        which ^= 1;
+    }
+    return which;
+}
+
+void launch_join_count(ucl_ctx *ctx, const uint64_t *jku, int64_t nu, const uint64_t *jkv, int64_t nv,
+                       int64_t *cnt, uint32_t *lo) {
+    if (nu <= 0) return;
+    join_count_kernel<<<grid_for(ctx, nu), kThreads, 0, ctx->stream>>>(jku, nu, jkv, nv, cnt, lo);
+    ctx->launches++;
+}
+
+void launch_expand(ucl_ctx *ctx, const int64_t *off, int64_t nu, const uint32_t *lo, const uint64_t *perm_u,
+                   const uint64_t *perm_v, const uint64_t *ko_u, const uint64_t *ko_v, int64_t P, uint64_t *pk,
+                   uint64_t *pv) {
+    if (P <= 0) return;
+    expand_kernel<<<grid_for(ctx, P), kThreads, 0, ctx->stream>>>(off, nu, lo, perm_u, perm_v, ko_u, ko_v, P, pk,
+                                                                  pv);
+    ctx->launches++;
+}
+
+void launch_unary_pairs(ucl_ctx *ctx, const uint64_t *ko_u, int64_t n, uint64_t *pk, uint64_t *pv) {
+    if (n <= 0) return;
+    unary_pairs_kernel<<<grid_for(ctx, n), kThreads, 0, ctx->stream>>>(ko_u, n, pk, pv);
+    ctx->launches++;
+}
+
+void launch_heads(ucl_ctx *ctx, const uint64_t *pk, int64_t P, int64_t *flag) {
+    if (P <= 0) return;
+    heads_kernel<<<grid_for(ctx, P), kThreads, 0, ctx->stream>>>(pk, P, flag);
+    ctx->launches++;
+}
+
+void launch_segments(ucl_ctx *ctx, const uint64_t *pk, const uint64_t *pv, const int64_t *seg_excl, int64_t P,
+                     int64_t S, KeyUnpack un, int32_t *out_keys, int64_t *seg_start, uint32_t *pu, uint32_t *pvi) {
+    if (P <= 0) return;
+    segments_kernel<<<grid_for(ctx, P), kThreads, 0, ctx->stream>>>(pk, pv, seg_excl, P, S, un, out_keys,
+                                                                    seg_start, pu, pvi);
+    ctx->launches++;
+}
+
+}  // namespace ucl

@@ -1,0 +1,227 @@
+"""Python binding of the UCL EinSum executor: argument marshalling only.
+
+Every step of an EinSum runs inside libucl.so on the GPU; this module turns
+torch tensors into pointers and sizes, calls the C ABI (include/ucl.h) and
+wraps the returned handles.  PyTorch provides device memory (its caching
+allocator backs the executor's workspace and outputs) and the stream.
+"""
+from __future__ import annotations
+
+import ctypes
+
+import numpy as np
+import torch
+
+from . import _lib
+
+BF16, F32 = 0, 1
+_DTYPES = {torch.bfloat16: BF16, torch.float32: F32}
+_TORCH = {BF16: torch.bfloat16, F32: torch.float32}
+EPI = {"none": 0, "relu": 1}
+PATH = {"auto": 0, "simt": 1, "tc": 2}
+OUT = {"bf16": BF16, "f32": F32, torch.bfloat16: BF16, torch.float32: F32}
+MEM_BORROW, MEM_DEVICE_COPY, MEM_HOST_COPY = 0, 1, 2
+
+
+class UclError(RuntimeError):
+    def __init__(self, status: int, detail: str = ""):
+        self.status = status
+        self.name = _lib.STATUS_NAMES.get(status, f"status {status}")
+        self.detail = detail
+        super().__init__(f"{self.name}: {detail}" if detail else self.name)
+
+
+class _DevArray:
+    """Minimal __cuda_array_interface__ holder for a zero-copy torch view."""
+
+    def __init__(self, ptr, shape, typestr, owner):
+        self.__cuda_array_interface__ = {
+            "shape": tuple(int(s) for s in shape),
+            "typestr": typestr,
+            "data": (int(ptr), False),
+            "version": 3,
+            "strides": None,
+        }
+        self._owner = owner
+
+
+class Context:
+    """An executor context bound to one device and one CUDA stream."""
+
+    def __init__(self, device: int = 0, stream: torch.cuda.Stream | None = None, torch_allocator: bool = True):
+        self.lib = _lib.load()
+        self.device = int(device)
+        self.stream = stream if stream is not None else torch.cuda.current_stream(self.device)
+        h = ctypes.c_void_p()
+        if torch_allocator:
+            dev, s = self.device, self.stream.cuda_stream
+
+            def _alloc(nbytes, user):
+                try:
+                    return torch.cuda.caching_allocator_alloc(int(nbytes), dev, s)
+                except Exception:  # noqa: BLE001 -- reported to C as NULL -> UCL_ERR_OOM
+                    return None
+
+            def _free(ptr, nbytes, user):
+                torch.cuda.caching_allocator_delete(int(ptr))
+
+            self._alloc_cb = _lib.ALLOC_FN(_alloc)
+            self._free_cb = _lib.FREE_FN(_free)
+        else:
+            self._alloc_cb = ctypes.cast(None, _lib.ALLOC_FN)
+            self._free_cb = ctypes.cast(None, _lib.FREE_FN)
+        self._check(self.lib.ucl_ctx_create(self.device, ctypes.c_void_p(self.stream.cuda_stream), self._alloc_cb,
+                                            self._free_cb, None, ctypes.byref(h)), ctx=None)
+        self.handle = h
+        self._rels = set()
+
+    # ------------------------------------------------------------ helpers
+    def _check(self, st, ctx="self"):
+        if st != 0:
+            detail = ""
+            if ctx == "self" and getattr(self, "handle", None):
+                detail = (self.lib.ucl_last_error(self.handle) or b"").decode()
+            raise UclError(st, detail)
+
+    def close(self):
+        if getattr(self, "handle", None):
+            for r in list(self._rels):
+                r.destroy()
+            self.lib.ucl_ctx_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:  # noqa: BLE001
+            pass
+
+    def synchronize(self):
+        self._check(self.lib.ucl_ctx_synchronize(self.handle))
+
+    def set_timing(self, on: bool):
+        self._check(self.lib.ucl_ctx_set_timing(self.handle, 1 if on else 0))
+
+    def timings(self, reset: bool = True, max_calls: int = 4096):
+        """Per-call stage times [calls, 4] (ms) of timed einsums since the last reset."""
+        buf = (ctypes.c_float * (max_calls * _lib.UCL_NSTAGES))()
+        n = ctypes.c_int()
+        self._check(self.lib.ucl_ctx_timings(self.handle, buf, max_calls, ctypes.byref(n), 1 if reset else 0))
+        k = min(n.value, max_calls)
+        return np.frombuffer(buf, dtype=np.float32, count=k * _lib.UCL_NSTAGES).reshape(k, _lib.UCL_NSTAGES).copy()
+
+    def last_stats(self) -> dict:
+        st = _lib.Stats()
+        self._check(self.lib.ucl_get_last_stats(self.handle, ctypes.byref(st)))
+        return {
+            "n_pairs": st.n_pairs,
+            "n_segments": st.n_segments,
+            "flops": st.flops,
+            "bytes_contract": st.bytes_contract,
+            "path": {1: "simt", 2: "tc"}.get(st.path, "none"),
+            "launches": st.launches,
+            "stage_ms": list(st.stage_ms) if st.timed else None,
+        }
+
+    # ---------------------------------------------------------- relations
+    def relation(self, keys, bounds, tiles, *, copy: bool = False) -> "Relation":
+        """Tensor-relation from device tensors: keys int32 [n, u], tiles
+        [n, *shape] bf16/fp32.  Borrowed (zero copy) unless copy=True."""
+        keys = torch.as_tensor(keys)
+        if keys.dtype != torch.int32:
+            raise TypeError("keys must be int32")
+        if tiles.dtype not in _DTYPES:
+            raise TypeError("tiles must be bfloat16 or float32")
+        n = tiles.shape[0]
+        bounds = [int(b) for b in bounds]
+        keys = keys.reshape(n, len(bounds))
+        host = keys.device.type == "cpu"
+        if host != (tiles.device.type == "cpu"):
+            raise ValueError("keys and tiles must both be on the host or both on the device")
+        if not host and (keys.device.index != self.device or tiles.device.index != self.device):
+            raise ValueError("tensors live on another device than the context")
+        keys = keys.contiguous()
+        tiles = tiles.contiguous()
+        mem = MEM_HOST_COPY if host else (MEM_DEVICE_COPY if copy else MEM_BORROW)
+        shape = list(tiles.shape[1:])
+        b_arr = (ctypes.c_int64 * max(1, len(bounds)))(*bounds)
+        s_arr = (ctypes.c_int64 * max(1, len(shape)))(*shape)
+        h = ctypes.c_void_p()
+        self._check(self.lib.ucl_relation_create(
+            self.handle, n, len(bounds), ctypes.c_void_p(keys.data_ptr() if keys.numel() else 0), b_arr,
+            len(shape), s_arr, _DTYPES[tiles.dtype], ctypes.c_void_p(tiles.data_ptr() if tiles.numel() else 0),
+            mem, ctypes.byref(h)))
+        rel = Relation(self, h, borrowed=(keys, tiles) if mem == MEM_BORROW else None)
+        return rel
+
+    def einsum(self, spec: str, *rels: "Relation", out_dtype="f32", epi="none", scale: float = 1.0,
+               path="auto") -> "Relation":
+        """Evaluate one UCL EinSum (see include/ucl.h for the grammar)."""
+        opts = _lib.EinsumOpts(OUT[out_dtype], EPI[epi], float(scale), PATH[path])
+        arr = (ctypes.c_void_p * len(rels))(*[r.handle for r in rels])
+        h = ctypes.c_void_p()
+        self._check(self.lib.ucl_einsum(self.handle, spec.encode(), len(rels), arr, ctypes.byref(opts),
+                                        ctypes.byref(h)))
+        return Relation(self, h)
+
+
+class Relation:
+    """Handle of a tensor-relation living on the GPU."""
+
+    def __init__(self, ctx: Context, handle: ctypes.c_void_p, borrowed=None):
+        self.ctx = ctx
+        self.handle = handle
+        self._borrowed = borrowed
+        n, u, r, dt = ctypes.c_int64(), ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+        kb = (ctypes.c_int64 * 16)()
+        ts = (ctypes.c_int64 * 16)()
+        ctx._check(ctx.lib.ucl_relation_info(handle, ctypes.byref(n), ctypes.byref(u), ctypes.byref(r), kb, ts,
+                                             ctypes.byref(dt)))
+        self.n, self.u, self.r = n.value, u.value, r.value
+        self.bounds = tuple(kb[i] for i in range(self.u))
+        self.shape = tuple(ts[i] for i in range(self.r))
+        self.dtype = _TORCH[dt.value]
+        ctx._rels.add(self)
+
+    def destroy(self):
+        if self.handle:
+            self.ctx.lib.ucl_relation_destroy(self.handle)
+            self.ctx._rels.discard(self)
+            self.handle = None
+            self._borrowed = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:  # noqa: BLE001
+            pass
+
+    def _ptrs(self):
+        k, t = ctypes.c_void_p(), ctypes.c_void_p()
+        self.ctx._check(self.ctx.lib.ucl_relation_data(self.handle, ctypes.byref(k), ctypes.byref(t)))
+        return k.value or 0, t.value or 0
+
+    def device_tensors(self):
+        """Zero-copy torch views (keys int32 [n, u], tiles [n, *shape]) of the
+        relation's device buffers; valid while the relation lives."""
+        kp, tp = self._ptrs()
+        dev = torch.device("cuda", self.ctx.device)
+        if self.n == 0:
+            return (torch.zeros((0, self.u), dtype=torch.int32, device=dev),
+                    torch.zeros((0,) + self.shape, dtype=self.dtype, device=dev))
+        keys = torch.as_tensor(_DevArray(kp, (self.n, self.u), "<i4", self), device=dev) if self.u else \
+            torch.zeros((self.n, 0), dtype=torch.int32, device=dev)
+        ts = "<i2" if self.dtype == torch.bfloat16 else "<f4"
+        tiles = torch.as_tensor(_DevArray(tp, (self.n,) + self.shape, ts, self), device=dev)
+        if self.dtype == torch.bfloat16:
+            tiles = tiles.view(torch.bfloat16)
+        return keys, tiles
+
+    def download(self):
+        """Copy to the host through the C ABI: (keys np.int32 [n, u], tiles torch CPU [n, *shape])."""
+        keys = np.zeros((self.n, self.u), dtype=np.int32)
+        tiles = torch.empty((self.n,) + self.shape, dtype=self.dtype)
+        self.ctx._check(self.ctx.lib.ucl_relation_download(
+            self.handle, ctypes.c_void_p(keys.ctypes.data if keys.size else 0),
+            ctypes.c_void_p(tiles.data_ptr() if tiles.numel() else 0)))
+        return keys, tiles

@@ -1,0 +1,282 @@
+"""GPU parity: the executor (through the C ABI) against the CPU oracle on the
+same seeded inputs.  Every test here needs a GB300 and the built library."""
+import itertools
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads
+from paper_2603_08957_gb300 import Context, UclError
+from tests.parity import TOL, assert_parity, gpu_rel, oracle_ref
+from tests.ucl_testutil import decompose, golden, random_sparse, ucl_operand
+
+pytestmark = pytest.mark.gpu
+
+GOLD = golden(os.path.join(os.path.dirname(__file__), "golden", "worked_example.txt"))
+
+
+@pytest.fixture(scope="module")
+def ctx():
+    c = Context(0)
+    yield c
+    c.close()
+
+
+def _bf16_exact(a):
+    """Round a float64 array to bf16 values (both sides then see the same inputs)."""
+    return torch.from_numpy(np.asarray(a)).to(torch.bfloat16).to(torch.float64).numpy()
+
+
+# ------------------------------------------------------ paper's worked example
+
+
+@pytest.mark.parametrize("path", ["simt", "auto"])
+def test_worked_example(ctx, path):
+    U, V = GOLD["U"], GOLD["V"]
+    relU = (np.array([[0], [2]], np.int32), (4,), torch.tensor(U[[0, 2]], dtype=torch.float32))
+    relV = (np.array([[0], [2]], np.int32), (4,), torch.tensor(V[:, [0, 2]].T.copy(), dtype=torch.float32))
+    out = ctx.einsum("Ij,jK->IK", gpu_rel(ctx, relU), gpu_rel(ctx, relV), path=path)
+    keys, tiles = out.download()
+    want = GOLD["W_scalars"]
+    assert keys.tolist() == want[:, :2].astype(int).tolist()
+    np.testing.assert_allclose(tiles.numpy(), want[:, 2], rtol=1e-6)
+    assert ctx.last_stats()["n_pairs"] == 4
+    vt = GOLD["V_relational_tuples"]
+    relU2 = (np.arange(4, dtype=np.int32)[:, None], (4,), torch.tensor(U.T.copy(), dtype=torch.float32))
+    relV2 = (vt[:, :2].astype(np.int32), (4, 4), torch.tensor(vt[:, 2], dtype=torch.float32))
+    out = ctx.einsum("iJ,JK->iK", gpu_rel(ctx, relU2), gpu_rel(ctx, relV2), path=path)
+    keys, tiles = out.download()
+    want = GOLD["W_colvec"]
+    assert keys[:, 0].tolist() == want[:, 0].astype(int).tolist()
+    np.testing.assert_allclose(tiles.numpy(), want[:, 1:], rtol=1e-6, atol=1e-7)
+    assert ctx.last_stats()["n_pairs"] == 6
+
+
+# ---------------------------------------------------------- random small specs
+
+SPECS = [
+    ("ij,jk->ik", {"i": 5, "j": 7, "k": 6}),
+    ("ij,jk->ki", {"i": 4, "j": 3, "k": 5}),
+    ("ijb,jbk->ik", {"i": 3, "j": 4, "b": 2, "k": 5}),
+    ("bij,bjk->bik", {"b": 3, "i": 4, "j": 5, "k": 2}),
+    ("ij,j->i", {"i": 6, "j": 5}),
+    ("i,j->ij", {"i": 5, "j": 4}),
+    ("ij,ij->i", {"i": 5, "j": 3}),
+    ("ijk->ki", {"i": 3, "j": 4, "k": 5}),
+]
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("spec,ext", SPECS)
+def test_random_splits(ctx, spec, ext, dtype):
+    rng = np.random.default_rng(abs(hash(spec)) % 2**31)
+    lhs, out = spec.split("->")
+    ops = lhs.split(",")
+    arrs = [random_sparse(rng, [ext[c] for c in op], density=0.6, block_axes=range(len(op))) for op in ops]
+    if dtype == torch.bfloat16:
+        arrs = [_bf16_exact(a) for a in arrs]
+    labels = sorted(ext)
+    subsets = [set(s) for k in range(len(labels) + 1) for s in itertools.combinations(labels, k)]
+    for promoted in subsets:
+        rels = [decompose(a, op, promoted) for op, a in zip(ops, arrs)]
+        rels = [(k, tuple(b), torch.from_numpy(t).to(dtype)) for k, b, t in rels]
+        uspec = ",".join(ucl_operand(op, promoted) for op in ops) + "->" + ucl_operand(out, promoted)
+        ref = oracle_ref(uspec, rels)
+        got = ctx.einsum(uspec, *[gpu_rel(ctx, r) for r in rels])
+        assert_parity(got, ref, dtype)
+
+
+# ------------------------------------------------------------------ workloads
+
+
+def test_blocksparse_fp32_full(ctx):
+    """Block-sparse fp32 matmul, 1024 x 1024 at 10% tile density times a dense
+    1024 x 256, 32 x 32 tiles, seed 0: the whole output checked."""
+    w = workloads.blocksparse_matmul(seed=0)
+    ref = oracle_ref(w["spec"], [w["A"], w["B"]])
+    out = ctx.einsum(w["spec"], gpu_rel(ctx, w["A"]), gpu_rel(ctx, w["B"]))
+    assert_parity(out, ref, torch.float32)
+    st = ctx.last_stats()
+    assert st["n_pairs"] == ref["n_pairs"] == 102 * 8
+
+
+def test_blocksparse_fp32_unsorted_inputs(ctx):
+    """Same workload with the tuples of both inputs shuffled: the sort path."""
+    w = workloads.blocksparse_matmul(seed=1)
+    rng = np.random.default_rng(0)
+    shuf = []
+    for k, b, t in (w["A"], w["B"]):
+        p = rng.permutation(len(k))
+        shuf.append((k[p], b, t[torch.from_numpy(p)]))
+    ref = oracle_ref(w["spec"], shuf)
+    out = ctx.einsum(w["spec"], gpu_rel(ctx, shuf[0]), gpu_rel(ctx, shuf[1]))
+    assert_parity(out, ref, torch.float32)
+
+
+@pytest.mark.parametrize("path", ["simt", "auto"])
+def test_gnn_chain_small(ctx, path):
+    """(X x Y)^T x Z on a 4096-vertex R-MAT graph, 64 x 64 tiles, bf16:
+    stage-local parity for both steps (the second step's oracle input is the
+    GPU's first-step output)."""
+    w = workloads.gnn_chain(seed=3, n=4096, degree=16)
+    X, Y, Z = (gpu_rel(ctx, w[k]) for k in ("X", "Y", "Z"))
+    T = ctx.einsum(w["spec1"], X, Y, out_dtype="bf16", path=path)
+    ref1 = oracle_ref(w["spec1"], [w["X"], w["Y"]])
+    assert_parity(T, ref1, torch.bfloat16)
+    keys_t, tiles_t = T.download()
+    out = ctx.einsum(w["spec2"], T, Z, path=path)
+    ref2 = oracle_ref(w["spec2"], [(keys_t, T.bounds, tiles_t), w["Z"]])
+    assert_parity(out, ref2, torch.bfloat16)
+
+
+def test_spgemm_small(ctx):
+    """Block-sparse x block-sparse, 128 x 128 bf16 tiles, band + uniform, fp32 out."""
+    w = workloads.spgemm(seed=2, n=8192, density=0.05)
+    ref = oracle_ref(w["spec"], [w["A"], w["B"]])
+    out = ctx.einsum(w["spec"], gpu_rel(ctx, w["A"]), gpu_rel(ctx, w["B"]))
+    assert_parity(out, ref, torch.bfloat16)
+
+
+def _sample_rows(n, k, seed, must=()):
+    rng = np.random.default_rng(seed)
+    pick = set(rng.choice(n, size=min(k, n), replace=False).tolist()) | set(int(m) for m in must)
+    return np.array(sorted(pick))
+
+
+def test_gnn_full_size_sampled(ctx):
+    """The full message-passing workload (100000 vertices, 1.6M R-MAT edges,
+    358k Y tiles): every output key checked, values checked on sampled keys
+    (including the largest segment) against the oracle with all their pairs."""
+    w = workloads.gnn_chain(seed=0, device="cuda")
+    X, Y, Z = (gpu_rel(ctx, w[k]) for k in ("X", "Y", "Z"))
+    T = ctx.einsum(w["spec1"], X, Y, out_dtype="bf16")
+    keys_t, _ = T.download()
+    ky = w["Y"][0]
+    want_keys = np.unique(ky[:, 1])[:, None].astype(np.int32)
+    assert np.array_equal(keys_t, want_keys)
+    biggest = np.argmax(np.bincount(ky[:, 1]))
+    sel = _sample_rows(len(keys_t), 24, 0, must=[int(np.searchsorted(want_keys[:, 0], biggest))])
+    sk = keys_t[sel]
+    ysel = np.isin(ky[:, 1], sk[:, 0])
+    yk = ky[ysel]
+    yt = workloads.adjacency_tiles_subset(w["edges"][0], w["edges"][1], w["n"], w["t"], yk)
+    ref = oracle_ref(w["spec1"], [w["X"], (yk, w["Y"][1], yt)], sample_keys=sk)
+    assert_parity(T, ref, torch.bfloat16, select=sel)
+
+
+def test_spgemm_full_size_sampled(ctx):
+    w = workloads.spgemm(seed=0)
+    out = ctx.einsum(w["spec"], gpu_rel(ctx, w["A"]), gpu_rel(ctx, w["B"]))
+    keys, _ = out.download()
+    ka, kb = w["A"][0], w["B"][0]
+    # full key set: (I, K) for every A(I, J), B(J, K)
+    want = set()
+    byJ = {}
+    for J, K in kb:
+        byJ.setdefault(int(J), []).append(int(K))
+    for I, J in ka:
+        for K in byJ.get(int(J), []):
+            want.add((int(I), K))
+    assert keys.tolist() == [list(k) for k in sorted(want)]
+    sel = _sample_rows(len(keys), 32, 1)
+    ref = oracle_ref(w["spec"], [w["A"], w["B"]], sample_keys=keys[sel])
+    assert_parity(out, ref, torch.bfloat16, select=sel)
+
+
+# ------------------------------------------------------------------ edge cases
+
+
+def test_empty_relation_and_empty_join(ctx):
+    e = (np.zeros((0, 1), np.int32), (4,), torch.zeros((0, 2, 3)))
+    f = (np.array([[1]], np.int32), (4,), torch.ones((1, 3, 2)))
+    out = ctx.einsum("Jij,Jjk->ik", gpu_rel(ctx, e), gpu_rel(ctx, f))
+    assert out.n == 0 and out.shape == (2, 2)
+    g = (np.array([[2]], np.int32), (4,), torch.ones((1, 2, 3)))
+    out = ctx.einsum("Jij,Jjk->Jik", gpu_rel(ctx, g), gpu_rel(ctx, f))
+    assert out.n == 0 and ctx.last_stats()["n_pairs"] == 0
+
+
+def test_one_segment_across_all_units(ctx):
+    """All pairs share one output key (a key-less output summed over J): the
+    segment is split across every work unit and reassembled by the fixup."""
+    rng = np.random.default_rng(4)
+    nJ = 3000
+    ka = np.arange(nJ, dtype=np.int32)[:, None]
+    A = (ka, (nJ,), torch.from_numpy(rng.standard_normal((nJ, 8, 5)).astype(np.float32)))
+    B = (ka.copy(), (nJ,), torch.from_numpy(rng.standard_normal((nJ, 5, 6)).astype(np.float32)))
+    ref = oracle_ref("Jij,Jjk->ik", [A, B])
+    out = ctx.einsum("Jij,Jjk->ik", gpu_rel(ctx, A), gpu_rel(ctx, B))
+    assert_parity(out, ref, torch.float32)
+
+
+def test_unary_relu_scale_bf16_out(ctx):
+    """Unary EinSum (Sec. 3's ReLU as a sum over the empty set, here also
+    summing an upper label), scale and relu after the sum, bf16 output."""
+    rng = np.random.default_rng(5)
+    k = np.array([(i, j) for i in range(6) for j in range(4) if (i + j) % 3], np.int32)
+    t = torch.from_numpy(rng.standard_normal((len(k), 3, 7)).astype(np.float32))
+    rel = (k, (6, 4), t)
+    ref = oracle_ref("IJab->Ib", [rel], epi="relu", scale=0.5)
+    out = ctx.einsum("IJab->Ib", gpu_rel(ctx, rel), epi="relu", scale=0.5, out_dtype="bf16")
+    assert_parity(out, ref, torch.float32, scale=0.5)
+
+
+def test_wide_keys_64_bits(ctx):
+    """Three key columns of 2^20 values each pack into 60 bits."""
+    rng = np.random.default_rng(6)
+    n = 500
+    kx = np.unique(rng.integers(0, 2**20, size=(n, 3)), axis=0).astype(np.int32)
+    ky = kx[rng.permutation(len(kx))[: len(kx) // 2]][:, [1, 2]]
+    ky = np.unique(ky, axis=0)
+    X = (kx, (2**20,) * 3, torch.from_numpy(rng.standard_normal((len(kx), 4)).astype(np.float32)))
+    Y = (ky, (2**20,) * 2, torch.from_numpy(rng.standard_normal((len(ky), 4)).astype(np.float32)))
+    ref = oracle_ref("IJKa,JKa->IK", [X, Y])
+    out = ctx.einsum("IJKa,JKa->IK", gpu_rel(ctx, X), gpu_rel(ctx, Y))
+    assert_parity(out, ref, torch.float32)
+
+
+def test_host_copy_and_download(ctx):
+    w = workloads.blocksparse_matmul(seed=2)
+    ka, ba, ta = w["A"]
+    A = ctx.relation(torch.from_numpy(ka), ba, ta)           # host tensors -> UCL_MEM_HOST_COPY
+    B = ctx.relation(torch.from_numpy(w["B"][0]), w["B"][1], w["B"][2])
+    out = ctx.einsum(w["spec"], A, B)
+    assert_parity(out, oracle_ref(w["spec"], [w["A"], w["B"]]), torch.float32)
+
+
+def test_deterministic(ctx):
+    w = workloads.gnn_chain(seed=5, n=8192, degree=16)
+    X, Y = gpu_rel(ctx, w["X"]), gpu_rel(ctx, w["Y"])
+    a = ctx.einsum(w["spec1"], X, Y).download()[1]
+    b = ctx.einsum(w["spec1"], X, Y).download()[1]
+    assert torch.equal(a, b)
+
+
+# ---------------------------------------------------------------------- errors
+
+
+def test_errors(ctx):
+    v = (np.array([[1]], np.int32), (2,), torch.ones((1, 3)))
+    with pytest.raises(UclError, match="UCL_ERR_DUP_KEY"):
+        gpu_rel(ctx, (np.array([[0], [1], [0]], np.int32), (2,), torch.ones((3, 3))))
+    with pytest.raises(UclError, match="UCL_ERR_KEY_RANGE"):
+        gpu_rel(ctx, (np.array([[2]], np.int32), (2,), torch.ones((1, 3))))
+    with pytest.raises(UclError, match="UCL_ERR_KEY_RANGE"):
+        gpu_rel(ctx, (np.array([[-1]], np.int32), (2,), torch.ones((1, 3))))
+    R = gpu_rel(ctx, v)
+    with pytest.raises(UclError, match="UCL_ERR_SPEC"):
+        ctx.einsum("Ij,jK", R, R)
+    with pytest.raises(UclError, match="UCL_ERR_SPEC"):
+        ctx.einsum("Ij,jK->IQ", R, R)
+    with pytest.raises(UclError, match="UCL_ERR_SHAPE"):
+        ctx.einsum("Iij,jK->IK", R, R)
+    W = gpu_rel(ctx, (np.array([[1]], np.int32), (2,), torch.ones((1, 4))))
+    with pytest.raises(UclError, match="UCL_ERR_SHAPE"):
+        ctx.einsum("Ij,jK->IK", R, W)
+    # the context stays usable after errors
+    out = ctx.einsum("Ij,Ij->I", R, R)
+    assert out.download()[1].tolist() == [3.0]
+    ctx.synchronize()

@@ -1,0 +1,183 @@
+"""Seeded synthetic inputs shaped like the paper's workloads.
+
+This module only draws random tensors and cuts them into tensor-relations
+(keys + tiles); it holds none of the EinSum arithmetic.  Both the GPU tests
+and the oracle tests consume what it returns, so neither side depends on the
+other.  The paper's datasets (ogbn-*, friendster, Planetoid, QASMBench) are
+not available; these inputs stand in for them.
+
+A relation is returned as ``(keys, bounds, tiles)``: keys int32 [n, u] (numpy),
+bounds a tuple, tiles a torch tensor [n, *shape] (CPU unless built on the GPU).
+Keys are emitted in ascending lexicographic order.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+import torch
+
+# ------------------------------------------------------------------ helpers
+
+
+def _tiles_of_dense(dense: torch.Tensor, tr: int, tc: int):
+    """Cut a dense [R, C] matrix into [tr x tc] tiles keyed (I, J), zero-padding
+    the ragged edge; every tile is kept (dense operand)."""
+    R, C = dense.shape
+    nr, nc = -(-R // tr), -(-C // tc)
+    pad = torch.zeros((nr * tr, nc * tc), dtype=dense.dtype, device=dense.device)
+    pad[:R, :C] = dense
+    tiles = pad.reshape(nr, tr, nc, tc).permute(0, 2, 1, 3).reshape(nr * nc, tr, tc).contiguous()
+    I, J = np.meshgrid(np.arange(nr), np.arange(nc), indexing="ij")
+    keys = np.stack([I.ravel(), J.ravel()], axis=1).astype(np.int32)
+    return keys, (nr, nc), tiles
+
+
+def rmat_edges(n: int, n_edges: int, a=0.57, b=0.19, c=0.19, seed=0, batch=1 << 22):
+    """R-MAT edge list (Chakrabarti et al.) on 2^ceil(log2 n) vertices; edges
+    with an endpoint >= n are rejected and redrawn until n_edges remain, then
+    duplicates are removed (self-loops kept).  Returns (src, dst) int64
+    sorted by (src, dst)."""
+    rng = np.random.default_rng(seed)
+    levels = max(1, math.ceil(math.log2(n)))
+    srcs, dsts, have = [], [], 0
+    while have < n_edges:
+        m = min(batch, 2 * (n_edges - have) + 1024)
+        s = np.zeros(m, dtype=np.int64)
+        d = np.zeros(m, dtype=np.int64)
+        for _ in range(levels):
+            r = rng.random(m)
+            sb = r >= a + b                       # quadrants c, d: lower half of the rows
+            db = ((r >= a) & (r < a + b)) | (r >= a + b + c)  # quadrants b, d: right half
+            s = (s << 1) | sb
+            d = (d << 1) | db
+        ok = (s < n) & (d < n)
+        s, d = s[ok], d[ok]
+        take = min(len(s), n_edges - have)
+        srcs.append(s[:take])
+        dsts.append(d[:take])
+        have += take
+    s = np.concatenate(srcs)
+    d = np.concatenate(dsts)
+    code = np.unique(s * n + d)
+    return code // n, code % n
+
+
+def adjacency_tiles(src, dst, n: int, t: int, device="cpu", dtype=torch.bfloat16):
+    """0/1 adjacency Y[src, dst] = 1 stored as only-nonempty [t x t] tiles
+    keyed (J = src // t, K = dst // t), ascending."""
+    nt = -(-n // t)
+    tcode = (src // t) * nt + (dst // t)
+    ukeys, inv = np.unique(tcode, return_inverse=True)
+    keys = np.stack([ukeys // nt, ukeys % nt], axis=1).astype(np.int32)
+    tiles = torch.zeros((len(ukeys), t, t), dtype=dtype, device=device)
+    idx = torch.as_tensor(inv, device=device)
+    r = torch.as_tensor(src % t, device=device)
+    q = torch.as_tensor(dst % t, device=device)
+    tiles[idx, r, q] = 1
+    return keys, (nt, nt), tiles
+
+
+def adjacency_tiles_subset(src, dst, n: int, t: int, keys_wanted: np.ndarray):
+    """The same tiles as adjacency_tiles, only for the (J, K) keys given, as a
+    float64 CPU array (for the oracle on sampled output keys)."""
+    nt = -(-n // t)
+    want = keys_wanted[:, 0].astype(np.int64) * nt + keys_wanted[:, 1]
+    tcode = (src // t) * nt + (dst // t)
+    pos = {int(c): i for i, c in enumerate(want)}
+    tiles = np.zeros((len(want), t, t))
+    sel = np.isin(tcode, want)
+    for s, d, c in zip(src[sel], dst[sel], tcode[sel]):
+        tiles[pos[int(c)], s % t, d % t] = 1.0
+    return tiles
+
+
+# ----------------------------------------------------------------- workloads
+
+
+def blocksparse_matmul(seed=0, n=1024, m=256, t=32, density=0.10):
+    """Block-sparse C[I,K] = sum_J A[I,J] B[J,K] over t x t fp32 tiles: A
+    n x n with round(density * (n/t)^2) tiles drawn uniformly without
+    replacement, B dense n x m, values U[-1, 1].  Spec IiJj,JjKk->IiKk."""
+    rng = np.random.default_rng(seed)
+    g = n // t
+    nnz = round(density * g * g)
+    pick = np.sort(rng.choice(g * g, size=nnz, replace=False))
+    ka = np.stack([pick // g, pick % g], axis=1).astype(np.int32)
+    ta = torch.from_numpy(rng.uniform(-1, 1, size=(nnz, t, t)).astype(np.float32))
+    B = torch.from_numpy(rng.uniform(-1, 1, size=(n, m)).astype(np.float32))
+    kb, bb, tb = _tiles_of_dense(B, t, t)
+    return {
+        "spec": "IiJj,JjKk->IiKk",
+        "A": (ka, (g, g), ta),
+        "B": (kb, bb, tb),
+    }
+
+
+def gnn_chain(seed=0, n=100_000, feat=128, out_feat=128, degree=16, t=64, device="cpu", z_std=0.1):
+    """Message passing (X x Y)^T x Z: X feat x n bf16 N(0,1) stored per vertex
+    tile J as [f x j] tiles; Y an R-MAT adjacency (a,b,c = .57,.19,.19, n*degree
+    edges) as only-nonempty t x t 0/1 tiles keyed (J, K); Z feat x out_feat
+    bf16 N(0, z_std^2) as one key-less tuple.
+    Specs: fJj,JjKk->Kkf (T = (X Y)^T), then Kkf,fg->Kkg (T Z)."""
+    g = torch.Generator().manual_seed(seed)
+    X = torch.randn((feat, n), generator=g).to(torch.bfloat16)
+    nt = -(-n // t)
+    Xp = torch.zeros((feat, nt * t), dtype=torch.bfloat16)
+    Xp[:, :n] = X
+    xt = Xp.reshape(feat, nt, t).permute(1, 0, 2).contiguous()   # [J][f][j]
+    kx = np.arange(nt, dtype=np.int32)[:, None]
+    src, dst = rmat_edges(n, n * degree, seed=seed + 1)
+    ky, by, ty = adjacency_tiles(src, dst, n, t, device=device)
+    Z = (torch.randn((feat, out_feat), generator=g) * z_std).to(torch.bfloat16)
+    return {
+        "spec1": "fJj,JjKk->Kkf",
+        "spec2": "Kkf,fg->Kkg",
+        "X": (kx, (nt,), xt.to(device)),
+        "Y": (ky, by, ty),
+        "Z": (np.zeros((1, 0), np.int32), (), Z[None].to(device)),
+        "edges": (src, dst),
+        "n": n,
+        "t": t,
+    }
+
+
+def spgemm(seed=0, n=65536, t=128, density=0.005, band=(-1, 0, 1, 2)):
+    """Block-sparse x block-sparse: A and B n x n with t x t bf16 N(0,1) tiles
+    at the given tile density, half of the tiles on the band J - I in `band`,
+    half uniform among the off-band tiles; drawn independently for A and B.
+    Spec IiJj,JjKk->IiKk (fp32 output)."""
+    rng = np.random.default_rng(seed)
+    g = n // t
+    nnz = round(density * g * g)
+    n_band = nnz // 2
+
+    def draw():
+        I = np.arange(g)
+        bi = np.concatenate([I for _ in band])
+        bj = np.concatenate([I + d for d in band])
+        ok = (bj >= 0) & (bj < g)
+        bcodes = (bi * g + bj)[ok]
+        bsel = rng.choice(bcodes, size=n_band, replace=False)
+        rest = nnz - n_band
+        chosen = set(bsel.tolist())
+        bandset = set(bcodes.tolist())
+        out = []
+        while len(out) < rest:
+            c = int(rng.integers(0, g * g))
+            if c in bandset or c in chosen:
+                continue
+            chosen.add(c)
+            out.append(c)
+        codes = np.sort(np.concatenate([bsel, np.array(out, dtype=np.int64)]))
+        keys = np.stack([codes // g, codes % g], axis=1).astype(np.int32)
+        tiles = torch.from_numpy(rng.standard_normal((len(codes), t, t)).astype(np.float32)).to(torch.bfloat16)
+        return keys, (g, g), tiles
+
+    return {"spec": "IiJj,JjKk->IiKk", "A": draw(), "B": draw()}
+
+
+def to_oracle(rel):
+    """(keys, bounds, tiles) with tiles converted exactly to float64 numpy."""
+    keys, bounds, tiles = rel
+    return keys, bounds, tiles.detach().to("cpu", torch.float64).numpy()
