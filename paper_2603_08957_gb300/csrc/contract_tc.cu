@@ -1,17 +1,579 @@
-// contract_tc.cu -- tcgen05 tile contraction (placeholder until the kernel lands).
+// contract_tc.cu -- tcgen05 tile contraction with the segmented group-by sum
+// fused into its epilogue (paper Sec. 5: the kernel K applied to every joined
+// pair, then SUM ... GROUP BY up(W)).
+//
+// Applies when the lower-case EinSum of one pair is a bf16 GEMM,
+//     D[M x N] += A[M x K] * B[K x N],
+// with A and B the two joined tiles (either operand order) and the output
+// tile equal to D up to a transpose.  One CTA per SM processes a contiguous
+// unit of the pair list, which is ordered by output key:
+//
+//   warp 0      TMA producer: gathers the A and B tiles of consecutive pairs
+//               (tile index = tuple index, from the pair list) into a ring of
+//               shared-memory stages, 128B/64B/32B-swizzled;
+//   warp 1      MMA issuer: one thread issues tcgen05.mma per 16-deep K step
+//               into a TMEM accumulator, accumulating across all pairs of one
+//               output key (one segment); the warp owns the TMEM allocation;
+//   warps 2-5   epilogue: when a segment's accumulator is complete, drain it
+//               from TMEM (tcgen05.ld), apply scale / relu, cast and store the
+//               output tile -- or, for a segment that continues in another
+//               unit, store an fp32 partial for the fixup kernel.
+//
+// Accumulators are multi-buffered in TMEM so the epilogue of one segment
+// overlaps the MMAs of the next.  Every wait on an mbarrier is bounded (1 s of
+// globaltimer); on expiry the CTA raises kStTimeout, every role leaves its
+// loop, in-flight TMA copies and MMAs are drained (again with a bound), TMEM
+// is freed and the kernel returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
 #include "internal.cuh"
 
 namespace ucl {
 
-bool tc_supported(const TcPlan &, const ContractArgs &, std::string *why) {
-    *why = "tcgen05 kernel not built";
-    return false;
+namespace {
+
+constexpr int kTcThreads = 192;
+constexpr uint64_t kWaitLimitNs = 1000000000ull;
+constexpr int kMaxStages = 8;
+constexpr int kMaxAcc = 4;
+constexpr uint32_t kSmemLimit = 227 * 1024;
+
+struct TcArgs {
+    const uint32_t *pa;   // [P] A tuple of each pair
+    const uint32_t *pb;   // [P] B tuple of each pair
+    int64_t nA, nB;
+    const int64_t *seg_start;
+    int64_t S;
+    Units units;
+    void *out;
+    int dout, epi;
+    float scale;
+    float *partials;
+    int64_t tile_w;
+    int64_t sWm, sWn;
+    int N, K, m_blocks;
+    int a_kmajor, b_kmajor;
+    int wa, wb;                  // sub-tile width (elements) of the A / B boxes
+    uint32_t a_sub, b_sub;       // bytes per sub-tile (multiple of 1024)
+    uint32_t a_bytes;            // A part of a stage
+    uint32_t stage_bytes;
+    uint32_t tx_bytes;           // bytes one stage receives from TMA
+    int na_sub, nb_sub;
+    int ns, nacc;
+    uint32_t tmem_cols;
+    uint32_t idesc;
+    uint32_t *status;
+};
+
+// ------------------------------------------------------------- PTX wrappers
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t globaltimer() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait for the phase of `parity` to complete.  Gives up when another
+// role of the CTA has aborted, or after kWaitLimitNs (then raises the abort
+// and the device status).  Returns false when it gave up.
+__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile uint32_t *abort_flag,
+                                       uint32_t *status) {
+    if (mbar_try(bar, parity)) return true;
+    const uint64_t t0 = globaltimer();
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_try(bar, parity)) return true;
+        if ((i & 31) == 0) {
+            if (*abort_flag) return false;
+            if (globaltimer() - t0 > kWaitLimitNs) {
+                *abort_flag = 1;
+                atomicOr(status, kStTimeout);
+                return false;
+            }
+        }
+    }
+}
+
+// Bounded wait used while draining after an abort (ignores the abort flag).
+__device__ __noinline__ void mbar_drain(uint32_t bar, uint32_t parity) {
+    const uint64_t t0 = globaltimer();
+    while (!mbar_try(bar, parity))
+        if (globaltimer() - t0 > kWaitLimitNs) return;
+}
+
+__device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, int x, int y, int z, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
+        "[%5];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
+        : "memory");
+}
+
+// Shared-memory matrix descriptor of tcgen05 (start, leading / stride byte
+// offsets, fixed version 1, swizzle layout).
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo, uint32_t layout) {
+    return (uint64_t)((addr >> 4) & 0x3FFFu) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+           ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | (1ull << 46) | ((uint64_t)layout << 61);
+}
+
+__device__ __forceinline__ uint32_t swz_layout(int width_elems) {
+    const int bytes = width_elems * 2;
+    return bytes == 128 ? 2u : (bytes == 64 ? 4u : 6u);   // SW128 / SW64 / SW32
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(acc)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float *v) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ int64_t find_seg(const int64_t *seg_start, int64_t S, int64_t p) {
+    int64_t a = 0, b = S;
+    while (a < b) {
+        int64_t mid = (a + b) >> 1;
+        if (seg_start[mid] <= p) a = mid + 1; else b = mid;
+    }
+    return a - 1;
+}
+
+__device__ __forceinline__ float epilogue(float x, int epi, float scale) {
+    x *= scale;
+    if (epi == UCL_EPI_RELU) x = fmaxf(x, 0.0f);
+    return x;
+}
+
+// A operand descriptor for K step kk and M block mb.
+__device__ __forceinline__ uint64_t a_desc(const TcArgs &a, uint32_t base, int kk, int mb) {
+    if (a.a_kmajor) {
+        const int k0 = kk * 16;
+        const uint32_t addr = base + (uint32_t)(k0 / a.wa) * a.a_sub + (uint32_t)mb * 128u * (uint32_t)a.wa * 2u +
+                              (uint32_t)(k0 % a.wa) * 2u;
+        return smem_desc(addr, 16, 8u * a.wa * 2u, swz_layout(a.wa));
+    }
+    const uint32_t addr = base + (uint32_t)mb * (uint32_t)(128 / a.wa) * a.a_sub + (uint32_t)kk * 16u * a.wa * 2u;
+    return smem_desc(addr, a.a_sub, 8u * a.wa * 2u, swz_layout(a.wa));
+}
+
+__device__ __forceinline__ uint64_t b_desc(const TcArgs &a, uint32_t base, int kk) {
+    if (a.b_kmajor) {
+        const int k0 = kk * 16;
+        const uint32_t addr = base + (uint32_t)(k0 / a.wb) * a.b_sub + (uint32_t)(k0 % a.wb) * 2u;
+        return smem_desc(addr, 16, 8u * a.wb * 2u, swz_layout(a.wb));
+    }
+    const uint32_t addr = base + (uint32_t)kk * 16u * a.wb * 2u;
+    return smem_desc(addr, a.b_sub, 8u * a.wb * 2u, swz_layout(a.wb));
+}
+
+// ------------------------------------------------------------------ kernel
+
+__global__ void __launch_bounds__(kTcThreads, 1)
+    tc_contract_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                       const TcArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    const uint32_t sbase = smem_u32(smem);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)a.ns * a.stage_bytes);
+    const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8u * a.ns, accf0 = empty0 + 8u * a.ns,
+                   acce0 = accf0 + 8u * a.nacc, done_bar = acce0 + 8u * a.nacc;
+    uint32_t *misc = reinterpret_cast<uint32_t *>(bars + 2 * a.ns + 2 * a.nacc + 1);
+    // misc[0] TMEM base, [1] abort flag, [2] stages consumed by the MMA warp, [3] stages issued by TMA
+    volatile uint32_t *abort_flag = misc + 1;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < a.ns; ++i) {
+            mbar_init(full0 + 8u * i, 1);
+            mbar_init(empty0 + 8u * i, 1);
+        }
+        for (int i = 0; i < a.nacc; ++i) {
+            mbar_init(accf0 + 8u * i, 1);
+            mbar_init(acce0 + 8u * i, 4);
+        }
+        mbar_init(done_bar, 1);
+        misc[1] = 0;
+        misc[2] = 0;
+        misc[3] = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(misc)),
+                     "r"(a.tmem_cols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = misc[0];
+
+    const int unit = blockIdx.x;
+    const int64_t pb = a.units.begin(unit), pe = a.units.begin(unit + 1);
+    const int64_t s_first = pe > pb ? find_seg(a.seg_start, a.S, pb) : 0;
+    const int64_t s_last = pe > pb ? find_seg(a.seg_start, a.S, pe - 1) : -1;
+    const uint32_t acc_cols = (uint32_t)(a.N * a.m_blocks);
+
+    if (warp == 0) {
+        // ------------------------------------------------------- producer
+        uint32_t it = 0;
+        for (int64_t base = pb; base < pe; base += 32) {
+            const int64_t p = base + lane;
+            uint32_t ia = 0, ib = 0;
+            if (p < pe) {
+                ia = a.pa[p];
+                ib = a.pb[p];
+                if ((int64_t)ia >= a.nA || (int64_t)ib >= a.nB) {
+                    atomicOr(a.status, kStBadIndex);
+                    ia = 0;
+                    ib = 0;
+                }
+            }
+            const int cnt = (int)(pe - base < 32 ? pe - base : 32);
+            uint32_t stop = 0;
+            for (int j = 0; j < cnt; ++j) {
+                const uint32_t xa = __shfl_sync(0xffffffffu, ia, j), xb = __shfl_sync(0xffffffffu, ib, j);
+                if (lane == 0) {
+                    const uint32_t st = it % a.ns, ph = (it / a.ns) & 1u;
+                    if (!mbar_wait(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status)) {
+                        stop = 1;
+                    } else {
+                        const uint32_t fb = full0 + 8u * st;
+                        mbar_arrive_tx(fb, a.tx_bytes);
+                        const uint32_t sa = sbase + st * a.stage_bytes, sb = sa + a.a_bytes;
+                        for (int q = 0; q < a.na_sub; ++q) tma_load_3d(sa + q * a.a_sub, &tmA, q * a.wa, 0, (int)xa, fb);
+                        for (int q = 0; q < a.nb_sub; ++q) tma_load_3d(sb + q * a.b_sub, &tmB, q * a.wb, 0, (int)xb, fb);
+                        ++it;
+                    }
+                }
+                if (__shfl_sync(0xffffffffu, stop, 0)) break;
+            }
+            if (__shfl_sync(0xffffffffu, stop, 0)) break;
+        }
+        if (lane == 0) misc[3] = it;
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA
+        if (lane == 0) {
+            uint32_t it = 0;
+            int64_t t = 0;
+            bool ok = true;
+            for (int64_t s = s_first; s <= s_last && ok; ++s, ++t) {
+                const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
+                const int64_t p0 = ss > pb ? ss : pb, p1 = se < pe ? se : pe;
+                const uint32_t b = (uint32_t)(t % a.nacc), ph = (uint32_t)((t / a.nacc) & 1);
+                if (!mbar_wait(acce0 + 8u * b, ph ^ 1u, abort_flag, a.status)) break;
+                tc_fence_after();
+                const uint32_t dcol = tmem + b * acc_cols;
+                for (int64_t p = p0; p < p1; ++p) {
+                    const uint32_t st = it % a.ns, sph = (it / a.ns) & 1u;
+                    if (!mbar_wait(full0 + 8u * st, sph, abort_flag, a.status)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = sbase + st * a.stage_bytes, sb = sa + a.a_bytes;
+                    for (int kk = 0; kk < a.K / 16; ++kk) {
+                        const uint64_t bd = b_desc(a, sb, kk);
+                        for (int mb = 0; mb < a.m_blocks; ++mb)
+                            mma_bf16(dcol + (uint32_t)(mb * a.N), a_desc(a, sa, kk, mb), bd, a.idesc,
+                                     (p > p0 || kk > 0) ? 1u : 0u);
+                    }
+                    mma_commit(empty0 + 8u * st);
+                    ++it;
+                }
+                if (ok) mma_commit(accf0 + 8u * b);
+            }
+            misc[2] = it;
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------- epilogue
+        const int q = warp & 3;   // TMEM lane quadrant this warp may access
+        int64_t t = 0;
+        for (int64_t s = s_first; s <= s_last; ++s, ++t) {
+            const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
+            const uint32_t b = (uint32_t)(t % a.nacc), ph = (uint32_t)((t / a.nacc) & 1);
+            if (!mbar_wait(accf0 + 8u * b, ph, abort_flag, a.status)) break;
+            tc_fence_after();
+            const int kind = (ss >= pb && se <= pe) ? 0 : (ss < pb ? 1 : 2);
+            float *part = a.partials + ((int64_t)unit * 2 + (kind == 1 ? 0 : 1)) * a.tile_w;
+            for (int mb = 0; mb < a.m_blocks; ++mb) {
+                const int64_t m = (int64_t)mb * 128 + q * 32 + lane;
+                for (int c = 0; c < a.N / 16; ++c) {
+                    float v[16];
+                    tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + b * acc_cols + (uint32_t)(mb * a.N + c * 16), v);
+                    const int64_t base_off = m * a.sWm + (int64_t)c * 16 * a.sWn;
+                    if (kind == 0) {
+                        if (a.dout == UCL_BF16) {
+                            __nv_bfloat16 *o = reinterpret_cast<__nv_bfloat16 *>(a.out) + s * a.tile_w + base_off;
+#pragma unroll
+                            for (int j = 0; j < 16; ++j) o[j * a.sWn] = __float2bfloat16_rn(epilogue(v[j], a.epi, a.scale));
+                        } else {
+                            float *o = reinterpret_cast<float *>(a.out) + s * a.tile_w + base_off;
+#pragma unroll
+                            for (int j = 0; j < 16; ++j) o[j * a.sWn] = epilogue(v[j], a.epi, a.scale);
+                        }
+                    } else {
+                        float *o = part + base_off;
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) o[j * a.sWn] = v[j];
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(acce0 + 8u * b);
+        }
+    }
+
+    // ---------------------------------------------------------- teardown
+    __syncthreads();
+    if (*abort_flag) {
+        if (warp == 0 && lane == 0) {
+            // copies still in flight write into this CTA's shared memory: wait for them
+            for (uint32_t it = misc[2]; it < misc[3]; ++it) mbar_drain(full0 + 8u * (it % a.ns), (it / a.ns) & 1u);
+        }
+        if (warp == 1 && lane == 0) {
+            mma_commit(done_bar);   // tracks every MMA this thread issued
+            mbar_drain(done_bar, 0);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(a.tmem_cols)
+                     : "memory");
+    }
+}
+
+// ------------------------------------------------------------------- host
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+        else
+            cudaGetLastError();
+    });
+    return fn;
+}
+
+// Operand geometry: the tile is [rows][cols] row-major; it is fetched as
+// cols / w boxes of {w, rows}, each landing in its own swizzled sub-tile.
+struct Operand {
+    int rows, cols, w, nsub;
+    uint32_t sub_bytes;
+};
+
+bool operand_geometry(int rows, int cols, Operand *op, std::string *why) {
+    if (rows < 16 || rows > 256 || rows % 16) {
+        *why = "tile rows must be a multiple of 16 up to 256";
+        return false;
+    }
+    if (!(cols == 16 || cols == 32 || (cols % 64 == 0 && cols <= 256))) {
+        *why = "tile row length must be 16, 32 or a multiple of 64 elements";
+        return false;
+    }
+    op->rows = rows;
+    op->cols = cols;
+    op->w = cols < 64 ? cols : 64;
+    op->nsub = cols / op->w;
+    uint32_t b = (uint32_t)rows * op->w * 2;
+    op->sub_bytes = (b + 1023u) & ~1023u;
+    return true;
+}
+
+struct TcGeometry {
+    Operand A, B;
+    uint32_t stage_bytes, a_bytes, tx_bytes, smem_bytes, tmem_cols;
+    int ns, nacc;
+};
+
+bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why) {
+    // A: K-major tiles are [M][K], MN-major [K][M]; same for B with N
+    if (!operand_geometry(tp.a_kmajor ? tp.M : tp.K, tp.a_kmajor ? tp.K : tp.M, &g->A, why)) return false;
+    if (!operand_geometry(tp.b_kmajor ? tp.N : tp.K, tp.b_kmajor ? tp.K : tp.N, &g->B, why)) return false;
+    g->a_bytes = g->A.sub_bytes * g->A.nsub;
+    g->stage_bytes = g->a_bytes + g->B.sub_bytes * g->B.nsub;
+    g->tx_bytes = (uint32_t)(tp.M * tp.K * 2 + tp.N * tp.K * 2);
+    const uint32_t bar_bytes = 8u * (2 * kMaxStages + 2 * kMaxAcc + 1) + 64;
+    int ns = (int)((kSmemLimit - 1024 - bar_bytes) / g->stage_bytes);
+    if (ns > kMaxStages) ns = kMaxStages;
+    if (ns < 2) {
+        *why = "tiles too large for two shared-memory stages";
+        return false;
+    }
+    g->ns = ns;
+    const int acc_cols = tp.N * tp.m_blocks;
+    g->nacc = 512 / acc_cols < kMaxAcc ? 512 / acc_cols : kMaxAcc;
+    if (g->nacc < 1) {
+        *why = "accumulator does not fit TMEM";
+        return false;
+    }
+    uint32_t need = (uint32_t)(g->nacc * acc_cols), cols = 32;
+    while (cols < need) cols <<= 1;
+    g->tmem_cols = cols;
+    g->smem_bytes = 1024 + ns * g->stage_bytes + bar_bytes;
+    return true;
+}
+
+bool make_map(CUtensorMap *m, const ucl_rel *R, const Operand &op, std::string *why) {
+    auto enc = encode_fn();
+    if (!enc) {
+        *why = "cuTensorMapEncodeTiled unavailable";
+        return false;
+    }
+    cuuint64_t dims[3] = {(cuuint64_t)op.cols, (cuuint64_t)op.rows, (cuuint64_t)R->n};
+    cuuint64_t strides[2] = {(cuuint64_t)op.cols * 2, (cuuint64_t)op.rows * op.cols * 2};
+    cuuint32_t box[3] = {(cuuint32_t)op.w, (cuuint32_t)op.rows, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUtensorMapSwizzle swz = op.w == 64 ? CU_TENSOR_MAP_SWIZZLE_128B
+                                        : (op.w == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B);
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, R->tiles, dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        *why = "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")";
+        return false;
+    }
+    return true;
+}
+
+}  // namespace
+
+bool tc_supported(const TcPlan &tp, const ContractArgs &a, std::string *why) {
+    TcGeometry g;
+    if (!geometry(tp, &g, why)) return false;
+    const void *pa = tp.a_is_u ? a.U : a.V, *pb = tp.a_is_u ? a.V : a.U;
+    if ((reinterpret_cast<uintptr_t>(pa) | reinterpret_cast<uintptr_t>(pb)) & 15) {
+        *why = "tile arrays not 16-byte aligned";
+        return false;
+    }
+    if (!encode_fn()) {
+        *why = "cuTensorMapEncodeTiled unavailable";
+        return false;
+    }
+    return true;
 }
 
 int tc_units(ucl_ctx *ctx, const TcPlan &, int64_t P) { return (int)(P < ctx->sm_count ? P : ctx->sm_count); }
 
-ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &, const TcPlan &, const ucl_rel *, const ucl_rel *) {
-    return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 kernel not built");
+ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan &tp, const ucl_rel *ra,
+                              const ucl_rel *rb) {
+    TcGeometry g;
+    std::string why;
+    if (!geometry(tp, &g, &why)) return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why);
+    CUtensorMap mA, mB;
+    if (!make_map(&mA, ra, g.A, &why) || !make_map(&mB, rb, g.B, &why))
+        return fail(ctx, UCL_ERR_CUDA, "tcgen05 path: " + why);
+    TcArgs k{};
+    k.pa = tp.a_is_u ? a.pu : a.pv;
+    k.pb = tp.a_is_u ? a.pv : a.pu;
+    k.nA = ra->n;
+    k.nB = rb->n;
+    k.seg_start = a.seg_start;
+    k.S = a.S;
+    k.units = a.units;
+    k.out = a.out;
+    k.dout = a.dout;
+    k.epi = a.epi;
+    k.scale = a.scale;
+    k.partials = a.partials;
+    k.tile_w = a.tile_w;
+    k.sWm = tp.sWm;
+    k.sWn = tp.sWn;
+    k.N = tp.N;
+    k.K = tp.K;
+    k.m_blocks = tp.m_blocks;
+    k.a_kmajor = tp.a_kmajor;
+    k.b_kmajor = tp.b_kmajor;
+    k.wa = g.A.w;
+    k.wb = g.B.w;
+    k.a_sub = g.A.sub_bytes;
+    k.b_sub = g.B.sub_bytes;
+    k.na_sub = g.A.nsub;
+    k.nb_sub = g.B.nsub;
+    k.a_bytes = g.a_bytes;
+    k.stage_bytes = g.stage_bytes;
+    k.tx_bytes = g.tx_bytes;
+    k.ns = g.ns;
+    k.nacc = g.nacc;
+    k.tmem_cols = g.tmem_cols;
+    // instruction descriptor, kind::f16: D fp32, A and B bf16, majors, N >> 3, M >> 4 (M = 128 per MMA)
+    k.idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(tp.a_kmajor ? 0 : 1) << 15) |
+              ((uint32_t)(tp.b_kmajor ? 0 : 1) << 16) | ((uint32_t)(tp.N >> 3) << 17) | ((128u >> 4) << 24);
+    k.status = ctx->d_status;
+    static int configured_smem = 0;
+    if ((int)g.smem_bytes > configured_smem) {
+        ucl_status st = cuda_check(ctx,
+                                   cudaFuncSetAttribute(tc_contract_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                        (int)g.smem_bytes),
+                                   "cudaFuncSetAttribute");
+        if (st) return st;
+        configured_smem = (int)g.smem_bytes;
+    }
+    tc_contract_kernel<<<a.units.G, kTcThreads, g.smem_bytes, ctx->stream>>>(mA, mB, k);
+    ctx->launches++;
+    return cuda_check(ctx, cudaGetLastError(), "tcgen05 kernel launch");
 }
 
 }  // namespace ucl

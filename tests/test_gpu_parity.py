@@ -55,6 +55,49 @@ def test_worked_example(ctx, path):
     assert ctx.last_stats()["n_pairs"] == 6
 
 
+# ------------------------------------------------- tcgen05 operand layouts
+
+TC_CASES = [
+    # (U operand, V operand, output, extents)  U/V tiles in every major order
+    ("IJmk", "JKkn", "IKmn", {"m": 128, "k": 64, "n": 64}),    # A K-major, B MN-major
+    ("IJmk", "JKnk", "IKmn", {"m": 128, "k": 64, "n": 64}),    # B K-major
+    ("IJkm", "JKkn", "IKmn", {"m": 128, "k": 64, "n": 64}),    # A MN-major
+    ("IJkm", "JKnk", "IKnm", {"m": 128, "k": 64, "n": 64}),    # both MN/K swapped, transposed output
+    ("IJmk", "JKkn", "IKmn", {"m": 128, "k": 16, "n": 16}),    # 32-byte swizzle
+    ("IJmk", "JKkn", "IKnm", {"m": 128, "k": 32, "n": 32}),    # 64-byte swizzle
+    ("IJmk", "JKkn", "IKmn", {"m": 128, "k": 128, "n": 128}),  # two boxes per row
+    ("IJkm", "JKkn", "IKmn", {"m": 128, "k": 128, "n": 256}),  # N = 256
+    ("IJmk", "JKkn", "IKmn", {"m": 256, "k": 64, "n": 64}),    # two M blocks
+    ("IJkm", "JKkn", "IKnm", {"m": 256, "k": 64, "n": 32}),    # two M blocks, MN-major A
+    ("IJnk", "JKmk", "IKnm", {"m": 128, "k": 64, "n": 48}),    # A comes from V
+]
+
+
+@pytest.mark.parametrize("ou,ov,ow,ext", TC_CASES)
+def test_tc_gemm_layouts(ctx, ou, ov, ow, ext):
+    """Block-sparse tiled matmul whose tile kernel is a bf16 GEMM in every
+    operand major order, output transpose and swizzle width: 3 x 40 x 2 key
+    grid, 240 pairs over 6 output keys (segments split across work units)."""
+    rng = np.random.default_rng(hash((ou, ov, ow)) % 2**31)
+    nI, nJ, nK = 3, 40, 2
+
+    def rel(op, keys, bounds):
+        shape = [ext[c] for c in op if c.islower()]
+        t = torch.randn([len(keys)] + shape, generator=torch.Generator().manual_seed(int(rng.integers(1 << 30))))
+        return (np.array(keys, np.int32), bounds, t.to(torch.bfloat16))
+
+    U = rel(ou, [(i, j) for i in range(nI) for j in range(nJ)], (nI, nJ))
+    V = rel(ov, [(j, k) for j in range(nJ) for k in range(nK)], (nJ, nK))
+    spec = f"{ou},{ov}->{ow}"
+    ref = oracle_ref(spec, [U, V])
+    out = ctx.einsum(spec, gpu_rel(ctx, U), gpu_rel(ctx, V), path="tc")
+    assert ctx.last_stats()["path"] == "tc"
+    assert_parity(out, ref, torch.bfloat16)
+    out16 = ctx.einsum(spec, gpu_rel(ctx, U), gpu_rel(ctx, V), path="tc", out_dtype="bf16", epi="relu", scale=2.0)
+    ref16 = oracle_ref(spec, [U, V], epi="relu", scale=2.0)
+    assert_parity(out16, ref16, torch.bfloat16, scale=2.0)
+
+
 # ---------------------------------------------------------- random small specs
 
 SPECS = [
