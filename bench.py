@@ -42,6 +42,13 @@ WORKLOAD = ("gnn-message-passing (XxY)^T x Z: X 128x100000 bf16, Y R-MAT 100000 
             "as 358136 nonempty 64x64 bf16 tiles, Z 128x128 bf16; specs fJj,JjKk->Kkf then Kkf,fg->Kkg")
 
 
+def workload_name(vertices):
+    if vertices == 100_000:
+        return WORKLOAD
+    return (f"gnn-message-passing (XxY)^T x Z, reduced: X 128x{vertices} bf16, Y R-MAT {vertices} vertices / "
+            f"{16 * vertices} edges as 64x64 bf16 tiles, Z 128x128 bf16")
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -205,7 +212,7 @@ def run_ucl(args, world, rank, local):
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    w = workloads.gnn_chain(seed=0, device=dev)
+    w = workloads.gnn_chain(seed=0, n=args.vertices, device=dev)
     ctx = Context(local)
 
     def rel(r):
@@ -278,7 +285,7 @@ def run_ucl(args, world, rank, local):
 
     # end to end through the C ABI with host buffers
     e2e = None
-    if rank == 0 or world > 1:
+    if not args.no_e2e:
         hx = [torch.as_tensor(w["X"][0]).pin_memory(), w["X"][2].cpu().pin_memory()]
         hy = [torch.as_tensor(w["Y"][0]).pin_memory(), w["Y"][2].cpu().pin_memory()]
         hz = [torch.as_tensor(w["Z"][0]).pin_memory(), w["Z"][2].cpu().pin_memory()]
@@ -316,7 +323,7 @@ def run_ucl(args, world, rank, local):
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps,
                 "warmup": args.warmup, "ms_per_step": ms_max / steps, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-                "config": {"workload": WORKLOAD, "pairs": [s1["n_pairs"], s2["n_pairs"]],
+                "config": {"workload": workload_name(args.vertices), "pairs": [s1["n_pairs"], s2["n_pairs"]],
                            "segments": [s1["n_segments"], s2["n_segments"]], "flops_per_step": flops_step,
                            "l2": "inputs larger than L2 (Y 2.9 GB); no flush", "path": s1["path"],
                            "parallelism": f"replicas x{world}"},
@@ -336,6 +343,8 @@ def main():
     ap.add_argument("--impl", choices=["ucl", "reference"], default="ucl")
     ap.add_argument("--path", choices=["auto", "simt", "tc"], default="auto")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--vertices", type=int, default=100_000, help="graph size (reduced sizes for profiling)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-step-seconds", type=float, default=3.0)
     args = ap.parse_args()
