@@ -20,10 +20,13 @@
 //               unit, store an fp32 partial for the fixup kernel.
 //
 // Accumulators are multi-buffered in TMEM so the epilogue of one segment
-// overlaps the MMAs of the next.  Every wait on an mbarrier is bounded (1 s of
-// globaltimer); on expiry the CTA raises kStTimeout, every role leaves its
-// loop, in-flight TMA copies and MMAs are drained (again with a bound), TMEM
-// is freed and the kernel returns.
+// overlaps the MMAs of the next.  A pipeline stage holds the tiles of `pps`
+// consecutive pairs, so that barrier traffic is paid once per stage.  The
+// producer and MMA warps run warp-uniform loops and issue through one elected
+// lane; descriptors are precomputed so that one MMA costs a few integer adds.
+// Every wait on an mbarrier is bounded (about 1 s of SM clock); on expiry the
+// CTA raises kStTimeout, every role leaves its loop, in-flight TMA copies and
+// MMAs are drained (again with a bound), TMEM is freed and the kernel returns.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -36,7 +39,7 @@ namespace ucl {
 namespace {
 
 constexpr int kTcThreads = 192;
-constexpr uint64_t kWaitLimitNs = 1000000000ull;
+constexpr long long kWaitLimitCycles = 2500000000ll;   // ~1.2 s at 2.07 GHz
 constexpr int kMaxStages = 8;
 constexpr int kMaxAcc = 4;
 constexpr uint32_t kSmemLimit = 227 * 1024;
@@ -55,16 +58,21 @@ struct TcArgs {
     int64_t tile_w;
     int64_t sWm, sWn;
     int N, K, m_blocks;
-    int a_kmajor, b_kmajor;
     int wa, wb;                  // sub-tile width (elements) of the A / B boxes
+    int na_sub, nb_sub;          // boxes per tile
     uint32_t a_sub, b_sub;       // bytes per sub-tile (multiple of 1024)
-    uint32_t a_bytes;            // A part of a stage
-    uint32_t stage_bytes;
-    uint32_t tx_bytes;           // bytes one stage receives from TMA
-    int na_sub, nb_sub;
+    uint32_t a_pair, b_pair;     // bytes of one pair's A / B tile in a stage
+    uint32_t stage_bytes;        // pps * (a_pair + b_pair)
+    uint32_t pair_tx;            // bytes TMA delivers per pair
+    int pps;                     // pairs per stage
     int ns, nacc;
     uint32_t tmem_cols;
     uint32_t idesc;
+    // descriptor templates (stage 0, slot 0, k step 0) and per-step offsets in
+    // 16-byte units: off(kk, mb) = (kk >> lg) * sub16 + (kk & mask) * k16 + mb * mb16
+    uint64_t a_desc0, b_desc0;   // start address field left 0; the kernel adds the smem base
+    int a_lg, a_mask, a_sub16, a_k16, a_mb16;
+    int b_lg, b_mask, b_sub16, b_k16;
     uint32_t *status;
 };
 
@@ -72,12 +80,6 @@ struct TcArgs {
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ uint64_t globaltimer() {
-    uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
 }
 
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
@@ -97,17 +99,18 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
 }
 
 // Bounded wait for the phase of `parity` to complete.  Gives up when another
-// role of the CTA has aborted, or after kWaitLimitNs (then raises the abort
-// and the device status).  Returns false when it gave up.
-__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile uint32_t *abort_flag,
-                                       uint32_t *status) {
-    if (mbar_try(bar, parity)) return true;
-    const uint64_t t0 = globaltimer();
+// role of the CTA has aborted, or after kWaitLimitCycles (then raises the
+// abort and the device status).  Returns false when it gave up.  Lanes of one
+// warp may decide differently at the limit, so callers combine the result
+// with __all_sync before any warp-collective instruction.
+__device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, volatile uint32_t *abort_flag,
+                                            uint32_t *status) {
+    const long long t0 = clock64();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try(bar, parity)) return true;
-        if ((i & 31) == 0) {
+        if ((i & 255) == 0) {
             if (*abort_flag) return false;
-            if (globaltimer() - t0 > kWaitLimitNs) {
+            if (clock64() - t0 > kWaitLimitCycles) {
                 *abort_flag = 1;
                 atomicOr(status, kStTimeout);
                 return false;
@@ -116,11 +119,26 @@ __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile u
     }
 }
 
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile uint32_t *abort_flag,
+                                          uint32_t *status) {
+    return mbar_try(bar, parity) || mbar_wait_slow(bar, parity, abort_flag, status);
+}
+
 // Bounded wait used while draining after an abort (ignores the abort flag).
 __device__ __noinline__ void mbar_drain(uint32_t bar, uint32_t parity) {
-    const uint64_t t0 = globaltimer();
+    const long long t0 = clock64();
     while (!mbar_try(bar, parity))
-        if (globaltimer() - t0 > kWaitLimitNs) return;
+        if (clock64() - t0 > kWaitLimitCycles) return;
+}
+
+__device__ __forceinline__ bool elect_one() {
+    uint32_t pred;
+    asm volatile(
+        "{\n\t.reg .b32 r;\n\t.reg .pred p;\n\t"
+        "elect.sync r|p, 0xffffffff;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(pred));
+    return pred != 0;
 }
 
 __device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes) {
@@ -137,18 +155,6 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map
         "[%5];" ::"r"(dst),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
         : "memory");
-}
-
-// Shared-memory matrix descriptor of tcgen05 (start, leading / stride byte
-// offsets, fixed version 1, swizzle layout).
-__device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo, uint32_t layout) {
-    return (uint64_t)((addr >> 4) & 0x3FFFu) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
-           ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | (1ull << 46) | ((uint64_t)layout << 61);
-}
-
-__device__ __forceinline__ uint32_t swz_layout(int width_elems) {
-    const int bytes = width_elems * 2;
-    return bytes == 128 ? 2u : (bytes == 64 ? 4u : 6u);   // SW128 / SW64 / SW32
 }
 
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
@@ -196,28 +202,6 @@ __device__ __forceinline__ float epilogue(float x, int epi, float scale) {
     return x;
 }
 
-// A operand descriptor for K step kk and M block mb.
-__device__ __forceinline__ uint64_t a_desc(const TcArgs &a, uint32_t base, int kk, int mb) {
-    if (a.a_kmajor) {
-        const int k0 = kk * 16;
-        const uint32_t addr = base + (uint32_t)(k0 / a.wa) * a.a_sub + (uint32_t)mb * 128u * (uint32_t)a.wa * 2u +
-                              (uint32_t)(k0 % a.wa) * 2u;
-        return smem_desc(addr, 16, 8u * a.wa * 2u, swz_layout(a.wa));
-    }
-    const uint32_t addr = base + (uint32_t)mb * (uint32_t)(128 / a.wa) * a.a_sub + (uint32_t)kk * 16u * a.wa * 2u;
-    return smem_desc(addr, a.a_sub, 8u * a.wa * 2u, swz_layout(a.wa));
-}
-
-__device__ __forceinline__ uint64_t b_desc(const TcArgs &a, uint32_t base, int kk) {
-    if (a.b_kmajor) {
-        const int k0 = kk * 16;
-        const uint32_t addr = base + (uint32_t)(k0 / a.wb) * a.b_sub + (uint32_t)(k0 % a.wb) * 2u;
-        return smem_desc(addr, 16, 8u * a.wb * 2u, swz_layout(a.wb));
-    }
-    const uint32_t addr = base + (uint32_t)kk * 16u * a.wb * 2u;
-    return smem_desc(addr, a.b_sub, 8u * a.wb * 2u, swz_layout(a.wb));
-}
-
 // ------------------------------------------------------------------ kernel
 
 __global__ void __launch_bounds__(kTcThreads, 1)
@@ -230,7 +214,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8u * a.ns, accf0 = empty0 + 8u * a.ns,
                    acce0 = accf0 + 8u * a.nacc, done_bar = acce0 + 8u * a.nacc;
     uint32_t *misc = reinterpret_cast<uint32_t *>(bars + 2 * a.ns + 2 * a.nacc + 1);
-    // misc[0] TMEM base, [1] abort flag, [2] stages consumed by the MMA warp, [3] stages issued by TMA
+    // misc[0] TMEM base, [1] abort flag, [2] stages consumed by the MMA warp, [3] stages filled by TMA
     volatile uint32_t *abort_flag = misc + 1;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -268,8 +252,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
     if (warp == 0) {
         // ------------------------------------------------------- producer
-        uint32_t it = 0;
-        for (int64_t base = pb; base < pe; base += 32) {
+        uint32_t stage_it = 0, st = 0;
+        int j = 0;
+        bool stop = false;
+        for (int64_t base = pb; base < pe && !stop; base += 32) {
             const int64_t p = base + lane;
             uint32_t ia = 0, ib = 0;
             if (p < pe) {
@@ -282,62 +268,88 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 }
             }
             const int cnt = (int)(pe - base < 32 ? pe - base : 32);
-            uint32_t stop = 0;
-            for (int j = 0; j < cnt; ++j) {
-                const uint32_t xa = __shfl_sync(0xffffffffu, ia, j), xb = __shfl_sync(0xffffffffu, ib, j);
-                if (lane == 0) {
-                    const uint32_t st = it % a.ns, ph = (it / a.ns) & 1u;
-                    if (!mbar_wait(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status)) {
-                        stop = 1;
-                    } else {
-                        const uint32_t fb = full0 + 8u * st;
-                        mbar_arrive_tx(fb, a.tx_bytes);
-                        const uint32_t sa = sbase + st * a.stage_bytes, sb = sa + a.a_bytes;
-                        for (int q = 0; q < a.na_sub; ++q) tma_load_3d(sa + q * a.a_sub, &tmA, q * a.wa, 0, (int)xa, fb);
-                        for (int q = 0; q < a.nb_sub; ++q) tma_load_3d(sb + q * a.b_sub, &tmB, q * a.wb, 0, (int)xb, fb);
-                        ++it;
+            for (int jj = 0; jj < cnt; ++jj) {
+                const uint32_t xa = __shfl_sync(0xffffffffu, ia, jj), xb = __shfl_sync(0xffffffffu, ib, jj);
+                if (j == 0) {
+                    st = stage_it % a.ns;
+                    if (!__all_sync(0xffffffffu,
+                                    mbar_wait(empty0 + 8u * st, ((stage_it / a.ns) & 1u) ^ 1u, abort_flag, a.status))) {
+                        stop = true;
+                        break;
                     }
+                    const int64_t left = pe - (base + jj);
+                    const uint32_t np = (uint32_t)(left < a.pps ? left : a.pps);
+                    if (elect_one()) mbar_arrive_tx(full0 + 8u * st, np * a.pair_tx);
+                    __syncwarp();
                 }
-                if (__shfl_sync(0xffffffffu, stop, 0)) break;
+                if (elect_one()) {
+                    const uint32_t fb = full0 + 8u * st;
+                    const uint32_t sa = sbase + st * a.stage_bytes + (uint32_t)j * a.a_pair;
+                    const uint32_t sb = sbase + st * a.stage_bytes + (uint32_t)a.pps * a.a_pair + (uint32_t)j * a.b_pair;
+                    for (int q = 0; q < a.na_sub; ++q) tma_load_3d(sa + q * a.a_sub, &tmA, q * a.wa, 0, (int)xa, fb);
+                    for (int q = 0; q < a.nb_sub; ++q) tma_load_3d(sb + q * a.b_sub, &tmB, q * a.wb, 0, (int)xb, fb);
+                }
+                __syncwarp();
+                if (++j == a.pps) {
+                    j = 0;
+                    ++stage_it;
+                }
             }
-            if (__shfl_sync(0xffffffffu, stop, 0)) break;
         }
-        if (lane == 0) misc[3] = it;
+        if (j != 0) ++stage_it;   // a partly filled last stage
+        if (lane == 0) misc[3] = stage_it;
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA
-        if (lane == 0) {
-            uint32_t it = 0;
-            int64_t t = 0;
-            bool ok = true;
-            for (int64_t s = s_first; s <= s_last && ok; ++s, ++t) {
-                const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
-                const int64_t p0 = ss > pb ? ss : pb, p1 = se < pe ? se : pe;
-                const uint32_t b = (uint32_t)(t % a.nacc), ph = (uint32_t)((t / a.nacc) & 1);
-                if (!mbar_wait(acce0 + 8u * b, ph ^ 1u, abort_flag, a.status)) break;
-                tc_fence_after();
-                const uint32_t dcol = tmem + b * acc_cols;
-                for (int64_t p = p0; p < p1; ++p) {
-                    const uint32_t st = it % a.ns, sph = (it / a.ns) & 1u;
-                    if (!mbar_wait(full0 + 8u * st, sph, abort_flag, a.status)) {
+        const uint64_t adesc0 = a.a_desc0 + (sbase >> 4), bdesc0 = a.b_desc0 + (sbase >> 4);
+        const int ksteps = a.K / 16;
+        uint32_t stage_it = 0, st = 0;
+        int j = 0;
+        int64_t t = 0;
+        bool ok = true;
+        for (int64_t s = s_first; s <= s_last && ok; ++s, ++t) {
+            const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
+            const int64_t p0 = ss > pb ? ss : pb, p1 = se < pe ? se : pe;
+            const uint32_t b = (uint32_t)(t % a.nacc);
+            if (!__all_sync(0xffffffffu,
+                            mbar_wait(acce0 + 8u * b, ((uint32_t)((t / a.nacc) & 1)) ^ 1u, abort_flag, a.status)))
+                break;
+            tc_fence_after();
+            const uint32_t dcol = tmem + b * acc_cols;
+            for (int64_t p = p0; p < p1; ++p) {
+                if (j == 0) {
+                    st = stage_it % a.ns;
+                    if (!__all_sync(0xffffffffu, mbar_wait(full0 + 8u * st, (stage_it / a.ns) & 1u, abort_flag, a.status))) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t sa = sbase + st * a.stage_bytes, sb = sa + a.a_bytes;
-                    for (int kk = 0; kk < a.K / 16; ++kk) {
-                        const uint64_t bd = b_desc(a, sb, kk);
-                        for (int mb = 0; mb < a.m_blocks; ++mb)
-                            mma_bf16(dcol + (uint32_t)(mb * a.N), a_desc(a, sa, kk, mb), bd, a.idesc,
-                                     (p > p0 || kk > 0) ? 1u : 0u);
-                    }
-                    mma_commit(empty0 + 8u * st);
-                    ++it;
                 }
-                if (ok) mma_commit(accf0 + 8u * b);
+                if (elect_one()) {
+                    const uint32_t soff = (st * a.stage_bytes) >> 4;
+                    const uint64_t ad = adesc0 + soff + (((uint32_t)j * a.a_pair) >> 4);
+                    const uint64_t bd = bdesc0 + soff + (((uint32_t)a.pps * a.a_pair + (uint32_t)j * a.b_pair) >> 4);
+                    for (int kk = 0; kk < ksteps; ++kk) {
+                        const uint32_t ao = (uint32_t)((kk >> a.a_lg) * a.a_sub16 + (kk & a.a_mask) * a.a_k16);
+                        const uint32_t bo = (uint32_t)((kk >> a.b_lg) * a.b_sub16 + (kk & a.b_mask) * a.b_k16);
+                        const uint32_t acc = (p > p0 || kk > 0) ? 1u : 0u;
+                        mma_bf16(dcol, ad + ao, bd + bo, a.idesc, acc);
+                        if (a.m_blocks > 1) mma_bf16(dcol + (uint32_t)a.N, ad + ao + (uint32_t)a.a_mb16, bd + bo, a.idesc, acc);
+                    }
+                }
+                __syncwarp();
+                if (++j == a.pps || p == pe - 1) {
+                    if (elect_one()) mma_commit(empty0 + 8u * st);
+                    __syncwarp();
+                    j = 0;
+                    ++stage_it;
+                }
             }
-            misc[2] = it;
+            if (ok) {
+                if (elect_one()) mma_commit(accf0 + 8u * b);
+                __syncwarp();
+            }
         }
-        __syncwarp();
+        if (lane == 0) misc[2] = stage_it;
     } else {
         // ------------------------------------------------------- epilogue
         const int q = warp & 3;   // TMEM lane quadrant this warp may access
@@ -345,7 +357,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (int64_t s = s_first; s <= s_last; ++s, ++t) {
             const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
             const uint32_t b = (uint32_t)(t % a.nacc), ph = (uint32_t)((t / a.nacc) & 1);
-            if (!mbar_wait(accf0 + 8u * b, ph, abort_flag, a.status)) break;
+            if (!__all_sync(0xffffffffu, mbar_wait(accf0 + 8u * b, ph, abort_flag, a.status))) break;
             tc_fence_after();
             const int kind = (ss >= pb && se <= pe) ? 0 : (ss < pb ? 1 : 2);
             float *part = a.partials + ((int64_t)unit * 2 + (kind == 1 ? 0 : 1)) * a.tile_w;
@@ -359,16 +371,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         if (a.dout == UCL_BF16) {
                             __nv_bfloat16 *o = reinterpret_cast<__nv_bfloat16 *>(a.out) + s * a.tile_w + base_off;
 #pragma unroll
-                            for (int j = 0; j < 16; ++j) o[j * a.sWn] = __float2bfloat16_rn(epilogue(v[j], a.epi, a.scale));
+                            for (int jj = 0; jj < 16; ++jj) o[jj * a.sWn] = __float2bfloat16_rn(epilogue(v[jj], a.epi, a.scale));
                         } else {
                             float *o = reinterpret_cast<float *>(a.out) + s * a.tile_w + base_off;
 #pragma unroll
-                            for (int j = 0; j < 16; ++j) o[j * a.sWn] = epilogue(v[j], a.epi, a.scale);
+                            for (int jj = 0; jj < 16; ++jj) o[jj * a.sWn] = epilogue(v[jj], a.epi, a.scale);
                         }
                     } else {
                         float *o = part + base_off;
 #pragma unroll
-                        for (int j = 0; j < 16; ++j) o[j * a.sWn] = v[j];
+                        for (int jj = 0; jj < 16; ++jj) o[jj * a.sWn] = v[jj];
                     }
                 }
             }
@@ -444,19 +456,27 @@ bool operand_geometry(int rows, int cols, Operand *op, std::string *why) {
 
 struct TcGeometry {
     Operand A, B;
-    uint32_t stage_bytes, a_bytes, tx_bytes, smem_bytes, tmem_cols;
-    int ns, nacc;
+    uint32_t a_pair, b_pair, stage_bytes, pair_tx, smem_bytes, tmem_cols;
+    int pps, ns, nacc;
 };
 
-bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why) {
+// Pairs per stage: as many as keep a stage within 64 KB while leaving at
+// least three stages in flight.
+bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_override = 0) {
     // A: K-major tiles are [M][K], MN-major [K][M]; same for B with N
     if (!operand_geometry(tp.a_kmajor ? tp.M : tp.K, tp.a_kmajor ? tp.K : tp.M, &g->A, why)) return false;
     if (!operand_geometry(tp.b_kmajor ? tp.N : tp.K, tp.b_kmajor ? tp.K : tp.N, &g->B, why)) return false;
-    g->a_bytes = g->A.sub_bytes * g->A.nsub;
-    g->stage_bytes = g->a_bytes + g->B.sub_bytes * g->B.nsub;
-    g->tx_bytes = (uint32_t)(tp.M * tp.K * 2 + tp.N * tp.K * 2);
+    g->a_pair = g->A.sub_bytes * g->A.nsub;
+    g->b_pair = g->B.sub_bytes * g->B.nsub;
+    g->pair_tx = (uint32_t)(tp.M * tp.K * 2 + tp.N * tp.K * 2);
     const uint32_t bar_bytes = 8u * (2 * kMaxStages + 2 * kMaxAcc + 1) + 64;
-    int ns = (int)((kSmemLimit - 1024 - bar_bytes) / g->stage_bytes);
+    const uint32_t avail = kSmemLimit - 1024 - bar_bytes, per_pair = g->a_pair + g->b_pair;
+    int pps = 1;
+    while (pps < 4 && 2 * pps * per_pair <= 64u * 1024u && avail / (2 * pps * per_pair) >= 3) pps *= 2;
+    if (pps_override > 0) pps = pps_override;
+    g->pps = pps;
+    g->stage_bytes = pps * per_pair;
+    int ns = (int)(avail / g->stage_bytes);
     if (ns > kMaxStages) ns = kMaxStages;
     if (ns < 2) {
         *why = "tiles too large for two shared-memory stages";
@@ -474,6 +494,34 @@ bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why) {
     g->tmem_cols = cols;
     g->smem_bytes = 1024 + ns * g->stage_bytes + bar_bytes;
     return true;
+}
+
+// Shared-memory matrix descriptor of tcgen05 with the start address left 0:
+// leading / stride byte offsets, fixed version 1 (bits 46-47), swizzle mode
+// (bits 61-63: 2 = 128B, 4 = 64B, 6 = 32B).
+uint64_t desc_template(const Operand &op, bool kmajor) {
+    const uint64_t sbo = 8ull * op.w * 2;   // next group of 8 rows
+    const uint64_t lbo = kmajor ? 16 : op.sub_bytes;   // MN-major: next swizzle atom along M / N
+    const uint64_t layout = op.w == 64 ? 2 : (op.w == 32 ? 4 : 6);
+    return ((lbo >> 4) << 16) | ((sbo >> 4) << 32) | (1ull << 46) | (layout << 61);
+}
+
+// Offsets (16-byte units) of K step kk: K-major tiles advance 32 bytes inside
+// a swizzle row and jump to the next box every w/16 steps; MN-major tiles
+// advance 16 rows.
+void kstep_offsets(const Operand &op, bool kmajor, int *lg, int *mask, int *sub16, int *k16) {
+    if (kmajor) {
+        const int steps = op.w / 16;   // 1, 2 or 4
+        *lg = steps == 4 ? 2 : (steps == 2 ? 1 : 0);
+        *mask = steps - 1;
+        *sub16 = (int)(op.sub_bytes >> 4);
+        *k16 = 2;
+    } else {
+        *lg = 16;   // kk < 16: never reaches the next box
+        *mask = 0xFFFF;
+        *sub16 = 0;
+        *k16 = 2 * op.w;   // 16 rows of w * 2 bytes
+    }
 }
 
 bool make_map(CUtensorMap *m, const ucl_rel *R, const Operand &op, std::string *why) {
@@ -544,23 +592,30 @@ ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan 
     k.N = tp.N;
     k.K = tp.K;
     k.m_blocks = tp.m_blocks;
-    k.a_kmajor = tp.a_kmajor;
-    k.b_kmajor = tp.b_kmajor;
     k.wa = g.A.w;
     k.wb = g.B.w;
-    k.a_sub = g.A.sub_bytes;
-    k.b_sub = g.B.sub_bytes;
     k.na_sub = g.A.nsub;
     k.nb_sub = g.B.nsub;
-    k.a_bytes = g.a_bytes;
+    k.a_sub = g.A.sub_bytes;
+    k.b_sub = g.B.sub_bytes;
+    k.a_pair = g.a_pair;
+    k.b_pair = g.b_pair;
     k.stage_bytes = g.stage_bytes;
-    k.tx_bytes = g.tx_bytes;
+    k.pair_tx = g.pair_tx;
+    k.pps = g.pps;
     k.ns = g.ns;
     k.nacc = g.nacc;
     k.tmem_cols = g.tmem_cols;
-    // instruction descriptor, kind::f16: D fp32, A and B bf16, majors, N >> 3, M >> 4 (M = 128 per MMA)
+    // instruction descriptor, kind::f16: D fp32 (bits 4-5), A and B bf16 (7-9, 10-12),
+    // A / B major (15, 16: 1 = MN-major), N >> 3 (17-22), M >> 4 (24-28), M = 128 per MMA
     k.idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(tp.a_kmajor ? 0 : 1) << 15) |
               ((uint32_t)(tp.b_kmajor ? 0 : 1) << 16) | ((uint32_t)(tp.N >> 3) << 17) | ((128u >> 4) << 24);
+    k.a_desc0 = desc_template(g.A, tp.a_kmajor);
+    k.b_desc0 = desc_template(g.B, tp.b_kmajor);
+    kstep_offsets(g.A, tp.a_kmajor, &k.a_lg, &k.a_mask, &k.a_sub16, &k.a_k16);
+    kstep_offsets(g.B, tp.b_kmajor, &k.b_lg, &k.b_mask, &k.b_sub16, &k.b_k16);
+    // second M block: 128 rows further (K-major) or 128 / w swizzle atoms further (MN-major)
+    k.a_mb16 = tp.a_kmajor ? (int)((128u * g.A.w * 2) >> 4) : (int)((128 / g.A.w) * (g.A.sub_bytes >> 4));
     k.status = ctx->d_status;
     static int configured_smem = 0;
     if ((int)g.smem_bytes > configured_smem) {
