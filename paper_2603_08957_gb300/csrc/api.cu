@@ -257,7 +257,10 @@ bool plan_tc(const Spec &s, ucl_rel *const *in, TcPlan &tp, std::string *why) {
     if (m_ok(Lu.ext) && n_ok(Lv.ext)) tp.a_is_u = 1;
     else if (m_ok(Lv.ext) && n_ok(Lu.ext)) tp.a_is_u = 0;
     else { *why = "M/N extents do not fit tcgen05 (M 128|256, N 16..256 step 16)"; return false; }
-    if (Lk.ext % 16 != 0 || Lk.ext > 256) { *why = "K extent not a multiple of 16 up to 256"; return false; }
+    if (Lk.ext != 16 && Lk.ext != 32 && Lk.ext != 64 && Lk.ext != 128 && Lk.ext != 256) {
+        *why = "K extent must be 16, 32, 64, 128 or 256";
+        return false;
+    }
     const int ka = tp.a_is_u ? 0 : 1, kb = 1 - ka;
     const Label &LM = tp.a_is_u ? Lu : Lv, &LN = tp.a_is_u ? Lv : Lu;
     tp.M = (int)LM.ext;

@@ -98,6 +98,21 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
+// try_wait with a suspend-time hint: the thread sleeps in hardware until the
+// phase completes or about `hint_ns` pass, instead of spinning (spinning
+// warps would flood the shared-memory pipe every other role depends on).
+__device__ __forceinline__ bool mbar_try_sleep(uint32_t bar, uint32_t parity, uint32_t hint_ns) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity), "r"(hint_ns)
+        : "memory");
+    return ok != 0;
+}
+
 // Bounded wait for the phase of `parity` to complete.  Gives up when another
 // role of the CTA has aborted, or after kWaitLimitCycles (then raises the
 // abort and the device status).  Returns false when it gave up.  Lanes of one
@@ -106,15 +121,13 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
 __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, volatile uint32_t *abort_flag,
                                             uint32_t *status) {
     const long long t0 = clock64();
-    for (uint32_t i = 1;; ++i) {
-        if (mbar_try(bar, parity)) return true;
-        if ((i & 255) == 0) {
-            if (*abort_flag) return false;
-            if (clock64() - t0 > kWaitLimitCycles) {
-                *abort_flag = 1;
-                atomicOr(status, kStTimeout);
-                return false;
-            }
+    for (;;) {
+        if (mbar_try_sleep(bar, parity, 100000u)) return true;
+        if (*abort_flag) return false;
+        if (clock64() - t0 > kWaitLimitCycles) {
+            *abort_flag = 1;
+            atomicOr(status, kStTimeout);
+            return false;
         }
     }
 }
@@ -127,18 +140,8 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
 // Bounded wait used while draining after an abort (ignores the abort flag).
 __device__ __noinline__ void mbar_drain(uint32_t bar, uint32_t parity) {
     const long long t0 = clock64();
-    while (!mbar_try(bar, parity))
+    while (!mbar_try_sleep(bar, parity, 100000u))
         if (clock64() - t0 > kWaitLimitCycles) return;
-}
-
-__device__ __forceinline__ bool elect_one() {
-    uint32_t pred;
-    asm volatile(
-        "{\n\t.reg .b32 r;\n\t.reg .pred p;\n\t"
-        "elect.sync r|p, 0xffffffff;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(pred));
-    return pred != 0;
 }
 
 __device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes) {
@@ -204,6 +207,7 @@ __device__ __forceinline__ float epilogue(float x, int epi, float scale) {
 
 // ------------------------------------------------------------------ kernel
 
+template <int KSTEPS>
 __global__ void __launch_bounds__(kTcThreads, 1)
     tc_contract_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                        const TcArgs a) {
@@ -214,7 +218,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8u * a.ns, accf0 = empty0 + 8u * a.ns,
                    acce0 = accf0 + 8u * a.nacc, done_bar = acce0 + 8u * a.nacc;
     uint32_t *misc = reinterpret_cast<uint32_t *>(bars + 2 * a.ns + 2 * a.nacc + 1);
-    // misc[0] TMEM base, [1] abort flag, [2] stages consumed by the MMA warp, [3] stages filled by TMA
+    // misc[0] TMEM base, [1] abort flag, [2] stages consumed by the MMA warp, [3] stages filled by TMA,
+    // [16..48) / [48..80) tile indices of the producer's current 32 pairs
     volatile uint32_t *abort_flag = misc + 1;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -252,9 +257,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
     if (warp == 0) {
         // ------------------------------------------------------- producer
-        uint32_t stage_it = 0, st = 0;
+        // All lanes stage 32 pairs' tile indices in shared memory; one lane
+        // then walks them with no warp-collective work per pair.
+        uint32_t *s_ia = misc + 16, *s_ib = misc + 48;
+        uint32_t st = 0, ph = 0, filled = 0;
         int j = 0;
-        bool stop = false;
+        uint32_t stop = 0;
         for (int64_t base = pb; base < pe && !stop; base += 32) {
             const int64_t p = base + lane;
             uint32_t ia = 0, ib = 0;
@@ -267,96 +275,112 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     ib = 0;
                 }
             }
-            const int cnt = (int)(pe - base < 32 ? pe - base : 32);
-            for (int jj = 0; jj < cnt; ++jj) {
-                const uint32_t xa = __shfl_sync(0xffffffffu, ia, jj), xb = __shfl_sync(0xffffffffu, ib, jj);
-                if (j == 0) {
-                    st = stage_it % a.ns;
-                    if (!__all_sync(0xffffffffu,
-                                    mbar_wait(empty0 + 8u * st, ((stage_it / a.ns) & 1u) ^ 1u, abort_flag, a.status))) {
-                        stop = true;
-                        break;
+            s_ia[lane] = ia;
+            s_ib[lane] = ib;
+            __syncwarp();
+            if (lane == 0) {
+                const int cnt = (int)(pe - base < 32 ? pe - base : 32);
+                for (int jj = 0; jj < cnt; ++jj) {
+                    if (j == 0) {
+                        if (!mbar_wait(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status)) {
+                            stop = 1;
+                            break;
+                        }
+                        const int64_t left = pe - (base + jj);
+                        const uint32_t np = (uint32_t)(left < a.pps ? left : a.pps);
+                        mbar_arrive_tx(full0 + 8u * st, np * a.pair_tx);
+                        ++filled;
                     }
-                    const int64_t left = pe - (base + jj);
-                    const uint32_t np = (uint32_t)(left < a.pps ? left : a.pps);
-                    if (elect_one()) mbar_arrive_tx(full0 + 8u * st, np * a.pair_tx);
-                    __syncwarp();
-                }
-                if (elect_one()) {
                     const uint32_t fb = full0 + 8u * st;
                     const uint32_t sa = sbase + st * a.stage_bytes + (uint32_t)j * a.a_pair;
                     const uint32_t sb = sbase + st * a.stage_bytes + (uint32_t)a.pps * a.a_pair + (uint32_t)j * a.b_pair;
-                    for (int q = 0; q < a.na_sub; ++q) tma_load_3d(sa + q * a.a_sub, &tmA, q * a.wa, 0, (int)xa, fb);
-                    for (int q = 0; q < a.nb_sub; ++q) tma_load_3d(sb + q * a.b_sub, &tmB, q * a.wb, 0, (int)xb, fb);
-                }
-                __syncwarp();
-                if (++j == a.pps) {
-                    j = 0;
-                    ++stage_it;
+                    const int xa = (int)s_ia[jj], xb = (int)s_ib[jj];
+                    for (int q = 0; q < a.na_sub; ++q) tma_load_3d(sa + q * a.a_sub, &tmA, q * a.wa, 0, xa, fb);
+                    for (int q = 0; q < a.nb_sub; ++q) tma_load_3d(sb + q * a.b_sub, &tmB, q * a.wb, 0, xb, fb);
+                    if (++j == a.pps) {
+                        j = 0;
+                        if (++st == (uint32_t)a.ns) {
+                            st = 0;
+                            ph ^= 1u;
+                        }
+                    }
                 }
             }
+            stop = __shfl_sync(0xffffffffu, stop, 0);
+            __syncwarp();
         }
-        if (j != 0) ++stage_it;   // a partly filled last stage
-        if (lane == 0) misc[3] = stage_it;
+        if (lane == 0) misc[3] = filled;
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA
-        const uint64_t adesc0 = a.a_desc0 + (sbase >> 4), bdesc0 = a.b_desc0 + (sbase >> 4);
-        const int ksteps = a.K / 16;
-        uint32_t stage_it = 0, st = 0;
-        int j = 0;
-        int64_t t = 0;
-        bool ok = true;
-        for (int64_t s = s_first; s <= s_last && ok; ++s, ++t) {
-            const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
-            const int64_t p0 = ss > pb ? ss : pb, p1 = se < pe ? se : pe;
-            const uint32_t b = (uint32_t)(t % a.nacc);
-            if (!__all_sync(0xffffffffu,
-                            mbar_wait(acce0 + 8u * b, ((uint32_t)((t / a.nacc) & 1)) ^ 1u, abort_flag, a.status)))
-                break;
-            tc_fence_after();
-            const uint32_t dcol = tmem + b * acc_cols;
-            for (int64_t p = p0; p < p1; ++p) {
-                if (j == 0) {
-                    st = stage_it % a.ns;
-                    if (!__all_sync(0xffffffffu, mbar_wait(full0 + 8u * st, (stage_it / a.ns) & 1u, abort_flag, a.status))) {
-                        ok = false;
-                        break;
+        // One thread issues every MMA; descriptor offsets of the K steps are
+        // computed once, the stage / accumulator rings advance by counters.
+        if (lane == 0) {
+            uint32_t aoff[KSTEPS], boff[KSTEPS];
+#pragma unroll
+            for (int kk = 0; kk < KSTEPS; ++kk) {
+                aoff[kk] = (uint32_t)((kk >> a.a_lg) * a.a_sub16 + (kk & a.a_mask) * a.a_k16);
+                boff[kk] = (uint32_t)((kk >> a.b_lg) * a.b_sub16 + (kk & a.b_mask) * a.b_k16);
+            }
+            const uint64_t adesc0 = a.a_desc0 + (sbase >> 4);
+            const uint64_t bdesc0 = a.b_desc0 + ((sbase + (uint32_t)a.pps * a.a_pair) >> 4);
+            const uint32_t stage16 = a.stage_bytes >> 4, apair16 = a.a_pair >> 4, bpair16 = a.b_pair >> 4;
+            const uint32_t mb16 = (uint32_t)a.a_mb16, ncol = (uint32_t)a.N;
+            uint32_t st = 0, ph = 0, b = 0, aph = 0, consumed = 0;
+            int j = 0;
+            uint64_t ad = adesc0, bd = bdesc0;
+            bool ok = true;
+            for (int64_t s = s_first; s <= s_last && ok; ++s) {
+                const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
+                const int64_t p0 = ss > pb ? ss : pb, p1 = se < pe ? se : pe;
+                if (!mbar_wait(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status)) break;
+                tc_fence_after();
+                const uint32_t dcol = tmem + b * acc_cols;
+                for (int64_t p = p0; p < p1; ++p) {
+                    if (j == 0) {
+                        if (!mbar_wait(full0 + 8u * st, ph, abort_flag, a.status)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        ad = adesc0 + st * stage16;
+                        bd = bdesc0 + st * stage16;
                     }
-                    tc_fence_after();
-                }
-                if (elect_one()) {
-                    const uint32_t soff = (st * a.stage_bytes) >> 4;
-                    const uint64_t ad = adesc0 + soff + (((uint32_t)j * a.a_pair) >> 4);
-                    const uint64_t bd = bdesc0 + soff + (((uint32_t)a.pps * a.a_pair + (uint32_t)j * a.b_pair) >> 4);
-                    for (int kk = 0; kk < ksteps; ++kk) {
-                        const uint32_t ao = (uint32_t)((kk >> a.a_lg) * a.a_sub16 + (kk & a.a_mask) * a.a_k16);
-                        const uint32_t bo = (uint32_t)((kk >> a.b_lg) * a.b_sub16 + (kk & a.b_mask) * a.b_k16);
-                        const uint32_t acc = (p > p0 || kk > 0) ? 1u : 0u;
-                        mma_bf16(dcol, ad + ao, bd + bo, a.idesc, acc);
-                        if (a.m_blocks > 1) mma_bf16(dcol + (uint32_t)a.N, ad + ao + (uint32_t)a.a_mb16, bd + bo, a.idesc, acc);
+                    const uint32_t acc0 = p > p0 ? 1u : 0u;
+#pragma unroll
+                    for (int kk = 0; kk < KSTEPS; ++kk) {
+                        const uint32_t acc = kk > 0 ? 1u : acc0;
+                        mma_bf16(dcol, ad + aoff[kk], bd + boff[kk], a.idesc, acc);
+                        if (a.m_blocks > 1) mma_bf16(dcol + ncol, ad + aoff[kk] + mb16, bd + boff[kk], a.idesc, acc);
+                    }
+                    ad += apair16;
+                    bd += bpair16;
+                    if (++j == a.pps || p == pe - 1) {
+                        mma_commit(empty0 + 8u * st);
+                        ++consumed;
+                        j = 0;
+                        if (++st == (uint32_t)a.ns) {
+                            st = 0;
+                            ph ^= 1u;
+                        }
                     }
                 }
-                __syncwarp();
-                if (++j == a.pps || p == pe - 1) {
-                    if (elect_one()) mma_commit(empty0 + 8u * st);
-                    __syncwarp();
-                    j = 0;
-                    ++stage_it;
+                if (ok) {
+                    mma_commit(accf0 + 8u * b);
+                    if (++b == (uint32_t)a.nacc) {
+                        b = 0;
+                        aph ^= 1u;
+                    }
                 }
             }
-            if (ok) {
-                if (elect_one()) mma_commit(accf0 + 8u * b);
-                __syncwarp();
-            }
+            misc[2] = consumed;
         }
-        if (lane == 0) misc[2] = stage_it;
+        __syncwarp();
     } else {
         // ------------------------------------------------------- epilogue
         const int q = warp & 3;   // TMEM lane quadrant this warp may access
-        int64_t t = 0;
-        for (int64_t s = s_first; s <= s_last; ++s, ++t) {
+        uint32_t b = 0, ph = 0;
+        for (int64_t s = s_first; s <= s_last; ++s) {
             const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
-            const uint32_t b = (uint32_t)(t % a.nacc), ph = (uint32_t)((t / a.nacc) & 1);
             if (!__all_sync(0xffffffffu, mbar_wait(accf0 + 8u * b, ph, abort_flag, a.status))) break;
             tc_fence_after();
             const int kind = (ss >= pb && se <= pe) ? 0 : (ss < pb ? 1 : 2);
@@ -387,6 +411,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(acce0 + 8u * b);
+            if (++b == (uint32_t)a.nacc) {
+                b = 0;
+                ph ^= 1u;
+            }
         }
     }
 
@@ -469,7 +497,7 @@ bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_overrid
     g->a_pair = g->A.sub_bytes * g->A.nsub;
     g->b_pair = g->B.sub_bytes * g->B.nsub;
     g->pair_tx = (uint32_t)(tp.M * tp.K * 2 + tp.N * tp.K * 2);
-    const uint32_t bar_bytes = 8u * (2 * kMaxStages + 2 * kMaxAcc + 1) + 64;
+    const uint32_t bar_bytes = 8u * (2 * kMaxStages + 2 * kMaxAcc + 1) + 512;
     const uint32_t avail = kSmemLimit - 1024 - bar_bytes, per_pair = g->a_pair + g->b_pair;
     int pps = 1;
     while (pps < 4 && 2 * pps * per_pair <= 64u * 1024u && avail / (2 * pps * per_pair) >= 3) pps *= 2;
@@ -617,16 +645,20 @@ ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan 
     // second M block: 128 rows further (K-major) or 128 / w swizzle atoms further (MN-major)
     k.a_mb16 = tp.a_kmajor ? (int)((128u * g.A.w * 2) >> 4) : (int)((128 / g.A.w) * (g.A.sub_bytes >> 4));
     k.status = ctx->d_status;
-    static int configured_smem = 0;
-    if ((int)g.smem_bytes > configured_smem) {
-        ucl_status st = cuda_check(ctx,
-                                   cudaFuncSetAttribute(tc_contract_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                        (int)g.smem_bytes),
-                                   "cudaFuncSetAttribute");
-        if (st) return st;
-        configured_smem = (int)g.smem_bytes;
+    void (*kern)(const CUtensorMap, const CUtensorMap, const TcArgs) = nullptr;
+    switch (tp.K / 16) {
+        case 1: kern = tc_contract_kernel<1>; break;
+        case 2: kern = tc_contract_kernel<2>; break;
+        case 4: kern = tc_contract_kernel<4>; break;
+        case 8: kern = tc_contract_kernel<8>; break;
+        case 16: kern = tc_contract_kernel<16>; break;
+        default: return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: K must be 16, 32, 64, 128 or 256");
     }
-    tc_contract_kernel<<<a.units.G, kTcThreads, g.smem_bytes, ctx->stream>>>(mA, mB, k);
+    ucl_status st = cuda_check(
+        ctx, cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem_bytes),
+        "cudaFuncSetAttribute");
+    if (st) return st;
+    kern<<<a.units.G, kTcThreads, g.smem_bytes, ctx->stream>>>(mA, mB, k);
     ctx->launches++;
     return cuda_check(ctx, cudaGetLastError(), "tcgen05 kernel launch");
 }
