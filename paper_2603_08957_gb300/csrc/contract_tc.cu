@@ -38,7 +38,8 @@ namespace ucl {
 
 namespace {
 
-constexpr int kTcThreads = 192;
+constexpr int kProducers = 2;                  // TMA warps
+constexpr int kTcThreads = 32 * (kProducers + 5);  // + MMA warp + 4 epilogue warps
 constexpr long long kWaitLimitCycles = 2500000000ll;   // ~1.2 s at 2.07 GHz
 constexpr int kMaxStages = 8;
 constexpr int kMaxAcc = 4;
@@ -144,6 +145,16 @@ __device__ __noinline__ void mbar_drain(uint32_t bar, uint32_t parity) {
         if (clock64() - t0 > kWaitLimitCycles) return;
 }
 
+__device__ __forceinline__ bool elect_one() {
+    uint32_t pred;
+    asm volatile(
+        "{\n\t.reg .b32 r;\n\t.reg .pred p;\n\t"
+        "elect.sync r|p, 0xffffffff;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(pred));
+    return pred != 0;
+}
+
 __device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
@@ -218,8 +229,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8u * a.ns, accf0 = empty0 + 8u * a.ns,
                    acce0 = accf0 + 8u * a.nacc, done_bar = acce0 + 8u * a.nacc;
     uint32_t *misc = reinterpret_cast<uint32_t *>(bars + 2 * a.ns + 2 * a.nacc + 1);
-    // misc[0] TMEM base, [1] abort flag, [2] stages consumed by the MMA warp, [3] stages filled by TMA,
-    // [16..48) / [48..80) tile indices of the producer's current 32 pairs
+    // misc[0] TMEM base, [1] abort flag, [2] stages consumed by the MMA warp, [4 + w] stages filled
+    // by producer w, [16 + 64 w, 80 + 64 w) tile indices of producer w's current 32 pairs
     volatile uint32_t *abort_flag = misc + 1;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -233,12 +244,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             mbar_init(acce0 + 8u * i, 4);
         }
         mbar_init(done_bar, 1);
-        misc[1] = 0;
-        misc[2] = 0;
-        misc[3] = 0;
+        for (int i = 1; i < 16; ++i) misc[i] = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    if (warp == 1) {
+    if (warp == kProducers) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(misc)),
                      "r"(a.tmem_cols)
                      : "memory");
@@ -255,12 +264,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const int64_t s_last = pe > pb ? find_seg(a.seg_start, a.S, pe - 1) : -1;
     const uint32_t acc_cols = (uint32_t)(a.N * a.m_blocks);
 
-    if (warp == 0) {
-        // ------------------------------------------------------- producer
-        // All lanes stage 32 pairs' tile indices in shared memory; one lane
-        // then walks them with no warp-collective work per pair.
-        uint32_t *s_ia = misc + 16, *s_ib = misc + 48;
-        uint32_t st = 0, ph = 0, filled = 0;
+    if (warp < kProducers) {
+        // ------------------------------------------------------ producers
+        // Producer warp w fills the stages of fill number w, w + kProducers,
+        // ...  Its lanes stage 32 pairs' tile indices in shared memory; one
+        // lane then walks them with no warp-collective work per pair.
+        uint32_t *s_ia = misc + 16 + 64 * warp, *s_ib = s_ia + 32;
+        uint32_t st = 0, ph = 0, fill = 0, mine = 0;
         int j = 0;
         uint32_t stop = 0;
         for (int64_t base = pb; base < pe && !stop; base += 32) {
@@ -281,7 +291,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if (lane == 0) {
                 const int cnt = (int)(pe - base < 32 ? pe - base : 32);
                 for (int jj = 0; jj < cnt; ++jj) {
-                    if (j == 0) {
+                    const bool own = (fill % kProducers) == (uint32_t)warp;
+                    if (j == 0 && own) {
                         if (!mbar_wait(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status)) {
                             stop = 1;
                             break;
@@ -289,16 +300,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         const int64_t left = pe - (base + jj);
                         const uint32_t np = (uint32_t)(left < a.pps ? left : a.pps);
                         mbar_arrive_tx(full0 + 8u * st, np * a.pair_tx);
-                        ++filled;
+                        ++mine;
                     }
-                    const uint32_t fb = full0 + 8u * st;
-                    const uint32_t sa = sbase + st * a.stage_bytes + (uint32_t)j * a.a_pair;
-                    const uint32_t sb = sbase + st * a.stage_bytes + (uint32_t)a.pps * a.a_pair + (uint32_t)j * a.b_pair;
-                    const int xa = (int)s_ia[jj], xb = (int)s_ib[jj];
-                    for (int q = 0; q < a.na_sub; ++q) tma_load_3d(sa + q * a.a_sub, &tmA, q * a.wa, 0, xa, fb);
-                    for (int q = 0; q < a.nb_sub; ++q) tma_load_3d(sb + q * a.b_sub, &tmB, q * a.wb, 0, xb, fb);
+                    if (own) {
+                        const uint32_t fb = full0 + 8u * st;
+                        const uint32_t sa = sbase + st * a.stage_bytes + (uint32_t)j * a.a_pair;
+                        const uint32_t sb =
+                            sbase + st * a.stage_bytes + (uint32_t)a.pps * a.a_pair + (uint32_t)j * a.b_pair;
+                        const int xa = (int)s_ia[jj], xb = (int)s_ib[jj];
+                        for (int q = 0; q < a.na_sub; ++q) tma_load_3d(sa + q * a.a_sub, &tmA, q * a.wa, 0, xa, fb);
+                        for (int q = 0; q < a.nb_sub; ++q) tma_load_3d(sb + q * a.b_sub, &tmB, q * a.wb, 0, xb, fb);
+                    }
                     if (++j == a.pps) {
                         j = 0;
+                        ++fill;
                         if (++st == (uint32_t)a.ns) {
                             st = 0;
                             ph ^= 1u;
@@ -309,72 +324,75 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             stop = __shfl_sync(0xffffffffu, stop, 0);
             __syncwarp();
         }
-        if (lane == 0) misc[3] = filled;
-    } else if (warp == 1) {
+        if (lane == 0) misc[4 + warp] = mine;
+    } else if (warp == kProducers) {
         // ------------------------------------------------------------ MMA
-        // One thread issues every MMA; descriptor offsets of the K steps are
-        // computed once, the stage / accumulator rings advance by counters.
-        if (lane == 0) {
-            uint32_t aoff[KSTEPS], boff[KSTEPS];
+        // Warp-uniform loop; one elected lane issues.  Descriptor offsets of
+        // the K steps are computed once; stage / accumulator rings advance by
+        // counters.
+        uint32_t aoff[KSTEPS], boff[KSTEPS];
 #pragma unroll
-            for (int kk = 0; kk < KSTEPS; ++kk) {
-                aoff[kk] = (uint32_t)((kk >> a.a_lg) * a.a_sub16 + (kk & a.a_mask) * a.a_k16);
-                boff[kk] = (uint32_t)((kk >> a.b_lg) * a.b_sub16 + (kk & a.b_mask) * a.b_k16);
-            }
-            const uint64_t adesc0 = a.a_desc0 + (sbase >> 4);
-            const uint64_t bdesc0 = a.b_desc0 + ((sbase + (uint32_t)a.pps * a.a_pair) >> 4);
-            const uint32_t stage16 = a.stage_bytes >> 4, apair16 = a.a_pair >> 4, bpair16 = a.b_pair >> 4;
-            const uint32_t mb16 = (uint32_t)a.a_mb16, ncol = (uint32_t)a.N;
-            uint32_t st = 0, ph = 0, b = 0, aph = 0, consumed = 0;
-            int j = 0;
-            uint64_t ad = adesc0, bd = bdesc0;
-            bool ok = true;
-            for (int64_t s = s_first; s <= s_last && ok; ++s) {
-                const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
-                const int64_t p0 = ss > pb ? ss : pb, p1 = se < pe ? se : pe;
-                if (!mbar_wait(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status)) break;
-                tc_fence_after();
-                const uint32_t dcol = tmem + b * acc_cols;
-                for (int64_t p = p0; p < p1; ++p) {
-                    if (j == 0) {
-                        if (!mbar_wait(full0 + 8u * st, ph, abort_flag, a.status)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-                        ad = adesc0 + st * stage16;
-                        bd = bdesc0 + st * stage16;
+        for (int kk = 0; kk < KSTEPS; ++kk) {
+            aoff[kk] = (uint32_t)((kk >> a.a_lg) * a.a_sub16 + (kk & a.a_mask) * a.a_k16);
+            boff[kk] = (uint32_t)((kk >> a.b_lg) * a.b_sub16 + (kk & a.b_mask) * a.b_k16);
+        }
+        const uint64_t adesc0 = a.a_desc0 + (sbase >> 4);
+        const uint64_t bdesc0 = a.b_desc0 + ((sbase + (uint32_t)a.pps * a.a_pair) >> 4);
+        const uint32_t stage16 = a.stage_bytes >> 4, apair16 = a.a_pair >> 4, bpair16 = a.b_pair >> 4;
+        const uint32_t mb16 = (uint32_t)a.a_mb16, ncol = (uint32_t)a.N;
+        const bool two_m = a.m_blocks > 1;
+        uint32_t st = 0, ph = 0, b = 0, aph = 0, consumed = 0;
+        int j = 0;
+        uint64_t ad = adesc0, bd = bdesc0;
+        bool ok = true;
+        for (int64_t s = s_first; s <= s_last && ok; ++s) {
+            const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
+            const int64_t p0 = ss > pb ? ss : pb, p1 = se < pe ? se : pe;
+            if (!__all_sync(0xffffffffu, mbar_wait(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status))) break;
+            tc_fence_after();
+            const uint32_t dcol = tmem + b * acc_cols;
+            for (int64_t p = p0; p < p1; ++p) {
+                if (j == 0) {
+                    if (!__all_sync(0xffffffffu, mbar_wait(full0 + 8u * st, ph, abort_flag, a.status))) {
+                        ok = false;
+                        break;
                     }
-                    const uint32_t acc0 = p > p0 ? 1u : 0u;
+                    tc_fence_after();
+                    ad = adesc0 + st * stage16;
+                    bd = bdesc0 + st * stage16;
+                }
+                const uint32_t acc0 = p > p0 ? 1u : 0u;
+                if (elect_one()) {
 #pragma unroll
                     for (int kk = 0; kk < KSTEPS; ++kk) {
-                        const uint32_t acc = kk > 0 ? 1u : acc0;
-                        mma_bf16(dcol, ad + aoff[kk], bd + boff[kk], a.idesc, acc);
-                        if (a.m_blocks > 1) mma_bf16(dcol + ncol, ad + aoff[kk] + mb16, bd + boff[kk], a.idesc, acc);
-                    }
-                    ad += apair16;
-                    bd += bpair16;
-                    if (++j == a.pps || p == pe - 1) {
-                        mma_commit(empty0 + 8u * st);
-                        ++consumed;
-                        j = 0;
-                        if (++st == (uint32_t)a.ns) {
-                            st = 0;
-                            ph ^= 1u;
-                        }
+                        mma_bf16(dcol, ad + aoff[kk], bd + boff[kk], a.idesc, kk > 0 ? 1u : acc0);
+                        if (two_m) mma_bf16(dcol + ncol, ad + aoff[kk] + mb16, bd + boff[kk], a.idesc, kk > 0 ? 1u : acc0);
                     }
                 }
-                if (ok) {
-                    mma_commit(accf0 + 8u * b);
-                    if (++b == (uint32_t)a.nacc) {
-                        b = 0;
-                        aph ^= 1u;
+                __syncwarp();
+                ad += apair16;
+                bd += bpair16;
+                if (++j == a.pps || p == pe - 1) {
+                    if (elect_one()) mma_commit(empty0 + 8u * st);
+                    __syncwarp();
+                    ++consumed;
+                    j = 0;
+                    if (++st == (uint32_t)a.ns) {
+                        st = 0;
+                        ph ^= 1u;
                     }
                 }
             }
-            misc[2] = consumed;
+            if (ok) {
+                if (elect_one()) mma_commit(accf0 + 8u * b);
+                __syncwarp();
+                if (++b == (uint32_t)a.nacc) {
+                    b = 0;
+                    aph ^= 1u;
+                }
+            }
         }
-        __syncwarp();
+        if (lane == 0) misc[2] = consumed;
     } else {
         // ------------------------------------------------------- epilogue
         const int q = warp & 3;   // TMEM lane quadrant this warp may access
@@ -421,18 +439,22 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // ---------------------------------------------------------- teardown
     __syncthreads();
     if (*abort_flag) {
-        if (warp == 0 && lane == 0) {
-            // copies still in flight write into this CTA's shared memory: wait for them
-            for (uint32_t it = misc[2]; it < misc[3]; ++it) mbar_drain(full0 + 8u * (it % a.ns), (it / a.ns) & 1u);
+        if (warp < kProducers && lane == 0) {
+            // copies still in flight write into this CTA's shared memory: wait
+            // for every stage this producer filled that the MMA warp did not consume
+            for (uint32_t k = 0; k < misc[4 + warp]; ++k) {
+                const uint32_t it = (uint32_t)warp + k * kProducers;   // fills this producer issued
+                if (it >= misc[2]) mbar_drain(full0 + 8u * (it % a.ns), (it / a.ns) & 1u);
+            }
         }
-        if (warp == 1 && lane == 0) {
+        if (warp == kProducers && lane == 0) {
             mma_commit(done_bar);   // tracks every MMA this thread issued
             mbar_drain(done_bar, 0);
         }
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 1) {
+    if (warp == kProducers) {
         tc_fence_after();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(a.tmem_cols)
                      : "memory");
@@ -497,7 +519,7 @@ bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_overrid
     g->a_pair = g->A.sub_bytes * g->A.nsub;
     g->b_pair = g->B.sub_bytes * g->B.nsub;
     g->pair_tx = (uint32_t)(tp.M * tp.K * 2 + tp.N * tp.K * 2);
-    const uint32_t bar_bytes = 8u * (2 * kMaxStages + 2 * kMaxAcc + 1) + 512;
+    const uint32_t bar_bytes = 8u * (2 * kMaxStages + 2 * kMaxAcc + 1) + 64 + 256u * kProducers + 64;
     const uint32_t avail = kSmemLimit - 1024 - bar_bytes, per_pair = g->a_pair + g->b_pair;
     int pps = 1;
     while (pps < 4 && 2 * pps * per_pair <= 64u * 1024u && avail / (2 * pps * per_pair) >= 3) pps *= 2;
