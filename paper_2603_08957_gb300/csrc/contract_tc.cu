@@ -327,9 +327,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (lane == 0) misc[4 + warp] = mine;
     } else if (warp == kProducers) {
         // ------------------------------------------------------------ MMA
-        // Warp-uniform loop; one elected lane issues.  Descriptor offsets of
-        // the K steps are computed once; stage / accumulator rings advance by
-        // counters.
+        // Warp-uniform loop over stages; one elected lane issues.  In the
+        // common case a whole stage lies inside the current segment and one
+        // elected region issues all of its MMAs and the stage's commit (the
+        // tensor pipe is fed back to back); segment starts and ends take the
+        // per-pair path.  Descriptor offsets of the K steps are computed once.
         uint32_t aoff[KSTEPS], boff[KSTEPS];
 #pragma unroll
         for (int kk = 0; kk < KSTEPS; ++kk) {
@@ -339,57 +341,94 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const uint64_t adesc0 = a.a_desc0 + (sbase >> 4);
         const uint64_t bdesc0 = a.b_desc0 + ((sbase + (uint32_t)a.pps * a.a_pair) >> 4);
         const uint32_t stage16 = a.stage_bytes >> 4, apair16 = a.a_pair >> 4, bpair16 = a.b_pair >> 4;
-        const uint32_t mb16 = (uint32_t)a.a_mb16, ncol = (uint32_t)a.N;
+        const uint32_t mb16 = (uint32_t)a.a_mb16, ncol = (uint32_t)a.N, idesc = a.idesc;
         const bool two_m = a.m_blocks > 1;
-        uint32_t st = 0, ph = 0, b = 0, aph = 0, consumed = 0;
-        int j = 0;
-        uint64_t ad = adesc0, bd = bdesc0;
-        bool ok = true;
-        for (int64_t s = s_first; s <= s_last && ok; ++s) {
-            const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
-            const int64_t p0 = ss > pb ? ss : pb, p1 = se < pe ? se : pe;
-            if (!__all_sync(0xffffffffu, mbar_wait(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status))) break;
+        const int n = (int)(pe - pb), pps = a.pps;
+        uint32_t st = 0, ph = 0, b = 0, aph = 0, consumed = 0, dcol = tmem;
+        int64_t s = s_first;
+        int i = 0;   // pairs of this unit issued so far
+        int seg_end = n > 0 ? (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) : 0;
+        bool fresh = true, ok = true;
+        while (i < n) {
+            const int np = n - i < pps ? n - i : pps;
+            if (!__all_sync(0xffffffffu, mbar_wait(full0 + 8u * st, ph, abort_flag, a.status))) {
+                ok = false;
+                break;
+            }
             tc_fence_after();
-            const uint32_t dcol = tmem + b * acc_cols;
-            for (int64_t p = p0; p < p1; ++p) {
-                if (j == 0) {
-                    if (!__all_sync(0xffffffffu, mbar_wait(full0 + 8u * st, ph, abort_flag, a.status))) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    ad = adesc0 + st * stage16;
-                    bd = bdesc0 + st * stage16;
-                }
-                const uint32_t acc0 = p > p0 ? 1u : 0u;
+            uint64_t ad = adesc0 + st * stage16, bd = bdesc0 + st * stage16;
+            if (!fresh && i + np <= seg_end) {
+                // fast path: the whole stage accumulates into the open accumulator
                 if (elect_one()) {
+                    for (int jj = 0; jj < np; ++jj) {
 #pragma unroll
-                    for (int kk = 0; kk < KSTEPS; ++kk) {
-                        mma_bf16(dcol, ad + aoff[kk], bd + boff[kk], a.idesc, kk > 0 ? 1u : acc0);
-                        if (two_m) mma_bf16(dcol + ncol, ad + aoff[kk] + mb16, bd + boff[kk], a.idesc, kk > 0 ? 1u : acc0);
+                        for (int kk = 0; kk < KSTEPS; ++kk) {
+                            mma_bf16(dcol, ad + aoff[kk], bd + boff[kk], idesc, 1u);
+                            if (two_m) mma_bf16(dcol + ncol, ad + aoff[kk] + mb16, bd + boff[kk], idesc, 1u);
+                        }
+                        ad += apair16;
+                        bd += bpair16;
                     }
+                    mma_commit(empty0 + 8u * st);
                 }
                 __syncwarp();
-                ad += apair16;
-                bd += bpair16;
-                if (++j == a.pps || p == pe - 1) {
-                    if (elect_one()) mma_commit(empty0 + 8u * st);
+                i += np;
+            } else {
+                for (int jj = 0; jj < np; ++jj, ++i) {
+                    if (fresh) {
+                        if (!__all_sync(0xffffffffu, mbar_wait(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status))) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        dcol = tmem + b * acc_cols;
+                    }
+                    const uint32_t acc0 = fresh ? 0u : 1u;
+                    if (elect_one()) {
+#pragma unroll
+                        for (int kk = 0; kk < KSTEPS; ++kk) {
+                            const uint32_t acc = kk > 0 ? 1u : acc0;
+                            mma_bf16(dcol, ad + aoff[kk], bd + boff[kk], idesc, acc);
+                            if (two_m) mma_bf16(dcol + ncol, ad + aoff[kk] + mb16, bd + boff[kk], idesc, acc);
+                        }
+                    }
                     __syncwarp();
-                    ++consumed;
-                    j = 0;
-                    if (++st == (uint32_t)a.ns) {
-                        st = 0;
-                        ph ^= 1u;
+                    fresh = false;
+                    ad += apair16;
+                    bd += bpair16;
+                    if (i + 1 == seg_end) {
+                        // the segment's last pair in this unit: hand the accumulator to the epilogue
+                        if (elect_one()) mma_commit(accf0 + 8u * b);
+                        __syncwarp();
+                        if (++b == (uint32_t)a.nacc) {
+                            b = 0;
+                            aph ^= 1u;
+                        }
+                        ++s;
+                        if (i + 1 < n) seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
+                        fresh = true;
                     }
                 }
+                if (!ok) break;
+                if (elect_one()) mma_commit(empty0 + 8u * st);
+                __syncwarp();
             }
-            if (ok) {
+            // a fast-path stage may also end exactly at the segment's end
+            if (!fresh && i == seg_end) {
                 if (elect_one()) mma_commit(accf0 + 8u * b);
                 __syncwarp();
                 if (++b == (uint32_t)a.nacc) {
                     b = 0;
                     aph ^= 1u;
                 }
+                ++s;
+                if (i < n) seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
+                fresh = true;
+            }
+            ++consumed;
+            if (++st == (uint32_t)a.ns) {
+                st = 0;
+                ph ^= 1u;
             }
         }
         if (lane == 0) misc[2] = consumed;
