@@ -38,8 +38,9 @@ namespace ucl {
 
 namespace {
 
-constexpr int kProducers = 2;                  // TMA warps
-constexpr int kTcThreads = 32 * (kProducers + 5);  // + MMA warp + 4 epilogue warps
+constexpr int kProducers = 2;                                 // TMA warps
+constexpr int kMmaWarps = 2;                                  // MMA-issuing warps (the first also owns TMEM)
+constexpr int kTcThreads = 32 * (kProducers + kMmaWarps + 4);  // + 4 epilogue warps
 constexpr long long kWaitLimitCycles = 2500000000ll;   // ~1.2 s at 2.07 GHz
 constexpr int kMaxStages = 8;
 constexpr int kMaxAcc = 4;
@@ -66,7 +67,7 @@ struct TcArgs {
     uint32_t stage_bytes;        // pps * (a_pair + b_pair)
     uint32_t pair_tx;            // bytes TMA delivers per pair
     int pps;                     // pairs per stage
-    int ns, nacc;
+    int ns, nacc, nmma;
     uint32_t tmem_cols;
     uint32_t idesc;
     // descriptor templates (stage 0, slot 0, k step 0) and per-step offsets in
@@ -218,6 +219,14 @@ __device__ __forceinline__ float epilogue(float x, int epi, float scale) {
 
 // ------------------------------------------------------------------ kernel
 
+__device__ __forceinline__ void tmem_st16_zero(uint32_t taddr) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %1, %1, %1, %1, %1, %1, %1, %1, %1, %1, %1, %1, %1, %1, "
+        "%1};" ::"r"(taddr),
+        "r"(0u)
+        : "memory");
+}
+
 template <int KSTEPS>
 __global__ void __launch_bounds__(kTcThreads, 1)
     tc_contract_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -229,10 +238,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8u * a.ns, accf0 = empty0 + 8u * a.ns,
                    acce0 = accf0 + 8u * a.nacc, done_bar = acce0 + 8u * a.nacc;
     uint32_t *misc = reinterpret_cast<uint32_t *>(bars + 2 * a.ns + 2 * a.nacc + 1);
-    // misc[0] TMEM base, [1] abort flag, [2] stages consumed by the MMA warp, [4 + w] stages filled
-    // by producer w, [16 + 64 w, 80 + 64 w) tile indices of producer w's current 32 pairs
+    // misc[0] TMEM base, [1] abort flag, [2 + w] stage fills MMA warp w has walked past,
+    // [4 + w] stages filled by producer w, [16 + 64 w, 80 + 64 w) tile indices staged by producer w
     volatile uint32_t *abort_flag = misc + 1;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nmma = a.nmma;
+    const uint32_t acc_cols = (uint32_t)(a.N * a.m_blocks), buf_cols = acc_cols * (uint32_t)nmma;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < a.ns; ++i) {
@@ -240,10 +251,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             mbar_init(empty0 + 8u * i, 1);
         }
         for (int i = 0; i < a.nacc; ++i) {
-            mbar_init(accf0 + 8u * i, 1);
+            mbar_init(accf0 + 8u * i, (uint32_t)nmma);
             mbar_init(acce0 + 8u * i, 4);
         }
-        mbar_init(done_bar, 1);
+        mbar_init(done_bar, (uint32_t)nmma);
         for (int i = 1; i < 16; ++i) misc[i] = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -257,12 +268,21 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = misc[0];
+    if (warp >= kProducers + kMmaWarps) {
+        // accumulators start at zero: every MMA accumulates, and the epilogue
+        // re-zeroes a buffer after draining it
+        const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+        for (uint32_t c = 0; c < a.tmem_cols; c += 16) tmem_st16_zero(tmem + lane_base + c);
+        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
 
     const int unit = blockIdx.x;
     const int64_t pb = a.units.begin(unit), pe = a.units.begin(unit + 1);
     const int64_t s_first = pe > pb ? find_seg(a.seg_start, a.S, pb) : 0;
     const int64_t s_last = pe > pb ? find_seg(a.seg_start, a.S, pe - 1) : -1;
-    const uint32_t acc_cols = (uint32_t)(a.N * a.m_blocks);
 
     if (warp < kProducers) {
         // ------------------------------------------------------ producers
@@ -325,116 +345,150 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             __syncwarp();
         }
         if (lane == 0) misc[4 + warp] = mine;
-    } else if (warp == kProducers) {
+    } else if (warp < kProducers + kMmaWarps) {
         // ------------------------------------------------------------ MMA
-        // Warp-uniform loop over stages; one elected lane issues.  In the
-        // common case a whole stage lies inside the current segment and one
-        // elected region issues all of its MMAs and the stage's commit (the
-        // tensor pipe is fed back to back); segment starts and ends take the
-        // per-pair path.  Descriptor offsets of the K steps are computed once.
-        uint32_t aoff[KSTEPS], boff[KSTEPS];
+        // MMA warp w consumes the stages of fill number w, w + nmma, ... and
+        // accumulates into its own half of each TMEM accumulator buffer, so
+        // that one warp's bookkeeping overlaps the other's MMAs.  Every warp
+        // walks all stages and segments to keep the buffer ring in step.
+        // Loops are warp-uniform; descriptors are formed in uniform code and
+        // one elected lane issues.
+        const int w = warp - kProducers;
+        if (w < nmma) {
+            uint32_t aoff[KSTEPS], boff[KSTEPS];
 #pragma unroll
-        for (int kk = 0; kk < KSTEPS; ++kk) {
-            aoff[kk] = (uint32_t)((kk >> a.a_lg) * a.a_sub16 + (kk & a.a_mask) * a.a_k16);
-            boff[kk] = (uint32_t)((kk >> a.b_lg) * a.b_sub16 + (kk & a.b_mask) * a.b_k16);
-        }
-        const uint64_t adesc0 = a.a_desc0 + (sbase >> 4);
-        const uint64_t bdesc0 = a.b_desc0 + ((sbase + (uint32_t)a.pps * a.a_pair) >> 4);
-        const uint32_t stage16 = a.stage_bytes >> 4, apair16 = a.a_pair >> 4, bpair16 = a.b_pair >> 4;
-        const uint32_t mb16 = (uint32_t)a.a_mb16, ncol = (uint32_t)a.N, idesc = a.idesc;
-        const bool two_m = a.m_blocks > 1;
-        const int n = (int)(pe - pb), pps = a.pps;
-        uint32_t st = 0, ph = 0, b = 0, aph = 0, consumed = 0, dcol = tmem;
-        int64_t s = s_first;
-        int i = 0;   // pairs of this unit issued so far
-        int seg_end = n > 0 ? (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) : 0;
-        bool fresh = true, ok = true;
-        while (i < n) {
-            const int np = n - i < pps ? n - i : pps;
-            if (!__all_sync(0xffffffffu, mbar_wait(full0 + 8u * st, ph, abort_flag, a.status))) {
-                ok = false;
-                break;
+            for (int kk = 0; kk < KSTEPS; ++kk) {
+                aoff[kk] = (uint32_t)((kk >> a.a_lg) * a.a_sub16 + (kk & a.a_mask) * a.a_k16);
+                boff[kk] = (uint32_t)((kk >> a.b_lg) * a.b_sub16 + (kk & a.b_mask) * a.b_k16);
             }
-            tc_fence_after();
-            uint64_t ad = adesc0 + st * stage16, bd = bdesc0 + st * stage16;
-            if (!fresh && i + np <= seg_end) {
-                // fast path: the whole stage accumulates into the open accumulator
-                if (elect_one()) {
-                    for (int jj = 0; jj < np; ++jj) {
+            const uint64_t adesc0 = a.a_desc0 + (sbase >> 4);
+            const uint64_t bdesc0 = a.b_desc0 + ((sbase + (uint32_t)a.pps * a.a_pair) >> 4);
+            const uint32_t stage16 = a.stage_bytes >> 4, apair16 = a.a_pair >> 4, bpair16 = a.b_pair >> 4;
+            const uint32_t mb16 = (uint32_t)a.a_mb16, ncol = (uint32_t)a.N, idesc = a.idesc;
+            const bool two_m = a.m_blocks > 1;
+            const int n = (int)(pe - pb), pps = a.pps;
+            uint32_t st = 0, ph = 0, b = 0, aph = 0, dcol = tmem;
+            uint32_t fill = 0;
+            int64_t s = s_first;
+            int i = 0;
+            int seg_end = n > 0 ? (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) : 0;
+            bool fresh = true, ok = true;
+            while (i < n) {
+                const int np = n - i < pps ? n - i : pps;
+                const bool own = (int)(fill % (uint32_t)nmma) == w;
+                if (own) {
+                    if (!__all_sync(0xffffffffu, mbar_wait(full0 + 8u * st, ph, abort_flag, a.status))) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                }
+                uint64_t ad = adesc0 + st * stage16, bd = bdesc0 + st * stage16;
+                if (!fresh && i + np <= seg_end) {
+                    // the whole stage accumulates into the open buffer
+                    if (own) {
+                        const uint64_t ad1 = ad + apair16, bd1 = bd + bpair16;
+                        const uint64_t ad2 = ad1 + apair16, bd2 = bd1 + bpair16;
+                        const uint64_t ad3 = ad2 + apair16, bd3 = bd2 + bpair16;
+                        if (elect_one()) {
 #pragma unroll
-                        for (int kk = 0; kk < KSTEPS; ++kk) {
-                            mma_bf16(dcol, ad + aoff[kk], bd + boff[kk], idesc, 1u);
-                            if (two_m) mma_bf16(dcol + ncol, ad + aoff[kk] + mb16, bd + boff[kk], idesc, 1u);
+                            for (int kk = 0; kk < KSTEPS; ++kk) {
+                                mma_bf16(dcol, ad + aoff[kk], bd + boff[kk], idesc, 1u);
+                                if (two_m) mma_bf16(dcol + ncol, ad + aoff[kk] + mb16, bd + boff[kk], idesc, 1u);
+                            }
+                            if (np > 1) {
+#pragma unroll
+                                for (int kk = 0; kk < KSTEPS; ++kk) {
+                                    mma_bf16(dcol, ad1 + aoff[kk], bd1 + boff[kk], idesc, 1u);
+                                    if (two_m) mma_bf16(dcol + ncol, ad1 + aoff[kk] + mb16, bd1 + boff[kk], idesc, 1u);
+                                }
+                            }
+                            if (np > 2) {
+#pragma unroll
+                                for (int kk = 0; kk < KSTEPS; ++kk) {
+                                    mma_bf16(dcol, ad2 + aoff[kk], bd2 + boff[kk], idesc, 1u);
+                                    if (two_m) mma_bf16(dcol + ncol, ad2 + aoff[kk] + mb16, bd2 + boff[kk], idesc, 1u);
+                                }
+                            }
+                            if (np > 3) {
+#pragma unroll
+                                for (int kk = 0; kk < KSTEPS; ++kk) {
+                                    mma_bf16(dcol, ad3 + aoff[kk], bd3 + boff[kk], idesc, 1u);
+                                    if (two_m) mma_bf16(dcol + ncol, ad3 + aoff[kk] + mb16, bd3 + boff[kk], idesc, 1u);
+                                }
+                            }
+                            mma_commit(empty0 + 8u * st);
+                        }
+                        __syncwarp();
+                    }
+                    i += np;
+                } else {
+                    // segment boundaries inside the stage: pair by pair
+                    for (int jj = 0; jj < np; ++jj, ++i) {
+                        if (fresh) {
+                            if (!__all_sync(0xffffffffu, mbar_wait(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status))) {
+                                ok = false;
+                                break;
+                            }
+                            tc_fence_after();
+                            dcol = tmem + b * buf_cols + (uint32_t)w * acc_cols;
+                            fresh = false;
+                        }
+                        if (own) {
+                            if (elect_one()) {
+#pragma unroll
+                                for (int kk = 0; kk < KSTEPS; ++kk) {
+                                    mma_bf16(dcol, ad + aoff[kk], bd + boff[kk], idesc, 1u);
+                                    if (two_m) mma_bf16(dcol + ncol, ad + aoff[kk] + mb16, bd + boff[kk], idesc, 1u);
+                                }
+                            }
+                            __syncwarp();
                         }
                         ad += apair16;
                         bd += bpair16;
-                    }
-                    mma_commit(empty0 + 8u * st);
-                }
-                __syncwarp();
-                i += np;
-            } else {
-                for (int jj = 0; jj < np; ++jj, ++i) {
-                    if (fresh) {
-                        if (!__all_sync(0xffffffffu, mbar_wait(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status))) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-                        dcol = tmem + b * acc_cols;
-                    }
-                    const uint32_t acc0 = fresh ? 0u : 1u;
-                    if (elect_one()) {
-#pragma unroll
-                        for (int kk = 0; kk < KSTEPS; ++kk) {
-                            const uint32_t acc = kk > 0 ? 1u : acc0;
-                            mma_bf16(dcol, ad + aoff[kk], bd + boff[kk], idesc, acc);
-                            if (two_m) mma_bf16(dcol + ncol, ad + aoff[kk] + mb16, bd + boff[kk], idesc, acc);
+                        if (i + 1 == seg_end) {
+                            // the segment's last pair in this unit: hand the buffer to the epilogue
+                            if (elect_one()) mma_commit(accf0 + 8u * b);
+                            __syncwarp();
+                            if (++b == (uint32_t)a.nacc) {
+                                b = 0;
+                                aph ^= 1u;
+                            }
+                            ++s;
+                            if (i + 1 < n) seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
+                            fresh = true;
                         }
                     }
-                    __syncwarp();
-                    fresh = false;
-                    ad += apair16;
-                    bd += bpair16;
-                    if (i + 1 == seg_end) {
-                        // the segment's last pair in this unit: hand the accumulator to the epilogue
-                        if (elect_one()) mma_commit(accf0 + 8u * b);
+                    if (!ok) break;
+                    if (own) {
+                        if (elect_one()) mma_commit(empty0 + 8u * st);
                         __syncwarp();
-                        if (++b == (uint32_t)a.nacc) {
-                            b = 0;
-                            aph ^= 1u;
-                        }
-                        ++s;
-                        if (i + 1 < n) seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
-                        fresh = true;
                     }
                 }
-                if (!ok) break;
-                if (elect_one()) mma_commit(empty0 + 8u * st);
-                __syncwarp();
-            }
-            // a fast-path stage may also end exactly at the segment's end
-            if (!fresh && i == seg_end) {
-                if (elect_one()) mma_commit(accf0 + 8u * b);
-                __syncwarp();
-                if (++b == (uint32_t)a.nacc) {
-                    b = 0;
-                    aph ^= 1u;
+                // a fast-path stage may end exactly at the segment's end
+                if (!fresh && i == seg_end) {
+                    if (elect_one()) mma_commit(accf0 + 8u * b);
+                    __syncwarp();
+                    if (++b == (uint32_t)a.nacc) {
+                        b = 0;
+                        aph ^= 1u;
+                    }
+                    ++s;
+                    if (i < n) seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
+                    fresh = true;
                 }
-                ++s;
-                if (i < n) seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
-                fresh = true;
+                ++fill;
+                if (++st == (uint32_t)a.ns) {
+                    st = 0;
+                    ph ^= 1u;
+                }
             }
-            ++consumed;
-            if (++st == (uint32_t)a.ns) {
-                st = 0;
-                ph ^= 1u;
-            }
+            if (lane == 0) misc[2 + w] = ok ? 0xFFFFFFFFu : fill;
         }
-        if (lane == 0) misc[2] = consumed;
     } else {
         // ------------------------------------------------------- epilogue
         const int q = warp & 3;   // TMEM lane quadrant this warp may access
+        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         uint32_t b = 0, ph = 0;
         for (int64_t s = s_first; s <= s_last; ++s) {
             const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
@@ -442,11 +496,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             tc_fence_after();
             const int kind = (ss >= pb && se <= pe) ? 0 : (ss < pb ? 1 : 2);
             float *part = a.partials + ((int64_t)unit * 2 + (kind == 1 ? 0 : 1)) * a.tile_w;
+            const uint32_t bcol = tmem + lane_base + b * buf_cols;
             for (int mb = 0; mb < a.m_blocks; ++mb) {
                 const int64_t m = (int64_t)mb * 128 + q * 32 + lane;
                 for (int c = 0; c < a.N / 16; ++c) {
                     float v[16];
-                    tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + b * acc_cols + (uint32_t)(mb * a.N + c * 16), v);
+                    const uint32_t col = (uint32_t)(mb * a.N + c * 16);
+                    tmem_ld16(bcol + col, v);
+                    if (nmma > 1) {
+                        float v2[16];
+                        tmem_ld16(bcol + acc_cols + col, v2);
+#pragma unroll
+                        for (int jj = 0; jj < 16; ++jj) v[jj] += v2[jj];
+                    }
                     const int64_t base_off = m * a.sWm + (int64_t)c * 16 * a.sWn;
                     if (kind == 0) {
                         if (a.dout == UCL_BF16) {
@@ -465,6 +527,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     }
                 }
             }
+            for (uint32_t c = 0; c < buf_cols; c += 16) tmem_st16_zero(bcol + c);
+            asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(acce0 + 8u * b);
@@ -479,14 +543,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     __syncthreads();
     if (*abort_flag) {
         if (warp < kProducers && lane == 0) {
-            // copies still in flight write into this CTA's shared memory: wait
-            // for every stage this producer filled that the MMA warp did not consume
+            // copies still in flight write into this CTA's shared memory: wait for
+            // every stage this producer filled that its MMA warp did not consume
             for (uint32_t k = 0; k < misc[4 + warp]; ++k) {
                 const uint32_t it = (uint32_t)warp + k * kProducers;   // fills this producer issued
-                if (it >= misc[2]) mbar_drain(full0 + 8u * (it % a.ns), (it / a.ns) & 1u);
+                if (it >= misc[2 + it % (uint32_t)nmma]) mbar_drain(full0 + 8u * (it % a.ns), (it / a.ns) & 1u);
             }
         }
-        if (warp == kProducers && lane == 0) {
+        if (warp >= kProducers && warp < kProducers + nmma && lane == 0) {
             mma_commit(done_bar);   // tracks every MMA this thread issued
             mbar_drain(done_bar, 0);
         }
@@ -546,7 +610,7 @@ bool operand_geometry(int rows, int cols, Operand *op, std::string *why) {
 struct TcGeometry {
     Operand A, B;
     uint32_t a_pair, b_pair, stage_bytes, pair_tx, smem_bytes, tmem_cols;
-    int pps, ns, nacc;
+    int pps, ns, nacc, nmma;
 };
 
 // Pairs per stage: as many as keep a stage within 64 KB while leaving at
@@ -560,8 +624,16 @@ bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_overrid
     g->pair_tx = (uint32_t)(tp.M * tp.K * 2 + tp.N * tp.K * 2);
     const uint32_t bar_bytes = 8u * (2 * kMaxStages + 2 * kMaxAcc + 1) + 64 + 256u * kProducers + 64;
     const uint32_t avail = kSmemLimit - 1024 - bar_bytes, per_pair = g->a_pair + g->b_pair;
+    // Pairs per stage (1..4): the largest that keeps a stage within 72 KB and
+    // leaves an even number (>= 4) of stages.
     int pps = 1;
-    while (pps < 4 && 2 * pps * per_pair <= 64u * 1024u && avail / (2 * pps * per_pair) >= 3) pps *= 2;
+    for (int c = 4; c >= 2; --c) {
+        const uint32_t k = avail / (c * per_pair);
+        if (c * per_pair <= 72u * 1024u && (k < (uint32_t)kMaxStages ? k : (uint32_t)kMaxStages) / 2 * 2 >= 4) {
+            pps = c;
+            break;
+        }
+    }
     if (pps_override > 0) pps = pps_override;
     g->pps = pps;
     g->stage_bytes = pps * per_pair;
@@ -571,14 +643,31 @@ bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_overrid
         *why = "tiles too large for two shared-memory stages";
         return false;
     }
-    g->ns = ns;
     const int acc_cols = tp.N * tp.m_blocks;
-    g->nacc = 512 / acc_cols < kMaxAcc ? 512 / acc_cols : kMaxAcc;
+    // Two MMA warps (each with its own half accumulator) when two buffers of
+    // two halves fit TMEM and the stage count is even.  MMA warp w takes the
+    // stage fills w, w + 2, ...; the previous fill of a stage must belong to
+    // the same warp, or a warp could wait on a stage's full barrier while the
+    // other warp's older fill of that stage is still pending and the parity
+    // test would pass a phase early.  An even ring guarantees it.  One MMA
+    // warp consumes in order and is safe with any ring size.
+    const bool two_fit = 512 / (2 * acc_cols) >= 2;
+    if (two_fit && ns >= 4) {
+        ns &= ~1;
+        g->nmma = 2;
+    } else if (two_fit && ns == 2) {
+        g->nmma = 2;
+    } else {
+        g->nmma = 1;
+    }
+    g->ns = ns;
+    const int buf = acc_cols * g->nmma;
+    g->nacc = 512 / buf < kMaxAcc ? 512 / buf : kMaxAcc;
     if (g->nacc < 1) {
         *why = "accumulator does not fit TMEM";
         return false;
     }
-    uint32_t need = (uint32_t)(g->nacc * acc_cols), cols = 32;
+    uint32_t need = (uint32_t)(g->nacc * buf), cols = 32;
     while (cols < need) cols <<= 1;
     g->tmem_cols = cols;
     g->smem_bytes = 1024 + ns * g->stage_bytes + bar_bytes;
@@ -694,6 +783,7 @@ ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan 
     k.pps = g.pps;
     k.ns = g.ns;
     k.nacc = g.nacc;
+    k.nmma = g.nmma;
     k.tmem_cols = g.tmem_cols;
     // instruction descriptor, kind::f16: D fp32 (bits 4-5), A and B bf16 (7-9, 10-12),
     // A / B major (15, 16: 1 = MN-major), N >> 3 (17-22), M >> 4 (24-28), M = 128 per MMA
