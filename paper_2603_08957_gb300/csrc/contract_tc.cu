@@ -239,7 +239,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                    acce0 = accf0 + 8u * a.nacc, done_bar = acce0 + 8u * a.nacc;
     uint32_t *misc = reinterpret_cast<uint32_t *>(bars + 2 * a.ns + 2 * a.nacc + 1);
     // misc[0] TMEM base, [1] abort flag, [2 + w] stage fills MMA warp w has walked past,
-    // [4 + w] stages filled by producer w, [16 + 64 w, 80 + 64 w) tile indices staged by producer w
+    // [4 + w] stages filled by producer w
     volatile uint32_t *abort_flag = misc + 1;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nmma = a.nmma;
@@ -287,16 +287,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (warp < kProducers) {
         // ------------------------------------------------------ producers
         // Producer warp w fills the stages of fill number w, w + kProducers,
-        // ...  Its lanes stage 32 pairs' tile indices in shared memory; one
-        // lane then walks them with no warp-collective work per pair.
-        uint32_t *s_ia = misc + 16 + 64 * warp, *s_ib = s_ia + 32;
-        uint32_t st = 0, ph = 0, fill = 0, mine = 0;
-        int j = 0;
-        uint32_t stop = 0;
-        for (int64_t base = pb; base < pe && !stop; base += 32) {
-            const int64_t p = base + lane;
-            uint32_t ia = 0, ib = 0;
-            if (p < pe) {
+        // ...: lane j loads the tile indices of the stage's pair j (prefetched
+        // one own stage ahead), lane 0 waits for the slot and posts the
+        // expected bytes, then lane j issues the TMA copies of pair j.
+        const int n = (int)(pe - pb), pps = a.pps;
+        const int nfills = (n + pps - 1) / pps;
+        uint32_t mine = 0;
+        auto load_idx = [&](int f, uint32_t &ia, uint32_t &ib) {
+            ia = 0;
+            ib = 0;
+            const int64_t p = pb + (int64_t)f * pps + lane;
+            if (f < nfills && lane < pps && p < pe) {
                 ia = a.pa[p];
                 ib = a.pb[p];
                 if ((int64_t)ia >= a.nA || (int64_t)ib >= a.nB) {
@@ -305,44 +306,36 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     ib = 0;
                 }
             }
-            s_ia[lane] = ia;
-            s_ib[lane] = ib;
-            __syncwarp();
+        };
+        uint32_t ia, ib;
+        load_idx(warp, ia, ib);
+        uint32_t st = (uint32_t)(warp % a.ns), ph = (uint32_t)((warp / a.ns) & 1);
+        for (int f = warp; f < nfills; f += kProducers) {
+            uint32_t nia, nib;
+            load_idx(f + kProducers, nia, nib);
+            const int np = n - f * pps < pps ? n - f * pps : pps;
+            uint32_t okw = 1;
             if (lane == 0) {
-                const int cnt = (int)(pe - base < 32 ? pe - base : 32);
-                for (int jj = 0; jj < cnt; ++jj) {
-                    const bool own = (fill % kProducers) == (uint32_t)warp;
-                    if (j == 0 && own) {
-                        if (!mbar_wait(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status)) {
-                            stop = 1;
-                            break;
-                        }
-                        const int64_t left = pe - (base + jj);
-                        const uint32_t np = (uint32_t)(left < a.pps ? left : a.pps);
-                        mbar_arrive_tx(full0 + 8u * st, np * a.pair_tx);
-                        ++mine;
-                    }
-                    if (own) {
-                        const uint32_t fb = full0 + 8u * st;
-                        const uint32_t sa = sbase + st * a.stage_bytes + (uint32_t)j * a.a_pair;
-                        const uint32_t sb =
-                            sbase + st * a.stage_bytes + (uint32_t)a.pps * a.a_pair + (uint32_t)j * a.b_pair;
-                        const int xa = (int)s_ia[jj], xb = (int)s_ib[jj];
-                        for (int q = 0; q < a.na_sub; ++q) tma_load_3d(sa + q * a.a_sub, &tmA, q * a.wa, 0, xa, fb);
-                        for (int q = 0; q < a.nb_sub; ++q) tma_load_3d(sb + q * a.b_sub, &tmB, q * a.wb, 0, xb, fb);
-                    }
-                    if (++j == a.pps) {
-                        j = 0;
-                        ++fill;
-                        if (++st == (uint32_t)a.ns) {
-                            st = 0;
-                            ph ^= 1u;
-                        }
-                    }
-                }
+                okw = mbar_wait(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status) ? 1u : 0u;
+                if (okw) mbar_arrive_tx(full0 + 8u * st, (uint32_t)np * a.pair_tx);
             }
-            stop = __shfl_sync(0xffffffffu, stop, 0);
+            if (!__shfl_sync(0xffffffffu, okw, 0)) break;
+            if (lane < np) {
+                const uint32_t fb = full0 + 8u * st;
+                const uint32_t sa = sbase + st * a.stage_bytes + (uint32_t)lane * a.a_pair;
+                const uint32_t sb = sbase + st * a.stage_bytes + (uint32_t)a.pps * a.a_pair + (uint32_t)lane * a.b_pair;
+                for (int q = 0; q < a.na_sub; ++q) tma_load_3d(sa + q * a.a_sub, &tmA, q * a.wa, 0, (int)ia, fb);
+                for (int q = 0; q < a.nb_sub; ++q) tma_load_3d(sb + q * a.b_sub, &tmB, q * a.wb, 0, (int)ib, fb);
+            }
             __syncwarp();
+            ++mine;
+            ia = nia;
+            ib = nib;
+            st += kProducers;
+            if (st >= (uint32_t)a.ns) {
+                st -= (uint32_t)a.ns;
+                ph ^= 1u;
+            }
         }
         if (lane == 0) misc[4 + warp] = mine;
     } else if (warp < kProducers + kMmaWarps) {
@@ -367,123 +360,128 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const uint32_t mb16 = (uint32_t)a.a_mb16, ncol = (uint32_t)a.N, idesc = a.idesc;
             const bool two_m = a.m_blocks > 1;
             const int n = (int)(pe - pb), pps = a.pps;
-            uint32_t st = 0, ph = 0, b = 0, aph = 0, dcol = tmem;
-            uint32_t fill = 0;
+            uint32_t b = 0, aph = 0, dcol = tmem;
             int64_t s = s_first;
-            int i = 0;
             int seg_end = n > 0 ? (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) : 0;
             bool fresh = true, ok = true;
-            while (i < n) {
-                const int np = n - i < pps ? n - i : pps;
-                const bool own = (int)(fill % (uint32_t)nmma) == w;
-                if (own) {
-                    if (!__all_sync(0xffffffffu, mbar_wait(full0 + 8u * st, ph, abort_flag, a.status))) {
+            // Segment events: before the warp's first MMA into a segment it waits
+            // for the accumulator buffer (open); at the segment's end it commits
+            // the buffer to the epilogue (close).  Both warps open and close every
+            // segment, in order, also segments whose pairs all lie in the other
+            // warp's stages.
+            auto open_seg = [&]() -> bool {
+                if (!__all_sync(0xffffffffu, mbar_wait(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status))) return false;
+                tc_fence_after();
+                dcol = tmem + b * buf_cols + (uint32_t)w * acc_cols;
+                fresh = false;
+                return true;
+            };
+            auto close_seg = [&](int pos) {
+                if (elect_one()) mma_commit(accf0 + 8u * b);
+                __syncwarp();
+                if (++b == (uint32_t)a.nacc) {
+                    b = 0;
+                    aph ^= 1u;
+                }
+                ++s;
+                if (pos < n) seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
+                fresh = true;
+            };
+            uint32_t st = (uint32_t)(w % a.ns), ph = (uint32_t)((w / a.ns) & 1);
+            int f = w;
+            for (; f * pps < n; f += nmma) {
+                const int start = f * pps;
+                const int np = n - start < pps ? n - start : pps;
+                // segments that end inside the other warp's stages before this one
+                while (seg_end <= start) {
+                    if (fresh && !open_seg()) {
                         ok = false;
                         break;
                     }
-                    tc_fence_after();
+                    close_seg(seg_end);
                 }
+                if (!ok) break;
+                if (!__all_sync(0xffffffffu, mbar_wait(full0 + 8u * st, ph, abort_flag, a.status))) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
                 uint64_t ad = adesc0 + st * stage16, bd = bdesc0 + st * stage16;
-                if (!fresh && i + np <= seg_end) {
+                if (!fresh && start + np <= seg_end) {
                     // the whole stage accumulates into the open buffer
-                    if (own) {
-                        const uint64_t ad1 = ad + apair16, bd1 = bd + bpair16;
-                        const uint64_t ad2 = ad1 + apair16, bd2 = bd1 + bpair16;
-                        const uint64_t ad3 = ad2 + apair16, bd3 = bd2 + bpair16;
+                    const uint64_t ad1 = ad + apair16, bd1 = bd + bpair16;
+                    const uint64_t ad2 = ad1 + apair16, bd2 = bd1 + bpair16;
+                    const uint64_t ad3 = ad2 + apair16, bd3 = bd2 + bpair16;
+                    if (elect_one()) {
+#pragma unroll
+                        for (int kk = 0; kk < KSTEPS; ++kk) {
+                            mma_bf16(dcol, ad + aoff[kk], bd + boff[kk], idesc, 1u);
+                            if (two_m) mma_bf16(dcol + ncol, ad + aoff[kk] + mb16, bd + boff[kk], idesc, 1u);
+                        }
+                        if (np > 1) {
+#pragma unroll
+                            for (int kk = 0; kk < KSTEPS; ++kk) {
+                                mma_bf16(dcol, ad1 + aoff[kk], bd1 + boff[kk], idesc, 1u);
+                                if (two_m) mma_bf16(dcol + ncol, ad1 + aoff[kk] + mb16, bd1 + boff[kk], idesc, 1u);
+                            }
+                        }
+                        if (np > 2) {
+#pragma unroll
+                            for (int kk = 0; kk < KSTEPS; ++kk) {
+                                mma_bf16(dcol, ad2 + aoff[kk], bd2 + boff[kk], idesc, 1u);
+                                if (two_m) mma_bf16(dcol + ncol, ad2 + aoff[kk] + mb16, bd2 + boff[kk], idesc, 1u);
+                            }
+                        }
+                        if (np > 3) {
+#pragma unroll
+                            for (int kk = 0; kk < KSTEPS; ++kk) {
+                                mma_bf16(dcol, ad3 + aoff[kk], bd3 + boff[kk], idesc, 1u);
+                                if (two_m) mma_bf16(dcol + ncol, ad3 + aoff[kk] + mb16, bd3 + boff[kk], idesc, 1u);
+                            }
+                        }
+                        mma_commit(empty0 + 8u * st);
+                    }
+                    __syncwarp();
+                } else {
+                    // segment boundaries inside the stage: pair by pair
+                    for (int jj = 0; jj < np; ++jj) {
+                        if (fresh && !open_seg()) {
+                            ok = false;
+                            break;
+                        }
                         if (elect_one()) {
 #pragma unroll
                             for (int kk = 0; kk < KSTEPS; ++kk) {
                                 mma_bf16(dcol, ad + aoff[kk], bd + boff[kk], idesc, 1u);
                                 if (two_m) mma_bf16(dcol + ncol, ad + aoff[kk] + mb16, bd + boff[kk], idesc, 1u);
                             }
-                            if (np > 1) {
-#pragma unroll
-                                for (int kk = 0; kk < KSTEPS; ++kk) {
-                                    mma_bf16(dcol, ad1 + aoff[kk], bd1 + boff[kk], idesc, 1u);
-                                    if (two_m) mma_bf16(dcol + ncol, ad1 + aoff[kk] + mb16, bd1 + boff[kk], idesc, 1u);
-                                }
-                            }
-                            if (np > 2) {
-#pragma unroll
-                                for (int kk = 0; kk < KSTEPS; ++kk) {
-                                    mma_bf16(dcol, ad2 + aoff[kk], bd2 + boff[kk], idesc, 1u);
-                                    if (two_m) mma_bf16(dcol + ncol, ad2 + aoff[kk] + mb16, bd2 + boff[kk], idesc, 1u);
-                                }
-                            }
-                            if (np > 3) {
-#pragma unroll
-                                for (int kk = 0; kk < KSTEPS; ++kk) {
-                                    mma_bf16(dcol, ad3 + aoff[kk], bd3 + boff[kk], idesc, 1u);
-                                    if (two_m) mma_bf16(dcol + ncol, ad3 + aoff[kk] + mb16, bd3 + boff[kk], idesc, 1u);
-                                }
-                            }
-                            mma_commit(empty0 + 8u * st);
                         }
                         __syncwarp();
-                    }
-                    i += np;
-                } else {
-                    // segment boundaries inside the stage: pair by pair
-                    for (int jj = 0; jj < np; ++jj, ++i) {
-                        if (fresh) {
-                            if (!__all_sync(0xffffffffu, mbar_wait(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status))) {
-                                ok = false;
-                                break;
-                            }
-                            tc_fence_after();
-                            dcol = tmem + b * buf_cols + (uint32_t)w * acc_cols;
-                            fresh = false;
-                        }
-                        if (own) {
-                            if (elect_one()) {
-#pragma unroll
-                                for (int kk = 0; kk < KSTEPS; ++kk) {
-                                    mma_bf16(dcol, ad + aoff[kk], bd + boff[kk], idesc, 1u);
-                                    if (two_m) mma_bf16(dcol + ncol, ad + aoff[kk] + mb16, bd + boff[kk], idesc, 1u);
-                                }
-                            }
-                            __syncwarp();
-                        }
                         ad += apair16;
                         bd += bpair16;
-                        if (i + 1 == seg_end) {
-                            // the segment's last pair in this unit: hand the buffer to the epilogue
-                            if (elect_one()) mma_commit(accf0 + 8u * b);
-                            __syncwarp();
-                            if (++b == (uint32_t)a.nacc) {
-                                b = 0;
-                                aph ^= 1u;
-                            }
-                            ++s;
-                            if (i + 1 < n) seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
-                            fresh = true;
-                        }
+                        if (start + jj + 1 == seg_end) close_seg(start + jj + 1);
                     }
                     if (!ok) break;
-                    if (own) {
-                        if (elect_one()) mma_commit(empty0 + 8u * st);
-                        __syncwarp();
-                    }
+                    if (elect_one()) mma_commit(empty0 + 8u * st);
+                    __syncwarp();
                 }
                 // a fast-path stage may end exactly at the segment's end
-                if (!fresh && i == seg_end) {
-                    if (elect_one()) mma_commit(accf0 + 8u * b);
-                    __syncwarp();
-                    if (++b == (uint32_t)a.nacc) {
-                        b = 0;
-                        aph ^= 1u;
-                    }
-                    ++s;
-                    if (i < n) seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
-                    fresh = true;
-                }
-                ++fill;
-                if (++st == (uint32_t)a.ns) {
-                    st = 0;
+                if (!fresh && start + np == seg_end) close_seg(seg_end);
+                st += (uint32_t)nmma;
+                if (st >= (uint32_t)a.ns) {
+                    st -= (uint32_t)a.ns;
                     ph ^= 1u;
                 }
             }
-            if (lane == 0) misc[2 + w] = ok ? 0xFFFFFFFFu : fill;
+            // segments that end after this warp's last stage
+            while (ok && s <= s_last) {
+                if (fresh && !open_seg()) {
+                    ok = false;
+                    break;
+                }
+                close_seg(seg_end);
+            }
+            if (lane == 0) misc[2 + w] = ok ? 0xFFFFFFFFu : (uint32_t)f;
         }
     } else {
         // ------------------------------------------------------- epilogue
@@ -622,7 +620,7 @@ bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_overrid
     g->a_pair = g->A.sub_bytes * g->A.nsub;
     g->b_pair = g->B.sub_bytes * g->B.nsub;
     g->pair_tx = (uint32_t)(tp.M * tp.K * 2 + tp.N * tp.K * 2);
-    const uint32_t bar_bytes = 8u * (2 * kMaxStages + 2 * kMaxAcc + 1) + 64 + 256u * kProducers + 64;
+    const uint32_t bar_bytes = 8u * (2 * kMaxStages + 2 * kMaxAcc + 1) + 64 + 64;
     const uint32_t avail = kSmemLimit - 1024 - bar_bytes, per_pair = g->a_pair + g->b_pair;
     // Pairs per stage (1..4): the largest that keeps a stage within 72 KB and
     // leaves an even number (>= 4) of stages.
