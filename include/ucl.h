@@ -199,6 +199,33 @@ ucl_status ucl_relation_download(const ucl_rel *rel, int32_t *keys_host, void *t
 ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec, int n_in, ucl_rel *const *in, const ucl_einsum_opts *opts,
                       ucl_rel **out);
 
+/* ------------------------------------------------------- no allocation */
+
+/* Largest key array ucl_keys_check_noalloc accepts (tuples). */
+#define UCL_NOALLOC_MAX_TUPLES (1 << 20)
+
+/* The key checks of ucl_relation_create -- every key in [0, bound), no key
+ * twice (UCL_ERR_KEY_RANGE / UCL_ERR_DUP_KEY), ascending order reported in
+ * *sorted -- for callers that cannot allocate device memory: code that runs
+ * under a device-memory budget owned by another component, or that must
+ * never call cudaMalloc because it can synchronise the device.  This call
+ * allocates nothing and needs no context: its scratch is a fixed array of
+ * about 16.3 MiB in the library's own device memory, which every GPU that
+ * loads the library holds until the process exits.  The paper has no
+ * counterpart; this is a service of this library.
+ *   device, stream  where the work runs (stream NULL = legacy default stream)
+ *   n, u, keys      int32 [n, u] key array in device memory, n <= UCL_NOALLOC_MAX_TUPLES
+ *   key_bounds      int64 [u] bounds (host memory)
+ *   sorted          optional; receives 1 if the keys are strictly ascending
+ * Returns UCL_ERR_UNSUPPORTED for n > UCL_NOALLOC_MAX_TUPLES or more than 64
+ * key bits.  Synchronises `stream` (once, or twice for unsorted keys).  The
+ * first call on a device looks up the scratch array's device address for
+ * that device; make that first call before any stream capture.  Every call
+ * shares the one scratch array: calls whose GPU work overlaps (e.g. on two
+ * streams) race on it and must be serialised by the caller. */
+ucl_status ucl_keys_check_noalloc(int device, void *stream, int64_t n, int u, const int32_t *keys,
+                                  const int64_t *key_bounds, int *sorted);
+
 /* ------------------------------------------------------------ diagnostics */
 
 const char *ucl_status_str(ucl_status st);
