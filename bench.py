@@ -49,6 +49,26 @@ def workload_name(vertices):
             f"{16 * vertices} edges as 64x64 bf16 tiles, Z 128x128 bf16")
 
 
+def contract_traffic(pairs):
+    """DRAM bytes of one contraction launch, scaled by pairs from the ncu capture in
+    profiles/contract_tc_traffic.txt; None once the kernel source changed since."""
+    import hashlib
+    p = os.path.join(ROOT, "profiles", "contract_tc_traffic.txt")
+    src = os.path.join(ROOT, "paper_2603_08957_gb300", "csrc", "contract_tc.cu")
+    if not os.path.exists(p):
+        return None
+    kv = {}
+    for line in open(p):
+        line = line.split("#", 1)[0].strip()
+        if ":" in line:
+            k, v = line.split(":", 1)
+            kv[k.strip()] = v.strip()
+    if hashlib.sha256(open(src, "rb").read()).hexdigest() != kv.get("source_sha256"):
+        return None
+    per_pair = (int(kv["dram_read_bytes"]) + int(kv["dram_write_bytes"])) / int(kv["pairs"])
+    return per_pair * pairs
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -276,7 +296,7 @@ def run_ucl(args, world, rank, local):
     pk = peaks()
     achieved = s1["bytes_contract"] / (avg_contract / 1e3) / 1e9
     roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
-            "frac": achieved / pk["hbm_gbs"], "traffic": None,
+            "frac": achieved / pk["hbm_gbs"], "traffic": contract_traffic(s1["n_pairs"]),
             "kernel": f"contract_{s1['path']} (fJj,JjKk->Kkf)", "avg_launch_ms": avg_contract,
             "alg_bytes_per_launch": s1["bytes_contract"], "peak_src": pk["src"],
             "tensor_frac": (s1["flops"] / (avg_contract / 1e3) / 1e12) / pk["bf16_tflops"]}
