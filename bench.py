@@ -233,7 +233,7 @@ def run_ucl(args, world, rank, local):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     w = workloads.gnn_chain(seed=0, n=args.vertices, device=dev)
-    ctx = Context(local)
+    ctx = Context(local, torch_allocator=(args.alloc == "torch"))
 
     def rel(r):
         return ctx.relation(torch.as_tensor(r[0]).to(dev), r[1], r[2].to(dev))
@@ -346,7 +346,7 @@ def run_ucl(args, world, rank, local):
                 "config": {"workload": workload_name(args.vertices), "pairs": [s1["n_pairs"], s2["n_pairs"]],
                            "segments": [s1["n_segments"], s2["n_segments"]], "flops_per_step": flops_step,
                            "l2": "inputs larger than L2 (Y 2.9 GB); no flush", "path": s1["path"],
-                           "parallelism": f"replicas x{world}"},
+                           "parallelism": f"replicas x{world}", "alloc": args.alloc},
                 "roofline": roof, "stage_ms": stages, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": int(launches_step * steps), "clocks": ck}
         print(json.dumps(line), flush=True)
@@ -364,6 +364,9 @@ def main():
     ap.add_argument("--path", choices=["auto", "simt", "tc"], default="auto")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--alloc", choices=["torch", "cuda"], default="torch",
+                    help="device memory for workspace and outputs: PyTorch's caching allocator (through the "
+                         "allocator hooks) or the library's cudaMallocAsync pool")
     ap.add_argument("--vertices", type=int, default=100_000, help="graph size (reduced sizes for profiling)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-step-seconds", type=float, default=3.0)

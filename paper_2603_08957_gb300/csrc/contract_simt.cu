@@ -155,9 +155,13 @@ __global__ void __launch_bounds__(kSimtThreads) fixup_kernel(ContractArgs a) {
     const int64_t s = find_seg(a.seg_start, a.S, p);
     const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
     if (ss >= p || ss < a.units.begin(c - 1)) return;
+    // units c .. u_end - 1 hold the segment's continuation partials (slot 0)
+    int u_end = c;
+    while (u_end < a.units.G && a.units.begin(u_end) < se) ++u_end;
+    const float *first = a.partials + ((int64_t)(c - 1) * 2 + 1) * a.tile_w;
     for (int64_t w = threadIdx.x; w < a.tile_w; w += blockDim.x) {
-        float acc = a.partials[((int64_t)(c - 1) * 2 + 1) * a.tile_w + w];
-        for (int u = c; u < a.units.G && a.units.begin(u) < se; ++u) acc += a.partials[((int64_t)u * 2) * a.tile_w + w];
+        float acc = first[w];
+        for (int u = c; u < u_end; ++u) acc += a.partials[((int64_t)u * 2) * a.tile_w + w];
         store_out(a.out, a.dout, s * a.tile_w + w, epilogue(acc, a.epi, a.scale));
     }
 }
