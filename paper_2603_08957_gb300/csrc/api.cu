@@ -464,6 +464,14 @@ ucl_status ucl_ctx_create(int device, void *stream, ucl_alloc_fn alloc, ucl_free
     ucl_status st = cuda_check(ctx, cudaSetDevice(device), "cudaSetDevice");
     if (!st) st = cuda_check(ctx, cudaDeviceGetAttribute(&ctx->sm_count, cudaDevAttrMultiProcessorCount, device),
                              "device attribute");
+    if (!st && !alloc) {
+        // default allocator: keep freed blocks in the device's pool across syncs
+        cudaMemPool_t pool;
+        st = cuda_check(ctx, cudaDeviceGetDefaultMemPool(&pool, device), "cudaDeviceGetDefaultMemPool");
+        uint64_t keep = ~0ull;
+        if (!st) st = cuda_check(ctx, cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep),
+                                 "cudaMemPoolSetAttribute");
+    }
     if (!st) st = cuda_check(ctx, cudaMalloc(&ctx->d_status, 256), "cudaMalloc status");
     if (!st) st = cuda_check(ctx, cudaMemset(ctx->d_status, 0, 256), "cudaMemset status");
     if (!st) st = cuda_check(ctx, cudaMallocHost(&ctx->h_pinned, 8 * sizeof(int64_t)), "cudaMallocHost");
