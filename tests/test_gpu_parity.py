@@ -323,3 +323,74 @@ def test_errors(ctx):
     out = ctx.einsum("Ij,Ij->I", R, R)
     assert out.download()[1].tolist() == [3.0]
     ctx.synchronize()
+
+
+def test_two_layer_gnn_full_size_sampled(ctx):
+    """Two-layer GNN at scale: R-MAT with 2M vertices / 40M drawn edges as
+    64x64 0/1 tiles (~16.6M tiles, ~136 GB), 256-wide embeddings, chained
+    T1=(XY)^T, H1=relu(T1 W1), T2=(H1 Y)^T, O=T2 W2.  Every step's key set
+    is checked in full; values stage-locally on sampled output keys (the
+    oracle gets exactly the tiles those keys join with)."""
+    w = workloads.gnn_two_layer(seed=0)
+    dev = torch.device("cuda", 0)
+    X, Y, W1, W2 = (gpu_rel(ctx, w[k]) for k in ("X", "Y", "W1", "W2"))
+    ky = w["Y"][0]
+    want_k = np.unique(ky[:, 1]).astype(np.int32)[:, None]
+    src, dst = w["edges"]
+    t, n = w["t"], w["n"]
+    cnt = np.bincount(ky[:, 1], minlength=want_k.max() + 1)
+    rng = np.random.default_rng(3)
+    small = np.nonzero((cnt > 0) & (cnt <= np.median(cnt[cnt > 0])))[0]
+    sk = np.sort(rng.choice(small, size=3, replace=False)).astype(np.int32)
+
+    def y_subset(kset):
+        m = torch.isin(dst // t, torch.as_tensor(kset, device=dst.device, dtype=torch.int64))
+        s, d = src[m].cpu().numpy(), dst[m].cpu().numpy()
+        yk = ky[np.isin(ky[:, 1], kset)]
+        return yk, workloads.adjacency_tiles_subset(s, d, n, t, yk)
+
+    def rows(rel, keys_sel):
+        k, tl = rel.device_tensors()
+        kk = k[:, 0].cpu().numpy()
+        idx = np.searchsorted(kk, keys_sel)
+        assert np.array_equal(kk[idx], keys_sel)
+        return keys_sel[:, None].astype(np.int32), tl[torch.as_tensor(idx, device=tl.device)].cpu()
+
+    yk, yt = y_subset(sk)
+    # step 1: T1 = (X Y)^T
+    T1 = ctx.einsum(w["spec1"], X, Y, out_dtype="bf16")
+    kt1, _ = T1.device_tensors()
+    assert np.array_equal(kt1.cpu().numpy(), want_k)
+    jneed = np.unique(yk[:, 0])
+    xrel = (jneed[:, None].astype(np.int32), w["X"][1], w["X"][2][torch.as_tensor(jneed, device=dev)].cpu())
+    ref = oracle_ref(w["spec1"], [xrel, (yk, w["Y"][1], yt)], sample_keys=sk[:, None])
+    sel = np.searchsorted(kt1[:, 0].cpu().numpy(), sk)
+    assert_parity(T1, ref, torch.bfloat16, select=sel)
+    # step 2: H1 = relu(T1 W1), stage-local
+    H1 = ctx.einsum(w["spec2"], T1, W1, out_dtype="bf16", epi="relu")
+    t1k, t1t = rows(T1, sk)
+    ref = oracle_ref(w["spec2"], [(t1k, T1.bounds, t1t), w["W1"]], epi="relu")
+    assert_parity(H1, ref, torch.bfloat16, select=sel)
+    # step 3: T2 = (H1 Y)^T with H1 keyed by J; only K reached from a J that
+    # H1 holds (a destination tile of some edge) appear
+    T2 = ctx.einsum(w["spec3"], H1, Y, out_dtype="bf16")
+    kt2 = T2.device_tensors()[0].cpu().numpy()
+    want_k2 = np.unique(ky[np.isin(ky[:, 0], want_k[:, 0]), 1]).astype(np.int32)[:, None]
+    assert np.array_equal(kt2, want_k2)
+    sk2 = sk[np.isin(sk, kt2[:, 0])]
+    assert len(sk2) > 0
+    yk2 = yk[np.isin(yk[:, 1], sk2) & np.isin(yk[:, 0], want_k[:, 0])]
+    yt2 = yt[np.isin(yk[:, 1], sk2) & np.isin(yk[:, 0], want_k[:, 0])]
+    hk, ht = rows(H1, np.unique(yk2[:, 0]))
+    ref = oracle_ref(w["spec3"], [(hk, H1.bounds, ht), (yk2, w["Y"][1], yt2)], sample_keys=sk2[:, None])
+    sel2 = np.searchsorted(kt2[:, 0], sk2)
+    assert_parity(T2, ref, torch.bfloat16, select=sel2)
+    # step 4: O = T2 W2
+    O = ctx.einsum(w["spec4"], T2, W2)
+    t2k, t2t = rows(T2, sk2)
+    ref = oracle_ref(w["spec4"], [(t2k, T2.bounds, t2t), w["W2"]])
+    assert_parity(O, ref, torch.bfloat16, select=sel2)
+    for r in (X, Y, W1, W2, T1, H1, T2, O):
+        r.destroy()
+    del w
+    torch.cuda.empty_cache()

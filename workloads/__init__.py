@@ -177,6 +177,76 @@ def spgemm(seed=0, n=65536, t=128, density=0.005, band=(-1, 0, 1, 2)):
     return {"spec": "IiJj,JjKk->IiKk", "A": draw(), "B": draw()}
 
 
+def rmat_edges_device(n: int, n_edges: int, a=0.57, b=0.19, c=0.19, seed=0, device="cuda", batch=1 << 25):
+    """rmat_edges drawn with torch on the GPU (for graphs too large for host
+    numpy): same model and rejection rule; returns (src, dst) int64 device
+    tensors, de-duplicated and sorted by (src, dst)."""
+    g = torch.Generator(device=device).manual_seed(seed)
+    levels = max(1, math.ceil(math.log2(n)))
+    parts, have = [], 0
+    while have < n_edges:
+        m = min(batch, int((n_edges - have) * 1.15) + 1024)
+        s = torch.zeros(m, dtype=torch.int64, device=device)
+        d = torch.zeros(m, dtype=torch.int64, device=device)
+        for _ in range(levels):
+            r = torch.rand(m, generator=g, device=device)
+            sb = (r >= a + b).long()
+            db = (((r >= a) & (r < a + b)) | (r >= a + b + c)).long()
+            s = s * 2 + sb
+            d = d * 2 + db
+        ok = (s < n) & (d < n)
+        code = (s * n + d)[ok][: n_edges - have]
+        parts.append(code)
+        have += code.numel()
+    code = torch.unique(torch.cat(parts))
+    return code // n, code % n
+
+
+def adjacency_tiles_device(src, dst, n: int, t: int, dtype=torch.bfloat16):
+    """adjacency_tiles for device edge tensors: only-nonempty [t x t] 0/1
+    tiles keyed (J = src // t, K = dst // t), ascending; keys returned as a
+    host int32 array, tiles on the device."""
+    nt = -(-n // t)
+    tcode = (src // t) * nt + (dst // t)
+    ukeys, inv = torch.unique(tcode, return_inverse=True)
+    tiles = torch.zeros((ukeys.numel(), t, t), dtype=dtype, device=src.device)
+    tiles[inv, src % t, dst % t] = 1
+    keys = torch.stack([ukeys // nt, ukeys % nt], dim=1).to(torch.int32).cpu().numpy()
+    return keys, (nt, nt), tiles
+
+
+def gnn_two_layer(seed=0, n=2_000_000, n_edges=40_000_000, feat=256, t=64, device="cuda", w_std=None):
+    """Two-layer GNN at scale: an R-MAT graph (a,b,c = .57,.19,.19) with
+    n_edges drawn edges as only-nonempty t x t 0/1 bf16 tiles Y keyed (J, K);
+    X feat x n bf16 N(0,1) as per-J tiles [f x j]; W1, W2 feat x feat bf16
+    N(0, 1/feat) (the config leaves their distribution open).  Chain:
+    T1 = (X Y)^T, H1 = relu(T1 W1), T2 = (H1 Y)^T, O = T2 W2."""
+    g = torch.Generator(device=device).manual_seed(seed)
+    nt = -(-n // t)
+    X = torch.randn((nt, feat, t), generator=g, device=device).to(torch.bfloat16)
+    if n % t:
+        X[-1, :, n % t:] = 0
+    std = w_std if w_std is not None else feat ** -0.5
+    W1 = (torch.randn((feat, feat), generator=g, device=device) * std).to(torch.bfloat16)
+    W2 = (torch.randn((feat, feat), generator=g, device=device) * std).to(torch.bfloat16)
+    src, dst = rmat_edges_device(n, n_edges, seed=seed + 1, device=device)
+    ky, by, ty = adjacency_tiles_device(src, dst, n, t)
+    nokey = np.zeros((1, 0), np.int32)
+    return {
+        "spec1": "fJj,JjKk->Kkf",
+        "spec2": "Kkf,fg->Kkg",
+        "spec3": "Jjg,JjKk->Kkg",
+        "spec4": "Kkg,gh->Kkh",
+        "X": (np.arange(nt, dtype=np.int32)[:, None], (nt,), X),
+        "Y": (ky, by, ty),
+        "W1": (nokey, (), W1[None]),
+        "W2": (nokey, (), W2[None]),
+        "edges": (src, dst),
+        "n": n,
+        "t": t,
+    }
+
+
 def to_oracle(rel):
     """(keys, bounds, tiles) with tiles converted exactly to float64 numpy."""
     keys, bounds, tiles = rel
