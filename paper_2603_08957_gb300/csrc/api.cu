@@ -49,7 +49,7 @@ bool is_upper(char c) { return c >= 'A' && c <= 'Z'; }
 
 ucl_status parse_spec(ucl_ctx *ctx, const char *text, int n_in, Spec &s) {
     if (!text) return fail(ctx, UCL_ERR_ARG, "spec is NULL");
-    if (n_in < 1 || n_in > 2) return fail(ctx, n_in == 3 ? UCL_ERR_UNSUPPORTED : UCL_ERR_ARG, "n_in must be 1 or 2");
+    if (n_in < 1 || n_in > 3) return fail(ctx, UCL_ERR_ARG, "n_in must be 1, 2 or 3");
     std::string t(text);
     size_t arrow = t.find("->");
     if (arrow == std::string::npos) return fail(ctx, UCL_ERR_SPEC, "spec has no '->'");
@@ -137,19 +137,55 @@ int64_t tile_stride(const Spec &s, int k, const Label &L) {
 }
 
 struct KeyPlan {
-    std::vector<int> join;   // label ids of the join attributes, U's order
+    // join order: (ord[0] JOIN ord[1]) JOIN ord[2]; inputs in spec order for
+    // one or two inputs
+    int ord[3] = {0, 1, 2};
+    std::vector<int> join;   // label ids of the first join's attributes, ord[0]'s order
     int join_bits = 0;
-    KeyPack join_u{}, join_v{};
-    KeyPack out_u{}, out_v{};
+    KeyPack join_u{}, join_v{};   // packers of the first join key for ord[0], ord[1]
+    // three inputs: the attributes ord[2] shares with ord[0] or ord[1], in
+    // ord[2]'s column order, each supplied by ord[0] if it has it, else ord[1]
+    std::vector<int> join2;
+    int join2_bits = 0;
+    KeyPack join2_a{}, join2_b{}, join2_c{};
+    KeyPack out_k[3]{};      // output-key bit fields each input supplies (spec order)
     int out_bits = 0;
     KeyUnpack unpack{};
     int64_t out_bounds[kMaxCols] = {};
     int uw = 0;
-    bool ident_u = false, ident_v = false;   // input already ordered by its join key
+    bool ident_u = false, ident_v = false, ident_c = false;   // input already ordered by its join key
 };
+
+// An input whose keys are sorted and whose leading key columns are the join
+// attributes, in order, is already grouped by join key.
+bool leading_cols(const Spec &s, const ucl_rel *R, int k, const std::vector<int> &labs) {
+    if (labs.empty()) return true;
+    if (!R->sorted) return false;
+    for (size_t q = 0; q < labs.size(); ++q)
+        if (s.labs[labs[q]].pos[k] != (int)q) return false;
+    return true;
+}
+
+int shared_bits(const Spec &s, int a, int b) {
+    int t = 0;
+    for (const Label &L : s.labs)
+        if (L.upper && L.pos[a] >= 0 && L.pos[b] >= 0) t += bit_width(L.ext);
+    return t;
+}
 
 ucl_status plan_keys(ucl_ctx *ctx, const Spec &s, ucl_rel *const *in, KeyPlan &kp) {
     const int n = s.n_in;
+    if (n == 3) {
+        // join first the two inputs that share the most key bits (a pair that
+        // shares none would be a cross product)
+        const int pairs[3][3] = {{0, 1, 2}, {0, 2, 1}, {1, 2, 0}};
+        int best = 0, bb = -1;
+        for (int q = 0; q < 3; ++q) {
+            int b = shared_bits(s, pairs[q][0], pairs[q][1]);
+            if (b > bb) { bb = b; best = q; }
+        }
+        for (int q = 0; q < 3; ++q) kp.ord[q] = pairs[best][q];
+    }
     // output key: W's upper labels, first most significant
     std::vector<int> wl;
     for (char c : s.out) {
@@ -170,17 +206,21 @@ ucl_status plan_keys(ucl_ctx *ctx, const Spec &s, ucl_rel *const *in, KeyPlan &k
         kp.unpack.shift[q] = shift;
         kp.unpack.bits[q] = b;
         kp.out_bounds[q] = L.ext;
-        // supplier: U if it has the label, else V
-        if (L.pos[0] >= 0)
-            kp.out_u.f[kp.out_u.nf++] = KeyField{L.pos[0], shift, b};
-        else
-            kp.out_v.f[kp.out_v.nf++] = KeyField{L.pos[1], shift, b};
+        // supplier: the first input in join order that has the label
+        for (int j = 0; j < n; ++j) {
+            const int k = kp.ord[j];
+            if (L.pos[k] >= 0) {
+                kp.out_k[k].f[kp.out_k[k].nf++] = KeyField{L.pos[k], shift, b};
+                break;
+            }
+        }
     }
     if (n < 2) return UCL_OK;
-    // join attributes: upper labels of both inputs, in U's order
-    for (char c : s.op[0]) {
+    const int ka = kp.ord[0], kb = kp.ord[1];
+    // first join: upper labels of both inputs, in ord[0]'s order
+    for (char c : s.op[ka]) {
         int L = s.find(c);
-        if (s.labs[L].upper && s.labs[L].pos[1] >= 0) kp.join.push_back(L);
+        if (s.labs[L].upper && s.labs[L].pos[kb] >= 0) kp.join.push_back(L);
     }
     total = 0;
     for (int L : kp.join) total += bit_width(s.labs[L].ext);
@@ -190,16 +230,33 @@ ucl_status plan_keys(ucl_ctx *ctx, const Spec &s, ucl_rel *const *in, KeyPlan &k
     for (int L : kp.join) {
         int b = bit_width(s.labs[L].ext);
         shift -= b;
-        kp.join_u.f[kp.join_u.nf++] = KeyField{s.labs[L].pos[0], shift, b};
-        kp.join_v.f[kp.join_v.nf++] = KeyField{s.labs[L].pos[1], shift, b};
+        kp.join_u.f[kp.join_u.nf++] = KeyField{s.labs[L].pos[ka], shift, b};
+        kp.join_v.f[kp.join_v.nf++] = KeyField{s.labs[L].pos[kb], shift, b};
     }
-    // an input whose keys are sorted and whose leading key columns are the
-    // join attributes in the same order is already grouped by join key
-    for (int k = 0; k < 2; ++k) {
-        bool ok = in[k]->sorted != 0;
-        for (size_t q = 0; q < kp.join.size() && ok; ++q) ok = s.labs[kp.join[q]].pos[k] == (int)q;
-        (k == 0 ? kp.ident_u : kp.ident_v) = ok || kp.join.empty();
+    kp.ident_u = leading_cols(s, in[ka], ka, kp.join);
+    kp.ident_v = leading_cols(s, in[kb], kb, kp.join);
+    if (n < 3) return UCL_OK;
+    const int kc = kp.ord[2];
+    for (char c : s.op[kc]) {
+        int L = s.find(c);
+        if (s.labs[L].upper && (s.labs[L].pos[ka] >= 0 || s.labs[L].pos[kb] >= 0)) kp.join2.push_back(L);
     }
+    total = 0;
+    for (int L : kp.join2) total += bit_width(s.labs[L].ext);
+    if (total > 64) return fail(ctx, UCL_ERR_UNSUPPORTED, "join key needs more than 64 bits");
+    kp.join2_bits = total;
+    shift = total;
+    for (int L : kp.join2) {
+        const Label &M = s.labs[L];
+        int b = bit_width(M.ext);
+        shift -= b;
+        kp.join2_c.f[kp.join2_c.nf++] = KeyField{M.pos[kc], shift, b};
+        if (M.pos[ka] >= 0)
+            kp.join2_a.f[kp.join2_a.nf++] = KeyField{M.pos[ka], shift, b};
+        else
+            kp.join2_b.f[kp.join2_b.nf++] = KeyField{M.pos[kb], shift, b};
+    }
+    kp.ident_c = leading_cols(s, in[kc], kc, kp.join2);
     return UCL_OK;
 }
 
@@ -207,6 +264,7 @@ ucl_status plan_lower(ucl_ctx *ctx, const Spec &s, ucl_rel *const *in, LowerPlan
     memset(&lp, 0, sizeof(lp));
     lp.tile_u = in[0]->tile;
     lp.tile_v = s.n_in > 1 ? in[1]->tile : 1;
+    lp.tile_x = s.n_in > 2 ? in[2]->tile : 1;
     lp.tile_w = 1;
     for (char c : s.out) {
         const Label &L = s.labs[s.find(c)];
@@ -214,6 +272,7 @@ ucl_status plan_lower(ucl_ctx *ctx, const Spec &s, ucl_rel *const *in, LowerPlan
         lp.w_ext[lp.nw] = (int)L.ext;
         lp.w_su[lp.nw] = (int)tile_stride(s, 0, L);
         lp.w_sv[lp.nw] = s.n_in > 1 ? (int)tile_stride(s, 1, L) : 0;
+        lp.w_sx[lp.nw] = s.n_in > 2 ? (int)tile_stride(s, 2, L) : 0;
         lp.tile_w *= L.ext;
         lp.nw++;
     }
@@ -224,10 +283,12 @@ ucl_status plan_lower(ucl_ctx *ctx, const Spec &s, ucl_rel *const *in, LowerPlan
         lp.c_ext[lp.nc] = (int)L.ext;
         lp.c_su[lp.nc] = (int)tile_stride(s, 0, L);
         lp.c_sv[lp.nc] = s.n_in > 1 ? (int)tile_stride(s, 1, L) : 0;
+        lp.c_sx[lp.nc] = s.n_in > 2 ? (int)tile_stride(s, 2, L) : 0;
         lp.n_c *= L.ext;
         lp.nc++;
     }
-    if (lp.tile_w >= (1ll << 31) || lp.tile_u >= (1ll << 31) || lp.tile_v >= (1ll << 31))
+    if (lp.tile_w >= (1ll << 31) || lp.tile_u >= (1ll << 31) || lp.tile_v >= (1ll << 31) ||
+        lp.tile_x >= (1ll << 31))
         return fail(ctx, UCL_ERR_UNSUPPORTED, "tile has 2^31 or more elements");
     return UCL_OK;
 }
@@ -237,7 +298,7 @@ ucl_status plan_lower(ucl_ctx *ctx, const Spec &s, ucl_rel *const *in, LowerPlan
 // operands bf16.  The operand giving the larger M-side extent becomes A.
 bool plan_tc(const Spec &s, ucl_rel *const *in, TcPlan &tp, std::string *why) {
     memset(&tp, 0, sizeof(tp));
-    if (s.n_in != 2) { *why = "unary"; return false; }
+    if (s.n_in != 2) { *why = "not a binary EinSum"; return false; }
     if (in[0]->dtype != UCL_BF16 || in[1]->dtype != UCL_BF16) { *why = "operands are not bf16"; return false; }
     int mu = -1, nv = -1, kk = -1;
     for (size_t i = 0; i < s.labs.size(); ++i) {
@@ -702,7 +763,11 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
 
     const ucl_rel *U = in[0];
     const ucl_rel *V = n_in > 1 ? in[1] : nullptr;
-    const int64_t nU = U->n, nV = V ? V->n : 1;
+    const ucl_rel *X = n_in > 2 ? in[2] : nullptr;
+    const int64_t nU = U->n, nV = V ? V->n : 1, nX = X ? X->n : 1;
+    // join order: A = ord[0], B = ord[1], C = ord[2] (spec order for < 3 inputs)
+    const ucl_rel *A = in[kp.ord[0]], *B = n_in > 1 ? in[kp.ord[1]] : nullptr, *C = n_in > 2 ? in[kp.ord[2]] : nullptr;
+    const int64_t nA = A->n, nB = B ? B->n : 1, nC = C ? C->n : 1;
     ucl_stats stats{};
     ctx->launches = 0;
     ucl_rel *R = nullptr;
@@ -712,50 +777,87 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
         record(ctx, 0);
         int64_t *d_scal = (int64_t *)ws_get(ctx, 8 * sizeof(int64_t));
         // ---------------------------------------------------------- stage 0
-        int64_t P = 0;
-        uint64_t *koU = nullptr, *koV = nullptr, *permU = nullptr, *permV = nullptr;
-        int64_t *off = nullptr;
-        uint32_t *lo = nullptr;
-        if (nU > 0 && nV > 0) {
-            koU = (uint64_t *)ws_get(ctx, 8 * nU);
-            uint64_t *jkU = V ? (uint64_t *)ws_get(ctx, 8 * nU) : nullptr;
-            launch_pack(ctx, U->keys, U->u, nU, kp.join_u, jkU, kp.out_u, koU);
-            if (V) {
-                koV = (uint64_t *)ws_get(ctx, 8 * nV);
-                uint64_t *jkV = (uint64_t *)ws_get(ctx, 8 * nV);
-                launch_pack(ctx, V->keys, V->u, nV, kp.join_v, jkV, kp.out_v, koV);
-                const bool join = !kp.join.empty();
-                if (join && !kp.ident_u) {
-                    uint64_t *vals = (uint64_t *)ws_get(ctx, 8 * nU), *ka = (uint64_t *)ws_get(ctx, 8 * nU),
-                             *va = (uint64_t *)ws_get(ctx, 8 * nU);
-                    launch_iota(ctx, vals, nU);
-                    int w = radix_sort(ctx, jkU, vals, ka, va, nU, kp.join_bits);
-                    if (w) { jkU = ka; permU = va; } else permU = vals;
-                }
-                if (join && !kp.ident_v) {
-                    uint64_t *vals = (uint64_t *)ws_get(ctx, 8 * nV), *ka = (uint64_t *)ws_get(ctx, 8 * nV),
-                             *va = (uint64_t *)ws_get(ctx, 8 * nV);
-                    launch_iota(ctx, vals, nV);
-                    int w = radix_sort(ctx, jkV, vals, ka, va, nV, kp.join_bits);
-                    if (w) { jkV = ka; permV = va; } else permV = vals;
-                }
-                int64_t *cnt = (int64_t *)ws_get(ctx, 8 * nU);
-                lo = (uint32_t *)ws_get(ctx, 4 * nU);
-                off = (int64_t *)ws_get(ctx, 8 * nU);
-                launch_join_count(ctx, join ? jkU : nullptr, nU, join ? jkV : nullptr, nV, cnt, lo);
-                scan_i64(ctx, cnt, off, nU, d_scal);
+        // pack keys; sort each side of a join by its join key unless it is
+        // already grouped; count the joined pairs (for three inputs: the
+        // pairs of the first join, then the triples)
+        int64_t P = 0, P1 = 0;
+        uint64_t *koA = nullptr, *koB = nullptr, *koC = nullptr;
+        uint64_t *permA = nullptr, *permB = nullptr, *permC = nullptr;
+        int64_t *off = nullptr, *off2 = nullptr;
+        uint32_t *lo = nullptr, *lo2 = nullptr;
+        uint64_t *pk1 = nullptr, *pv1 = nullptr;
+        auto sort_by = [&](uint64_t *&jk, int64_t cnt, int bits, uint64_t *&perm) {
+            uint64_t *vals = (uint64_t *)ws_get(ctx, 8 * cnt), *ka = (uint64_t *)ws_get(ctx, 8 * cnt),
+                     *va = (uint64_t *)ws_get(ctx, 8 * cnt);
+            launch_iota(ctx, vals, cnt);
+            if (radix_sort(ctx, jk, vals, ka, va, cnt, bits)) { jk = ka; perm = va; } else perm = vals;
+        };
+        auto sync_count = [&](int64_t *dev) {
+            int64_t h;
+            check(sync_read(ctx, dev, 1, &h));
+            if (h >= (1ll << 31)) check(fail(ctx, UCL_ERR_UNSUPPORTED, "more than 2^31-1 joined pairs"));
+            return h;
+        };
+        if (nA > 0 && nB > 0 && nC > 0) {
+            koA = (uint64_t *)ws_get(ctx, 8 * nA);
+            uint64_t *jkA = B ? (uint64_t *)ws_get(ctx, 8 * nA) : nullptr;
+            launch_pack(ctx, A->keys, A->u, nA, kp.join_u, jkA, kp.out_k[kp.ord[0]], koA);
+            if (!B) {
                 record(ctx, 1);
-                int64_t h;
-                check(sync_read(ctx, d_scal, 1, &h));
-                P = h;
+                P = nA;
             } else {
-                record(ctx, 1);
-                P = nU;
+                koB = (uint64_t *)ws_get(ctx, 8 * nB);
+                uint64_t *jkB = (uint64_t *)ws_get(ctx, 8 * nB);
+                launch_pack(ctx, B->keys, B->u, nB, kp.join_v, jkB, kp.out_k[kp.ord[1]], koB);
+                const bool join = !kp.join.empty();
+                if (join && !kp.ident_u) sort_by(jkA, nA, kp.join_bits, permA);
+                if (join && !kp.ident_v) sort_by(jkB, nB, kp.join_bits, permB);
+                int64_t *cnt = (int64_t *)ws_get(ctx, 8 * nA);
+                lo = (uint32_t *)ws_get(ctx, 4 * nA);
+                off = (int64_t *)ws_get(ctx, 8 * nA);
+                launch_join_count(ctx, join ? jkA : nullptr, nA, join ? jkB : nullptr, nB, cnt, lo);
+                scan_i64(ctx, cnt, off, nA, d_scal);
+                if (!C) {
+                    record(ctx, 1);
+                    P = sync_count(d_scal);
+                } else if ((P1 = sync_count(d_scal)) > 0) {
+                    // second join: each pair's key on the attributes C shares
+                    pk1 = (uint64_t *)ws_get(ctx, 8 * P1);
+                    pv1 = (uint64_t *)ws_get(ctx, 8 * P1);
+                    launch_expand(ctx, off, nA, lo, permA, permB, koA, koB, P1, pk1, pv1);
+                    koC = (uint64_t *)ws_get(ctx, 8 * nC);
+                    uint64_t *jkC = (uint64_t *)ws_get(ctx, 8 * nC);
+                    launch_pack(ctx, C->keys, C->u, nC, kp.join2_c, jkC, kp.out_k[kp.ord[2]], koC);
+                    const bool join2 = !kp.join2.empty();
+                    uint64_t *jkP = nullptr;
+                    if (join2) {
+                        uint64_t *ja = nullptr, *jb = nullptr;
+                        if (kp.join2_a.nf) {
+                            ja = (uint64_t *)ws_get(ctx, 8 * nA);
+                            launch_pack(ctx, A->keys, A->u, nA, kp.join2_a, ja, KeyPack{}, nullptr);
+                        }
+                        if (kp.join2_b.nf) {
+                            jb = (uint64_t *)ws_get(ctx, 8 * nB);
+                            launch_pack(ctx, B->keys, B->u, nB, kp.join2_b, jb, KeyPack{}, nullptr);
+                        }
+                        jkP = (uint64_t *)ws_get(ctx, 8 * P1);
+                        launch_pair_keys(ctx, pv1, P1, ja, jb, jkP);
+                        if (!kp.ident_c) sort_by(jkC, nC, kp.join2_bits, permC);
+                    }
+                    int64_t *cnt2 = (int64_t *)ws_get(ctx, 8 * P1);
+                    lo2 = (uint32_t *)ws_get(ctx, 4 * P1);
+                    off2 = (int64_t *)ws_get(ctx, 8 * P1);
+                    launch_join_count(ctx, jkP, P1, join2 ? jkC : nullptr, nC, cnt2, lo2);
+                    scan_i64(ctx, cnt2, off2, P1, d_scal + 2);
+                    record(ctx, 1);
+                    P = sync_count(d_scal + 2);
+                } else {
+                    record(ctx, 1);
+                }
             }
         } else {
             record(ctx, 1);
         }
-        if (P >= (1ll << 31)) check(fail(ctx, UCL_ERR_UNSUPPORTED, "more than 2^31-1 joined pairs"));
 
         // ---------------------------------------------------------- stage 1
         int64_t S = 0;
@@ -765,10 +867,12 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             pk = (uint64_t *)ws_get(ctx, 8 * P);
             pv = (uint64_t *)ws_get(ctx, 8 * P);
             uint64_t *pk2 = (uint64_t *)ws_get(ctx, 8 * P), *pv2 = (uint64_t *)ws_get(ctx, 8 * P);
-            if (V)
-                launch_expand(ctx, off, nU, lo, permU, permV, koU, koV, P, pk, pv);
+            if (C)
+                launch_expand3(ctx, off2, P1, lo2, permC, pk1, koC, P, pk, pv);
+            else if (B)
+                launch_expand(ctx, off, nA, lo, permA, permB, koA, koB, P, pk, pv);
             else
-                launch_unary_pairs(ctx, koU, P, pk, pv);
+                launch_unary_pairs(ctx, koA, P, pk, pv);
             if (radix_sort(ctx, pk, pv, pk2, pv2, P, kp.out_bits)) { pk = pk2; pv = pv2; }
             int64_t *flag = (int64_t *)ws_get(ctx, 8 * P);
             seg_excl = (int64_t *)ws_get(ctx, 8 * P);
@@ -806,17 +910,27 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
         if (P > 0) {
             int64_t *seg_start = (int64_t *)ws_get(ctx, 8 * (S + 1));
             uint32_t *pu = (uint32_t *)ws_get(ctx, 4 * P), *pvi = (uint32_t *)ws_get(ctx, 4 * P);
-            launch_segments(ctx, pk, pv, seg_excl, P, S, kp.unpack, R->keys, seg_start, pu, pvi);
+            uint32_t *pxi = X ? (uint32_t *)ws_get(ctx, 4 * P) : nullptr;
+            if (X) {
+                uint32_t *const idx[3] = {pu, pvi, pxi};
+                launch_segments3(ctx, pk, pv, pv1, seg_excl, P, S, kp.unpack, kp.ord, R->keys, seg_start, idx);
+            } else {
+                launch_segments(ctx, pk, pv, seg_excl, P, S, kp.unpack, R->keys, seg_start, pu, pvi);
+            }
             record(ctx, 2);
             ContractArgs a{};
             a.U = U->tiles;
             a.V = V ? V->tiles : nullptr;
+            a.X = X ? X->tiles : nullptr;
             a.du = U->dtype;
             a.dv = V ? V->dtype : U->dtype;
+            a.dx = X ? X->dtype : U->dtype;
             a.nU = nU;
             a.nV = V ? nV : 0;
+            a.nX = X ? nX : 0;
             a.pu = pu;
             a.pv = pvi;
+            a.px = pxi;
             a.seg_start = seg_start;
             a.S = S;
             a.out = R->tiles;
@@ -856,8 +970,10 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
         stats.n_pairs = P;
         stats.n_segments = S;
         stats.flops = 2.0 * (double)P * (double)lp.tile_w * (double)lp.n_c;
-        stats.bytes_contract = (double)nU * U->tile * dsize(U->dtype) + (V ? (double)nV * V->tile * dsize(V->dtype) : 0.0) +
-                               (double)S * lp.tile_w * dsize(o.out_dtype) + 8.0 * (double)P;
+        stats.bytes_contract = (double)nU * U->tile * dsize(U->dtype) +
+                               (V ? (double)nV * V->tile * dsize(V->dtype) : 0.0) +
+                               (X ? (double)nX * X->tile * dsize(X->dtype) : 0.0) +
+                               (double)S * lp.tile_w * dsize(o.out_dtype) + 4.0 * n_in * (double)P;
         stats.path = path;
         stats.launches = ctx->launches;
         stats.timed = ctx->cur_ev != nullptr;

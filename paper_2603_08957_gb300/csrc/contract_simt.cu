@@ -145,6 +145,92 @@ __global__ void __launch_bounds__(kSimtThreads) simt_contract_kernel(ContractArg
     if (bad) atomicOr(status, bad);
 }
 
+__device__ __forceinline__ float ld_any(const void *base, int64_t i, bool bf16) {
+    return bf16 ? __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(base)[i])
+                : __ldg(reinterpret_cast<const float *>(base) + i);
+}
+
+// Three-way EinSum (a star join such as MTTKRP): the product of the three
+// tiles' entries summed over the contracted lower labels.  Operand dtypes are
+// read at run time; the partial/fixup protocol is the binary kernel's.
+__global__ void __launch_bounds__(kSimtThreads) simt_contract3_kernel(ContractArgs a, LowerPlan lp,
+                                                                      uint32_t *status) {
+    __shared__ int s_c[3][kMaxTab];
+    const bool tab = lp.n_c <= kMaxTab;
+    const bool bu = a.du == UCL_BF16, bv = a.dv == UCL_BF16, bx = a.dx == UCL_BF16;
+    if (tab) {
+        for (int64_t c = threadIdx.x; c < lp.n_c; c += blockDim.x) {
+            int64_t rem = c;
+            int ou = 0, ov = 0, ox = 0;
+            for (int q = lp.nc - 1; q >= 0; --q) {
+                int idx = (int)(rem % lp.c_ext[q]);
+                rem /= lp.c_ext[q];
+                ou += idx * lp.c_su[q];
+                ov += idx * lp.c_sv[q];
+                ox += idx * lp.c_sx[q];
+            }
+            s_c[0][c] = ou;
+            s_c[1][c] = ov;
+            s_c[2][c] = ox;
+        }
+    }
+    __syncthreads();
+    const int unit = blockIdx.x;
+    const int64_t pb = a.units.begin(unit), pe = a.units.begin(unit + 1);
+    uint32_t bad = 0;
+    for (int64_t s = find_seg(a.seg_start, a.S, pb); s < a.S; ++s) {
+        const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
+        if (ss >= pe) break;
+        const int64_t p0 = ss > pb ? ss : pb, p1 = se < pe ? se : pe;
+        const int kind = (ss >= pb && se <= pe) ? 0 : (ss < pb ? 1 : 2);
+        for (int64_t w = threadIdx.x; w < a.tile_w; w += blockDim.x) {
+            int64_t rem = w;
+            int64_t ou = 0, ov = 0, ox = 0;
+            for (int q = lp.nw - 1; q >= 0; --q) {
+                int idx = (int)(rem % lp.w_ext[q]);
+                rem /= lp.w_ext[q];
+                ou += idx * lp.w_su[q];
+                ov += idx * lp.w_sv[q];
+                ox += idx * lp.w_sx[q];
+            }
+            float acc = 0.0f;
+            for (int64_t p = p0; p < p1; ++p) {
+                const uint32_t iu = a.pu[p], iv = a.pv[p], ix = a.px[p];
+                if (iu >= a.nU || iv >= a.nV || ix >= a.nX) {
+                    bad = kStBadIndex;
+                    continue;
+                }
+                const int64_t bu0 = (int64_t)iu * lp.tile_u + ou, bv0 = (int64_t)iv * lp.tile_v + ov,
+                              bx0 = (int64_t)ix * lp.tile_x + ox;
+                for (int64_t c = 0; c < lp.n_c; ++c) {
+                    int cu, cv, cx;
+                    if (tab) {
+                        cu = s_c[0][c];
+                        cv = s_c[1][c];
+                        cx = s_c[2][c];
+                    } else {
+                        int64_t rem2 = c;
+                        cu = cv = cx = 0;
+                        for (int q = lp.nc - 1; q >= 0; --q) {
+                            int idx = (int)(rem2 % lp.c_ext[q]);
+                            rem2 /= lp.c_ext[q];
+                            cu += idx * lp.c_su[q];
+                            cv += idx * lp.c_sv[q];
+                            cx += idx * lp.c_sx[q];
+                        }
+                    }
+                    acc = fmaf(ld_any(a.U, bu0 + cu, bu) * ld_any(a.V, bv0 + cv, bv), ld_any(a.X, bx0 + cx, bx), acc);
+                }
+            }
+            if (kind == 0)
+                store_out(a.out, a.dout, s * a.tile_w + w, epilogue(acc, a.epi, a.scale));
+            else
+                a.partials[((int64_t)unit * 2 + (kind == 1 ? 0 : 1)) * a.tile_w + w] = acc;
+        }
+    }
+    if (bad) atomicOr(status, bad);
+}
+
 // Boundary c (between units c-1 and c) owns the segment that crosses it if
 // that segment starts inside unit c-1; it sums the segment's partials in unit
 // order and writes the output tile.
@@ -171,6 +257,11 @@ __global__ void __launch_bounds__(kSimtThreads) fixup_kernel(ContractArgs a) {
 void launch_contract_simt(ucl_ctx *ctx, const ContractArgs &a, const LowerPlan &lp) {
     const int G = a.units.G;
     if (G <= 0) return;
+    if (a.X) {
+        simt_contract3_kernel<<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status);
+        ctx->launches++;
+        return;
+    }
     if (a.du == UCL_F32 && (!a.V || a.dv == UCL_F32))
         simt_contract_kernel<float, float><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status);
     else if (a.du == UCL_F32)

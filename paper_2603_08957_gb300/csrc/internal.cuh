@@ -45,20 +45,22 @@ struct KeyUnpack {
     int bits[kMaxCols];
 };
 
-// Generic lower-label contraction of one pair (FFMA path):
-//   W[w] += sum_c U[offU(w) + cU(c)] * V[offV(w) + cV(c)]
+// Generic lower-label contraction of one joined pair (FFMA path):
+//   W[w] += sum_c U[offU(w) + cU(c)] * V[offV(w) + cV(c)] (* X[offX(w) + cX(c)])
 // w runs over W's lower labels (row-major, W's order), c over the lower
-// labels absent from W.
+// labels absent from W; X is the third input of a three-way EinSum.
 struct LowerPlan {
     int nw;
     int w_ext[kMaxCols];
     int w_su[kMaxCols];
     int w_sv[kMaxCols];
+    int w_sx[kMaxCols];
     int nc;
     int c_ext[kMaxLow];
     int c_su[kMaxLow];
     int c_sv[kMaxLow];
-    int64_t tile_u, tile_v, tile_w, n_c;
+    int c_sx[kMaxLow];
+    int64_t tile_u, tile_v, tile_x, tile_w, n_c;
 };
 
 // tcgen05 contraction shape: D[M x N] += A[M x K] * B[K x N] per pair, with
@@ -176,6 +178,19 @@ void launch_heads(ucl_ctx *ctx, const uint64_t *pk, int64_t P, int64_t *flag);
 // Segment starts, output keys, pair index arrays.
 void launch_segments(ucl_ctx *ctx, const uint64_t *pk, const uint64_t *pv, const int64_t *seg_excl, int64_t P,
                      int64_t S, KeyUnpack un, int32_t *out_keys, int64_t *seg_start, uint32_t *pu, uint32_t *pvi);
+// Three-way join, second step.  pair_keys: jk[p] = jk_a[a] | jk_b[b] for
+// each first-step pair pv1[p] = (a << 32) | b (either table may be NULL).
+void launch_pair_keys(ucl_ctx *ctx, const uint64_t *pv1, int64_t P1, const uint64_t *jk_a, const uint64_t *jk_b,
+                      uint64_t *jk);
+// expand3: triple t of pair p (found in off2) and the third input's row c:
+// pk[t] = pk1[p] | ko_c[c], pv[t] = (p << 32) | c.
+void launch_expand3(ucl_ctx *ctx, const int64_t *off2, int64_t P1, const uint32_t *lo2, const uint64_t *perm_c,
+                    const uint64_t *pk1, const uint64_t *ko_c, int64_t P, uint64_t *pk, uint64_t *pv);
+// segments3: as launch_segments, with each triple's three row indices written
+// in spec order: idx[ord[0]] = a, idx[ord[1]] = b, idx[ord[2]] = c.
+void launch_segments3(ucl_ctx *ctx, const uint64_t *pk, const uint64_t *pv, const uint64_t *pv1,
+                      const int64_t *seg_excl, int64_t P, int64_t S, KeyUnpack un, const int ord[3],
+                      int32_t *out_keys, int64_t *seg_start, uint32_t *const idx[3]);
 
 // ---- contraction (contract_simt.cu / contract_tc.cu)
 struct ContractArgs {
@@ -185,6 +200,10 @@ struct ContractArgs {
     int64_t nU, nV;
     const uint32_t *pu;    // [P] U tuple of each pair
     const uint32_t *pv;    // [P] V tuple of each pair
+    const void *X;         // third input of a three-way EinSum, else NULL
+    ucl_dtype dx;
+    int64_t nX;
+    const uint32_t *px;    // [P] X tuple of each triple
     const int64_t *seg_start;  // [S + 1]
     int64_t S;
     Units units;

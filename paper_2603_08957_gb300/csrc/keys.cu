@@ -311,6 +311,64 @@ __global__ void segments_kernel(const uint64_t *__restrict__ pk, const uint64_t 
     }
 }
 
+// Last row i of a monotone offset table with off[i] <= p.
+__device__ __forceinline__ int64_t owner_row(const int64_t *off, int64_t n, int64_t p) {
+    int64_t a = 0, b = n;
+    while (a < b) {
+        int64_t mid = (a + b) >> 1;
+        if (off[mid] <= p) a = mid + 1; else b = mid;
+    }
+    return a - 1;
+}
+
+__global__ void pair_keys_kernel(const uint64_t *__restrict__ pv1, int64_t P1, const uint64_t *__restrict__ jk_a,
+                                 const uint64_t *__restrict__ jk_b, uint64_t *jk) {
+    for (int64_t p = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; p < P1; p += (int64_t)gridDim.x * blockDim.x) {
+        const uint64_t v = pv1[p];
+        jk[p] = (jk_a ? jk_a[v >> 32] : 0ull) | (jk_b ? jk_b[(uint32_t)v] : 0ull);
+    }
+}
+
+__global__ void expand3_kernel(const int64_t *__restrict__ off2, int64_t P1, const uint32_t *__restrict__ lo2,
+                               const uint64_t *__restrict__ perm_c, const uint64_t *__restrict__ pk1,
+                               const uint64_t *__restrict__ ko_c, int64_t P, uint64_t *pk, uint64_t *pv) {
+    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < P; t += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t p = owner_row(off2, P1, t);
+        const int64_t cpos = (int64_t)lo2[p] + (t - off2[p]);
+        const uint64_t c = perm_c ? perm_c[cpos] : (uint64_t)cpos;
+        pk[t] = pk1[p] | ko_c[c];
+        pv[t] = ((uint64_t)p << 32) | c;
+    }
+}
+
+struct Ord3 {
+    int o[3];
+};
+
+__global__ void segments3_kernel(const uint64_t *__restrict__ pk, const uint64_t *__restrict__ pv,
+                                 const uint64_t *__restrict__ pv1, const int64_t *__restrict__ seg_excl, int64_t P,
+                                 int64_t S, KeyUnpack un, Ord3 ord, int32_t *out_keys, int64_t *seg_start,
+                                 uint32_t *i0, uint32_t *i1, uint32_t *i2) {
+    uint32_t *idx[3] = {i0, i1, i2};
+    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < P; t += (int64_t)gridDim.x * blockDim.x) {
+        const uint64_t v = pv[t];
+        const uint64_t ab = pv1[v >> 32];
+        idx[ord.o[0]][t] = (uint32_t)(ab >> 32);
+        idx[ord.o[1]][t] = (uint32_t)ab;
+        idx[ord.o[2]][t] = (uint32_t)v;
+        const uint64_t k = pk[t];
+        if (t == 0 || k != pk[t - 1]) {
+            const int64_t s = seg_excl[t];
+            seg_start[s] = t;
+            for (int c = 0; c < un.uw; ++c) {
+                uint64_t mask = un.bits[c] ? ((~0ull) >> (64 - un.bits[c])) : 0ull;
+                out_keys[s * un.uw + c] = (int32_t)((k >> un.shift[c]) & mask);
+            }
+        }
+        if (t == 0) seg_start[S] = P;
+    }
+}
+
 }  // namespace
 
 // ------------------------------------------------------------ launchers
@@ -400,6 +458,30 @@ void launch_segments(ucl_ctx *ctx, const uint64_t *pk, const uint64_t *pv, const
     if (P <= 0) return;
     segments_kernel<<<grid_for(ctx, P), kThreads, 0, ctx->stream>>>(pk, pv, seg_excl, P, S, un, out_keys,
                                                                     seg_start, pu, pvi);
+    ctx->launches++;
+}
+
+void launch_pair_keys(ucl_ctx *ctx, const uint64_t *pv1, int64_t P1, const uint64_t *jk_a, const uint64_t *jk_b,
+                      uint64_t *jk) {
+    if (P1 <= 0) return;
+    pair_keys_kernel<<<grid_for(ctx, P1), kThreads, 0, ctx->stream>>>(pv1, P1, jk_a, jk_b, jk);
+    ctx->launches++;
+}
+
+void launch_expand3(ucl_ctx *ctx, const int64_t *off2, int64_t P1, const uint32_t *lo2, const uint64_t *perm_c,
+                    const uint64_t *pk1, const uint64_t *ko_c, int64_t P, uint64_t *pk, uint64_t *pv) {
+    if (P <= 0) return;
+    expand3_kernel<<<grid_for(ctx, P), kThreads, 0, ctx->stream>>>(off2, P1, lo2, perm_c, pk1, ko_c, P, pk, pv);
+    ctx->launches++;
+}
+
+void launch_segments3(ucl_ctx *ctx, const uint64_t *pk, const uint64_t *pv, const uint64_t *pv1,
+                      const int64_t *seg_excl, int64_t P, int64_t S, KeyUnpack un, const int ord[3],
+                      int32_t *out_keys, int64_t *seg_start, uint32_t *const idx[3]) {
+    if (P <= 0) return;
+    Ord3 o{{ord[0], ord[1], ord[2]}};
+    segments3_kernel<<<grid_for(ctx, P), kThreads, 0, ctx->stream>>>(pk, pv, pv1, seg_excl, P, S, un, o, out_keys,
+                                                                     seg_start, idx[0], idx[1], idx[2]);
     ctx->launches++;
 }
 

@@ -109,6 +109,9 @@ SPECS = [
     ("i,j->ij", {"i": 5, "j": 4}),
     ("ij,ij->i", {"i": 5, "j": 3}),
     ("ijk->ki", {"i": 3, "j": 4, "k": 5}),
+    ("ijk,jr,kr->ir", {"i": 3, "j": 4, "k": 2, "r": 5}),   # MTTKRP: star join
+    ("ij,jk,kl->il", {"i": 3, "j": 4, "k": 3, "l": 2}),    # chain: C joins through B
+    ("i,j,k->ijk", {"i": 3, "j": 2, "k": 4}),               # no shared labels: cross products
 ]
 
 
@@ -391,6 +394,56 @@ def test_two_layer_gnn_full_size_sampled(ctx):
     ref = oracle_ref(w["spec4"], [(t2k, T2.bounds, t2t), w["W2"]])
     assert_parity(O, ref, torch.bfloat16, select=sel2)
     for r in (X, Y, W1, W2, T1, H1, T2, O):
+        r.destroy()
+    del w
+    torch.cuda.empty_cache()
+
+
+# ------------------------------------------------------------ three inputs
+
+
+@pytest.mark.parametrize("path", ["simt", "auto"])
+def test_mttkrp_small(ctx, path):
+    """MTTKRP over a 1000^3 Zipf(1.1) tensor with 5000 nonzeros in 16^3 tiles,
+    rank 64, bf16: the whole output checked."""
+    w = workloads.mttkrp(seed=0, n=1000, nnz=5000)
+    ref = oracle_ref(w["spec"], [w["T"], w["B"], w["C"]])
+    out = ctx.einsum(w["spec"], *(gpu_rel(ctx, w[k]) for k in ("T", "B", "C")), path=path)
+    assert_parity(out, ref, torch.bfloat16)
+    assert ctx.last_stats()["n_pairs"] == ref["n_pairs"] == len(w["T"][0])
+    # operands in another order: the join order is chosen from the keys
+    out2 = ctx.einsum("Jjr,IJKijk,Kkr->Iir", *(gpu_rel(ctx, w[k]) for k in ("B", "T", "C")), path=path)
+    assert_parity(out2, ref, torch.bfloat16)
+
+
+def test_mttkrp_full_size_sampled(ctx):
+    """MTTKRP at full size: a 100000^3 tensor with 1e7 Zipf(1.1) nonzeros in
+    16^3 tiles (~3.9M tiles, ~32 GB bf16), rank-64 factors.  The whole output
+    key set is checked, values on sampled output keys (the oracle gets the T
+    tiles of those keys and the factor tiles they join with)."""
+    w = workloads.mttkrp(seed=0, device="cuda")
+    dev = torch.device("cuda", 0)
+    rels = [gpu_rel(ctx, w[k]) for k in ("T", "B", "C")]
+    out = ctx.einsum(w["spec"], *rels)
+    kt = w["T"][0]
+    got = out.device_tensors()[0].cpu().numpy()
+    assert np.array_equal(got, np.unique(kt[:, 0]).astype(np.int32)[:, None])
+    assert ctx.last_stats()["n_pairs"] == len(kt)
+    cnt = np.bincount(kt[:, 0])
+    rng = np.random.default_rng(5)
+    small = np.nonzero((cnt > 0) & (cnt <= np.median(cnt[cnt > 0])))[0]
+    sk = np.sort(rng.choice(small, size=3, replace=False)).astype(np.int32)
+    m = np.nonzero(np.isin(kt[:, 0], sk))[0]
+    tsub = (kt[m], w["T"][1], w["T"][2][torch.as_tensor(m, device=dev)].cpu())
+
+    def factor_rows(f, rows):
+        rows = np.unique(rows)
+        return (rows[:, None].astype(np.int32), f[1], f[2][torch.as_tensor(rows, device=dev)].cpu())
+
+    ref = oracle_ref(w["spec"], [tsub, factor_rows(w["B"], kt[m, 1]), factor_rows(w["C"], kt[m, 2])],
+                     sample_keys=sk[:, None])
+    assert_parity(out, ref, torch.bfloat16, select=np.searchsorted(got[:, 0], sk))
+    for r in rels + [out]:
         r.destroy()
     del w
     torch.cuda.empty_cache()

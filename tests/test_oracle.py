@@ -13,6 +13,7 @@ import numpy as np
 import pytest
 
 import oracle
+import workloads
 from tests.ucl_testutil import brute_force, decompose, golden, random_sparse, recompose, ucl_operand
 
 GOLD = golden(os.path.join(os.path.dirname(__file__), "golden", "worked_example.txt"))
@@ -177,6 +178,29 @@ def test_tiled_reshape_matches_dense():
     cnt_a = np.bincount(ka[:, 1], minlength=ba[1])
     cnt_b = np.bincount(kb[:, 0], minlength=bb[0])
     assert r["n_pairs"] == int((cnt_a * cnt_b).sum())
+
+
+def test_mttkrp_workload_matches_dense():
+    """The sparse MTTKRP workload (Zipf coordinates in t^3 tiles, ragged last
+    tile row of the factors) evaluated by the oracle equals the dense
+    MTTKRP of the same values; one triple per nonempty T tile."""
+    n, t, rank = 42, 4, 3
+    w = workloads.mttkrp(seed=2, n=n, nnz=300, t=t, rank=rank)
+    T, B, C = (workloads.to_oracle(w[k]) for k in ("T", "B", "C"))
+    assert np.unique(w["coords"].numpy()).size == 300
+    dense = np.zeros((len(B[2]) * t,) * 3)
+    for (I, J, K), tile in zip(T[0], T[2]):
+        dense[I * t:(I + 1) * t, J * t:(J + 1) * t, K * t:(K + 1) * t] = tile
+    assert np.count_nonzero(dense) <= 300 and not dense[n:].any()
+    Bd, Cd = B[2].reshape(-1, rank), C[2].reshape(-1, rank)
+    assert not Bd[n:].any() and not Cd[n:].any()
+    want = np.einsum("ijk,jr,kr->ir", dense, Bd, Cd)
+    r = oracle.einsum(w["spec"], [T, B, C])
+    assert r["n_pairs"] == len(T[0])
+    got = np.zeros_like(want)
+    for (I,), tile in zip(r["keys"], r["acc"]):
+        got[I * t:(I + 1) * t] = tile
+    np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-12)
 
 
 # ------------------------------------------------------ cardinalities (Sec. 1)

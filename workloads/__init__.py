@@ -247,6 +247,68 @@ def gnn_two_layer(seed=0, n=2_000_000, n_edges=40_000_000, feat=256, t=64, devic
     }
 
 
+def zipf_coords(n: int, nnz: int, order=3, s=1.1, seed=0, device="cpu", batch=1 << 23):
+    """nnz distinct order-`order` coordinates over [0, n)^order, each mode
+    drawn independently from a Zipf law over ranks 1..n (P(rank) ~ rank^-s,
+    index = rank - 1); draws continue until nnz distinct coordinates have
+    appeared and the first nnz in draw order are kept.  Returns the sorted
+    row-major codes (int64 tensor on `device`)."""
+    g = torch.Generator(device=device).manual_seed(seed)
+    w = torch.arange(1, n + 1, dtype=torch.float64, device=device) ** -s
+    cdf = torch.cumsum(w, 0)
+    cdf = cdf / cdf[-1]
+    draws = []
+    while True:
+        m = batch if draws else max(1024, min(batch, int(nnz * 1.3)))
+        code = torch.zeros(m, dtype=torch.int64, device=device)
+        for _ in range(order):
+            u = torch.rand(m, generator=g, device=device, dtype=torch.float64)
+            code = code * n + torch.searchsorted(cdf, u, right=True).clamp_(max=n - 1)
+        draws.append(code)
+        if torch.unique(torch.cat(draws)).numel() >= nnz:
+            break
+    allc = torch.cat(draws)
+    uniq, inv = torch.unique(allc, return_inverse=True)
+    pos = torch.arange(allc.numel(), device=device)
+    first = torch.full((uniq.numel(),), allc.numel(), dtype=torch.int64, device=device)
+    first.scatter_reduce_(0, inv, pos, reduce="amin")
+    keep = torch.argsort(first)[:nnz]
+    return torch.sort(uniq[keep]).values
+
+
+def mttkrp(seed=0, n=100_000, nnz=10_000_000, t=16, rank=64, s=1.1, device="cpu"):
+    """MTTKRP M[i,r] = sum_{j,k} T[i,j,k] B[j,r] C[k,r]: T sparse n^3 with nnz
+    Zipf(s) coordinates (zipf_coords), values U[-1,1), grouped into only-
+    nonempty t^3 bf16 tiles keyed (I, J, K); B and C dense n x rank bf16
+    U[-1,1) as per-tile-row relations keyed J (resp. K) with [t x rank] tiles
+    (rows past n zero).  Spec "IJKijk,Jjr,Kkr->Iir"."""
+    codes = zipf_coords(n, nnz, 3, s, seed, device)
+    g = torch.Generator(device=device).manual_seed(seed + 1)
+    vals = torch.rand(codes.numel(), generator=g, device=device) * 2 - 1
+    i, j, k = codes // (n * n), (codes // n) % n, codes % n
+    nt = -(-n // t)
+    tcode = ((i // t) * nt + j // t) * nt + k // t
+    ukeys, inv = torch.unique(tcode, return_inverse=True)
+    tiles = torch.zeros((ukeys.numel(), t, t, t), dtype=torch.bfloat16, device=device)
+    tiles[inv, i % t, j % t, k % t] = vals.to(torch.bfloat16)
+    keys = torch.stack([ukeys // (nt * nt), (ukeys // nt) % nt, ukeys % nt], 1).to(torch.int32).cpu().numpy()
+
+    def factor():
+        f = torch.zeros((nt * t, rank), device=device)
+        f[:n] = torch.rand((n, rank), generator=g, device=device) * 2 - 1
+        return (np.arange(nt, dtype=np.int32)[:, None], (nt,), f.view(nt, t, rank).to(torch.bfloat16))
+
+    return {
+        "spec": "IJKijk,Jjr,Kkr->Iir",
+        "T": (keys, (nt, nt, nt), tiles),
+        "B": factor(),
+        "C": factor(),
+        "coords": codes,
+        "n": n,
+        "t": t,
+    }
+
+
 def to_oracle(rel):
     """(keys, bounds, tiles) with tiles converted exactly to float64 numpy."""
     keys, bounds, tiles = rel
