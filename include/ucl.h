@@ -43,7 +43,7 @@ typedef enum {
     UCL_ERR_KEY_RANGE = 5,   /* a key value outside [0, bound) */
     UCL_ERR_OOM = 6,         /* the allocator returned NULL */
     UCL_ERR_CUDA = 7,        /* a CUDA runtime call failed */
-    UCL_ERR_UNSUPPORTED = 8, /* valid but outside this build (e.g. > 64 key bits, > 3 inputs) */
+    UCL_ERR_UNSUPPORTED = 8, /* valid but outside this build (e.g. > 64 key bits) */
     UCL_ERR_TIMEOUT = 9      /* a device-side wait ran out; the context stays usable */
 } ucl_status;
 
@@ -172,7 +172,7 @@ ucl_status ucl_relation_download(const ucl_rel *rel, int32_t *keys_host, void *t
 
 /* Evaluate one UCL EinSum (Sec. 4.3 notation, Sec. 5 Eq. eqn-TRA).
  *
- * Spec grammar: "<op>,<op>->" "<out>" with 1 or 2 input operands (n_in).
+ * Spec grammar: "<op>,<op>->" "<out>" with 1, 2 or 3 input operands (n_in).
  * Each operand is a string of letters, one letter per label; an upper-case
  * letter is a promoted label (a key column, in the order the upper-case
  * letters appear), a lower-case letter a demoted label (a tile dimension, in
@@ -184,6 +184,10 @@ ucl_status ucl_relation_download(const ucl_rel *rel, int32_t *keys_host, void *t
  * ones inside the tile kernel.  Shared upper labels are the join attributes;
  * with none the join is a cross product (Sec. 6.2).  n_in = 1 is a unary
  * EinSum (a group-by sum over one relation, e.g. with the relu epilogue).
+ * n_in = 3 joins all three inputs (tuples agree on every shared upper label)
+ * and multiplies the three tiles' entries, as in MTTKRP
+ * "IJKijk,Jjr,Kkr->Iir"; the two inputs sharing the most key bits are joined
+ * first, so a star join never forms a cross product of its factors.
  *
  * Output: a new relation owned by the library (destroy it with
  * ucl_relation_destroy), one tuple per distinct output key produced by at
@@ -191,7 +195,8 @@ ucl_status ucl_relation_download(const ucl_rel *rel, int32_t *keys_host, void *t
  * lexicographic key order; tiles row-major over the output's lower labels.
  *
  * Synchronises the stream twice (after the join count and after the segment
- * count: both sizes depend on the data).  The contraction is deterministic:
+ * count: both sizes depend on the data; three inputs add one sync after the
+ * first join's count).  The contraction is deterministic:
  * pairs of one output key are summed in a fixed order.
  * Errors: UCL_ERR_SPEC / SHAPE for spec-relation mismatches, UCL_ERR_OOM,
  * UCL_ERR_UNSUPPORTED (more than 2^31-1 joined pairs, > 64 key bits),
