@@ -336,6 +336,67 @@ bool plan_tc(const Spec &s, ucl_rel *const *in, TcPlan &tp, std::string *why) {
     return true;
 }
 
+// Three inputs of the MTTKRP shape: T with lower labels (i, e, f) in that
+// tile order, factor E with e and r, factor F with f and r laid out [f][r],
+// output with i and r; no other lower label; extents i = e = f = 16,
+// r = 64; all bf16.  E is the factor of the first join when T is in it (its
+// tuple changes least often along the pair list).
+bool plan_tc3(const Spec &s, ucl_rel *const *in, const KeyPlan &kp, Tc3Plan &tp, std::string *why) {
+    memset(&tp, 0, sizeof(tp));
+    if (s.n_in != 3) { *why = "not a three-input EinSum"; return false; }
+    for (int k = 0; k < 3; ++k)
+        if (in[k]->dtype != UCL_BF16) { *why = "operands are not bf16"; return false; }
+    tp.t = -1;
+    for (int k = 0; k < 3; ++k)
+        if (in[k]->r == 3) tp.t = k;
+    if (tp.t < 0 || in[(tp.t + 1) % 3]->r != 2 || in[(tp.t + 2) % 3]->r != 2) {
+        *why = "not one 3-d tile and two 2-d factor tiles";
+        return false;
+    }
+    const int t = tp.t;
+    // the label at each T tile position; the factor holding each
+    int lab[3] = {-1, -1, -1};
+    for (size_t i = 0; i < s.labs.size(); ++i)
+        if (!s.labs[i].upper && s.labs[i].pos[t] >= 0) lab[s.labs[i].pos[t]] = (int)i;
+    const Label &Li = s.labs[lab[0]], &Le = s.labs[lab[1]], &Lf = s.labs[lab[2]];
+    int fe = -1, ff = -1;
+    for (int k = 0; k < 3; ++k) {
+        if (k == t) continue;
+        if (Le.pos[k] >= 0) fe = k;
+        if (Lf.pos[k] >= 0) ff = k;
+    }
+    if (Li.pos[3] < 0 || Le.pos[3] >= 0 || Lf.pos[3] >= 0 || fe < 0 || ff < 0 || fe == ff ||
+        Li.pos[fe] >= 0 || Li.pos[ff] >= 0 || Le.pos[ff] >= 0 || Lf.pos[fe] >= 0) {
+        *why = "tile kernel is not MTTKRP-shaped";
+        return false;
+    }
+    int rl = -1;
+    for (size_t i = 0; i < s.labs.size(); ++i) {
+        const Label &L = s.labs[i];
+        if (L.upper || (int)i == lab[0] || (int)i == lab[1] || (int)i == lab[2]) continue;
+        if (rl >= 0 || L.pos[fe] < 0 || L.pos[ff] < 0 || L.pos[3] < 0) {
+            *why = "tile kernel is not MTTKRP-shaped";
+            return false;
+        }
+        rl = (int)i;
+    }
+    if (rl < 0) { *why = "no rank label"; return false; }
+    const Label &Lr = s.labs[rl];
+    if (Li.ext != 16 || Le.ext != 16 || Lf.ext != 16 || Lr.ext != 64) {
+        *why = "extents must be i = j = k = 16, r = 64";
+        return false;
+    }
+    if (Lf.pos[ff] != 0 || Lr.pos[ff] != 1) { *why = "F tile must be laid out [k][r]"; return false; }
+    (void)kp;
+    tp.e = fe;
+    tp.f = ff;
+    tp.sEj = tile_stride(s, fe, Le);
+    tp.sEr = tile_stride(s, fe, Lr);
+    tp.sWi = tile_stride(s, 3, Li);
+    tp.sWr = tile_stride(s, 3, Lr);
+    return true;
+}
+
 // --------------------------------------------------------------- helpers
 
 size_t dsize(ucl_dtype d) { return d == UCL_BF16 ? 2 : 4; }
@@ -756,8 +817,9 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
     LowerPlan lp;
     if ((st = plan_lower(ctx, s, in, lp))) return st;
     TcPlan tp;
+    Tc3Plan tp3;
     std::string why;
-    bool tc_ok = plan_tc(s, in, tp, &why);
+    const bool tc_ok = n_in == 3 ? plan_tc3(s, in, kp, tp3, &why) : plan_tc(s, in, tp, &why);
     if (o.path == UCL_PATH_TC && !tc_ok) return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why);
     cudaSetDevice(ctx->device);
 
@@ -939,18 +1001,22 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             a.scale = o.scale;
             a.tile_w = lp.tile_w;
             bool use_tc = tc_ok && o.path != UCL_PATH_SIMT;
-            if (use_tc) {
+            if (use_tc && n_in < 3) {
                 std::string why2;
                 if (!tc_supported(tp, a, &why2)) {
                     if (o.path == UCL_PATH_TC) check(fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why2));
                     use_tc = false;
                 }
             }
-            int G = use_tc ? tc_units(ctx, tp, P) : (int)std::min<int64_t>(P, (int64_t)ctx->sm_count * 4);
+            int G = use_tc ? (n_in == 3 ? tc3_units(ctx, P) : tc_units(ctx, tp, P))
+                           : (int)std::min<int64_t>(P, (int64_t)ctx->sm_count * 4);
             a.units.P = P;
             a.units.G = G;
             a.partials = (float *)ws_get(ctx, sizeof(float) * 2 * (size_t)G * lp.tile_w);
-            if (use_tc) {
+            if (use_tc && n_in == 3) {
+                check(launch_contract_tc3(ctx, a, tp3, in));
+                path = UCL_PATH_TC;
+            } else if (use_tc) {
                 const ucl_rel *ra = tp.a_is_u ? U : V, *rb = tp.a_is_u ? V : U;
                 check(launch_contract_tc(ctx, a, tp, ra, rb));
                 path = UCL_PATH_TC;

@@ -74,6 +74,15 @@ struct TcPlan {
     int64_t sWm, sWn;    // output tile strides of the M and N indices
 };
 
+// tcgen05 three-way contraction of the MTTKRP shape (one label of each
+// kind): W[i][r] += sum_{j,k} T[i][j][k] * E[j][r] * F[k][r], with the T
+// tile laid out [i][j][k] and the F tile [k][r]; i = j = k = 16, r = 64.
+struct Tc3Plan {
+    int t, e, f;             // spec positions of T, the epilogue factor E, the MMA factor F
+    int64_t sEj, sEr;        // E tile strides of j and r
+    int64_t sWi, sWr;        // output tile strides of i and r
+};
+
 // Partition of the pair list into G contiguous units (one CTA each).
 struct Units {
     int64_t P;
@@ -221,5 +230,7 @@ bool tc_supported(const TcPlan &tp, const ContractArgs &a, std::string *why);
 ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan &tp, const ucl_rel *ra,
                               const ucl_rel *rb);
 int tc_units(ucl_ctx *ctx, const TcPlan &tp, int64_t P);
+ucl_status launch_contract_tc3(ucl_ctx *ctx, const ContractArgs &a, const Tc3Plan &tp, const ucl_rel *const *in);
+int tc3_units(ucl_ctx *ctx, int64_t P);
 
 }  // namespace ucl

@@ -402,7 +402,7 @@ def test_two_layer_gnn_full_size_sampled(ctx):
 # ------------------------------------------------------------ three inputs
 
 
-@pytest.mark.parametrize("path", ["simt", "auto"])
+@pytest.mark.parametrize("path", ["simt", "auto", "tc"])
 def test_mttkrp_small(ctx, path):
     """MTTKRP over a 1000^3 Zipf(1.1) tensor with 5000 nonzeros in 16^3 tiles,
     rank 64, bf16: the whole output checked."""
@@ -411,6 +411,7 @@ def test_mttkrp_small(ctx, path):
     out = ctx.einsum(w["spec"], *(gpu_rel(ctx, w[k]) for k in ("T", "B", "C")), path=path)
     assert_parity(out, ref, torch.bfloat16)
     assert ctx.last_stats()["n_pairs"] == ref["n_pairs"] == len(w["T"][0])
+    assert ctx.last_stats()["path"] == ("simt" if path == "simt" else "tc")
     # operands in another order: the join order is chosen from the keys
     out2 = ctx.einsum("Jjr,IJKijk,Kkr->Iir", *(gpu_rel(ctx, w[k]) for k in ("B", "T", "C")), path=path)
     assert_parity(out2, ref, torch.bfloat16)
@@ -447,3 +448,34 @@ def test_mttkrp_full_size_sampled(ctx):
         r.destroy()
     del w
     torch.cuda.empty_cache()
+
+
+TC3_CASES = [
+    # (spec, T tile permutation, factor order, E layout [j][r] or [r][j])
+    ("IJKijk,Jjr,Kkr->Iir", (0, 1, 2), "BC", "jr"),   # E = B, groups of equal J
+    ("IJKijk,Jjr,Kkr->rIi", (0, 1, 2), "BC", "jr"),   # transposed output tile
+    ("IJKijk,Kkr,Jjr->Iir", (0, 1, 2), "CB", "jr"),   # first join on K: E changes every triple
+    ("IJKikj,Kkr,Jjr->Iir", (0, 2, 1), "CB", "jr"),   # T laid out [i][k][j]: E = C, F = B
+    ("IJKijk,Jrj,Kkr->Iir", (0, 1, 2), "BC", "rj"),   # E stored [r][j]
+]
+
+
+@pytest.mark.parametrize("spec,perm,order,elay", TC3_CASES)
+def test_tc3_layouts(ctx, spec, perm, order, elay):
+    """The tcgen05 MTTKRP path for every operand arrangement it accepts, with
+    bf16 / relu / scale epilogues; 2000^3 tensor, 20000 Zipf nonzeros."""
+    w = workloads.mttkrp(seed=4, n=2000, nnz=20000)
+    kt, bt, tt = w["T"]
+    T = (kt, bt, tt.permute(0, *[1 + p for p in perm]).contiguous())
+    fac = {"B": w["B"], "C": w["C"]}
+    if elay == "rj":
+        kb, bb, tb = fac["B"]
+        fac["B"] = (kb, bb, tb.transpose(1, 2).contiguous())
+    rels = [T, fac[order[0]], fac[order[1]]]
+    ref = oracle_ref(spec, rels)
+    out = ctx.einsum(spec, *(gpu_rel(ctx, r) for r in rels), path="tc")
+    assert ctx.last_stats()["path"] == "tc"
+    assert_parity(out, ref, torch.bfloat16)
+    ref2 = oracle_ref(spec, rels, epi="relu", scale=0.5)
+    out2 = ctx.einsum(spec, *(gpu_rel(ctx, r) for r in rels), path="tc", out_dtype="bf16", epi="relu", scale=0.5)
+    assert_parity(out2, ref2, torch.bfloat16, scale=0.5)
