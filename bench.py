@@ -1,19 +1,31 @@
-"""Benchmark: GNN message passing (X x Y)^T x Z as two chained UCL EinSums.
+"""Benchmark: UCL EinSum workloads on one GPU (or N replicas under torchrun).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ucl|reference]
+                    [--workload gnn|blocksparse|mttkrp|spgemm|gnn2]
 
-Workload (seed 0): X 128 x 100000 bf16 N(0,1) as 1563 per-vertex-block tiles
-[f=128 x j=64]; Y an R-MAT graph on 100000 vertices (a,b,c = .57,.19,.19,
-1.6M drawn edges, 1.49M after dedupe) stored as its 358136 nonempty 64 x 64
-0/1 bf16 tiles keyed (J, K); Z 128 x 128 bf16 N(0, 0.1^2), one key-less tuple.
-One step = ucl_einsum("fJj,JjKk->Kkf", X, Y) -> T (bf16) followed by
+Default workload (``gnn``, seed 0): GNN message passing (X x Y)^T x Z.  X
+128 x 100000 bf16 N(0,1) as 1563 per-vertex-block tiles [f=128 x j=64]; Y an
+R-MAT graph on 100000 vertices (a,b,c = .57,.19,.19, 1.6M drawn edges, 1.49M
+after dedupe) stored as its 358136 nonempty 64 x 64 0/1 bf16 tiles keyed
+(J, K); Z 128 x 128 bf16 N(0, 0.1^2), one key-less tuple.  One step =
+ucl_einsum("fJj,JjKk->Kkf", X, Y) -> T (bf16) followed by
 ucl_einsum("Kkf,fg->Kkg", T, Z) -> out (fp32): join, group-by and tile
 contraction all on the GPU.
 
-Metric: effective TFLOP/s over nonzero tiles = sum over the two EinSums of
-2 * (joined pairs) * prod(lower extents), divided by the wall time of the
-step (CUDA events, host sizing syncs included).  Inputs are device resident
-and larger than L2 (Y alone is 2.9 GB), so no L2 flush is needed.
+The other workloads (one step = the EinSum chain listed):
+  blocksparse  IiJj,JjKk->IiKk: A 1024^2 fp32 at 10% of 32x32 tiles, B dense 1024x256
+  mttkrp       IJKijk,Jjr,Kkr->Iir: T 100000^3, 1e7 Zipf(1.1) nonzeros in 16^3 bf16
+               tiles; B, C 100000 x 64 bf16
+  spgemm       IiJj,JjKk->IiKk: A, B 65536^2 at 0.5% of 128x128 bf16 tiles (half banded)
+  gnn2         two-layer GNN: R-MAT 2M vertices / 40M edges as 64x64 tiles, 256-wide
+               bf16 embeddings and weights, T1=(XY)^T, H1=relu(T1 W1), T2=(H1 Y)^T, O=T2 W2
+
+Metric: effective TFLOP/s over nonzero tiles = sum over the step's EinSums of
+2 * (joined tuples) * prod(lower extents), divided by the device time of the
+step (CUDA events; the host sizing syncs inside each EinSum are included).
+Inputs are device resident.  Workloads whose inputs exceed L2 (gnn, mttkrp,
+gnn2) run back to back; the others flush L2 (a 256 MB write) before every
+timed step, outside its events.
 
 Under torchrun (N > 1) every rank runs its own replica of the workload
 (weak scaling, no data-path collective); value = all ranks' FLOPs / the
@@ -38,24 +50,212 @@ sys.path.insert(0, ROOT)
 
 METRIC = "effective TFLOP/s over nonzero tiles per EinSum"
 UNIT = "TFLOP/s"
-WORKLOAD = ("gnn-message-passing (XxY)^T x Z: X 128x100000 bf16, Y R-MAT 100000 vertices / 1.6M edges "
-            "as 358136 nonempty 64x64 bf16 tiles, Z 128x128 bf16; specs fJj,JjKk->Kkf then Kkf,fg->Kkg")
+STAGES = ["keys_join", "pairs_segments", "contract", "fixup"]
 
 
-def workload_name(vertices):
-    if vertices == 100_000:
-        return WORKLOAD
-    return (f"gnn-message-passing (XxY)^T x Z, reduced: X 128x{vertices} bf16, Y R-MAT {vertices} vertices / "
-            f"{16 * vertices} edges as 64x64 bf16 tiles, Z 128x128 bf16")
+# ---------------------------------------------------------------- workloads
 
 
-def contract_traffic(pairs):
-    """DRAM bytes of one contraction launch, scaled by pairs from the ncu capture in
-    profiles/contract_tc_traffic.txt; None once the kernel source changed since."""
+class Workload:
+    """inputs: name -> (keys, bounds, tiles on the device); chain: list of
+    (output name, spec, input names, einsum options); sample(target, seed) ->
+    (spec, host relations, sample keys, joined tuples) for the oracle's timing
+    of the first EinSum on a subset of its output keys."""
+
+    name = ""
+    desc = ""
+    dtype = "bf16"
+    big = True          # inputs larger than L2 (no flush needed)
+    hostable = True     # inputs small enough to stage through pinned host memory every step
+    flops_per_tuple = 0.0
+
+    def __init__(self, dev, args):
+        self.dev = dev
+        self.args = args
+        self.inputs = {}
+        self.chain = []
+
+    def sample(self, target, seed):
+        raise NotImplementedError
+
+
+def _pick_keys(counts, target, seed):
+    """Random output keys (indices into counts) whose tuple counts total
+    about `target`."""
+    nz = np.nonzero(counts)[0]
+    order = np.random.default_rng(seed).permutation(nz)
+    take, tot = [], 0
+    for k in order:
+        take.append(int(k))
+        tot += int(counts[k])
+        if tot >= target:
+            break
+    return np.array(sorted(take), dtype=np.int64), tot
+
+
+def _host64(t):
+    return t.detach().to("cpu", torch.float64).numpy()
+
+
+class GnnChain(Workload):
+    name = "gnn"
+
+    def __init__(self, dev, args):
+        super().__init__(dev, args)
+        import workloads
+        n = args.vertices
+        self.w = w = workloads.gnn_chain(seed=0, n=n, device=dev)
+        self.inputs = {k: (w[k][0], w[k][1], w[k][2].to(dev)) for k in ("X", "Y", "Z")}
+        self.chain = [("T", w["spec1"], ["X", "Y"], {"out_dtype": "bf16"}),
+                      ("O", w["spec2"], ["T", "Z"], {"out_dtype": "f32"})]
+        self.flops_per_tuple = 2.0 * 128 * 64 * 64
+        if n == 100_000:
+            self.desc = ("gnn-message-passing (XxY)^T x Z: X 128x100000 bf16, Y R-MAT 100000 vertices / 1.6M edges "
+                         "as 358136 nonempty 64x64 bf16 tiles, Z 128x128 bf16; specs fJj,JjKk->Kkf then Kkf,fg->Kkg")
+        else:
+            self.desc = (f"gnn-message-passing (XxY)^T x Z, reduced: X 128x{n} bf16, Y R-MAT {n} vertices / "
+                         f"{16 * n} edges as 64x64 bf16 tiles, Z 128x128 bf16")
+        self.l2 = f"inputs larger than L2 (Y {self.inputs['Y'][2].numel() * 2 / 1e9:.1f} GB); no flush"
+
+    def sample(self, target, seed):
+        import workloads
+        w = self.w
+        ky = w["Y"][0]
+        sk, tot = _pick_keys(np.bincount(ky[:, 1]), target, seed)
+        yk = ky[np.isin(ky[:, 1], sk)]
+        if not hasattr(self, "_edges"):
+            self._edges = [e.cpu().numpy() if torch.is_tensor(e) else e for e in w["edges"]]
+        yt = workloads.adjacency_tiles_subset(self._edges[0], self._edges[1], w["n"], w["t"], yk)
+        jn = np.unique(yk[:, 0])
+        xt = w["X"][2]
+        xr = (jn[:, None].astype(np.int32), w["X"][1], _host64(xt[torch.as_tensor(jn, device=xt.device)]))
+        return w["spec1"], [xr, (yk, w["Y"][1], yt)], sk[:, None].astype(np.int32), tot
+
+
+class Gnn2(GnnChain):
+    name = "gnn2"
+    hostable = False
+
+    def __init__(self, dev, args):
+        Workload.__init__(self, dev, args)
+        import workloads
+        self.w = w = workloads.gnn_two_layer(seed=0, device=dev)
+        self.inputs = {k: w[k] for k in ("X", "Y", "W1", "W2")}
+        self.chain = [("T1", w["spec1"], ["X", "Y"], {"out_dtype": "bf16"}),
+                      ("H1", w["spec2"], ["T1", "W1"], {"out_dtype": "bf16", "epi": "relu"}),
+                      ("T2", w["spec3"], ["H1", "Y"], {"out_dtype": "bf16"}),
+                      ("O", w["spec4"], ["T2", "W2"], {"out_dtype": "f32"})]
+        self.flops_per_tuple = 2.0 * 256 * 64 * 64
+        ny = len(w["Y"][0])
+        self.desc = (f"two-layer GNN at scale: R-MAT 2M vertices / 40M drawn edges as {ny} nonempty 64x64 bf16 "
+                     f"tiles, X 256x2M bf16, W1, W2 256x256 bf16; T1=(XY)^T, H1=relu(T1 W1), T2=(H1 Y)^T, O=T2 W2")
+        self.l2 = f"inputs larger than L2 (Y {ny * 8192 / 1e9:.0f} GB); no flush"
+
+
+class Mttkrp(Workload):
+    name = "mttkrp"
+    hostable = False
+
+    def __init__(self, dev, args):
+        super().__init__(dev, args)
+        import workloads
+        self.w = w = workloads.mttkrp(seed=0, device=dev)
+        self.inputs = {k: w[k] for k in ("T", "B", "C")}
+        self.chain = [("M", w["spec"], ["T", "B", "C"], {"out_dtype": "f32"})]
+        self.flops_per_tuple = 2.0 * 16 * 16 * 16 * 64
+        nt = len(w["T"][0])
+        self.desc = (f"MTTKRP M[i,r]=sum T[i,j,k] B[j,r] C[k,r]: T 100000^3 with 1e7 Zipf(1.1) nonzeros in {nt} "
+                     f"nonempty 16^3 bf16 tiles, B, C 100000x64 bf16; spec IJKijk,Jjr,Kkr->Iir")
+        self.l2 = f"inputs larger than L2 (T {nt * 8192 / 1e9:.1f} GB); no flush"
+
+    def sample(self, target, seed):
+        w = self.w
+        kt = w["T"][0]
+        sk, tot = _pick_keys(np.bincount(kt[:, 0]), target, seed)
+        m = np.nonzero(np.isin(kt[:, 0], sk))[0]
+        dev = w["T"][2].device
+        tr = (kt[m], w["T"][1], _host64(w["T"][2][torch.as_tensor(m, device=dev)]))
+
+        def rows(f, r):
+            r = np.unique(r)
+            return (r[:, None].astype(np.int32), f[1], _host64(f[2][torch.as_tensor(r, device=dev)]))
+
+        return w["spec"], [tr, rows(w["B"], kt[m, 1]), rows(w["C"], kt[m, 2])], sk[:, None].astype(np.int32), tot
+
+
+class _Binary(Workload):
+    """Block-sparse matmul-shaped workloads (IiJj,JjKk->IiKk), inputs fit L2."""
+    big = False
+
+    def _setup(self, w, tile):
+        self.w = w
+        self.inputs = {k: (w[k][0], w[k][1], w[k][2].to(self.dev)) for k in ("A", "B")}
+        self.chain = [("C", w["spec"], ["A", "B"], {"out_dtype": "f32"})]
+        self.flops_per_tuple = 2.0 * tile ** 3
+        # tuples per output key (I, K): join of A and B on J
+        ka, kb = w["A"][0], w["B"][0]
+        g = int(max(w["A"][1][0], w["B"][1][1]))
+        byj = {}
+        for j, k in kb:
+            byj.setdefault(int(j), []).append(int(k))
+        cnt = {}
+        for i, j in ka:
+            for k in byj.get(int(j), ()):
+                cnt[int(i) * g + k] = cnt.get(int(i) * g + k, 0) + 1
+        self._codes = np.array(sorted(cnt), dtype=np.int64)
+        self._counts = np.array([cnt[c] for c in self._codes], dtype=np.int64)
+        self._g = g
+        self._host = None
+
+    def sample(self, target, seed):
+        pick, tot = _pick_keys(self._counts, target, seed)
+        codes = self._codes[pick]
+        sk = np.stack([codes // self._g, codes % self._g], 1).astype(np.int32)
+        if self._host is None:
+            self._host = [(self.w[k][0], self.w[k][1], _host64(self.w[k][2])) for k in ("A", "B")]
+        return self.w["spec"], self._host, sk, tot
+
+
+class Blocksparse(_Binary):
+    name = "blocksparse"
+    dtype = "f32"
+
+    def __init__(self, dev, args):
+        super().__init__(dev, args)
+        import workloads
+        self._setup(workloads.blocksparse_matmul(seed=0), 32)
+        self.desc = ("block-sparse matmul C[I,K]=sum A[I,J] B[J,K]: A 1024x1024 fp32 at 10% of 32x32 tiles "
+                     "(102 tiles), B dense 1024x256 fp32; spec IiJj,JjKk->IiKk")
+        self.l2 = "inputs smaller than L2: 256 MB L2 flush before every timed step (outside the events)"
+
+
+class Spgemm(_Binary):
+    name = "spgemm"
+
+    def __init__(self, dev, args):
+        super().__init__(dev, args)
+        import workloads
+        self._setup(workloads.spgemm(seed=0), 128)
+        n = len(self.w["A"][0])
+        self.desc = (f"block-sparse x block-sparse SpGEMM: A, B 65536x65536 at 0.5% of 128x128 bf16 tiles ({n} "
+                     f"tiles each, half on a 4-tile band); spec IiJj,JjKk->IiKk")
+        self.l2 = "inputs smaller than L2: 256 MB L2 flush before every timed step (outside the events)"
+
+
+WORKLOADS = {"gnn": GnnChain, "blocksparse": Blocksparse, "mttkrp": Mttkrp, "spgemm": Spgemm, "gnn2": Gnn2}
+
+
+# ---------------------------------------------------------------- helpers
+
+
+def contract_traffic(kernel_file, workload, units):
+    """DRAM bytes of one contraction launch, scaled by `units` (joined tuples)
+    from an ncu capture summarised in profiles/<kernel>_traffic.txt; None if
+    there is no capture for this workload or the kernel source changed since."""
     import hashlib
-    p = os.path.join(ROOT, "profiles", "contract_tc_traffic.txt")
-    src = os.path.join(ROOT, "paper_2603_08957_gb300", "csrc", "contract_tc.cu")
-    if not os.path.exists(p):
+    p = os.path.join(ROOT, "profiles", f"{kernel_file}_traffic.txt")
+    src = os.path.join(ROOT, "paper_2603_08957_gb300", "csrc", f"{kernel_file}.cu")
+    if not os.path.exists(p) or not os.path.exists(src):
         return None
     kv = {}
     for line in open(p):
@@ -65,8 +265,10 @@ def contract_traffic(pairs):
             kv[k.strip()] = v.strip()
     if hashlib.sha256(open(src, "rb").read()).hexdigest() != kv.get("source_sha256"):
         return None
-    per_pair = (int(kv["dram_read_bytes"]) + int(kv["dram_write_bytes"])) / int(kv["pairs"])
-    return per_pair * pairs
+    if kv.get("workload", "gnn") != workload:
+        return None
+    per = (int(kv["dram_read_bytes"]) + int(kv["dram_write_bytes"])) / int(kv["pairs"])
+    return per * units
 
 
 def peaks():
@@ -147,77 +349,55 @@ def allreduce_max(x, world, device):
 # ----------------------------------------------------------- CPU oracle leg
 
 
-def oracle_sample(w, target_pairs, seed=0):
-    """Output keys K whose pairs total about target_pairs, with the oracle's
-    inputs for them (X whole, only the Y tiles of those K)."""
-    import workloads
-    ky = w["Y"][0]
-    cnt = np.bincount(ky[:, 1])
-    ks = np.nonzero(cnt)[0]
-    rng = np.random.default_rng(seed)
-    order = rng.permutation(ks)
-    take, tot = [], 0
-    for k in order:
-        take.append(k)
-        tot += cnt[k]
-        if tot >= target_pairs:
-            break
-    sk = np.array(sorted(take), dtype=np.int32)[:, None]
-    ysel = np.isin(ky[:, 1], sk[:, 0])
-    yk = ky[ysel]
-    yt = workloads.adjacency_tiles_subset(w["edges"][0], w["edges"][1], w["n"], w["t"], yk)
-    xk, xb, xt = w["X"]
-    return sk, (xk, xb, xt.to("cpu", torch.float64).numpy()), (yk, w["Y"][1], yt), int(tot)
-
-
-def time_oracle(w, target_pairs, seed):
+def time_oracle(W, target, seed):
+    """The oracle on the first EinSum restricted to random output keys holding
+    about `target` joined tuples: (FLOPs, seconds, tuples, keys)."""
     import oracle
-    sk, xr, yr, pairs = oracle_sample(w, target_pairs, seed)
+    spec, rels, sk, tuples = W.sample(target, seed)
     t0 = time.perf_counter()
-    r = oracle.einsum("fJj,JjKk->Kkf", [xr, yr], sample_keys=sk)
+    r = oracle.einsum(spec, rels, sample_keys=sk)
     dt = time.perf_counter() - t0
-    assert r["n_pairs"] >= pairs
-    flops = 2.0 * pairs * 128 * 64 * 64
-    return flops, dt, pairs, len(sk)
+    assert r["keys"].shape[0] == len(sk)
+    return W.flops_per_tuple * tuples, dt, tuples, len(sk)
 
 
-def calibrate_oracle(w):
-    flops, dt, pairs, _ = time_oracle(w, 64, seed=12345)
-    return pairs / dt  # pairs per second
+def oracle_rate(W):
+    _, dt, tuples, _ = time_oracle(W, 32, seed=12345)
+    return tuples / max(dt, 1e-6)
 
 
-def cpu_baseline(w, seconds=12.0):
-    rate = calibrate_oracle(w)
-    target = max(64, int(rate * seconds))
-    flops, dt, pairs, nk = time_oracle(w, target, seed=1)
+def cpu_baseline(W, seconds=12.0):
+    target = max(16, int(oracle_rate(W) * seconds))
+    flops, dt, tuples, nk = time_oracle(W, target, seed=1)
+    spec = W.chain[0][1]
     return {"value": flops / dt / 1e12, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"first EinSum fJj,JjKk->Kkf restricted to {nk} random output keys K ({pairs} joined pairs, "
-                      f"{dt:.1f} s single-threaded fp64 C); FLOPs of those pairs / time"}
+            "sample": f"first EinSum {spec} restricted to {nk} random output keys ({tuples} joined tuples, "
+                      f"{dt:.1f} s single-threaded fp64 C); FLOPs of those tuples / time"}
 
 
 def run_reference(args, world, rank):
     """The oracle as the reference arm: each step a bounded sample of the workload."""
     if rank != 0:
         return
-    import workloads
-    w = workloads.gnn_chain(seed=0, device="cpu")
-    rate = calibrate_oracle(w)
-    per_step = max(16, int(rate * args.ref_step_seconds))
+    dev = "cuda" if args.workload in ("mttkrp", "gnn2") and torch.cuda.is_available() else "cpu"
+    W = WORKLOADS[args.workload](dev, args)
+    per_step = max(16, int(oracle_rate(W) * args.ref_step_seconds))
     for i in range(args.warmup):
-        time_oracle(w, max(16, per_step // 4), seed=100 + i)
+        time_oracle(W, max(8, per_step // 4), seed=100 + i)
     tot_f, tot_t, tot_p = 0.0, 0.0, 0
     for i in range(args.steps):
-        f, dt, p, _ = time_oracle(w, per_step, seed=1000 + i)
+        f, dt, p, _ = time_oracle(W, per_step, seed=1000 + i)
         tot_f += f
         tot_t += dt
         tot_p += p
     v = tot_f / tot_t / 1e12
-    sample = (f"each step: first EinSum fJj,JjKk->Kkf on random output keys K totalling ~{per_step} joined pairs "
-              f"({tot_p} pairs over {args.steps} steps), single-threaded fp64 C oracle")
+    spec = W.chain[0][1]
+    sample = (f"each step: first EinSum {spec} on random output keys totalling ~{per_step} joined tuples "
+              f"({tot_p} over {args.steps} steps), single-threaded fp64 C oracle")
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": 1, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1e3 * tot_t / max(1, args.steps), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "l2": "n/a (CPU)"},
+            "config": {"workload": W.desc, "l2": "n/a (CPU)"},
             "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -226,48 +406,80 @@ def run_reference(args, world, rank):
 # ---------------------------------------------------------------- GPU leg
 
 
+def stage_roofline(W, arity, stats, tim, pk):
+    """Per EinSum of the chain: mean stage times and the achieved fraction of
+    the HBM roofline for the key/join stages (algorithmic bytes: read every
+    input key once, write and read back the 16-byte pair records once, write
+    the index arrays and output keys) and for the contraction (its
+    algorithmic bytes: every input tile once, the output once, the indices),
+    with the tensor-pipe fraction of the contraction's FLOPs."""
+    out = []
+    L = len(W.chain)
+    for c, (name, spec, ins, _) in enumerate(W.chain):
+        s = stats[c]
+        P, S = s["n_pairs"], s["n_segments"]
+        key_bytes = sum(arity[i][0] * arity[i][1] * 4 for i in ins)
+        uw = sum(ch.isupper() for ch in spec.split("->")[1])
+        sort_bytes = key_bytes + 32.0 * P + 4.0 * len(ins) * P + 4.0 * uw * S
+        ms = tim[c::L].mean(axis=0) if len(tim) else np.full(4, np.nan)
+        sj = float(ms[0] + ms[1])
+        ct = float(ms[2])
+        gbs_sj = sort_bytes / (sj / 1e3) / 1e9
+        gbs_c = s["bytes_contract"] / (ct / 1e3) / 1e9
+        tf_c = s["flops"] / (ct / 1e3) / 1e12
+        out.append({"spec": spec, "path": s["path"], "tuples": P, "segments": S,
+                    "sort_join": {"ms": sj, "alg_bytes": sort_bytes, "GB/s": gbs_sj, "frac": gbs_sj / pk["hbm_gbs"]},
+                    "contract": {"ms": ct, "alg_bytes": s["bytes_contract"], "GB/s": gbs_c,
+                                 "frac": gbs_c / pk["hbm_gbs"], "TFLOP/s": tf_c,
+                                 "tensor_frac": tf_c / pk["bf16_tflops"]},
+                    "fixup": {"ms": float(ms[3])}})
+    return out
+
+
 def run_ucl(args, world, rank, local):
-    import workloads
     from paper_2603_08957_gb300 import Context
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    w = workloads.gnn_chain(seed=0, n=args.vertices, device=dev)
+    W = WORKLOADS[args.workload](dev, args)
     ctx = Context(local, torch_allocator=(args.alloc == "torch"))
-
-    def rel(r):
-        return ctx.relation(torch.as_tensor(r[0]).to(dev), r[1], r[2].to(dev))
-
-    X, Y, Z = rel(w["X"]), rel(w["Y"]), rel(w["Z"])
+    rels = {k: ctx.relation(torch.as_tensor(r[0]).to(dev), r[1], r[2].to(dev)) for k, r in W.inputs.items()}
     path = args.path
+    flush = None if W.big else torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+
+    def run_chain(env, collect=None):
+        made = []
+        for name, spec, ins, opts in W.chain:
+            r = ctx.einsum(spec, *[env[i] for i in ins], path=path, **opts)
+            if collect is not None:
+                collect.append(ctx.last_stats())
+                arity[name] = (r.n, r.u)
+            env[name] = r
+            made.append(r)
+        return made
 
     def step():
-        T = ctx.einsum(w["spec1"], X, Y, out_dtype="bf16", path=path)
-        O = ctx.einsum(w["spec2"], T, Z, out_dtype="f32", path=path)
-        T.destroy()
-        return O
+        for r in run_chain(dict(rels)):
+            r.destroy()
 
-    # warm-up and per-step counters (deterministic)
-    T = ctx.einsum(w["spec1"], X, Y, out_dtype="bf16", path=path)
-    s1 = ctx.last_stats()
-    O = ctx.einsum(w["spec2"], T, Z, out_dtype="f32", path=path)
-    s2 = ctx.last_stats()
-    T.destroy()
-    O.destroy()
+    stats = []
+    arity = {k: (r.n, r.u) for k, r in rels.items()}
+    for r in run_chain(dict(rels), stats):
+        r.destroy()
     for _ in range(max(0, args.warmup - 1)):
-        step().destroy()
+        step()
     torch.cuda.synchronize()
-    flops_step = s1["flops"] + s2["flops"]
-    launches_step = s1["launches"] + s2["launches"]
+    flops_step = sum(s["flops"] for s in stats)
+    launches_step = sum(s["launches"] for s in stats)
 
     steps = args.steps
     if steps is None:
         t0 = time.perf_counter()
         for _ in range(3):
-            step().destroy()
+            step()
         torch.cuda.synchronize()
         per = (time.perf_counter() - t0) / 3
-        steps = int(min(2000, max(10, 3.0 / max(per, 1e-6))))
+        steps = int(min(2000, max(10, args.seconds / max(per, 1e-6))))
 
     clocks = Clocks(local)
     ctx.set_timing(True)
@@ -276,49 +488,57 @@ def run_ucl(args, world, rank, local):
     torch.cuda.synchronize()
     clocks.start()
     time.sleep(0.3)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for _ in range(steps):
-        step().destroy()
-    e1.record()
-    torch.cuda.synchronize()
+    if W.big:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(steps):
+            step()
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+    else:
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        for a, b in evs:
+            flush.fill_(1)
+            a.record()
+            step()
+            b.record()
+        torch.cuda.synchronize()
+        ms = sum(a.elapsed_time(b) for a, b in evs)
     barrier(world)
     ck = clocks.stop()
-    ms = e0.elapsed_time(e1)
     tim = ctx.timings(reset=True)
     ctx.set_timing(False)
     ms_max = allreduce_max(ms, world, dev)
     value = flops_step * steps * world / (ms_max / 1e3) / 1e12
 
-    # dominant kernel: the contraction of the first EinSum (stage 2 of every other call)
-    contract_ms = tim[0::2, 2]
-    avg_contract = float(contract_ms.mean()) if len(contract_ms) else float("nan")
     pk = peaks()
-    achieved = s1["bytes_contract"] / (avg_contract / 1e3) / 1e9
-    roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
-            "frac": achieved / pk["hbm_gbs"], "traffic": contract_traffic(s1["n_pairs"]),
-            "kernel": f"contract_{s1['path']} (fJj,JjKk->Kkf)", "avg_launch_ms": avg_contract,
-            "alg_bytes_per_launch": s1["bytes_contract"], "peak_src": pk["src"],
-            "tensor_frac": (s1["flops"] / (avg_contract / 1e3) / 1e12) / pk["bf16_tflops"]}
-    stages = {name: float(tim[0::2, i].mean()) for i, name in enumerate(["keys_join", "pairs_segments",
-                                                                           "contract", "fixup"])}
+    per_einsum = stage_roofline(W, arity, stats, tim, pk)
+    # dominant kernel: the contraction with the largest total time
+    dom = max(range(len(per_einsum)), key=lambda c: per_einsum[c]["contract"]["ms"])
+    d, s = per_einsum[dom], stats[dom]
+    kfile = {"tc": "contract_tc3" if len(W.chain[dom][2]) == 3 else "contract_tc",
+             "simt": "contract_simt"}.get(s["path"], "contract_simt")
+    roof = {"bound": "hbm", "achieved": d["contract"]["GB/s"], "peak": pk["hbm_gbs"], "unit": "GB/s",
+            "frac": d["contract"]["frac"], "traffic": contract_traffic(kfile, W.name, s["n_pairs"]),
+            "kernel": f"{kfile} ({d['spec']})", "avg_launch_ms": d["contract"]["ms"],
+            "alg_bytes_per_launch": s["bytes_contract"], "peak_src": pk["src"],
+            "tensor_frac": d["contract"]["tensor_frac"]}
+    stages = {name: float(tim[:, i].reshape(-1, len(W.chain)).sum(axis=1).mean()) if len(tim) else None
+              for i, name in enumerate(STAGES)}
 
     # end to end through the C ABI with host buffers
     e2e = None
-    if not args.no_e2e:
-        hx = [torch.as_tensor(w["X"][0]).pin_memory(), w["X"][2].cpu().pin_memory()]
-        hy = [torch.as_tensor(w["Y"][0]).pin_memory(), w["Y"][2].cpu().pin_memory()]
-        hz = [torch.as_tensor(w["Z"][0]).pin_memory(), w["Z"][2].cpu().pin_memory()]
-        h2d = sum(t.numel() * t.element_size() for t in hx + hy + hz)
+    if not args.no_e2e and W.hostable:
+        host = {k: (torch.as_tensor(r[0]).pin_memory(), r[1], r[2].cpu().pin_memory()) for k, r in W.inputs.items()}
+        h2d = sum(t[0].numel() * 4 + t[2].numel() * t[2].element_size() for t in host.values())
+        last = W.chain[-1][0]
 
         def e2e_step():
-            Xh = ctx.relation(hx[0], w["X"][1], hx[1])
-            Yh = ctx.relation(hy[0], w["Y"][1], hy[1])
-            Zh = ctx.relation(hz[0], w["Z"][1], hz[1])
-            T = ctx.einsum(w["spec1"], Xh, Yh, out_dtype="bf16", path=path)
-            O = ctx.einsum(w["spec2"], T, Zh, out_dtype="f32", path=path)
-            k, t = O.download()
-            for r in (Xh, Yh, Zh, T, O):
+            env = {k: ctx.relation(h[0], h[1], h[2]) for k, h in host.items()}
+            made = run_chain(env)
+            k, t = env[last].download()
+            for r in list(env.values()):
                 r.destroy()
             return k.nbytes + t.numel() * t.element_size()
 
@@ -334,23 +554,27 @@ def run_ucl(args, world, rank, local):
         te = allreduce_max(te, world, dev)
         e2e = {"value": flops_step * world / te / 1e12, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(d2h), "ms_per_step": te * 1e3}
+        del host
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(w, seconds=args.cpu_seconds)
+        cpu = cpu_baseline(W, seconds=args.cpu_seconds)
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps,
                 "warmup": args.warmup, "ms_per_step": ms_max / steps, "higher_is_better": True, "scaling": "weak",
-                "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-                "config": {"workload": workload_name(args.vertices), "pairs": [s1["n_pairs"], s2["n_pairs"]],
-                           "segments": [s1["n_segments"], s2["n_segments"]], "flops_per_step": flops_step,
-                           "l2": "inputs larger than L2 (Y 2.9 GB); no flush", "path": s1["path"],
+                "vs_baseline": None, "dtype": W.dtype, "data": "synthetic",
+                "config": {"workload": W.desc, "pairs": [s["n_pairs"] for s in stats],
+                           "segments": [s["n_segments"] for s in stats], "flops_per_step": flops_step,
+                           "l2": W.l2, "path": [s["path"] for s in stats],
                            "parallelism": f"replicas x{world}", "alloc": args.alloc},
-                "roofline": roof, "stage_ms": stages, "cpu_baseline": cpu, "e2e": e2e,
+                "roofline": roof, "stage_ms": stages, "stage_roofline": per_einsum, "cpu_baseline": cpu,
+                "e2e": e2e if e2e is not None else (None if W.hostable else
+                                                    {"value": None, "unit": UNIT,
+                                                     "skipped": "inputs too large to stage through host memory"}),
                 "gpu_launches": int(launches_step * steps), "clocks": ck}
         print(json.dumps(line), flush=True)
-    for r in (X, Y, Z):
+    for r in rels.values():
         r.destroy()
     ctx.close()
 
@@ -361,13 +585,15 @@ def main():
     ap.add_argument("--steps", type=int, default=None)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ucl", "reference"], default="ucl")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="gnn")
     ap.add_argument("--path", choices=["auto", "simt", "tc"], default="auto")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--alloc", choices=["torch", "cuda"], default="torch",
                     help="device memory for workspace and outputs: PyTorch's caching allocator (through the "
                          "allocator hooks) or the library's cudaMallocAsync pool")
-    ap.add_argument("--vertices", type=int, default=100_000, help="graph size (reduced sizes for profiling)")
+    ap.add_argument("--vertices", type=int, default=100_000, help="gnn graph size (reduced sizes for profiling)")
+    ap.add_argument("--seconds", type=float, default=3.0, help="timed seconds when --steps is not given")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-step-seconds", type=float, default=3.0)
     args = ap.parse_args()
