@@ -20,7 +20,10 @@
 //               unit, store an fp32 partial for the fixup kernel.
 //
 // Accumulators are multi-buffered in TMEM so the epilogue of one segment
-// overlaps the MMAs of the next.  A pipeline stage holds the tiles of `pps`
+// overlaps the MMAs of the next.  Tiles too large for a deep enough ring of
+// whole pairs are streamed in K chunks: a stage then holds one chunk of one
+// pair, and the pipeline runs over (pair, chunk) positions, kc per pair; all
+// chunks of a segment's pairs accumulate into its buffer.  A pipeline stage holds the tiles of `pps`
 // consecutive pairs, so that barrier traffic is paid once per stage.  The
 // producer and MMA warps run warp-uniform loops and issue through one elected
 // lane; descriptors are precomputed so that one MMA costs a few integer adds.
@@ -60,12 +63,14 @@ struct TcArgs {
     int64_t tile_w;
     int64_t sWm, sWn;
     int N, K, m_blocks;
+    int kc_lg;                   // log2 of the K chunks per pair
     int wa, wb;                  // sub-tile width (elements) of the A / B boxes
-    int na_sub, nb_sub;          // boxes per tile
+    int na_sub, nb_sub;          // boxes per chunk
+    int a_cx, a_cy, b_cx, b_cy;  // box coordinate step per K chunk (x: columns, y: rows)
     uint32_t a_sub, b_sub;       // bytes per sub-tile (multiple of 1024)
     uint32_t a_pair, b_pair;     // bytes of one pair's A / B tile in a stage
     uint32_t stage_bytes;        // pps * (a_pair + b_pair)
-    uint32_t pair_tx;            // bytes TMA delivers per pair
+    uint32_t pair_tx;            // bytes TMA delivers per pair chunk
     int pps;                     // pairs per stage
     int ns, nacc, nmma;
     uint32_t tmem_cols;
@@ -290,14 +295,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         // ...: lane j loads the tile indices of the stage's pair j (prefetched
         // one own stage ahead), lane 0 waits for the slot and posts the
         // expected bytes, then lane j issues the TMA copies of pair j.
-        const int n = (int)(pe - pb), pps = a.pps;
+        const int n = (int)(pe - pb) << a.kc_lg, pps = a.pps;
         const int nfills = (n + pps - 1) / pps;
+        const int kmask = (1 << a.kc_lg) - 1;
         uint32_t mine = 0;
         auto load_idx = [&](int f, uint32_t &ia, uint32_t &ib) {
             ia = 0;
             ib = 0;
-            const int64_t p = pb + (int64_t)f * pps + lane;
-            if (f < nfills && lane < pps && p < pe) {
+            const int v = f * pps + lane;
+            const int64_t p = pb + (v >> a.kc_lg);
+            if (f < nfills && lane < pps && v < n) {
                 ia = a.pa[p];
                 ib = a.pb[p];
                 if ((int64_t)ia >= a.nA || (int64_t)ib >= a.nB) {
@@ -324,8 +331,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 const uint32_t fb = full0 + 8u * st;
                 const uint32_t sa = sbase + st * a.stage_bytes + (uint32_t)lane * a.a_pair;
                 const uint32_t sb = sbase + st * a.stage_bytes + (uint32_t)a.pps * a.a_pair + (uint32_t)lane * a.b_pair;
-                for (int q = 0; q < a.na_sub; ++q) tma_load_3d(sa + q * a.a_sub, &tmA, q * a.wa, 0, (int)ia, fb);
-                for (int q = 0; q < a.nb_sub; ++q) tma_load_3d(sb + q * a.b_sub, &tmB, q * a.wb, 0, (int)ib, fb);
+                const int c = (f * pps + lane) & kmask;   // K chunk
+                for (int q = 0; q < a.na_sub; ++q)
+                    tma_load_3d(sa + q * a.a_sub, &tmA, q * a.wa + c * a.a_cx, c * a.a_cy, (int)ia, fb);
+                for (int q = 0; q < a.nb_sub; ++q)
+                    tma_load_3d(sb + q * a.b_sub, &tmB, q * a.wb + c * a.b_cx, c * a.b_cy, (int)ib, fb);
             }
             __syncwarp();
             ++mine;
@@ -359,10 +369,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const uint32_t stage16 = a.stage_bytes >> 4, apair16 = a.a_pair >> 4, bpair16 = a.b_pair >> 4;
             const uint32_t mb16 = (uint32_t)a.a_mb16, ncol = (uint32_t)a.N, idesc = a.idesc;
             const bool two_m = a.m_blocks > 1;
-            const int n = (int)(pe - pb), pps = a.pps;
+            // positions count (pair, K chunk) steps, kc per pair
+            const int n = (int)(pe - pb) << a.kc_lg, pps = a.pps;
             uint32_t b = 0, aph = 0, dcol = tmem;
             int64_t s = s_first;
-            int seg_end = n > 0 ? (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) : 0;
+            int seg_end = n > 0 ? (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) << a.kc_lg : 0;
             bool fresh = true, ok = true;
             // Segment events: before the warp's first MMA into a segment it waits
             // for the accumulator buffer (open); at the segment's end it commits
@@ -384,7 +395,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     aph ^= 1u;
                 }
                 ++s;
-                if (pos < n) seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
+                if (pos < n) seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) << a.kc_lg;
                 fresh = true;
             };
             uint32_t st = (uint32_t)(w % a.ns), ph = (uint32_t)((w / a.ns) & 1);
@@ -508,7 +519,33 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         for (int jj = 0; jj < 16; ++jj) v[jj] += v2[jj];
                     }
                     const int64_t base_off = m * a.sWm + (int64_t)c * 16 * a.sWn;
-                    if (kind == 0) {
+                    if (a.sWn == 1) {
+                        // N contiguous in the output: this lane's 16 values are
+                        // one 64-byte (fp32) or 32-byte (bf16) run
+                        if (kind == 0) {
+#pragma unroll
+                            for (int jj = 0; jj < 16; ++jj) v[jj] = epilogue(v[jj], a.epi, a.scale);
+                        }
+                        if (kind == 0 && a.dout == UCL_BF16) {
+                            uint32_t h[8];
+#pragma unroll
+                            for (int jj = 0; jj < 8; ++jj) {
+                                __nv_bfloat162 t = __floats2bfloat162_rn(v[2 * jj], v[2 * jj + 1]);
+                                h[jj] = *reinterpret_cast<uint32_t *>(&t);
+                            }
+                            uint4 *o = reinterpret_cast<uint4 *>(reinterpret_cast<__nv_bfloat16 *>(a.out) +
+                                                                 s * a.tile_w + base_off);
+                            o[0] = make_uint4(h[0], h[1], h[2], h[3]);
+                            o[1] = make_uint4(h[4], h[5], h[6], h[7]);
+                        } else {
+                            float *dst = kind == 0 ? reinterpret_cast<float *>(a.out) + s * a.tile_w + base_off
+                                                   : part + base_off;
+                            float4 *o = reinterpret_cast<float4 *>(dst);
+#pragma unroll
+                            for (int jj = 0; jj < 4; ++jj)
+                                o[jj] = make_float4(v[4 * jj], v[4 * jj + 1], v[4 * jj + 2], v[4 * jj + 3]);
+                        }
+                    } else if (kind == 0) {
                         if (a.dout == UCL_BF16) {
                             __nv_bfloat16 *o = reinterpret_cast<__nv_bfloat16 *>(a.out) + s * a.tile_w + base_off;
 #pragma unroll
@@ -580,14 +617,24 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-// Operand geometry: the tile is [rows][cols] row-major; it is fetched as
-// cols / w boxes of {w, rows}, each landing in its own swizzled sub-tile.
+// Operand geometry: the tile is [trows][tcols] row-major.  One stage holds a
+// K chunk of it, [rows][cols] (all rows and a column range for K-major tiles,
+// a row range for MN-major ones), fetched as cols / w boxes of {w, rows},
+// each landing in its own swizzled sub-tile.
 struct Operand {
-    int rows, cols, w, nsub;
+    int trows, tcols, rows, cols, w, nsub;
+    int cx, cy;   // box coordinate step per chunk
     uint32_t sub_bytes;
 };
 
-bool operand_geometry(int rows, int cols, Operand *op, std::string *why) {
+bool operand_geometry(int trows, int tcols, bool kmajor, int kc, Operand *op, std::string *why) {
+    op->trows = trows;
+    op->tcols = tcols;
+    op->rows = kmajor ? trows : trows / kc;
+    op->cols = kmajor ? tcols / kc : tcols;
+    op->cx = kmajor ? op->cols : 0;
+    op->cy = kmajor ? 0 : op->rows;
+    const int rows = op->rows, cols = op->cols;
     if (rows < 16 || rows > 256 || rows % 16) {
         *why = "tile rows must be a multiple of 16 up to 256";
         return false;
@@ -596,8 +643,6 @@ bool operand_geometry(int rows, int cols, Operand *op, std::string *why) {
         *why = "tile row length must be 16, 32 or a multiple of 64 elements";
         return false;
     }
-    op->rows = rows;
-    op->cols = cols;
     op->w = cols < 64 ? cols : 64;
     op->nsub = cols / op->w;
     uint32_t b = (uint32_t)rows * op->w * 2;
@@ -608,31 +653,49 @@ bool operand_geometry(int rows, int cols, Operand *op, std::string *why) {
 struct TcGeometry {
     Operand A, B;
     uint32_t a_pair, b_pair, stage_bytes, pair_tx, smem_bytes, tmem_cols;
-    int pps, ns, nacc, nmma;
+    int pps, ns, nacc, nmma, kc;
 };
 
-// Pairs per stage: as many as keep a stage within 64 KB while leaving at
-// least three stages in flight.
+// Ring of stages: whole pairs (kc = 1) when at least four stages of one pair
+// fit, else the fewest K chunks per pair that leave four.  With whole pairs, a
+// stage holds pps pairs (1..4): the largest pps that keeps a stage within
+// 72 KB and leaves an even number (>= 4) of stages.
 bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_override = 0) {
-    // A: K-major tiles are [M][K], MN-major [K][M]; same for B with N
-    if (!operand_geometry(tp.a_kmajor ? tp.M : tp.K, tp.a_kmajor ? tp.K : tp.M, &g->A, why)) return false;
-    if (!operand_geometry(tp.b_kmajor ? tp.N : tp.K, tp.b_kmajor ? tp.K : tp.N, &g->B, why)) return false;
-    g->a_pair = g->A.sub_bytes * g->A.nsub;
-    g->b_pair = g->B.sub_bytes * g->B.nsub;
-    g->pair_tx = (uint32_t)(tp.M * tp.K * 2 + tp.N * tp.K * 2);
     const uint32_t bar_bytes = 8u * (2 * kMaxStages + 2 * kMaxAcc + 1) + 64 + 64;
-    const uint32_t avail = kSmemLimit - 1024 - bar_bytes, per_pair = g->a_pair + g->b_pair;
-    // Pairs per stage (1..4): the largest that keeps a stage within 72 KB and
-    // leaves an even number (>= 4) of stages.
-    int pps = 1;
-    for (int c = 4; c >= 2; --c) {
-        const uint32_t k = avail / (c * per_pair);
-        if (c * per_pair <= 72u * 1024u && (k < (uint32_t)kMaxStages ? k : (uint32_t)kMaxStages) / 2 * 2 >= 4) {
-            pps = c;
+    const uint32_t avail = kSmemLimit - 1024 - bar_bytes;
+    bool found = false;
+    for (int kc = 1; kc <= 16 && tp.K / kc >= 16 && tp.K % kc == 0; kc *= 2) {
+        // A: K-major tiles are [M][K], MN-major [K][M]; same for B with N
+        if (!operand_geometry(tp.a_kmajor ? tp.M : tp.K, tp.a_kmajor ? tp.K : tp.M, tp.a_kmajor, kc, &g->A, why))
+            continue;
+        if (!operand_geometry(tp.b_kmajor ? tp.N : tp.K, tp.b_kmajor ? tp.K : tp.N, tp.b_kmajor, kc, &g->B, why))
+            continue;
+        g->a_pair = g->A.sub_bytes * g->A.nsub;
+        g->b_pair = g->B.sub_bytes * g->B.nsub;
+        if (avail / (g->a_pair + g->b_pair) >= 4) {
+            g->kc = kc;
+            found = true;
             break;
         }
     }
-    if (pps_override > 0) pps = pps_override;
+    if (!found) {
+        if (why->empty()) *why = "tiles too large for four shared-memory stages";
+        return false;
+    }
+    const int Kc = tp.K / g->kc;
+    g->pair_tx = (uint32_t)(tp.M * Kc * 2 + tp.N * Kc * 2);
+    const uint32_t per_pair = g->a_pair + g->b_pair;
+    int pps = 1;
+    if (g->kc == 1) {
+        for (int c = 4; c >= 2; --c) {
+            const uint32_t k = avail / (c * per_pair);
+            if (c * per_pair <= 72u * 1024u && (k < (uint32_t)kMaxStages ? k : (uint32_t)kMaxStages) / 2 * 2 >= 4) {
+                pps = c;
+                break;
+            }
+        }
+        if (pps_override > 0) pps = pps_override;
+    }
     g->pps = pps;
     g->stage_bytes = pps * per_pair;
     int ns = (int)(avail / g->stage_bytes);
@@ -706,8 +769,8 @@ bool make_map(CUtensorMap *m, const ucl_rel *R, const Operand &op, std::string *
         *why = "cuTensorMapEncodeTiled unavailable";
         return false;
     }
-    cuuint64_t dims[3] = {(cuuint64_t)op.cols, (cuuint64_t)op.rows, (cuuint64_t)R->n};
-    cuuint64_t strides[2] = {(cuuint64_t)op.cols * 2, (cuuint64_t)op.rows * op.cols * 2};
+    cuuint64_t dims[3] = {(cuuint64_t)op.tcols, (cuuint64_t)op.trows, (cuuint64_t)R->n};
+    cuuint64_t strides[2] = {(cuuint64_t)op.tcols * 2, (cuuint64_t)op.trows * op.tcols * 2};
     cuuint32_t box[3] = {(cuuint32_t)op.w, (cuuint32_t)op.rows, 1};
     cuuint32_t estr[3] = {1, 1, 1};
     CUtensorMapSwizzle swz = op.w == 64 ? CU_TENSOR_MAP_SWIZZLE_128B
@@ -768,6 +831,11 @@ ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan 
     k.N = tp.N;
     k.K = tp.K;
     k.m_blocks = tp.m_blocks;
+    k.kc_lg = g.kc == 1 ? 0 : (g.kc == 2 ? 1 : (g.kc == 4 ? 2 : (g.kc == 8 ? 3 : 4)));
+    k.a_cx = g.A.cx;
+    k.a_cy = g.A.cy;
+    k.b_cx = g.B.cx;
+    k.b_cy = g.B.cy;
     k.wa = g.A.w;
     k.wb = g.B.w;
     k.na_sub = g.A.nsub;
@@ -795,7 +863,7 @@ ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan 
     k.a_mb16 = tp.a_kmajor ? (int)((128u * g.A.w * 2) >> 4) : (int)((128 / g.A.w) * (g.A.sub_bytes >> 4));
     k.status = ctx->d_status;
     void (*kern)(const CUtensorMap, const CUtensorMap, const TcArgs) = nullptr;
-    switch (tp.K / 16) {
+    switch (tp.K / g.kc / 16) {
         case 1: kern = tc_contract_kernel<1>; break;
         case 2: kern = tc_contract_kernel<2>; break;
         case 4: kern = tc_contract_kernel<4>; break;

@@ -35,6 +35,11 @@
 //               end of an output key, store the output tile (or a partial for
 //               the fixup kernel when the key straddles two work units).
 //
+// When the MMA warp opens a group it also requests the group's E tile by TMA
+// into the buffer's E slot; when it closes the group it posts whether the
+// group ends its output key.  The epilogue thus never searches the pair list
+// nor waits on a global load.
+//
 // Every mbarrier wait is bounded; on expiry the CTA raises kStTimeout, all
 // roles leave their loops, in-flight copies and MMAs are drained (bounded),
 // TMEM is freed and the kernel returns.
@@ -59,16 +64,17 @@ constexpr uint32_t kFBytes = 16 * 64 * 2;    // F tile: 16 rows k x 64 r, bf16
 // stage: pps T tiles, then Z F0 Z F1 Z ... F(pps-1) Z (Z = zero block of kFBytes)
 constexpr uint32_t kFRegion = (2 * kPps3 + 1) * kFBytes;
 constexpr uint32_t kStageBytes = kPps3 * kTBytes + kFRegion;
-constexpr uint32_t kBarBytes = 8 * (2 * kStages3 + 2 * kAcc3 + 1) + 64;
-constexpr uint32_t kSmem3 = 1024 + kStages3 * kStageBytes + kBarBytes;
+constexpr uint32_t kEBytes = 16 * 64 * 2;    // E tile: 16 j x 64 r, bf16, one slot per accumulator buffer
+// barriers: full, empty (per stage); accf, acce, ef, infoc (per buffer); done
+constexpr uint32_t kBarBytes = 8 * (2 * kStages3 + 4 * kAcc3 + 1) + 64 + 8 * kAcc3;
+constexpr uint32_t kSmem3 = 1024 + kStages3 * kStageBytes + kAcc3 * kEBytes + kBarBytes;
 static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
 static_assert(kSmem3 <= 227 * 1024, "shared memory budget");
 
 struct Tc3Args {
     const uint32_t *idx_t, *idx_e, *idx_f;   // [P] T, E, F tuple of each triple
     int64_t nT, nE, nF;
-    const void *E;                  // E tiles (bf16), read by the epilogue
-    int64_t tileE, sEj, sEr;        // E tile size and strides of j and r
+    int64_t sEj, sEr;               // E tile strides of j and r
     const int64_t *seg_start;
     int64_t S;
     Units units;
@@ -115,6 +121,24 @@ __device__ __noinline__ bool wait3(uint32_t bar, uint32_t parity, volatile uint3
             return false;
         }
     }
+}
+
+__device__ __forceinline__ bool try3(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait with an inline first attempt.
+__device__ __forceinline__ bool wait3f(uint32_t bar, uint32_t parity, volatile uint32_t *abort_flag,
+                                       uint32_t *status) {
+    return try3(bar, parity) || wait3(bar, parity, abort_flag, status);
 }
 
 __device__ __noinline__ void drain3(uint32_t bar, uint32_t parity) {
@@ -166,17 +190,13 @@ __device__ __forceinline__ void commit(uint32_t bar) {
 __device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
-// 32 consecutive TMEM columns of this thread's lane.  The wait sits in the
-// same asm statement, so no use of the outputs can be scheduled before it.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t *r) {
+// 128 consecutive TMEM columns of this thread's lane, one load; the wait sits
+// in the same asm statement, so no use of the outputs is scheduled before it.
+__device__ __forceinline__ void tmem_ld128(uint32_t taddr, uint32_t *r) {
     asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
-        "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];\n\t"
+        "tcgen05.ld.sync.aligned.32x32b.x128.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63, %64, %65, %66, %67, %68, %69, %70, %71, %72, %73, %74, %75, %76, %77, %78, %79, %80, %81, %82, %83, %84, %85, %86, %87, %88, %89, %90, %91, %92, %93, %94, %95, %96, %97, %98, %99, %100, %101, %102, %103, %104, %105, %106, %107, %108, %109, %110, %111, %112, %113, %114, %115, %116, %117, %118, %119, %120, %121, %122, %123, %124, %125, %126, %127}, [%128];\n\t"
         "tcgen05.wait::ld.sync.aligned;"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63]), "=r"(r[64]), "=r"(r[65]), "=r"(r[66]), "=r"(r[67]), "=r"(r[68]), "=r"(r[69]), "=r"(r[70]), "=r"(r[71]), "=r"(r[72]), "=r"(r[73]), "=r"(r[74]), "=r"(r[75]), "=r"(r[76]), "=r"(r[77]), "=r"(r[78]), "=r"(r[79]), "=r"(r[80]), "=r"(r[81]), "=r"(r[82]), "=r"(r[83]), "=r"(r[84]), "=r"(r[85]), "=r"(r[86]), "=r"(r[87]), "=r"(r[88]), "=r"(r[89]), "=r"(r[90]), "=r"(r[91]), "=r"(r[92]), "=r"(r[93]), "=r"(r[94]), "=r"(r[95]), "=r"(r[96]), "=r"(r[97]), "=r"(r[98]), "=r"(r[99]), "=r"(r[100]), "=r"(r[101]), "=r"(r[102]), "=r"(r[103]), "=r"(r[104]), "=r"(r[105]), "=r"(r[106]), "=r"(r[107]), "=r"(r[108]), "=r"(r[109]), "=r"(r[110]), "=r"(r[111]), "=r"(r[112]), "=r"(r[113]), "=r"(r[114]), "=r"(r[115]), "=r"(r[116]), "=r"(r[117]), "=r"(r[118]), "=r"(r[119]), "=r"(r[120]), "=r"(r[121]), "=r"(r[122]), "=r"(r[123]), "=r"(r[124]), "=r"(r[125]), "=r"(r[126]), "=r"(r[127])
         : "r"(taddr)
         : "memory");
 }
@@ -198,17 +218,26 @@ __device__ __forceinline__ float epi3(float x, int epi, float scale) {
 
 __global__ void __launch_bounds__(kThreads3, 1)
     tc3_contract_kernel(const __grid_constant__ CUtensorMap tmT, const __grid_constant__ CUtensorMap tmF,
-                        const Tc3Args a) {
+                        const __grid_constant__ CUtensorMap tmE, const Tc3Args a) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     const uint32_t sbase = smem_u32(smem);
-    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)kStages3 * kStageBytes);
+    // E slot of buffer b: the group's E tile, fetched by TMA when the MMA warp
+    // opens the group (ef[b]), read by the epilogue before it frees the buffer
+    const __nv_bfloat16 *eslots = reinterpret_cast<const __nv_bfloat16 *>(smem + (size_t)kStages3 * kStageBytes);
+    const uint32_t eslot0 = sbase + kStages3 * kStageBytes;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)kStages3 * kStageBytes + kAcc3 * kEBytes);
     const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8u * kStages3, accf0 = empty0 + 8u * kStages3,
-                   acce0 = accf0 + 8u * kAcc3, done_bar = acce0 + 8u * kAcc3;
-    uint32_t *misc = reinterpret_cast<uint32_t *>(bars + 2 * kStages3 + 2 * kAcc3 + 1);
+                   acce0 = accf0 + 8u * kAcc3, done_bar = acce0 + 8u * kAcc3, ef0 = done_bar + 8u,
+                   infoc0 = ef0 + 8u * kAcc3;
+    uint32_t *misc = reinterpret_cast<uint32_t *>(bars + 2 * kStages3 + 4 * kAcc3 + 1);
     // misc[0] TMEM base, [1] abort flag, [2] stage fills the MMA warp consumed,
-    // [3] stage fills the producer issued
+    // [3] stage fills the producer issued, [4] E tiles requested, [5] E tiles
+    // the epilogue received
     volatile uint32_t *abort_flag = misc + 1;
+    // per accumulator buffer: [2b + 1] 1 if the group ends its output key
+    // (posted at close through infoc[b])
+    volatile uint32_t *info = misc + 16;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     // zero blocks around the F slots: written once, read by every MMA
@@ -228,6 +257,10 @@ __global__ void __launch_bounds__(kThreads3, 1)
             mbar_init(acce0 + 8u * i, 4);
         }
         mbar_init(done_bar, 1);
+        for (int i = 0; i < kAcc3; ++i) {
+            mbar_init(ef0 + 8u * i, 1);
+            mbar_init(infoc0 + 8u * i, 1);
+        }
         for (int i = 1; i < 16; ++i) misc[i] = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -275,7 +308,7 @@ __global__ void __launch_bounds__(kThreads3, 1)
             const int np = n - f * kPps3 < kPps3 ? n - f * kPps3 : kPps3;
             uint32_t okw = 1;
             if (lane == 0) {
-                okw = wait3(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status) ? 1u : 0u;
+                okw = wait3f(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status) ? 1u : 0u;
                 if (okw) arrive_tx(full0 + 8u * st, (uint32_t)np * (kTBytes + kFBytes));
             }
             if (!__shfl_sync(0xffffffffu, okw, 0)) break;
@@ -300,7 +333,7 @@ __global__ void __launch_bounds__(kThreads3, 1)
         // accumulates into one TMEM buffer; its first MMA overwrites.
         const uint64_t adesc = a.a_desc0, bdesc = a.b_desc0;
         const uint32_t idesc = a.idesc;
-        uint32_t b = 0, aph = 0, dcol = tmem, st = 0, ph = 0, consumed = 0;
+        uint32_t b = 0, aph = 0, dcol = tmem, st = 0, ph = 0, consumed = 0, opened = 0;
         bool open = false, ok = true;
         int64_t s = s_first;
         int seg_end = n > 0 ? (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) : 0;
@@ -309,11 +342,25 @@ __global__ void __launch_bounds__(kThreads3, 1)
             const int64_t p = pb + start + lane;
             return (start < n && lane < kPps3 && p < pe) ? a.idx_e[p] : 0u;
         };
+        // group close: post whether it ends its output key, then hand the
+        // buffer to the epilogue once its MMAs complete
+        auto close_grp = [&](uint32_t ends) {
+            if (lane == 0) {
+                info[2 * b + 1] = ends;
+                arrive(infoc0 + 8u * b);
+            }
+            if (elect1()) commit(accf0 + 8u * b);
+            __syncwarp();
+            if (++b == (uint32_t)kAcc3) {
+                b = 0;
+                aph ^= 1u;
+            }
+        };
         uint32_t ev = load_e(0);
         for (int start = 0; start < n; start += kPps3) {
             const int np = n - start < kPps3 ? n - start : kPps3;
             const uint32_t ev_next = load_e(start + kPps3);
-            if (!__all_sync(0xffffffffu, wait3(full0 + 8u * st, ph, abort_flag, a.status))) {
+            if (!__all_sync(0xffffffffu, wait3f(full0 + 8u * st, ph, abort_flag, a.status))) {
                 ok = false;
                 break;
             }
@@ -323,26 +370,31 @@ __global__ void __launch_bounds__(kThreads3, 1)
                 const int pos = start + jj;
                 const uint32_t ecur = __shfl_sync(0xffffffffu, ev, jj);
                 bool newgrp = !open || ecur != eprev;
-                if (pos == seg_end) {
+                const bool segbrk = pos == seg_end;
+                if (segbrk) {
                     ++s;
                     seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
                     newgrp = true;
                 }
                 if (newgrp) {
-                    if (open) {
-                        if (elect1()) commit(accf0 + 8u * b);
-                        __syncwarp();
-                        if (++b == (uint32_t)kAcc3) {
-                            b = 0;
-                            aph ^= 1u;
-                        }
-                    }
-                    if (!__all_sync(0xffffffffu, wait3(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status))) {
+                    if (open) close_grp(segbrk ? 1u : 0u);
+                    if (!__all_sync(0xffffffffu, wait3f(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status))) {
                         ok = false;
                         open = false;
                         break;
                     }
                     fence_after();
+                    if (lane == 0) {
+                        uint32_t ei = ecur;
+                        if ((int64_t)ei >= a.nE) {
+                            atomicOr(a.status, kStBadIndex);
+                            ei = 0;
+                        }
+                        arrive_tx(ef0 + 8u * b, kEBytes);
+                        tma3d(eslot0 + b * kEBytes, &tmE, (int)ei, ef0 + 8u * b);
+                    }
+                    __syncwarp();
+                    ++opened;
                     dcol = tmem + b * 128u;
                     open = true;
                 }
@@ -367,54 +419,37 @@ __global__ void __launch_bounds__(kThreads3, 1)
                 ph ^= 1u;
             }
         }
-        if (open) {
-            if (elect1()) commit(accf0 + 8u * b);
-            __syncwarp();
+        if (open) close_grp(1u);
+        if (lane == 0) {
+            misc[2] = ok ? 0xFFFFFFFFu : consumed;
+            misc[4] = opened;
         }
-        if (lane == 0) misc[2] = ok ? 0xFFFFFFFFu : consumed;
     } else {
         // ------------------------------------------------------- epilogue
         const int q = warp & 3;   // TMEM lane quadrant of this warp
         const int l = q * 32 + lane, x = l >> 6, r = l & 63;
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
-        const __nv_bfloat16 *E = reinterpret_cast<const __nv_bfloat16 *>(a.E);
         float acc[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) acc[i] = 0.0f;
-        uint32_t b = 0, ph = 0;
-        int64_t p = pb, s = s_first;
-        int64_t seg_stop = n > 0 ? (a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) : pe;
-        while (p < pe) {
-            // the group starting at p: same E tuple, up to the end of the key
-            const uint32_t e0 = a.idx_e[p];
-            int64_t qe = p + 1;
-            while (qe < seg_stop) {
-                const int64_t idx = qe + lane;
-                const bool diff = idx < seg_stop ? a.idx_e[idx] != e0 : true;
-                const unsigned m = __ballot_sync(0xffffffffu, diff);
-                if (m) {
-                    qe += __ffs(m) - 1;
-                    break;
-                }
-                qe += 32;
-            }
-            uint32_t ei = e0;
-            if ((int64_t)ei >= a.nE) {
-                if (lane == 0) atomicOr(a.status, kStBadIndex);
-                ei = 0;
-            }
+        uint32_t b = 0, ph = 0, got_e = 0;
+        int64_t s = s_first;
+        const int64_t s_last = n > 0 ? seg_of(a.seg_start, a.S, pe - 1) : s_first - 1;
+        while (s <= s_last) {
+            // the group's E tile was requested when the MMA warp opened it
+            if (!__all_sync(0xffffffffu, wait3f(ef0 + 8u * b, ph, abort_flag, a.status))) break;
+            ++got_e;
             float ef[16];
-            const __nv_bfloat16 *ep = E + (int64_t)ei * a.tileE + r * a.sEr;
+            const __nv_bfloat16 *ep = eslots + b * (kEBytes / 2) + r * a.sEr;
 #pragma unroll
             for (int j = 0; j < 16; ++j) ef[j] = __bfloat162float(ep[j * a.sEj]);
-            if (!__all_sync(0xffffffffu, wait3(accf0 + 8u * b, ph, abort_flag, a.status))) break;
+            if (!__all_sync(0xffffffffu, wait3f(infoc0 + 8u * b, ph, abort_flag, a.status))) break;
+            const uint32_t ends = info[2 * b + 1];
+            if (!__all_sync(0xffffffffu, wait3f(accf0 + 8u * b, ph, abort_flag, a.status))) break;
             fence_after();
             uint32_t v[128];
             const uint32_t bcol = tmem + lane_base + b * 128u;
-            tmem_ld32(bcol, v);
-            tmem_ld32(bcol + 32, v + 32);
-            tmem_ld32(bcol + 64, v + 64);
-            tmem_ld32(bcol + 96, v + 96);
+            tmem_ld128(bcol, v);
             fence_before();
             __syncwarp();
             if (lane == 0) arrive(acce0 + 8u * b);
@@ -426,8 +461,7 @@ __global__ void __launch_bounds__(kThreads3, 1)
             for (int i = 0; i < 8; ++i)
 #pragma unroll
                 for (int j = 0; j < 16; ++j) acc[i] = fmaf(ef[j], __uint_as_float(v[i * 16 + j]), acc[i]);
-            p = qe;
-            if (p == seg_stop) {
+            if (ends) {
                 const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
                 const int kind = (ss >= pb && se <= pe) ? 0 : (ss < pb ? 1 : 2);
 #pragma unroll
@@ -445,9 +479,9 @@ __global__ void __launch_bounds__(kThreads3, 1)
                     acc[i] = 0.0f;
                 }
                 ++s;
-                if (p < pe) seg_stop = a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe;
             }
         }
+        if (warp == 2 && lane == 0) misc[5] = got_e;
     }
 
     // ---------------------------------------------------------- teardown
@@ -458,6 +492,8 @@ __global__ void __launch_bounds__(kThreads3, 1)
             // every fill the MMA warp did not consume
             const uint32_t done = misc[2];
             for (uint32_t k = done; k < misc[3]; ++k) drain3(full0 + 8u * (k % kStages3), (k / kStages3) & 1u);
+            // E tiles requested for groups the epilogue did not reach
+            for (uint32_t k = misc[5]; k < misc[4]; ++k) drain3(ef0 + 8u * (k % kAcc3), (k / kAcc3) & 1u);
         }
         if (warp == 1 && lane == 0) {
             commit(done_bar);   // tracks every MMA this thread issued
@@ -519,9 +555,13 @@ ucl_status launch_contract_tc3(ucl_ctx *ctx, const ContractArgs &a, const Tc3Pla
     std::string why;
     if ((reinterpret_cast<uintptr_t>(T->tiles) | reinterpret_cast<uintptr_t>(F->tiles)) & 15)
         return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: tile arrays not 16-byte aligned");
-    CUtensorMap mT, mF;
+    if (reinterpret_cast<uintptr_t>(E->tiles) & 15)
+        return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: tile arrays not 16-byte aligned");
+    CUtensorMap mT, mF, mE;
+    // E is copied as stored (no swizzle): [shape0][shape1]
     if (!map3(&mT, T->tiles, T->n, 16, 256, CU_TENSOR_MAP_SWIZZLE_32B, &why) ||
-        !map3(&mF, F->tiles, F->n, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B, &why))
+        !map3(&mF, F->tiles, F->n, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B, &why) ||
+        !map3(&mE, E->tiles, E->n, (int)E->shape[1], (int)E->shape[0], CU_TENSOR_MAP_SWIZZLE_NONE, &why))
         return fail(ctx, UCL_ERR_CUDA, "tcgen05 path: " + why);
     Tc3Args k{};
     k.idx_t = idx[tp.t];
@@ -530,8 +570,6 @@ ucl_status launch_contract_tc3(ucl_ctx *ctx, const ContractArgs &a, const Tc3Pla
     k.nT = T->n;
     k.nE = E->n;
     k.nF = F->n;
-    k.E = E->tiles;
-    k.tileE = E->tile;
     k.sEj = tp.sEj;
     k.sEr = tp.sEr;
     k.seg_start = a.seg_start;
@@ -558,7 +596,7 @@ ucl_status launch_contract_tc3(ucl_ctx *ctx, const ContractArgs &a, const Tc3Pla
         ctx, cudaFuncSetAttribute(tc3_contract_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem3),
         "cudaFuncSetAttribute");
     if (st) return st;
-    tc3_contract_kernel<<<a.units.G, kThreads3, kSmem3, ctx->stream>>>(mT, mF, k);
+    tc3_contract_kernel<<<a.units.G, kThreads3, kSmem3, ctx->stream>>>(mT, mF, mE, k);
     ctx->launches++;
     return cuda_check(ctx, cudaGetLastError(), "tcgen05 kernel launch");
 }

@@ -70,6 +70,9 @@ TC_CASES = [
     ("IJmk", "JKkn", "IKmn", {"m": 256, "k": 64, "n": 64}),    # two M blocks
     ("IJkm", "JKkn", "IKnm", {"m": 256, "k": 64, "n": 32}),    # two M blocks, MN-major A
     ("IJnk", "JKmk", "IKnm", {"m": 128, "k": 64, "n": 48}),    # A comes from V
+    ("IJkm", "JKkn", "IKmn", {"m": 256, "k": 256, "n": 64}),   # K chunks, MN-major A (row ranges)
+    ("IJmk", "JKnk", "IKmn", {"m": 256, "k": 256, "n": 128}),  # K chunks, K-major A and B (column ranges)
+    ("IJmk", "JKkn", "IKnm", {"m": 128, "k": 128, "n": 256}),  # K chunks, transposed output
 ]
 
 
