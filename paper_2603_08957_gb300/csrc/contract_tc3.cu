@@ -28,8 +28,9 @@
 //   warp 0      TMA producer: T tile (16 x 256 rows, 32B swizzle) and F tile
 //               (64 x 16 rows, 128B swizzle) of each triple into a ring of
 //               stages of `pps` triples;
-//   warp 1      MMA issuer (owns TMEM): two tcgen05.mma per triple into the
-//               group's accumulator buffer;
+//   warp 1      MMA issuer (owns TMEM): one thread issues two tcgen05.mma per
+//               triple into the group's accumulator buffer, following a group
+//               plan the producer posts with each stage;
 //   warps 2-5   epilogue: per group, load E's 16 values for its r, drain the
 //               group's accumulator and fold it into 8 fp32 registers; at the
 //               end of an output key, store the output tile (or a partial for
@@ -66,7 +67,7 @@ constexpr uint32_t kFRegion = (2 * kPps3 + 1) * kFBytes;
 constexpr uint32_t kStageBytes = kPps3 * kTBytes + kFRegion;
 constexpr uint32_t kEBytes = 16 * 64 * 2;    // E tile: 16 j x 64 r, bf16, one slot per accumulator buffer
 // barriers: full, empty (per stage); accf, acce, ef, infoc (per buffer); done
-constexpr uint32_t kBarBytes = 8 * (2 * kStages3 + 4 * kAcc3 + 1) + 64 + 8 * kAcc3;
+constexpr uint32_t kBarBytes = 8 * (2 * kStages3 + 4 * kAcc3 + 1) + 64 + 8 * kAcc3 + 4 * kStages3 * (kPps3 + 1);
 constexpr uint32_t kSmem3 = 1024 + kStages3 * kStageBytes + kAcc3 * kEBytes + kBarBytes;
 static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
 static_assert(kSmem3 <= 227 * 1024, "shared memory budget");
@@ -145,16 +146,6 @@ __device__ __noinline__ void drain3(uint32_t bar, uint32_t parity) {
     const long long t0 = clock64();
     while (!mbar_try_sleep(bar, parity, 100000u))
         if (clock64() - t0 > kWait3) return;
-}
-
-__device__ __forceinline__ bool elect1() {
-    uint32_t pred;
-    asm volatile(
-        "{\n\t.reg .b32 r;\n\t.reg .pred p;\n\t"
-        "elect.sync r|p, 0xffffffff;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(pred));
-    return pred != 0;
 }
 
 __device__ __forceinline__ void arrive_tx(uint32_t bar, uint32_t bytes) {
@@ -238,6 +229,10 @@ __global__ void __launch_bounds__(kThreads3, 1)
     // per accumulator buffer: [2b + 1] 1 if the group ends its output key
     // (posted at close through infoc[b])
     volatile uint32_t *info = misc + 16;
+    // per stage: the E tuple of each triple, then a word whose bit j marks
+    // triple j as opening a group and bit 8 + j marks the group before it as
+    // ending its output key (written by the producer before its arrive)
+    volatile uint32_t *plan = info + 2 * kAcc3;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     // zero blocks around the F slots: written once, read by every MMA
@@ -282,16 +277,22 @@ __global__ void __launch_bounds__(kThreads3, 1)
 
     if (warp == 0) {
         // ------------------------------------------------------- producer
-        // lane j < pps issues the two copies of triple j of each stage; the
-        // tuple indices are loaded one stage ahead
+        // Lane j < pps handles triple j of each stage: its tuple indices are
+        // loaded one stage ahead; lane 0 posts the stage's group plan (each
+        // triple's E tuple, which triples open a group, which groups end their
+        // output key) in shared memory before its arrive, so the plan is
+        // visible to whoever observes the stage full; then lane j issues the
+        // two copies of triple j.
         const int nfills = (n + kPps3 - 1) / kPps3;
-        auto load_idx = [&](int f, uint32_t &it, uint32_t &iff) {
+        auto load_idx = [&](int f, uint32_t &it, uint32_t &iff, uint32_t &ie) {
             it = 0;
             iff = 0;
+            ie = 0;
             const int64_t p = pb + (int64_t)f * kPps3 + lane;
             if (f < nfills && lane < kPps3 && p < pe) {
                 it = a.idx_t[p];
                 iff = a.idx_f[p];
+                ie = a.idx_e[p];
                 if ((int64_t)it >= a.nT || (int64_t)iff >= a.nF) {
                     atomicOr(a.status, kStBadIndex);
                     it = 0;
@@ -299,17 +300,40 @@ __global__ void __launch_bounds__(kThreads3, 1)
                 }
             }
         };
-        uint32_t it, iff;
-        load_idx(0, it, iff);
-        uint32_t st = 0, ph = 0, mine = 0;
+        uint32_t it, iff, ie;
+        load_idx(0, it, iff, ie);
+        uint32_t st = 0, ph = 0, mine = 0, e_last = 0;
+        int64_t s = s_first;
+        int seg_end = n > 0 ? (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) : 0;
         for (int f = 0; f < nfills; ++f) {
-            uint32_t nit, niff;
-            load_idx(f + 1, nit, niff);
-            const int np = n - f * kPps3 < kPps3 ? n - f * kPps3 : kPps3;
+            uint32_t nit, niff, nie;
+            load_idx(f + 1, nit, niff, nie);
+            const int start = f * kPps3;
+            const int np = n - start < kPps3 ? n - start : kPps3;
+            // segment starts inside this stage (uniform; rare)
+            uint32_t brk = 0;
+            while (seg_end < start + np) {
+                brk |= 1u << (seg_end - start);
+                ++s;
+                seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
+            }
+            const uint32_t eup = __shfl_up_sync(0xffffffffu, ie, 1);
+            const uint32_t eprev = lane == 0 ? e_last : eup;
+            const bool newg = lane < np && (start + lane == 0 || ie != eprev || ((brk >> lane) & 1u));
+            const uint32_t gmask = __ballot_sync(0xffffffffu, newg) & 0xFu;
+            e_last = __shfl_sync(0xffffffffu, ie, np - 1);
+            uint32_t e4[kPps3];
+#pragma unroll
+            for (int j = 0; j < kPps3; ++j) e4[j] = __shfl_sync(0xffffffffu, ie, j);
             uint32_t okw = 1;
             if (lane == 0) {
                 okw = wait3f(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status) ? 1u : 0u;
-                if (okw) arrive_tx(full0 + 8u * st, (uint32_t)np * (kTBytes + kFBytes));
+                if (okw) {
+#pragma unroll
+                    for (int j = 0; j < kPps3; ++j) plan[st * (kPps3 + 1) + j] = e4[j];
+                    plan[st * (kPps3 + 1) + kPps3] = gmask | (brk << 8);
+                    arrive_tx(full0 + 8u * st, (uint32_t)np * (kTBytes + kFBytes));
+                }
             }
             if (!__shfl_sync(0xffffffffu, okw, 0)) break;
             if (lane < np) {
@@ -321,6 +345,7 @@ __global__ void __launch_bounds__(kThreads3, 1)
             ++mine;
             it = nit;
             iff = niff;
+            ie = nie;
             if (++st == (uint32_t)kStages3) {
                 st = 0;
                 ph ^= 1u;
@@ -329,101 +354,77 @@ __global__ void __launch_bounds__(kThreads3, 1)
         if (lane == 0) misc[3] = mine;
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA
+        // One thread issues everything, following the producer's group plan.
         // A group (a run of triples of one output key with the same E tuple)
         // accumulates into one TMEM buffer; its first MMA overwrites.
-        const uint64_t adesc = a.a_desc0, bdesc = a.b_desc0;
-        const uint32_t idesc = a.idesc;
-        uint32_t b = 0, aph = 0, dcol = tmem, st = 0, ph = 0, consumed = 0, opened = 0;
-        bool open = false, ok = true;
-        int64_t s = s_first;
-        int seg_end = n > 0 ? (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) : 0;
-        uint32_t eprev = 0;
-        auto load_e = [&](int start) -> uint32_t {
-            const int64_t p = pb + start + lane;
-            return (start < n && lane < kPps3 && p < pe) ? a.idx_e[p] : 0u;
-        };
-        // group close: post whether it ends its output key, then hand the
-        // buffer to the epilogue once its MMAs complete
-        auto close_grp = [&](uint32_t ends) {
-            if (lane == 0) {
+        if (lane == 0) {
+            const uint64_t adesc = a.a_desc0, bdesc = a.b_desc0;
+            const uint32_t idesc = a.idesc;
+            uint32_t b = 0, aph = 0, dcol = tmem, st = 0, ph = 0, consumed = 0, opened = 0;
+            bool open = false, ok = true;
+            // group close: post whether it ends its output key, then hand the
+            // buffer to the epilogue once its MMAs complete
+            auto close_grp = [&](uint32_t ends) {
                 info[2 * b + 1] = ends;
                 arrive(infoc0 + 8u * b);
-            }
-            if (elect1()) commit(accf0 + 8u * b);
-            __syncwarp();
-            if (++b == (uint32_t)kAcc3) {
-                b = 0;
-                aph ^= 1u;
-            }
-        };
-        uint32_t ev = load_e(0);
-        for (int start = 0; start < n; start += kPps3) {
-            const int np = n - start < kPps3 ? n - start : kPps3;
-            const uint32_t ev_next = load_e(start + kPps3);
-            if (!__all_sync(0xffffffffu, wait3f(full0 + 8u * st, ph, abort_flag, a.status))) {
-                ok = false;
-                break;
-            }
-            fence_after();
-            const uint32_t s0 = sbase + st * kStageBytes;
-            for (int jj = 0; jj < np; ++jj) {
-                const int pos = start + jj;
-                const uint32_t ecur = __shfl_sync(0xffffffffu, ev, jj);
-                bool newgrp = !open || ecur != eprev;
-                const bool segbrk = pos == seg_end;
-                if (segbrk) {
-                    ++s;
-                    seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
-                    newgrp = true;
+                commit(accf0 + 8u * b);
+                if (++b == (uint32_t)kAcc3) {
+                    b = 0;
+                    aph ^= 1u;
                 }
-                if (newgrp) {
-                    if (open) close_grp(segbrk ? 1u : 0u);
-                    if (!__all_sync(0xffffffffu, wait3f(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status))) {
-                        ok = false;
-                        open = false;
-                        break;
-                    }
-                    fence_after();
-                    if (lane == 0) {
-                        uint32_t ei = ecur;
+            };
+            for (int start = 0; start < n; start += kPps3) {
+                const int np = n - start < kPps3 ? n - start : kPps3;
+                if (!wait3f(full0 + 8u * st, ph, abort_flag, a.status)) {
+                    ok = false;
+                    break;
+                }
+                fence_after();
+                const uint32_t flags = plan[st * (kPps3 + 1) + kPps3];
+                const uint32_t s0 = sbase + st * kStageBytes;
+                const uint64_t bd0 = bdesc + (s0 >> 4), ad0 = adesc + ((s0 + kPps3 * kTBytes + kFBytes) >> 4);
+                for (int jj = 0; jj < np; ++jj) {
+                    const bool newgrp = (flags >> jj) & 1u;
+                    if (newgrp) {
+                        if (open) close_grp((flags >> (8 + jj)) & 1u);
+                        if (!wait3f(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status)) {
+                            ok = false;
+                            open = false;
+                            break;
+                        }
+                        fence_after();
+                        uint32_t ei = plan[st * (kPps3 + 1) + jj];
                         if ((int64_t)ei >= a.nE) {
                             atomicOr(a.status, kStBadIndex);
                             ei = 0;
                         }
                         arrive_tx(ef0 + 8u * b, kEBytes);
                         tma3d(eslot0 + b * kEBytes, &tmE, (int)ei, ef0 + 8u * b);
+                        ++opened;
+                        dcol = tmem + b * 128u;
+                        open = true;
                     }
-                    __syncwarp();
-                    ++opened;
-                    dcol = tmem + b * 128u;
-                    open = true;
-                }
-                const uint32_t fslot = s0 + kPps3 * kTBytes + (2u * jj + 1u) * kFBytes;
-                const uint32_t tslot = s0 + (uint32_t)jj * kTBytes;
-                if (elect1()) {
+                    // F slot jj at (2 jj + 1) blocks; T slot jj at jj tiles
+                    const uint64_t ad = ad0 + (uint64_t)(jj * (2 * kFBytes >> 4));
+                    const uint64_t bd = bd0 + (uint64_t)(jj * (kTBytes >> 4));
                     // x = 0: F^T in M rows 0-63 (zeros below), i in 0..7
-                    mma(dcol, adesc + (fslot >> 4), bdesc + (tslot >> 4), idesc, newgrp ? 0u : 1u);
+                    mma(dcol, ad, bd, idesc, newgrp ? 0u : 1u);
                     // x = 1: F^T in M rows 64-127 (zeros above), i in 8..15
-                    mma(dcol, adesc + ((fslot - kFBytes) >> 4), bdesc + ((tslot + kTBytes / 2) >> 4), idesc, 1u);
+                    mma(dcol, ad - (kFBytes >> 4), bd + ((kTBytes / 2) >> 4), idesc, 1u);
                 }
-                __syncwarp();
-                eprev = ecur;
+                if (!ok) break;
+                commit(empty0 + 8u * st);
+                ++consumed;
+                if (++st == (uint32_t)kStages3) {
+                    st = 0;
+                    ph ^= 1u;
+                }
             }
-            if (!ok) break;
-            if (elect1()) commit(empty0 + 8u * st);
-            __syncwarp();
-            ++consumed;
-            ev = ev_next;
-            if (++st == (uint32_t)kStages3) {
-                st = 0;
-                ph ^= 1u;
-            }
-        }
-        if (open) close_grp(1u);
-        if (lane == 0) {
+            if (open) close_grp(1u);
             misc[2] = ok ? 0xFFFFFFFFu : consumed;
             misc[4] = opened;
         }
+        __syncwarp();
     } else {
         // ------------------------------------------------------- epilogue
         const int q = warp & 3;   // TMEM lane quadrant of this warp
