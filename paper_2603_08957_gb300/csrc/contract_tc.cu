@@ -299,6 +299,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int nfills = (n + pps - 1) / pps;
         const int kmask = (1 << a.kc_lg) - 1;
         uint32_t mine = 0;
+        // raw index loads two own fills ahead, checked only when used, so a
+        // fill never waits on the latency of its own index loads
         auto load_idx = [&](int f, uint32_t &ia, uint32_t &ib) {
             ia = 0;
             ib = 0;
@@ -307,19 +309,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if (f < nfills && lane < pps && v < n) {
                 ia = a.pa[p];
                 ib = a.pb[p];
-                if ((int64_t)ia >= a.nA || (int64_t)ib >= a.nB) {
-                    atomicOr(a.status, kStBadIndex);
-                    ia = 0;
-                    ib = 0;
-                }
             }
         };
-        uint32_t ia, ib;
+        uint32_t ia, ib, ia1, ib1;
         load_idx(warp, ia, ib);
+        load_idx(warp + kProducers, ia1, ib1);
         uint32_t st = (uint32_t)(warp % a.ns), ph = (uint32_t)((warp / a.ns) & 1);
         for (int f = warp; f < nfills; f += kProducers) {
-            uint32_t nia, nib;
-            load_idx(f + kProducers, nia, nib);
+            uint32_t ia2, ib2;
+            load_idx(f + 2 * kProducers, ia2, ib2);
+            if ((int64_t)ia >= a.nA || (int64_t)ib >= a.nB) {
+                atomicOr(a.status, kStBadIndex);
+                ia = 0;
+                ib = 0;
+            }
             const int np = n - f * pps < pps ? n - f * pps : pps;
             uint32_t okw = 1;
             if (lane == 0) {
@@ -339,8 +342,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             __syncwarp();
             ++mine;
-            ia = nia;
-            ib = nib;
+            ia = ia1;
+            ib = ib1;
+            ia1 = ia2;
+            ib1 = ib2;
             st += kProducers;
             if (st >= (uint32_t)a.ns) {
                 st -= (uint32_t)a.ns;
