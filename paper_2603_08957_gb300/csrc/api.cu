@@ -935,7 +935,16 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
                 launch_expand(ctx, off, nA, lo, permA, permB, koA, koB, P, pk, pv);
             else
                 launch_unary_pairs(ctx, koA, P, pk, pv);
-            if (radix_sort(ctx, pk, pv, pk2, pv2, P, kp.out_bits)) { pk = pk2; pv = pv2; }
+            // Pairs are expanded in A's row order (each A row's partners
+            // contiguous).  When A is visited in its own ascending key order
+            // and alone supplies the output key, as its leading key columns,
+            // the pairs are already in output-key order: the stable sort
+            // would leave them as they are, so it is skipped.
+            bool presorted = A->sorted && permA == nullptr;
+            for (int k = 1; k < n_in && presorted; ++k) presorted = kp.out_k[kp.ord[k]].nf == 0;
+            for (int q = 0; q < kp.out_k[kp.ord[0]].nf && presorted; ++q)
+                presorted = kp.out_k[kp.ord[0]].f[q].col == q;
+            if (!presorted && radix_sort(ctx, pk, pv, pk2, pv2, P, kp.out_bits)) { pk = pk2; pv = pv2; }
             int64_t *flag = (int64_t *)ws_get(ctx, 8 * P);
             seg_excl = (int64_t *)ws_get(ctx, 8 * P);
             launch_heads(ctx, pk, P, flag);
