@@ -14,6 +14,7 @@ import pytest
 
 import oracle
 import workloads
+from oracle.repartition import RepartitionError, repartition
 from tests.ucl_testutil import brute_force, decompose, golden, random_sparse, recompose, ucl_operand
 
 GOLD = golden(os.path.join(os.path.dirname(__file__), "golden", "worked_example.txt"))
@@ -335,3 +336,69 @@ def test_relation_errors():
     x = (np.array([[1]], np.int32), [3], np.ones((1, 3)))  # bound of I disagrees
     with pytest.raises(oracle.OracleError, match="ERR_SHAPE"):
         oracle.einsum("Ij,Ij->I", [v, x])
+
+
+# ---------------------------------------------------- repartition (Sec. 5)
+
+
+
+def test_repartition_row_vectors_to_column_vectors():
+    """Sec. 5's example: T stored as row vectors (upper row index) becomes T
+    stored as column vectors (upper column index); every column index gets a
+    tuple (the decompose step ranges over the whole label)."""
+    T = np.array([[1.0, 0.0, 2.0, 0.0], [0.0, 0.0, 3.0, 0.0], [4.0, 0.0, 5.0, 0.0]])
+    rows = decompose(T, "ki", {"k"}, drop_zero=False)
+    keys, bounds, tiles = repartition("Ki->kI", rows)
+    assert bounds == (4,)
+    assert keys[:, 0].tolist() == [0, 1, 2, 3]
+    np.testing.assert_array_equal(tiles, T.T)
+
+
+@pytest.mark.parametrize("labels,ext,src,rhs", [
+    ("ij", {"i": 5, "j": 4}, {"i"}, "iJ"),             # rows -> columns
+    ("ijk", {"i": 3, "j": 4, "k": 2}, {"i"}, "IjK"),    # decompose only
+    ("ijk", {"i": 3, "j": 4, "k": 2}, {"i", "j"}, "iJk"),   # stack only
+    ("ijk", {"i": 3, "j": 4, "k": 2}, {"j", "k"}, "Ijk"),   # both
+    ("ijk", {"i": 3, "j": 4, "k": 2}, {"i"}, "Ikj"),    # tile dims reordered
+    ("ijk", {"i": 3, "j": 4, "k": 2}, {"j", "k"}, "KiJ"),   # keys reordered, i promoted
+    ("ijk", {"i": 3, "j": 4, "k": 2}, set(), "IJK"),    # dense -> scalars
+    ("ijk", {"i": 3, "j": 4, "k": 2}, {"i", "j", "k"}, "kji"),   # scalars -> one dense tuple, reversed
+])
+def test_repartition_keeps_the_tensor(labels, ext, src, rhs):
+    """The repartitioned relation denotes the same dense tensor, and its key
+    set is (kept key values present) x (full range of each promoted label),
+    in ascending order."""
+    rng = np.random.default_rng(len(labels) * 7 + len(src) + len(rhs))
+    dense = random_sparse(rng, [ext[c] for c in labels], density=0.5, block_axes=range(len(labels)))
+    rel = decompose(dense, labels, src)
+    lhs = "".join(c.upper() for c in labels if c in src) + "".join(c for c in labels if c not in src)
+    keys, bounds, tiles = repartition(lhs + "->" + rhs, rel)
+    dst = {c.lower() for c in rhs if c.isupper()}
+    out_order = rhs.lower()
+    back = recompose(keys, tiles, out_order, dst, ext)
+    np.testing.assert_array_equal(np.transpose(back, [out_order.index(c) for c in labels]), dense)
+    src_up = [c for c in labels if c in src]
+    out_up = [c.lower() for c in rhs if c.isupper()]
+    kept = [c for c in out_up if c in src]
+    prom = [c for c in out_up if c not in src]
+    kept_vals = {tuple(int(k[src_up.index(c)]) for c in kept) for k in rel[0]}
+    want = set()
+    for kv in kept_vals:
+        for pv in itertools.product(*[range(ext[c]) for c in prom]):
+            d = dict(zip(kept, kv))
+            d.update(zip(prom, pv))
+            want.add(tuple(d[c] for c in out_up))
+    assert set(map(tuple, keys.tolist())) == want
+    assert keys.tolist() == sorted(keys.tolist())
+    assert bounds == tuple(ext[c] for c in out_up)
+
+
+def test_repartition_identity_and_errors():
+    rng = np.random.default_rng(2)
+    rel = decompose(random_sparse(rng, [4, 3], density=0.6, block_axes=(0, 1)), "ij", {"i"})
+    k, b, t = repartition("Ij->Ij", rel)
+    np.testing.assert_array_equal(k, rel[0])
+    np.testing.assert_array_equal(t, rel[2])
+    for bad in ["Ij->Ik", "Ij->IJj", "Ij", "IJj->Ij", "Ij->I"]:
+        with pytest.raises(RepartitionError):
+            repartition(bad, rel)
