@@ -204,6 +204,38 @@ ucl_status ucl_relation_download(const ucl_rel *rel, int32_t *keys_host, void *t
 ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec, int n_in, ucl_rel *const *in, const ucl_einsum_opts *opts,
                       ucl_rel **out);
 
+/* ------------------------------------------------------------ repartition */
+
+/* Change a relation's upper/lower split without changing the tensor it
+ * denotes (Sec. 5, the representation change between two EinSums whose
+ * decompositions of a tensor differ: decompose every tuple over the full
+ * range of each label that becomes upper -- the ALLINTS step -- then stack
+ * the labels that become lower, grouped by the new upper labels -- the STACK
+ * aggregate).
+ *
+ * Spec: "<input labels>-><output>".  The input side lists the relation's
+ * labels, one letter each, upper case for key columns and lower case for tile
+ * dimensions, in order.  The output side is either
+ *   "<keys>|<tile dims>", the input's letters as written, or
+ *   the same letters with their case changed to give the new class (letters
+ *   then compare without case, so this form cannot tell J from j).
+ * Examples: "Ki->kI" (or "Ki->i|K") turns row vectors keyed by the row index
+ * into column vectors keyed by the column index; "Jfj->fJ|j" splits [f][j]
+ * tiles keyed by J into j-vectors keyed by (f, J).
+ *
+ * Output (owned by the library, destroy with ucl_relation_destroy): one tuple
+ * for every combination of a distinct value of the labels upper on both
+ * sides (as present in the input) with every index of the labels that become
+ * upper, in ascending key order; tiles row-major over the output's lower
+ * labels, the input's dtype, positions no input element maps to set to 0
+ * (tuples are never dropped, as the decompose step keeps every index).
+ * Values are copied, never rounded.  Synchronises the stream once when the
+ * input has key labels that stay upper.
+ * Errors: UCL_ERR_ARG, UCL_ERR_SPEC (labels), UCL_ERR_SHAPE (arity),
+ * UCL_ERR_UNSUPPORTED (> 64 output key bits, a tile or count of 2^31 or
+ * more), UCL_ERR_OOM, UCL_ERR_CUDA. */
+ucl_status ucl_repartition(ucl_ctx *ctx, const char *spec, const ucl_rel *in, ucl_rel **out);
+
 /* ------------------------------------------------------- no allocation */
 
 /* Largest key array ucl_keys_check_noalloc accepts (tuples). */

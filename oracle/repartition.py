@@ -16,11 +16,12 @@ This module follows those two steps tuple at a time, in fp64, with no
 blocking or fusion.  Only the tests, ``__graft_entry__.smoke`` and the CPU leg
 of ``bench.py`` may use it; it shares nothing with the GPU executor.
 
-Spec: ``"<input labels>-><output labels>"``, one letter per label, the case
-of a letter giving its class on that side (upper = key column, lower = tile
-dimension, in the order the letters appear).  A label is the same letter on
-both sides, compared without case, so one side may not hold two letters that
-differ only in case.
+Spec: ``"<input labels>-><output>"``.  The input side lists the relation's
+labels, one letter each, upper case for key columns and lower case for tile
+dimensions, in order.  The output side is either ``"<keys>|<tile dims>"``,
+the input's letters as written, or the same letters with their case changed
+to give the new class (letters then compare without case, so that form needs
+no two input letters that differ only in case).
 """
 from __future__ import annotations
 
@@ -34,24 +35,35 @@ class RepartitionError(ValueError):
 
 
 def _parse(spec, u, r):
+    """Labels are named by their input-side letter.  Returns the input's
+    upper and lower labels and the output's, each in order."""
     if "->" not in spec:
         raise RepartitionError("spec has no '->'")
     lhs, rhs = spec.split("->", 1)
-    for side in (lhs, rhs):
-        if not side.isalpha() and side != "":
-            raise RepartitionError("labels must be letters")
-        low = side.lower()
-        if len(set(low)) != len(low):
-            raise RepartitionError("a label appears twice on one side")
-    if sorted(lhs.lower()) != sorted(rhs.lower()):
-        raise RepartitionError("both sides must hold the same labels")
-    in_up = [c.lower() for c in lhs if c.isupper()]
+    if not lhs.isalpha() and lhs != "":
+        raise RepartitionError("labels must be letters")
+    if len(set(lhs)) != len(lhs):
+        raise RepartitionError("a label appears twice on the input side")
+    in_up = [c for c in lhs if c.isupper()]
     in_low = [c for c in lhs if c.islower()]
     if len(in_up) != u or len(in_low) != r:
         raise RepartitionError("input side does not match the relation's key/tile arity")
-    out_up = [c.lower() for c in rhs if c.isupper()]
-    out_low = [c for c in rhs if c.islower()]
-    return in_up, in_low, out_up, out_low
+    if "|" in rhs:
+        # explicit form: output keys | output tile dims, input letters as written
+        up, low = rhs.split("|", 1)
+        out = up + low
+        if (out and not out.isalpha()) or sorted(out) != sorted(lhs):
+            raise RepartitionError("both sides must hold the same labels")
+        return in_up, in_low, list(up), list(low)
+    # case form: the letter's case gives its output class; letters compare without case
+    if not rhs.isalpha() and rhs != "":
+        raise RepartitionError("labels must be letters")
+    if len(set(lhs.lower())) != len(lhs) or len(set(rhs.lower())) != len(rhs):
+        raise RepartitionError("a label appears twice on one side (letters compare without case)")
+    if sorted(lhs.lower()) != sorted(rhs.lower()):
+        raise RepartitionError("both sides must hold the same labels")
+    name = {c.lower(): c for c in lhs}
+    return in_up, in_low, [name[c.lower()] for c in rhs if c.isupper()], [name[c.lower()] for c in rhs if c.islower()]
 
 
 def repartition(spec, rel):

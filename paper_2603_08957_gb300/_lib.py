@@ -41,6 +41,7 @@ EXPORTS = [
     "ucl_relation_data",
     "ucl_relation_download",
     "ucl_einsum",
+    "ucl_repartition",
     "ucl_keys_check_noalloc",
     "ucl_status_str",
     "ucl_last_error",
@@ -93,6 +94,7 @@ def _declare(lib):
     lib.ucl_relation_data.argtypes = [vp, pp, pp]
     lib.ucl_relation_download.argtypes = [vp, vp, vp]
     lib.ucl_einsum.argtypes = [vp, c.c_char_p, i32, pp, c.POINTER(EinsumOpts), pp]
+    lib.ucl_repartition.argtypes = [vp, c.c_char_p, vp, pp]
     lib.ucl_keys_check_noalloc.argtypes = [i32, vp, i64, i32, vp, c.POINTER(i64), c.POINTER(i32)]
     lib.ucl_status_str.argtypes = [i32]
     lib.ucl_status_str.restype = c.c_char_p

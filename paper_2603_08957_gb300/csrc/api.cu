@@ -1065,4 +1065,249 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
     return st;
 }
 
+ucl_status ucl_repartition(ucl_ctx *ctx, const char *spec_text, const ucl_rel *in, ucl_rel **out) {
+    if (!out) return fail(ctx, UCL_ERR_ARG, "out is NULL");
+    *out = nullptr;
+    if (!ctx || !in || !spec_text) return fail(ctx, UCL_ERR_ARG, "NULL context, relation or spec");
+    if (in->ctx != ctx) return fail(ctx, UCL_ERR_ARG, "relation belongs to another context");
+    // ------------------------------------------------------------ plan
+    const std::string t(spec_text);
+    const size_t arrow = t.find("->");
+    if (arrow == std::string::npos) return fail(ctx, UCL_ERR_SPEC, "spec has no '->'");
+    const std::string lhs = t.substr(0, arrow), rhs = t.substr(arrow + 2);
+    auto lower = [](char c) { return (char)(c >= 'A' && c <= 'Z' ? c - 'A' + 'a' : c); };
+    // labels are named by their input-side letter; the output side is either
+    // "<keys>|<tile dims>" (input letters as written) or the input letters
+    // with their case changed to the new class (compared without case)
+    const size_t bar = rhs.find('|');
+    const bool explicit_form = bar != std::string::npos;
+    const std::string rhs_letters = explicit_form ? rhs.substr(0, bar) + rhs.substr(bar + 1) : rhs;
+    for (size_t a = 0; a < lhs.size(); ++a) {
+        if (!is_alpha(lhs[a])) return fail(ctx, UCL_ERR_SPEC, "labels must be letters");
+        for (size_t b = a + 1; b < lhs.size(); ++b)
+            if (lhs[a] == lhs[b] || (!explicit_form && lower(lhs[a]) == lower(lhs[b])))
+                return fail(ctx, UCL_ERR_SPEC,
+                            "a label appears twice on the input side (without '|' letters compare without case)");
+    }
+    for (char c : rhs_letters)
+        if (!is_alpha(c)) return fail(ctx, UCL_ERR_SPEC, "labels must be letters");
+    if (lhs.size() != rhs_letters.size()) return fail(ctx, UCL_ERR_SPEC, "both sides must hold the same labels");
+    struct RL {
+        char name;
+        bool in_up, out_up;
+        int in_pos, out_pos;
+        int64_t ext;
+    };
+    std::vector<RL> labs;
+    int iu = 0, il = 0;
+    for (char c : lhs) {
+        RL L{c, is_upper(c), false, is_upper(c) ? iu++ : il++, -1, 0};
+        labs.push_back(L);
+    }
+    if (iu != in->u || il != in->r)
+        return fail(ctx, UCL_ERR_SHAPE, "input side does not match the relation's key/tile arity");
+    int ou = 0, ol = 0;
+    for (size_t q = 0; q < rhs_letters.size(); ++q) {
+        const char c = rhs_letters[q];
+        RL *L = nullptr;
+        for (RL &M : labs)
+            if (explicit_form ? M.name == c : lower(M.name) == lower(c)) L = &M;
+        if (!L || L->out_pos >= 0) return fail(ctx, UCL_ERR_SPEC, "both sides must hold the same labels");
+        L->out_up = explicit_form ? q < bar : is_upper(c);
+        L->out_pos = L->out_up ? ou++ : ol++;
+    }
+    for (RL &L : labs) L.ext = L.in_up ? in->bounds[L.in_pos] : in->shape[L.in_pos];
+    auto by_out = [&](bool up) {
+        std::vector<const RL *> v(up ? ou : ol);
+        for (const RL &L : labs)
+            if (L.out_up == up) v[L.out_pos] = &L;
+        return v;
+    };
+    const std::vector<const RL *> oup = by_out(true), olow = by_out(false);
+    int64_t tile_out = 1, np = 1;
+    for (const RL *L : olow) tile_out *= L->ext;
+    for (const RL *L : oup)
+        if (!L->in_up) np *= L->ext;
+    if (tile_out >= (1ll << 31) || np >= (1ll << 31)) return fail(ctx, UCL_ERR_UNSUPPORTED, "output tile too large");
+    // output key packing (output order) and the kept-key packing (kept labels, output order)
+    KeyUnpack un{};
+    un.uw = ou;
+    int total = 0;
+    for (const RL *L : oup) total += bit_width(L->ext);
+    if (total > 64) return fail(ctx, UCL_ERR_UNSUPPORTED, "output key needs more than 64 bits");
+    RepartKeys rk{};
+    rk.uw = ou;
+    rk.np = np;
+    KeyPack kpack{};
+    int kbits_total = 0;
+    for (const RL *L : oup)
+        if (L->in_up) kbits_total += bit_width(L->ext);
+    {
+        int sh = total, ksh = kbits_total;
+        int64_t pdiv = np;
+        for (int q = 0; q < ou; ++q) {
+            const RL &L = *oup[q];
+            const int b = bit_width(L.ext);
+            sh -= b;
+            un.shift[q] = sh;
+            un.bits[q] = b;
+            rk.osh[q] = sh;
+            rk.promoted[q] = !L.in_up;
+            if (L.in_up) {
+                ksh -= b;
+                rk.ksh[q] = ksh;
+                rk.kbits[q] = b;
+                kpack.f[kpack.nf++] = KeyField{L.in_pos, ksh, b};
+            } else {
+                pdiv /= L.ext;
+                rk.pdiv[q] = pdiv;
+                rk.pext[q] = L.ext;
+            }
+        }
+    }
+    // element routing
+    RepartCopy pc{};
+    pc.r = in->r;
+    pc.u = in->u;
+    pc.tile_in = in->tile;
+    pc.tile_out = tile_out;
+    pc.np = np;
+    auto out_stride = [&](const RL &L) {
+        int64_t st = 1;
+        for (int q = ol - 1; q > L.out_pos; --q) st *= olow[q]->ext;
+        return st;
+    };
+    for (const RL &L : labs) {
+        if (L.in_up) {
+            pc.kstride[L.in_pos] = L.out_up ? 0 : out_stride(L);
+        } else {
+            pc.ext[L.in_pos] = L.ext;
+            pc.ostride[L.in_pos] = L.out_up ? 0 : out_stride(L);
+            if (L.out_up) pc.pstride[L.in_pos] = rk.pdiv[L.out_pos];
+        }
+    }
+    // kept labels lead the output key, in the input's leading columns' order?
+    bool kept_first = true, kept_leading = true;
+    {
+        bool seen_promoted = false;
+        int kq = 0;
+        for (const RL *L : oup) {
+            if (!L->in_up) seen_promoted = true;
+            else {
+                if (seen_promoted) kept_first = false;
+                if (L->in_pos != kq) kept_leading = false;
+                ++kq;
+            }
+        }
+    }
+    cudaSetDevice(ctx->device);
+    ucl_stats stats{};
+    ctx->launches = 0;
+    ucl_rel *R = nullptr;
+    ucl_status st;
+    if ((st = begin_timed_call(ctx))) return st;
+    try {
+        arena_reset(ctx);
+        record(ctx, 0);
+        int64_t *d_scal = (int64_t *)ws_get(ctx, 8 * sizeof(int64_t));
+        const int64_t n = in->n;
+        // distinct kept keys and each tuple's rank among them
+        int64_t kd = 0;
+        uint32_t *rank = nullptr;
+        uint64_t *dk = nullptr;
+        if (n > 0) {
+            rank = (uint32_t *)ws_get(ctx, 4 * n);
+            if (kpack.nf == 0) {
+                kd = 1;
+                check(cuda_check(ctx, cudaMemsetAsync(rank, 0, 4 * n, ctx->stream), "cudaMemsetAsync"));
+                record(ctx, 1);
+            } else {
+                uint64_t *kk = (uint64_t *)ws_get(ctx, 8 * n), *perm = nullptr;
+                launch_pack(ctx, in->keys, in->u, n, kpack, kk, KeyPack{}, nullptr);
+                if (!(in->sorted && kept_leading)) {
+                    uint64_t *vals = (uint64_t *)ws_get(ctx, 8 * n), *ka = (uint64_t *)ws_get(ctx, 8 * n),
+                             *va = (uint64_t *)ws_get(ctx, 8 * n);
+                    launch_iota(ctx, vals, n);
+                    if (radix_sort(ctx, kk, vals, ka, va, n, kbits_total)) { kk = ka; perm = va; } else perm = vals;
+                }
+                int64_t *flag = (int64_t *)ws_get(ctx, 8 * n), *excl = (int64_t *)ws_get(ctx, 8 * n);
+                launch_heads(ctx, kk, n, flag);
+                scan_i64(ctx, flag, excl, n, d_scal);
+                dk = (uint64_t *)ws_get(ctx, 8 * n);
+                launch_kept_rank(ctx, kk, flag, excl, perm, n, rank, dk);
+                record(ctx, 1);
+                check(sync_read(ctx, d_scal, 1, &kd));
+            }
+        } else {
+            record(ctx, 1);
+        }
+        const int64_t n_out = kd * np;
+        if (n_out >= (1ll << 31)) check(fail(ctx, UCL_ERR_UNSUPPORTED, "more than 2^31-1 output tuples"));
+        R = new_rel(ctx);
+        if (!R) check(fail(ctx, UCL_ERR_OOM, "host allocation failed"));
+        R->n = n_out;
+        R->u = ou;
+        R->r = ol;
+        for (int q = 0; q < ou; ++q) R->bounds[q] = oup[q]->ext;
+        for (int q = 0; q < ol; ++q) R->shape[q] = olow[q]->ext;
+        R->dtype = in->dtype;
+        R->tile = tile_out;
+        R->sorted = 1;
+        R->key_bits = total;
+        const size_t es = dsize(in->dtype);
+        if (n_out > 0) {
+            size_t tbytes = (size_t)n_out * tile_out * es;
+            size_t koff = (tbytes + 255) & ~(size_t)255;
+            R->own_bytes = koff + (size_t)n_out * ou * 4 + 4;
+            R->own_block = ctx_alloc(ctx, R->own_bytes);
+            if (!R->own_block) throw Oom();
+            R->tiles = R->own_block;
+            R->keys = (int32_t *)((char *)R->own_block + koff);
+            // output keys; slot order is key order when the kept labels lead
+            uint64_t *okey = (uint64_t *)ws_get(ctx, 8 * n_out);
+            uint32_t *pos = nullptr;
+            if (kept_first) {
+                launch_out_keys(ctx, dk, n_out, rk, okey, nullptr);
+                launch_out_place(ctx, okey, nullptr, n_out, un, nullptr, R->keys);
+            } else {
+                uint64_t *iota = (uint64_t *)ws_get(ctx, 8 * n_out), *ka = (uint64_t *)ws_get(ctx, 8 * n_out),
+                         *va = (uint64_t *)ws_get(ctx, 8 * n_out);
+                launch_out_keys(ctx, dk, n_out, rk, okey, iota);
+                if (radix_sort(ctx, okey, iota, ka, va, n_out, total)) { okey = ka; iota = va; }
+                pos = (uint32_t *)ws_get(ctx, 4 * n_out);
+                launch_out_place(ctx, okey, iota, n_out, un, pos, R->keys);
+            }
+            record(ctx, 2);
+            // zero-filled tiles, then every input element to its place
+            check(cuda_check(ctx, cudaMemsetAsync(R->tiles, 0, tbytes, ctx->stream), "cudaMemsetAsync"));
+            launch_repart_scatter(ctx, in->tiles, in->dtype, in->keys, rank, pos, n, pc, R->tiles);
+            record(ctx, 3);
+        } else {
+            record(ctx, 2);
+            record(ctx, 3);
+        }
+        record(ctx, 4);
+        check(cuda_check(ctx, cudaGetLastError(), "kernel launch"));
+        stats.n_pairs = n;
+        stats.n_segments = n_out;
+        stats.flops = 0.0;
+        stats.bytes_contract = (double)n * in->tile * es + (double)n_out * tile_out * es + 4.0 * n * in->u +
+                               4.0 * n_out * ou;
+        stats.path = UCL_PATH_SIMT;
+        stats.launches = ctx->launches;
+        stats.timed = ctx->cur_ev != nullptr;
+        ctx->last = stats;
+        *out = R;
+        R = nullptr;
+        ctx->err.clear();
+        st = UCL_OK;
+    } catch (Oom &) {
+        st = fail(ctx, UCL_ERR_OOM, "device allocation failed");
+    } catch (Fail &f) {
+        st = f.st;
+    }
+    if (R) ucl_relation_destroy(R);
+    return st;
+}
+
 }  // extern "C"

@@ -201,6 +201,34 @@ void launch_segments3(ucl_ctx *ctx, const uint64_t *pk, const uint64_t *pv, cons
                       const int64_t *seg_excl, int64_t P, int64_t S, KeyUnpack un, const int ord[3],
                       int32_t *out_keys, int64_t *seg_start, uint32_t *const idx[3]);
 
+// ---- repartition (repartition.cu)
+// Output key of slot r * np + p: field q (output order) is promoted label q's
+// mixed-radix digit of p (p / pdiv % pext) or a kept label's field of the r-th
+// distinct kept key (bits at ksh); it lands at osh in the packed output key.
+struct RepartKeys {
+    int uw;
+    int promoted[kMaxCols];
+    int ksh[kMaxCols], kbits[kMaxCols], osh[kMaxCols];
+    int64_t pdiv[kMaxCols], pext[kMaxCols];
+    int64_t np;
+};
+// Where an input element goes: per input tile dim its extent, its stride in
+// the output tile (kept-lower labels) and its weight in p (promoted labels);
+// per input key column its stride in the output tile (demoted labels, else 0).
+struct RepartCopy {
+    int r, u;
+    int64_t ext[kMaxCols], ostride[kMaxCols], pstride[kMaxCols], kstride[kMaxCols];
+    int64_t tile_in, tile_out, np;
+};
+void launch_kept_rank(ucl_ctx *ctx, const uint64_t *kk, const int64_t *flag, const int64_t *excl,
+                      const uint64_t *perm, int64_t n, uint32_t *rank, uint64_t *dk);
+void launch_out_keys(ucl_ctx *ctx, const uint64_t *dk, int64_t n_out, const RepartKeys &rk, uint64_t *okey,
+                     uint64_t *iota);
+void launch_out_place(ucl_ctx *ctx, const uint64_t *okey_sorted, const uint64_t *perm, int64_t n_out,
+                      const KeyUnpack &un, uint32_t *pos, int32_t *out_keys);
+void launch_repart_scatter(ucl_ctx *ctx, const void *in, ucl_dtype dt, const int32_t *keys, const uint32_t *rank,
+                           const uint32_t *pos, int64_t n, const RepartCopy &pc, void *out);
+
 // ---- contraction (contract_simt.cu / contract_tc.cu)
 struct ContractArgs {
     const void *U;

@@ -164,6 +164,12 @@ class Context:
                                         ctypes.byref(h)))
         return Relation(self, h)
 
+    def repartition(self, spec: str, rel: "Relation") -> "Relation":
+        """Change a relation's upper/lower split (see include/ucl.h)."""
+        h = ctypes.c_void_p()
+        self._check(self.lib.ucl_repartition(self.handle, spec.encode(), rel.handle, ctypes.byref(h)))
+        return Relation(self, h)
+
 
 class Relation:
     """Handle of a tensor-relation living on the GPU."""

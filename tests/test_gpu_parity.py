@@ -482,3 +482,82 @@ def test_tc3_layouts(ctx, spec, perm, order, elay):
     ref2 = oracle_ref(spec, rels, epi="relu", scale=0.5)
     out2 = ctx.einsum(spec, *(gpu_rel(ctx, r) for r in rels), path="tc", out_dtype="bf16", epi="relu", scale=0.5)
     assert_parity(out2, ref2, torch.bfloat16, scale=0.5)
+
+
+# ------------------------------------------------------------ repartition
+
+from oracle.repartition import repartition as oracle_repartition  # noqa: E402
+
+REPART_CASES = [
+    # (dense labels, extents, upper labels of the input, output side of the spec)
+    ("ij", {"i": 5, "j": 4}, {"i"}, "iJ"),                     # rows -> columns
+    ("ijk", {"i": 3, "j": 4, "k": 2}, {"i"}, "IjK"),            # decompose only
+    ("ijk", {"i": 3, "j": 4, "k": 2}, {"i", "j"}, "iJk"),       # stack only
+    ("ijk", {"i": 3, "j": 4, "k": 2}, {"j", "k"}, "Ijk"),       # both
+    ("ijk", {"i": 3, "j": 4, "k": 2}, {"i"}, "Ikj"),            # tile dims reordered
+    ("ijk", {"i": 3, "j": 4, "k": 2}, {"j", "k"}, "KiJ"),       # promoted label between kept ones
+    ("ijk", {"i": 3, "j": 4, "k": 2}, set(), "IJK"),            # one dense tuple -> scalars
+    ("ijk", {"i": 3, "j": 4, "k": 2}, {"i", "j", "k"}, "kji"),  # scalars -> one dense tuple
+    ("ijkl", {"i": 70, "j": 3, "k": 40, "l": 5}, {"i", "k"}, "KjIl"),   # several tiles' worth of keys
+]
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("labels,ext,src,rhs", REPART_CASES)
+def test_repartition_matches_oracle(ctx, labels, ext, src, rhs, dtype):
+    """Every output key and value bit-exact against the oracle (values are
+    copies), with the input's tuples in key order and shuffled."""
+    rng = np.random.default_rng(abs(hash((labels, rhs))) % 2**31)
+    dense = random_sparse(rng, [ext[c] for c in labels], density=0.4, block_axes=range(len(labels)))
+    # the oracle sees exactly the values the GPU holds
+    dense = _bf16_exact(dense) if dtype == torch.bfloat16 else dense.astype(np.float32).astype(np.float64)
+    keys, bounds, tiles = decompose(dense, labels, src)
+    lhs = "".join(c.upper() for c in labels if c in src) + "".join(c for c in labels if c not in src)
+    spec = lhs + "->" + rhs
+    want_k, want_b, want_t = oracle_repartition(spec, (keys, bounds, tiles))
+    perm = rng.permutation(len(keys))
+    for k, t in ((keys, tiles), (keys[perm], tiles[perm])):
+        rel = gpu_rel(ctx, (k.astype(np.int32), tuple(int(b) for b in bounds), torch.from_numpy(t).to(dtype)))
+        out = ctx.repartition(spec, rel)
+        gk, gt = out.download()
+        assert out.bounds == tuple(want_b)
+        assert np.array_equal(gk.reshape(want_k.shape), want_k)
+        np.testing.assert_array_equal(gt.to(torch.float64).numpy().reshape(want_t.shape), want_t)
+
+
+def test_repartition_empty_and_errors(ctx):
+    empty = gpu_rel(ctx, (np.zeros((0, 1), np.int32), (4,), torch.zeros((0, 3))))
+    out = ctx.repartition("Ij->iJ", empty)
+    assert out.n == 0 and out.bounds == (3,) and out.shape == (4,)
+    R = gpu_rel(ctx, (np.array([[1]], np.int32), (2,), torch.ones((1, 3))))
+    for bad, err in [("Ij->Ik", "UCL_ERR_SPEC"), ("IJj->IJj", "UCL_ERR_SPEC"), ("IJ->IJ", "UCL_ERR_SHAPE"),
+                     ("Ij", "UCL_ERR_SPEC"), ("Ij->I|jj", "UCL_ERR_SPEC"), ("Ij->I|j|", "UCL_ERR_SPEC")]:
+        with pytest.raises(UclError, match=err):
+            ctx.repartition(bad, R)
+    # no key labels stay upper: no sync, every promoted index gets a tuple
+    out = ctx.repartition("Ij->iJ", R)
+    k, t = out.download()
+    assert k[:, 0].tolist() == [0, 1, 2]
+    assert t.tolist() == [[0.0, 1.0]] * 3
+
+
+def test_repartition_round_trip_full_size(ctx):
+    """The message-passing X (128 x 100000 bf16 as 1563 tiles [f][j]) split
+    into 128-row vectors keyed (F, J) and stacked back: bit-identical, and
+    the split relation matches the oracle on sampled tuples."""
+    w = workloads.gnn_chain(seed=0, n=100_000, device="cpu")
+    kx, bx, tx = w["X"]
+    X = gpu_rel(ctx, w["X"])
+    V = ctx.repartition("Jfj->fJ|j", X)
+    assert V.n == 128 * len(kx) and V.shape == (64,)
+    back = ctx.repartition("FJj->J|Fj", V)
+    bk, bt = back.download()
+    assert np.array_equal(bk, kx)
+    assert torch.equal(bt, tx)
+    vk, vt = V.download()
+    rng = np.random.default_rng(1)
+    rows = np.sort(rng.choice(len(kx), size=6, replace=False))
+    want_k, _, want_t = oracle_repartition("Jfj->fJ|j", (kx[rows], bx, tx[rows].to(torch.float64).numpy()))
+    got = {tuple(k): t for k, t in zip(vk.tolist(), vt.to(torch.float64).numpy())}
+    for k, t in zip(want_k.tolist(), want_t):
+        np.testing.assert_array_equal(got[tuple(k)], t)

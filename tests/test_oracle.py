@@ -402,3 +402,25 @@ def test_repartition_identity_and_errors():
     for bad in ["Ij->Ik", "Ij->IJj", "Ij", "IJj->Ij", "Ij->I"]:
         with pytest.raises(RepartitionError):
             repartition(bad, rel)
+
+
+def test_repartition_explicit_form_with_tile_and_offset_labels():
+    """A reshaped dense index keeps its tile index J and offset j as two
+    labels; the explicit "<keys>|<tile dims>" form names them apart.  Here X
+    stored as [f][j] tiles keyed J becomes j-vectors keyed (f, J), and back."""
+    rng = np.random.default_rng(9)
+    dense = random_sparse(rng, [5, 3, 4], density=0.5, block_axes=(0, 1, 2))   # axes J, f, j
+    ext = {"J": 5, "f": 3, "j": 4}
+    rel = decompose(dense, "Jfj", {"J"})
+    keys, bounds, tiles = repartition("Jfj->fJ|j", rel)
+    assert bounds == (3, 5) and tiles.shape[1:] == (4,)
+    back = recompose(keys, tiles, "fJj", {"f", "J"}, ext)
+    np.testing.assert_array_equal(np.transpose(back, [1, 0, 2]), dense)
+    assert len(keys) == 3 * len(rel[0])    # every f for every J present
+    k2, b2, t2 = repartition("FJj->J|Fj", (keys, bounds, tiles))
+    np.testing.assert_array_equal(k2, rel[0])
+    np.testing.assert_array_equal(t2, rel[2])
+    with pytest.raises(RepartitionError):
+        repartition("Jfj->fJ", rel)      # case form cannot tell J from j
+    with pytest.raises(RepartitionError):
+        repartition("Jfj->fj|J|", rel)
