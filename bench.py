@@ -65,6 +65,7 @@ class Workload:
     name = ""
     desc = ""
     dtype = "bf16"
+    metric, unit, scale = None, None, 1e12   # None: the EinSum metric (TFLOP/s)
     big = True          # inputs larger than L2 (no flush needed)
     hostable = True     # inputs small enough to stage through pinned host memory every step
     flops_per_tuple = 0.0
@@ -242,7 +243,47 @@ class Spgemm(_Binary):
         self.l2 = "inputs smaller than L2: 256 MB L2 flush before every timed step (outside the events)"
 
 
-WORKLOADS = {"gnn": GnnChain, "blocksparse": Blocksparse, "mttkrp": Mttkrp, "spgemm": Spgemm, "gnn2": Gnn2}
+class Repart(Workload):
+    """Repartition (Sec. 5's representation change): the message-passing Y
+    (358136 64x64 bf16 tiles keyed (J, K)) split into 64-wide row vectors
+    keyed (J, K, j), then stacked back into tiles."""
+    name = "repart"
+    metric = "effective GB/s of tiles and keys moved per repartition"
+    unit = "GB/s"
+    scale = 1e9
+
+    def __init__(self, dev, args):
+        super().__init__(dev, args)
+        import workloads
+        self.w = w = workloads.gnn_chain(seed=0, n=args.vertices, device=dev)
+        self.inputs = {"Y": (w["Y"][0], w["Y"][1], w["Y"][2].to(dev))}
+        self.chain = [("V", "JKjk->JKj|k", ["Y"], {"op": "repartition"}),
+                      ("B", "JKLk->JK|Lk", ["V"], {"op": "repartition"})]
+        ny = len(w["Y"][0])
+        self.desc = (f"repartition of the message-passing Y ({ny} nonempty 64x64 bf16 tiles keyed (J, K)) into "
+                     f"{64 * ny} row vectors keyed (J, K, j) and back; specs JKjk->JKj|k then JKLk->JK|Lk")
+        self.l2 = f"inputs larger than L2 (Y {ny * 8192 / 1e9:.1f} GB); no flush"
+
+    def oracle_time(self, target, seed):
+        """The oracle's repartition of a random subset of Y's tuples: (bytes
+        moved, seconds, tuples, tuples)."""
+        from oracle.repartition import repartition
+        import workloads
+        w = self.w
+        ky = w["Y"][0]
+        rows = np.sort(np.random.default_rng(seed).choice(len(ky), size=min(len(ky), max(1, target)),
+                                                          replace=False))
+        if not hasattr(self, "_edges"):
+            self._edges = [e.cpu().numpy() if torch.is_tensor(e) else e for e in w["edges"]]
+        yt = workloads.adjacency_tiles_subset(self._edges[0], self._edges[1], w["n"], w["t"], ky[rows])
+        t0 = time.perf_counter()
+        repartition("JKjk->JKj|k", (ky[rows], w["Y"][1], yt))
+        dt = time.perf_counter() - t0
+        moved = len(rows) * (2 * 64 * 64 * 2 + 2 * 4 + 64 * 3 * 4)
+        return moved, dt, len(rows), len(rows)
+
+
+WORKLOADS = {"gnn": GnnChain, "repart": Repart, "blocksparse": Blocksparse, "mttkrp": Mttkrp, "spgemm": Spgemm, "gnn2": Gnn2}
 
 
 # ---------------------------------------------------------------- helpers
@@ -352,6 +393,8 @@ def allreduce_max(x, world, device):
 def time_oracle(W, target, seed):
     """The oracle on the first EinSum restricted to random output keys holding
     about `target` joined tuples: (FLOPs, seconds, tuples, keys)."""
+    if hasattr(W, "oracle_time"):
+        return W.oracle_time(target, seed)
     import oracle
     spec, rels, sk, tuples = W.sample(target, seed)
     t0 = time.perf_counter()
@@ -370,7 +413,7 @@ def cpu_baseline(W, seconds=12.0):
     target = max(16, int(oracle_rate(W) * seconds))
     flops, dt, tuples, nk = time_oracle(W, target, seed=1)
     spec = W.chain[0][1]
-    return {"value": flops / dt / 1e12, "unit": UNIT, "cores": 1, "kind": "oracle",
+    return {"value": flops / dt / W.scale, "unit": W.unit or UNIT, "cores": 1, "kind": "oracle",
             "sample": f"first EinSum {spec} restricted to {nk} random output keys ({tuples} joined tuples, "
                       f"{dt:.1f} s single-threaded fp64 C); FLOPs of those tuples / time"}
 
@@ -390,16 +433,17 @@ def run_reference(args, world, rank):
         tot_f += f
         tot_t += dt
         tot_p += p
-    v = tot_f / tot_t / 1e12
+    v = tot_f / tot_t / W.scale
     spec = W.chain[0][1]
     sample = (f"each step: first EinSum {spec} on random output keys totalling ~{per_step} joined tuples "
               f"({tot_p} over {args.steps} steps), single-threaded fp64 C oracle")
-    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+    unit = W.unit or UNIT
+    line = {"impl": "reference", "metric": W.metric or METRIC, "value": v, "unit": unit, "n_gpus": 1, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1e3 * tot_t / max(1, args.steps), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": W.desc, "l2": "n/a (CPU)"},
-            "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
-            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+            "cpu_baseline": {"value": v, "unit": unit, "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": v, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
 
@@ -419,7 +463,8 @@ def stage_roofline(W, arity, stats, tim, pk):
         s = stats[c]
         P, S = s["n_pairs"], s["n_segments"]
         key_bytes = sum(arity[i][0] * arity[i][1] * 4 for i in ins)
-        uw = sum(ch.isupper() for ch in spec.split("->")[1])
+        rhs = spec.split("->")[1]
+        uw = len(rhs.split("|")[0]) if "|" in rhs else sum(ch.isupper() for ch in rhs)
         sort_bytes = key_bytes + 32.0 * P + 4.0 * len(ins) * P + 4.0 * uw * S
         ms = tim[c::L].mean(axis=0) if len(tim) else np.full(4, np.nan)
         sj = float(ms[0] + ms[1])
@@ -450,7 +495,10 @@ def run_ucl(args, world, rank, local):
     def run_chain(env, collect=None):
         made = []
         for name, spec, ins, opts in W.chain:
-            r = ctx.einsum(spec, *[env[i] for i in ins], path=path, **opts)
+            if opts.get("op") == "repartition":
+                r = ctx.repartition(spec, env[ins[0]])
+            else:
+                r = ctx.einsum(spec, *[env[i] for i in ins], path=path, **opts)
             if collect is not None:
                 collect.append(ctx.last_stats())
                 arity[name] = (r.n, r.u)
@@ -470,6 +518,8 @@ def run_ucl(args, world, rank, local):
         step()
     torch.cuda.synchronize()
     flops_step = sum(s["flops"] for s in stats)
+    if W.metric:   # a data-movement workload: its unit is bytes moved
+        flops_step = sum(s["bytes_contract"] for s in stats)
     launches_step = sum(s["launches"] for s in stats)
 
     steps = args.steps
@@ -510,7 +560,7 @@ def run_ucl(args, world, rank, local):
     tim = ctx.timings(reset=True)
     ctx.set_timing(False)
     ms_max = allreduce_max(ms, world, dev)
-    value = flops_step * steps * world / (ms_max / 1e3) / 1e12
+    value = flops_step * steps * world / (ms_max / 1e3) / W.scale
 
     pk = peaks()
     per_einsum = stage_roofline(W, arity, stats, tim, pk)
@@ -519,6 +569,8 @@ def run_ucl(args, world, rank, local):
     d, s = per_einsum[dom], stats[dom]
     kfile = {"tc": "contract_tc3" if len(W.chain[dom][2]) == 3 else "contract_tc",
              "simt": "contract_simt"}.get(s["path"], "contract_simt")
+    if W.chain[dom][3].get("op") == "repartition":
+        kfile = "repartition"
     roof = {"bound": "hbm", "achieved": d["contract"]["GB/s"], "peak": pk["hbm_gbs"], "unit": "GB/s",
             "frac": d["contract"]["frac"], "traffic": contract_traffic(kfile, W.name, s["n_pairs"]),
             "kernel": f"{kfile} ({d['spec']})", "avg_launch_ms": d["contract"]["ms"],
@@ -552,7 +604,7 @@ def run_ucl(args, world, rank, local):
         torch.cuda.synchronize()
         te = (time.perf_counter() - t0) / ne
         te = allreduce_max(te, world, dev)
-        e2e = {"value": flops_step * world / te / 1e12, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+        e2e = {"value": flops_step * world / te / W.scale, "unit": W.unit or UNIT, "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(d2h), "ms_per_step": te * 1e3}
         del host
 
@@ -561,7 +613,7 @@ def run_ucl(args, world, rank, local):
         cpu = cpu_baseline(W, seconds=args.cpu_seconds)
 
     if rank == 0:
-        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps,
+        line = {"metric": W.metric or METRIC, "value": value, "unit": W.unit or UNIT, "n_gpus": world, "steps": steps,
                 "warmup": args.warmup, "ms_per_step": ms_max / steps, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": W.dtype, "data": "synthetic",
                 "config": {"workload": W.desc, "pairs": [s["n_pairs"] for s in stats],

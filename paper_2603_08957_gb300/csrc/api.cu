@@ -1278,8 +1278,12 @@ ucl_status ucl_repartition(ucl_ctx *ctx, const char *spec_text, const ucl_rel *i
                 launch_out_place(ctx, okey, iota, n_out, un, pos, R->keys);
             }
             record(ctx, 2);
-            // zero-filled tiles, then every input element to its place
-            check(cuda_check(ctx, cudaMemsetAsync(R->tiles, 0, tbytes, ctx->stream), "cudaMemsetAsync"));
+            // every input element to its place; positions no element maps to
+            // exist only when labels are stacked, and are zero
+            bool stacked = false;
+            for (const RL &L : labs) stacked |= L.in_up && !L.out_up;
+            if (stacked)
+                check(cuda_check(ctx, cudaMemsetAsync(R->tiles, 0, tbytes, ctx->stream), "cudaMemsetAsync"));
             launch_repart_scatter(ctx, in->tiles, in->dtype, in->keys, rank, pos, n, pc, R->tiles);
             record(ctx, 3);
         } else {

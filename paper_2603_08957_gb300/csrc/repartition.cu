@@ -99,6 +99,42 @@ __global__ void scatter_kernel(const T *__restrict__ in, const int32_t *__restri
     }
 }
 
+// Fast path when the input's innermost tile dim stays the output's innermost
+// one: its runs of E elements are contiguous on both sides, so they move as
+// V-element vectors (VT).  A group of G lanes takes one tuple at a time: the
+// tuple's key offset and slot base are read once, then the lanes walk the
+// tile's vectors (32-bit index math inside a tile).
+template <typename VT, int G>
+__global__ void scatter_runs_kernel(const VT *__restrict__ in, const int32_t *__restrict__ keys,
+                                    const uint32_t *__restrict__ rank, const uint32_t *__restrict__ pos, int64_t n,
+                                    RepartCopy pc, int vpr, VT *out) {
+    const int sub = threadIdx.x % G;
+    const int64_t groups = ((int64_t)gridDim.x * blockDim.x) / G;
+    const uint32_t vecs = (uint32_t)(pc.tile_in / (pc.ext[pc.r - 1] / vpr));   // vectors per input tile
+    const int64_t vpo = pc.tile_out / (pc.ext[pc.r - 1] / vpr);                // vectors per output tile
+    const int64_t V = pc.ext[pc.r - 1] / vpr;                                  // elements per vector
+    for (int64_t t = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) / G; t < n; t += groups) {
+        int64_t koff = 0;
+        for (int c = 0; c < pc.u; ++c) koff += (int64_t)keys[t * pc.u + c] * pc.kstride[c];
+        const int64_t base = (int64_t)rank[t] * pc.np;
+        const VT *src = in + t * (int64_t)vecs;
+        for (uint32_t v = sub; v < vecs; v += G) {
+            uint32_t run = v / (uint32_t)vpr;
+            const uint32_t w = v - run * (uint32_t)vpr;
+            int64_t off = koff, p = 0;
+            for (int d = pc.r - 2; d >= 0; --d) {
+                const uint32_t e = (uint32_t)pc.ext[d];
+                const uint32_t idx = run % e;
+                run /= e;
+                off += (int64_t)idx * pc.ostride[d];
+                p += (int64_t)idx * pc.pstride[d];
+            }
+            const int64_t o = pos ? (int64_t)pos[base + p] : base + p;
+            out[o * vpo + off / V + w] = src[v];
+        }
+    }
+}
+
 }  // namespace
 
 void launch_kept_rank(ucl_ctx *ctx, const uint64_t *kk, const int64_t *flag, const int64_t *excl,
@@ -126,6 +162,44 @@ void launch_out_place(ucl_ctx *ctx, const uint64_t *okey_sorted, const uint64_t 
 void launch_repart_scatter(ucl_ctx *ctx, const void *in, ucl_dtype dt, const int32_t *keys, const uint32_t *rank,
                            const uint32_t *pos, int64_t n, const RepartCopy &pc, void *out) {
     if (n <= 0 || pc.tile_in <= 0) return;
+    if (pc.r > 0 && pc.ostride[pc.r - 1] == 1 && pc.pstride[pc.r - 1] == 0) {
+        // runs of the innermost dim: widest vector dividing the run (in bytes)
+        // that both tile arrays' alignment allows
+        const int es = dt == UCL_BF16 ? 2 : 4;
+        const int64_t run_bytes = pc.ext[pc.r - 1] * es;
+        const uintptr_t al = reinterpret_cast<uintptr_t>(in) | reinterpret_cast<uintptr_t>(out);
+        int vb = 16;
+        while (vb > es && (run_bytes % vb || al % vb)) vb >>= 1;
+        const int vpr = (int)(run_bytes / vb);   // vectors per run
+        const int64_t vecs = pc.tile_in * es / vb;
+        const int G = vecs >= 32 ? 32 : (vecs >= 16 ? 16 : (vecs >= 8 ? 8 : (vecs >= 4 ? 4 : (vecs >= 2 ? 2 : 1))));
+        const int64_t want = (n * G + kThreads - 1) / kThreads;
+        const int g = (int)(want < (int64_t)ctx->sm_count * 32 ? (want < 1 ? 1 : want) : (int64_t)ctx->sm_count * 32);
+#define UCL_RUNS(VT)                                                                                             \
+    switch (G) {                                                                                                 \
+        case 32: scatter_runs_kernel<VT, 32><<<g, kThreads, 0, ctx->stream>>>(                                   \
+            static_cast<const VT *>(in), keys, rank, pos, n, pc, vpr, static_cast<VT *>(out)); break;            \
+        case 16: scatter_runs_kernel<VT, 16><<<g, kThreads, 0, ctx->stream>>>(                                   \
+            static_cast<const VT *>(in), keys, rank, pos, n, pc, vpr, static_cast<VT *>(out)); break;            \
+        case 8: scatter_runs_kernel<VT, 8><<<g, kThreads, 0, ctx->stream>>>(                                     \
+            static_cast<const VT *>(in), keys, rank, pos, n, pc, vpr, static_cast<VT *>(out)); break;            \
+        case 4: scatter_runs_kernel<VT, 4><<<g, kThreads, 0, ctx->stream>>>(                                     \
+            static_cast<const VT *>(in), keys, rank, pos, n, pc, vpr, static_cast<VT *>(out)); break;            \
+        case 2: scatter_runs_kernel<VT, 2><<<g, kThreads, 0, ctx->stream>>>(                                     \
+            static_cast<const VT *>(in), keys, rank, pos, n, pc, vpr, static_cast<VT *>(out)); break;            \
+        default: scatter_runs_kernel<VT, 1><<<g, kThreads, 0, ctx->stream>>>(                                    \
+            static_cast<const VT *>(in), keys, rank, pos, n, pc, vpr, static_cast<VT *>(out)); break;            \
+    }
+        switch (vb) {
+            case 16: UCL_RUNS(uint4) break;
+            case 8: UCL_RUNS(uint2) break;
+            case 4: UCL_RUNS(uint32_t) break;
+            default: UCL_RUNS(uint16_t) break;
+        }
+#undef UCL_RUNS
+        ctx->launches++;
+        return;
+    }
     const int g = grid_for(ctx, n * pc.tile_in);
     if (dt == UCL_BF16)
         scatter_kernel<uint16_t><<<g, kThreads, 0, ctx->stream>>>(static_cast<const uint16_t *>(in), keys, rank, pos,
