@@ -561,3 +561,34 @@ def test_repartition_round_trip_full_size(ctx):
     got = {tuple(k): t for k, t in zip(vk.tolist(), vt.to(torch.float64).numpy())}
     for k, t in zip(want_k.tolist(), want_t):
         np.testing.assert_array_equal(got[tuple(k)], t)
+
+
+def test_random_graph_contraction_sampled(ctx):
+    """A message-passing-shaped EinSum on a uniform random graph: 600 vertex
+    blocks, ~90k random (J, K) tiles over 1000 destination blocks (one in five
+    empty).  The full key set and the values of 48 sampled keys (incl. the
+    largest) against the oracle; then a second run, bit-identical."""
+    rng = np.random.default_rng(11)
+    nJ, nK, f, t = 600, 1000, 128, 64
+    live = np.nonzero(rng.random(nK) < 0.8)[0]
+    codes = np.unique(rng.integers(0, nJ, 120_000) * nK + rng.choice(live, 120_000))
+    ky = np.stack([codes // nK, codes % nK], 1).astype(np.int32)
+    g = torch.Generator().manual_seed(5)
+    Xt = torch.randn((nJ, f, t), generator=g).to(torch.bfloat16)
+    Yt = (torch.rand((len(ky), t, t), generator=g) < 0.1).to(torch.bfloat16)
+    X = (np.arange(nJ, dtype=np.int32)[:, None], (nJ,), Xt)
+    Y = (ky, (nJ, nK), Yt)
+    spec = "fJj,JjKk->Kkf"
+    out = ctx.einsum(spec, gpu_rel(ctx, X), gpu_rel(ctx, Y), out_dtype="bf16")
+    assert ctx.last_stats()["n_pairs"] == len(ky) >= 1 << 16
+    keys, _ = out.download()
+    assert np.array_equal(keys[:, 0], np.unique(ky[:, 1]))
+    cnt = np.bincount(ky[:, 1], minlength=nK)
+    sk = np.unique(np.concatenate([rng.choice(np.nonzero(cnt)[0], 47, replace=False), [np.argmax(cnt)]]))
+    m = np.isin(ky[:, 1], sk)
+    ref = oracle_ref(spec, [X, (ky[m], (nJ, nK), Yt[torch.from_numpy(np.nonzero(m)[0])])],
+                     sample_keys=sk[:, None].astype(np.int32))
+    sel = np.searchsorted(keys[:, 0], sk)
+    assert_parity(out, ref, torch.bfloat16, select=sel)
+    out2 = ctx.einsum(spec, gpu_rel(ctx, X), gpu_rel(ctx, Y), out_dtype="bf16")
+    assert torch.equal(out.download()[1], out2.download()[1])
