@@ -401,8 +401,15 @@ bool plan_tc3(const Spec &s, ucl_rel *const *in, const KeyPlan &kp, Tc3Plan &tp,
 
 size_t dsize(ucl_dtype d) { return d == UCL_BF16 ? 2 : 4; }
 
-void arena_reset(ucl_ctx *ctx) {
-    Arena &A = ctx->arena;
+// Take the next workspace arena in turn.  The stream in use first waits until
+// main has finished the call that used it last; a grown arena is merged into
+// one block.
+int arena_begin(ucl_ctx *ctx) {
+    const int a = ctx->arena_next;
+    ctx->arena_next = (a + 1) % ucl_ctx::kArenas;
+    ctx->arena = &ctx->arenas[a];
+    if (ctx->stream != ctx->main) cudaStreamWaitEvent(ctx->stream, ctx->arena_done[a], 0);
+    Arena &A = *ctx->arena;
     if (A.blocks.size() > 1) {
         size_t total = A.total();
         for (auto &b : A.blocks) ctx_free(ctx, b.ptr, b.size);
@@ -411,7 +418,15 @@ void arena_reset(ucl_ctx *ctx) {
         if (p) A.blocks.push_back({p, total});
     }
     A.used = 0;
+    return a;
 }
+
+// Events of a timed call: [0] key stage start, [1] after the join count,
+// [2] after the segments (key stream), [3] before the contraction, [4] after
+// it, [5] after the fixup (main).  Stage s spans events kStageFrom[s] ..
+// kStageFrom[s] + 1.
+constexpr int kCallEvents = 6;
+constexpr int kStageFrom[UCL_NSTAGES] = {0, 1, 3, 4};
 
 void record(ucl_ctx *ctx, int i) {
     if (ctx->cur_ev) cudaEventRecord(ctx->cur_ev[i], ctx->stream);
@@ -421,7 +436,7 @@ void record(ucl_ctx *ctx, int i) {
 ucl_status begin_timed_call(ucl_ctx *ctx) {
     ctx->cur_ev = nullptr;
     if (!ctx->timing) return UCL_OK;
-    const size_t per = UCL_NSTAGES + 1, need = per * (ctx->ev_calls + 1);
+    const size_t per = kCallEvents, need = per * (ctx->ev_calls + 1);
     while (ctx->ev_pool.size() < need) {
         cudaEvent_t e;
         ucl_status st = cuda_check(ctx, cudaEventCreate(&e), "cudaEventCreate");
@@ -433,28 +448,60 @@ ucl_status begin_timed_call(ucl_ctx *ctx) {
     return UCL_OK;
 }
 
-// Read n int64 device scalars after draining the stream.  Word 0 of the
-// device status holds error bits raised by any earlier kernel of this context
-// (sticky until reported here); word 1 holds validation flags (returned in
-// *flags, cleared).
+// Read n int64 device scalars after draining the stream in use.  Word 1 of
+// the device status holds validation flags (returned in *flags, cleared);
+// word 2 holds error bits raised by earlier main-stream kernels of this
+// context, sticky until a read on main reports and clears them (a key-stream
+// read reports them if already set but leaves the word to main, whose kernels
+// may still be writing it).
 ucl_status sync_read(ucl_ctx *ctx, const int64_t *dev, int n, int64_t *host, uint32_t *flags = nullptr) {
     cudaError_t e = cudaSuccess;
     if (n > 0) e = cudaMemcpyAsync(ctx->h_pinned, dev, sizeof(int64_t) * n, cudaMemcpyDeviceToHost, ctx->stream);
     if (e == cudaSuccess)
-        e = cudaMemcpyAsync(ctx->h_pinned + 7, ctx->d_status, 2 * sizeof(uint32_t), cudaMemcpyDeviceToHost,
+        e = cudaMemcpyAsync(ctx->h_pinned + 6, ctx->d_status, 4 * sizeof(uint32_t), cudaMemcpyDeviceToHost,
                             ctx->stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize(ctx->stream);
     if (e != cudaSuccess) return cuda_check(ctx, e, "stream sync");
     e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_check(ctx, e, "kernel launch");
     for (int i = 0; i < n; ++i) host[i] = ctx->h_pinned[i];
-    uint32_t words[2];
-    memcpy(words, ctx->h_pinned + 7, sizeof(words));
+    uint32_t words[4];
+    memcpy(words, ctx->h_pinned + 6, sizeof(words));
     if (flags) *flags = words[1];
-    if (words[0] | words[1]) cudaMemsetAsync(ctx->d_status, 0, 2 * sizeof(uint32_t), ctx->stream);
-    if (words[0] & kStTimeout) return fail(ctx, UCL_ERR_TIMEOUT, "a device-side wait timed out");
-    if (words[0] & kStBadIndex) return fail(ctx, UCL_ERR_CUDA, "a device-side bounds check failed");
+    const bool on_main = ctx->stream == ctx->main;
+    if (words[1]) cudaMemsetAsync(ctx->d_status + 1, 0, sizeof(uint32_t), ctx->stream);
+    if (words[2] && on_main) cudaMemsetAsync(ctx->d_status + 2, 0, sizeof(uint32_t), ctx->stream);
+    if (words[2] & kStTimeout) return fail(ctx, UCL_ERR_TIMEOUT, "a device-side wait timed out");
+    if (words[2] & kStBadIndex) return fail(ctx, UCL_ERR_CUDA, "a device-side bounds check failed");
     return UCL_OK;
+}
+
+// Key stage of ucl_einsum on the key stream; back to main with main ordered
+// after everything the key stream did so far.
+void to_key_stream(ucl_ctx *ctx) { ctx->stream = ctx->kstream; }
+void to_main(ucl_ctx *ctx) {
+    if (ctx->stream == ctx->main) return;
+    cudaEventRecord(ctx->ev_order, ctx->kstream);
+    cudaStreamWaitEvent(ctx->main, ctx->ev_order, 0);
+    ctx->stream = ctx->main;
+}
+
+// Relation keys became valid at this point of main.
+void keys_ready(ucl_ctx *ctx, ucl_rel *R) {
+    if (!R->ev_keys && cudaEventCreateWithFlags(&R->ev_keys, cudaEventDisableTiming) != cudaSuccess) {
+        cudaGetLastError();
+        R->ev_keys = nullptr;
+        return;
+    }
+    cudaEventRecord(R->ev_keys, ctx->main);
+}
+
+// The stream in use waits until a relation's keys are valid (main order when
+// it has no event).
+void wait_keys(ucl_ctx *ctx, const ucl_rel *R) {
+    if (ctx->stream == ctx->main) return;
+    if (R->ev_keys) cudaStreamWaitEvent(ctx->stream, R->ev_keys, 0);
+    else order_after_main(ctx);
 }
 
 struct Fail {
@@ -512,15 +559,27 @@ ucl_status cuda_check(ucl_ctx *ctx, cudaError_t e, const char *what) {
     return fail(ctx, UCL_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
 }
 
+void order_after_main(ucl_ctx *ctx) {
+    if (ctx->stream == ctx->main) return;
+    cudaEventRecord(ctx->ev_order, ctx->main);
+    cudaStreamWaitEvent(ctx->stream, ctx->ev_order, 0);
+}
+
+// Device memory comes and goes in main's order (the allocator hooks' stream,
+// or the stream-ordered pool on main).  A block handed out while the key
+// stream is in use may have been freed on main with main's readers still
+// queued: the key stream is ordered after main first.
 void *ctx_alloc(ucl_ctx *ctx, size_t bytes) {
     if (bytes == 0) bytes = 256;
     bytes = (bytes + 255) & ~(size_t)255;
-    if (ctx->alloc) return ctx->alloc(bytes, ctx->user);
     void *p = nullptr;
-    if (cudaMallocAsync(&p, bytes, ctx->stream) != cudaSuccess) {
+    if (ctx->alloc) {
+        p = ctx->alloc(bytes, ctx->user);
+    } else if (cudaMallocAsync(&p, bytes, ctx->main) != cudaSuccess) {
         cudaGetLastError();
-        return nullptr;
+        p = nullptr;
     }
+    if (p) order_after_main(ctx);
     return p;
 }
 
@@ -528,11 +587,11 @@ void ctx_free(ucl_ctx *ctx, void *p, size_t bytes) {
     if (!p) return;
     bytes = (bytes + 255) & ~(size_t)255;
     if (ctx->free_fn) ctx->free_fn(p, bytes, ctx->user);
-    else cudaFreeAsync(p, ctx->stream);
+    else cudaFreeAsync(p, ctx->main);
 }
 
 void *ws_get(ucl_ctx *ctx, size_t bytes) {
-    Arena &A = ctx->arena;
+    Arena &A = *ctx->arena;
     bytes = (bytes + 255) & ~(size_t)255;
     if (bytes == 0) bytes = 256;
     if (A.blocks.empty() || A.used + bytes > A.blocks.back().size) {
@@ -579,7 +638,7 @@ ucl_status ucl_ctx_create(int device, void *stream, ucl_alloc_fn alloc, ucl_free
     ucl_ctx *ctx = new (std::nothrow) ucl_ctx();
     if (!ctx) return UCL_ERR_OOM;
     ctx->device = device;
-    ctx->stream = (cudaStream_t)stream;
+    ctx->stream = ctx->main = (cudaStream_t)stream;
     ctx->alloc = alloc;
     ctx->free_fn = free_fn;
     ctx->user = user;
@@ -597,9 +656,17 @@ ucl_status ucl_ctx_create(int device, void *stream, ucl_alloc_fn alloc, ucl_free
     if (!st) st = cuda_check(ctx, cudaMalloc(&ctx->d_status, 256), "cudaMalloc status");
     if (!st) st = cuda_check(ctx, cudaMemset(ctx->d_status, 0, 256), "cudaMemset status");
     if (!st) st = cuda_check(ctx, cudaMallocHost(&ctx->h_pinned, 8 * sizeof(int64_t)), "cudaMallocHost");
+    if (!st) st = cuda_check(ctx, cudaStreamCreateWithFlags(&ctx->kstream, cudaStreamNonBlocking), "cudaStreamCreate");
+    if (!st) st = cuda_check(ctx, cudaEventCreateWithFlags(&ctx->ev_order, cudaEventDisableTiming), "cudaEventCreate");
+    for (int i = 0; i < ucl_ctx::kArenas && !st; ++i)
+        st = cuda_check(ctx, cudaEventCreateWithFlags(&ctx->arena_done[i], cudaEventDisableTiming), "cudaEventCreate");
     if (st) {
         if (ctx->d_status) cudaFree(ctx->d_status);
         if (ctx->h_pinned) cudaFreeHost(ctx->h_pinned);
+        if (ctx->kstream) cudaStreamDestroy(ctx->kstream);
+        if (ctx->ev_order) cudaEventDestroy(ctx->ev_order);
+        for (cudaEvent_t e : ctx->arena_done)
+            if (e) cudaEventDestroy(e);
         delete ctx;
         return st;
     }
@@ -610,11 +677,17 @@ ucl_status ucl_ctx_create(int device, void *stream, ucl_alloc_fn alloc, ucl_free
 ucl_status ucl_ctx_destroy(ucl_ctx *ctx) {
     if (!ctx) return UCL_ERR_ARG;
     if (ctx->live_rels) return fail(ctx, UCL_ERR_ARG, "relations still alive on this context");
-    cudaStreamSynchronize(ctx->stream);
-    for (auto &b : ctx->arena.blocks) ctx_free(ctx, b.ptr, b.size);
-    cudaStreamSynchronize(ctx->stream);
+    cudaStreamSynchronize(ctx->kstream);
+    cudaStreamSynchronize(ctx->main);
+    ctx->stream = ctx->main;
+    for (Arena &A : ctx->arenas)
+        for (auto &b : A.blocks) ctx_free(ctx, b.ptr, b.size);
+    cudaStreamSynchronize(ctx->main);
     cudaFree(ctx->d_status);
     cudaFreeHost(ctx->h_pinned);
+    cudaStreamDestroy(ctx->kstream);
+    cudaEventDestroy(ctx->ev_order);
+    for (cudaEvent_t e : ctx->arena_done) cudaEventDestroy(e);
     for (cudaEvent_t e : ctx->ev_pool) cudaEventDestroy(e);
     delete ctx;
     return UCL_OK;
@@ -629,16 +702,19 @@ ucl_status ucl_ctx_set_timing(ucl_ctx *ctx, int enable) {
 ucl_status ucl_ctx_synchronize(ucl_ctx *ctx) {
     if (!ctx) return UCL_ERR_ARG;
     cudaSetDevice(ctx->device);
+    cudaError_t e = cudaStreamSynchronize(ctx->kstream);
+    if (e != cudaSuccess) return cuda_check(ctx, e, "stream sync");
+    ctx->stream = ctx->main;
     return sync_read(ctx, nullptr, 0, nullptr);
 }
 
 ucl_status ucl_get_last_stats(ucl_ctx *ctx, ucl_stats *out) {
     if (!ctx || !out) return UCL_ERR_ARG;
     if (ctx->last.timed && ctx->cur_ev) {
-        cudaError_t e = cudaEventSynchronize(ctx->cur_ev[UCL_NSTAGES]);
+        cudaError_t e = cudaEventSynchronize(ctx->cur_ev[kCallEvents - 1]);
         if (e != cudaSuccess) return cuda_check(ctx, e, "event sync");
         for (int i = 0; i < UCL_NSTAGES; ++i)
-            cudaEventElapsedTime(&ctx->last.stage_ms[i], ctx->cur_ev[i], ctx->cur_ev[i + 1]);
+            cudaEventElapsedTime(&ctx->last.stage_ms[i], ctx->cur_ev[kStageFrom[i]], ctx->cur_ev[kStageFrom[i] + 1]);
     }
     *out = ctx->last;
     return UCL_OK;
@@ -646,15 +722,15 @@ ucl_status ucl_get_last_stats(ucl_ctx *ctx, ucl_stats *out) {
 
 ucl_status ucl_ctx_timings(ucl_ctx *ctx, float *ms, int max_calls, int *n_calls, int reset) {
     if (!ctx || (max_calls > 0 && !ms)) return UCL_ERR_ARG;
-    const int per = UCL_NSTAGES + 1;
+    const int per = kCallEvents;
     if (n_calls) *n_calls = ctx->ev_calls;
     if (ctx->ev_calls > 0 && max_calls > 0) {
         cudaError_t e = cudaEventSynchronize(ctx->ev_pool[(size_t)per * ctx->ev_calls - 1]);
         if (e != cudaSuccess) return cuda_check(ctx, e, "event sync");
         for (int c = 0; c < ctx->ev_calls && c < max_calls; ++c)
             for (int i = 0; i < UCL_NSTAGES; ++i)
-                cudaEventElapsedTime(&ms[c * UCL_NSTAGES + i], ctx->ev_pool[(size_t)per * c + i],
-                                     ctx->ev_pool[(size_t)per * c + i + 1]);
+                cudaEventElapsedTime(&ms[c * UCL_NSTAGES + i], ctx->ev_pool[(size_t)per * c + kStageFrom[i]],
+                                     ctx->ev_pool[(size_t)per * c + kStageFrom[i] + 1]);
     }
     if (reset) {
         ctx->ev_calls = 0;
@@ -721,8 +797,8 @@ ucl_status ucl_relation_create(ucl_ctx *ctx, int64_t n, int u, const int32_t *ke
     tmp.sorted = 1;
     ucl_status st = UCL_OK;
     if (n > 0 && u > 0) {
+        const int arena = arena_begin(ctx);
         try {
-            arena_reset(ctx);
             uint64_t *packed = (uint64_t *)ws_get(ctx, sizeof(uint64_t) * n);
             launch_check_keys(ctx, tmp.keys, u, n, tmp.bounds, fp, packed);
             uint32_t flags = 0;
@@ -739,6 +815,7 @@ ucl_status ucl_relation_create(ucl_ctx *ctx, int64_t n, int u, const int32_t *ke
         } catch (Oom &) {
             st = fail(ctx, UCL_ERR_OOM, "workspace allocation failed");
         }
+        cudaEventRecord(ctx->arena_done[arena], ctx->main);
     }
     if (st) {
         if (tmp.own_block) ctx_free(ctx, tmp.own_block, tmp.own_bytes);
@@ -750,6 +827,7 @@ ucl_status ucl_relation_create(ucl_ctx *ctx, int64_t n, int u, const int32_t *ke
         return fail(ctx, UCL_ERR_OOM, "host allocation failed");
     }
     *R = tmp;
+    keys_ready(ctx, R);
     *out = R;
     ctx->err.clear();
     return UCL_OK;
@@ -759,6 +837,7 @@ ucl_status ucl_relation_destroy(ucl_rel *rel) {
     if (!rel) return UCL_ERR_ARG;
     ucl_ctx *ctx = rel->ctx;
     if (rel->own_block) ctx_free(ctx, rel->own_block, rel->own_bytes);
+    if (rel->ev_keys) cudaEventDestroy(rel->ev_keys);
     ctx->live_rels--;
     delete rel;
     return UCL_OK;
@@ -834,8 +913,14 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
     ctx->launches = 0;
     ucl_rel *R = nullptr;
     if ((st = begin_timed_call(ctx))) return st;
+    // The key stage (stages 0 and 1 and the segment pass) runs on the key
+    // stream, so that it overlaps the contraction of the previous call still
+    // queued on main; the output relation, the contraction and the fixup are
+    // on main.
+    to_key_stream(ctx);
+    const int arena = arena_begin(ctx);
+    for (int k = 0; k < n_in; ++k) wait_keys(ctx, in[k]);
     try {
-        arena_reset(ctx);
         record(ctx, 0);
         int64_t *d_scal = (int64_t *)ws_get(ctx, 8 * sizeof(int64_t));
         // ---------------------------------------------------------- stage 0
@@ -954,6 +1039,29 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             S = h;
         }
 
+        // ------------------------------------------------------ segments
+        // one pass over the sorted pairs: each segment's output key (into
+        // the workspace; copied into the output relation on main) and
+        // start, and each pair's input rows
+        int64_t *seg_start = nullptr;
+        uint32_t *pu = nullptr, *pvi = nullptr, *pxi = nullptr;
+        int32_t *okeys = nullptr;
+        if (P > 0) {
+            seg_start = (int64_t *)ws_get(ctx, 8 * (S + 1));
+            pu = (uint32_t *)ws_get(ctx, 4 * P);
+            pvi = (uint32_t *)ws_get(ctx, 4 * P);
+            pxi = X ? (uint32_t *)ws_get(ctx, 4 * P) : nullptr;
+            okeys = (int32_t *)ws_get(ctx, 4 * (size_t)S * kp.uw);
+            if (X) {
+                uint32_t *const idx[3] = {pu, pvi, pxi};
+                launch_segments3(ctx, pk, pv, pv1, seg_excl, P, S, kp.unpack, kp.ord, okeys, seg_start, idx);
+            } else {
+                launch_segments(ctx, pk, pv, seg_excl, P, S, kp.unpack, okeys, seg_start, pu, pvi);
+            }
+        }
+        record(ctx, 2);
+        to_main(ctx);
+
         // output relation: keys ascending by construction
         R = new_rel(ctx);
         if (!R) check(fail(ctx, UCL_ERR_OOM, "host allocation failed"));
@@ -974,21 +1082,16 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             if (!R->own_block) throw Oom();
             R->tiles = R->own_block;
             R->keys = (int32_t *)((char *)R->own_block + koff);
+            if (kp.uw > 0)
+                check(cuda_check(ctx, cudaMemcpyAsync(R->keys, okeys, (size_t)S * kp.uw * 4,
+                                                      cudaMemcpyDeviceToDevice, ctx->main), "copy of output keys"));
         }
+        keys_ready(ctx, R);
 
         // ------------------------------------------------------ stage 2, 3
+        record(ctx, 3);
         int path = UCL_PATH_SIMT;
         if (P > 0) {
-            int64_t *seg_start = (int64_t *)ws_get(ctx, 8 * (S + 1));
-            uint32_t *pu = (uint32_t *)ws_get(ctx, 4 * P), *pvi = (uint32_t *)ws_get(ctx, 4 * P);
-            uint32_t *pxi = X ? (uint32_t *)ws_get(ctx, 4 * P) : nullptr;
-            if (X) {
-                uint32_t *const idx[3] = {pu, pvi, pxi};
-                launch_segments3(ctx, pk, pv, pv1, seg_excl, P, S, kp.unpack, kp.ord, R->keys, seg_start, idx);
-            } else {
-                launch_segments(ctx, pk, pv, seg_excl, P, S, kp.unpack, R->keys, seg_start, pu, pvi);
-            }
-            record(ctx, 2);
             ContractArgs a{};
             a.U = U->tiles;
             a.V = V ? V->tiles : nullptr;
@@ -1032,13 +1135,12 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             } else {
                 launch_contract_simt(ctx, a, lp);
             }
-            record(ctx, 3);
+            record(ctx, 4);
             launch_fixup(ctx, a);
-            record(ctx, 4);
+            record(ctx, 5);
         } else {
-            record(ctx, 2);
-            record(ctx, 3);
             record(ctx, 4);
+            record(ctx, 5);
         }
         check(cuda_check(ctx, cudaGetLastError(), "kernel launch"));
 
@@ -1061,6 +1163,8 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
     } catch (Fail &f) {
         st = f.st;
     }
+    to_main(ctx);
+    cudaEventRecord(ctx->arena_done[arena], ctx->main);
     if (R) ucl_relation_destroy(R);
     return st;
 }
@@ -1206,8 +1310,8 @@ ucl_status ucl_repartition(ucl_ctx *ctx, const char *spec_text, const ucl_rel *i
     ucl_rel *R = nullptr;
     ucl_status st;
     if ((st = begin_timed_call(ctx))) return st;
+    const int arena = arena_begin(ctx);
     try {
-        arena_reset(ctx);
         record(ctx, 0);
         int64_t *d_scal = (int64_t *)ws_get(ctx, 8 * sizeof(int64_t));
         const int64_t n = in->n;
@@ -1278,6 +1382,7 @@ ucl_status ucl_repartition(ucl_ctx *ctx, const char *spec_text, const ucl_rel *i
                 launch_out_place(ctx, okey, iota, n_out, un, pos, R->keys);
             }
             record(ctx, 2);
+            record(ctx, 3);
             // every input element to its place; positions no element maps to
             // exist only when labels are stacked, and are zero
             bool stacked = false;
@@ -1285,12 +1390,14 @@ ucl_status ucl_repartition(ucl_ctx *ctx, const char *spec_text, const ucl_rel *i
             if (stacked)
                 check(cuda_check(ctx, cudaMemsetAsync(R->tiles, 0, tbytes, ctx->stream), "cudaMemsetAsync"));
             launch_repart_scatter(ctx, in->tiles, in->dtype, in->keys, rank, pos, n, pc, R->tiles);
-            record(ctx, 3);
+            record(ctx, 4);
         } else {
             record(ctx, 2);
             record(ctx, 3);
+            record(ctx, 4);
         }
-        record(ctx, 4);
+        record(ctx, 5);
+        keys_ready(ctx, R);
         check(cuda_check(ctx, cudaGetLastError(), "kernel launch"));
         stats.n_pairs = n;
         stats.n_segments = n_out;
@@ -1310,6 +1417,7 @@ ucl_status ucl_repartition(ucl_ctx *ctx, const char *spec_text, const ucl_rel *i
     } catch (Fail &f) {
         st = f.st;
     }
+    cudaEventRecord(ctx->arena_done[arena], ctx->main);
     if (R) ucl_relation_destroy(R);
     return st;
 }

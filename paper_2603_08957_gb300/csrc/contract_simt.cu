@@ -258,18 +258,18 @@ void launch_contract_simt(ucl_ctx *ctx, const ContractArgs &a, const LowerPlan &
     const int G = a.units.G;
     if (G <= 0) return;
     if (a.X) {
-        simt_contract3_kernel<<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status);
+        simt_contract3_kernel<<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status + 2);
         ctx->launches++;
         return;
     }
     if (a.du == UCL_F32 && (!a.V || a.dv == UCL_F32))
-        simt_contract_kernel<float, float><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status);
+        simt_contract_kernel<float, float><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status + 2);
     else if (a.du == UCL_F32)
-        simt_contract_kernel<float, __nv_bfloat16><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status);
+        simt_contract_kernel<float, __nv_bfloat16><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status + 2);
     else if (!a.V || a.dv == UCL_BF16)
-        simt_contract_kernel<__nv_bfloat16, __nv_bfloat16><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status);
+        simt_contract_kernel<__nv_bfloat16, __nv_bfloat16><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status + 2);
     else
-        simt_contract_kernel<__nv_bfloat16, float><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status);
+        simt_contract_kernel<__nv_bfloat16, float><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status + 2);
     ctx->launches++;
 }
 

@@ -866,7 +866,7 @@ ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan 
     kstep_offsets(g.B, tp.b_kmajor, &k.b_lg, &k.b_mask, &k.b_sub16, &k.b_k16);
     // second M block: 128 rows further (K-major) or 128 / w swizzle atoms further (MN-major)
     k.a_mb16 = tp.a_kmajor ? (int)((128u * g.A.w * 2) >> 4) : (int)((128 / g.A.w) * (g.A.sub_bytes >> 4));
-    k.status = ctx->d_status;
+    k.status = ctx->d_status + 2;
     void (*kern)(const CUtensorMap, const CUtensorMap, const TcArgs) = nullptr;
     switch (tp.K / g.kc / 16) {
         case 1: kern = tc_contract_kernel<1>; break;

@@ -592,7 +592,7 @@ ucl_status launch_contract_tc3(ucl_ctx *ctx, const ContractArgs &a, const Tc3Pla
     // core matrix group (SBO 256).
     k.a_desc0 = ((uint64_t)(kFBytes >> 4) << 16) | ((uint64_t)(1024 >> 4) << 32) | (1ull << 46) | (2ull << 61);
     k.b_desc0 = ((uint64_t)(16 >> 4) << 16) | ((uint64_t)(256 >> 4) << 32) | (1ull << 46) | (6ull << 61);
-    k.status = ctx->d_status;
+    k.status = ctx->d_status + 2;
     ucl_status st = cuda_check(
         ctx, cudaFuncSetAttribute(tc3_contract_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem3),
         "cudaFuncSetAttribute");

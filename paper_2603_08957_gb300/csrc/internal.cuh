@@ -109,16 +109,31 @@ struct Arena {
 
 struct ucl_ctx {
     int device = 0;
+    // Streams.  `main` is the caller's: relation storage, contractions and
+    // results live in its order.  The key stage of ucl_einsum (joins, sorts,
+    // sizing syncs) runs on `kstream`, so it overlaps the contractions still
+    // queued on main; `stream` is the one launches go to right now.
     cudaStream_t stream = nullptr;
+    cudaStream_t main = nullptr;
+    cudaStream_t kstream = nullptr;
+    cudaEvent_t ev_order = nullptr;   // scratch event for one-off stream ordering
     ucl_alloc_fn alloc = nullptr;
     ucl_free_fn free_fn = nullptr;
     void *user = nullptr;
     int sm_count = 0;
-    ucl::Arena arena;
-    uint32_t *d_status = nullptr;   // [0] sticky error bits, [1] validation flags
+    // Workspace arenas used by successive calls in turn; arena_done[i] is
+    // recorded on main when the call using arena i has finished with it.
+    static constexpr int kArenas = 4;
+    ucl::Arena arenas[kArenas];
+    cudaEvent_t arena_done[kArenas] = {};
+    int arena_next = 0;
+    ucl::Arena *arena = &arenas[0];
+    // [1] validation flags (main), [2] sticky error bits of main-stream kernels
+    uint32_t *d_status = nullptr;
     int64_t *h_pinned = nullptr;    // pinned host scratch for sizing syncs (8 words)
     int timing = 0;
-    // CUDA events of timed calls: UCL_NSTAGES + 1 per ucl_einsum, reused
+    // CUDA events of timed calls: six per call (stage boundaries on the key
+    // stream and on main), reused
     // after ucl_ctx_timings(..., reset = 1)
     std::vector<cudaEvent_t> ev_pool;
     int ev_calls = 0;      // calls recorded since the last reset
@@ -143,6 +158,7 @@ struct ucl_rel {
     size_t own_bytes = 0;
     int sorted = 0;              // keys strictly ascending lexicographically
     int key_bits = 0;            // sum of column bit widths
+    cudaEvent_t ev_keys = nullptr;   // recorded on main once keys are valid (key-stream readers wait on it)
 };
 
 namespace ucl {
@@ -150,7 +166,9 @@ namespace ucl {
 // ---- context helpers (api.cu)
 void *ctx_alloc(ucl_ctx *ctx, size_t bytes);
 void ctx_free(ucl_ctx *ctx, void *p, size_t bytes);
-void *ws_get(ucl_ctx *ctx, size_t bytes);   // arena workspace, valid until the next arena reset
+void *ws_get(ucl_ctx *ctx, size_t bytes);   // workspace of the current call's arena
+// Order the stream in use after everything enqueued on main so far (no-op on main).
+void order_after_main(ucl_ctx *ctx);
 ucl_status fail(ucl_ctx *ctx, ucl_status st, const std::string &msg);
 ucl_status cuda_check(ucl_ctx *ctx, cudaError_t e, const char *what);
 int bit_width(int64_t bound);   // bits to store values in [0, bound)
