@@ -1,0 +1,221 @@
+"""Pins of the planner oracle (oracle/planner.py) against brute force, closed
+forms and invariants that the paper's definitions fix (Sec. 6.1, 6.2, Alg. 1,
+Alg. 2).  CPU only."""
+from __future__ import annotations
+
+import itertools
+import math
+import random
+
+import numpy as np
+import pytest
+
+from oracle import planner as P
+
+
+# ----------------------------------------------------------- statistics
+
+def _brute_stats(arr, labels):
+    """T and V by visiting every index tuple (pure Python)."""
+    T = 0
+    seen = {l: set() for l in labels}
+    for idx in itertools.product(*[range(e) for e in arr.shape]):
+        if arr[idx] != 0:
+            T += 1
+            for q, l in enumerate(labels):
+                seen[l].add(idx[q])
+    return T, {l: len(s) for l, s in seen.items()}
+
+
+@pytest.mark.parametrize("shape", [(7,), (5, 6), (3, 4, 5), (2, 3, 2, 4)])
+@pytest.mark.parametrize("density", [0.0, 0.05, 0.4, 1.0])
+def test_dense_stats_brute_force(shape, density):
+    rng = np.random.default_rng(len(shape) * 100 + int(density * 10))
+    arr = rng.standard_normal(shape) * (rng.random(shape) < density)
+    labels = "abcd"[: len(shape)]
+    s = P.dense_stats(arr, labels)
+    T, V = _brute_stats(arr, labels)
+    assert s.T == T and s.V == V
+
+
+def test_relation_stats_any_decomposition():
+    # the statistics belong to the tensor, not to how it is decomposed
+    rng = np.random.default_rng(3)
+    dense = rng.standard_normal((4, 6, 5)) * (rng.random((4, 6, 5)) < 0.2)
+    ref = P.dense_stats(dense, "abc")
+    for up in range(1, 3):
+        keys = np.array(list(itertools.product(*[range(e) for e in dense.shape[:up]])), dtype=np.int32)
+        tiles = dense.reshape((-1,) + dense.shape[up:])
+        s = P.relation_stats(keys, dense.shape[:up], tiles, "abc")
+        assert s.T == ref.T and s.V == ref.V
+
+
+# ----------------------------------------------------- Eq. eqn-count
+
+def test_tuple_count_limits():
+    s = P.Stats(1e9, {"a": 10, "b": 20})
+    assert P.tuple_count(s, ("a", "b")) == pytest.approx(200.0)       # T ≫ n: every tuple present
+    s = P.Stats(5.0, {"a": 1e6, "b": 1e6})
+    assert P.tuple_count(s, ("a", "b")) == pytest.approx(5.0, rel=1e-9)  # n ≫ T: one tuple per entry
+    s = P.Stats(3.0, {"a": 4})
+    assert P.tuple_count(s, ()) == pytest.approx(1 - math.exp(-3.0))   # no promoted label: one tuple
+    assert P.tuple_count(P.Stats(0.0, {"a": 4}), ("a",)) == 0.0
+
+
+def test_tuple_count_uniform_monte_carlo():
+    # T non-zeros placed uniformly at random: the tuple count of a decomposition
+    # is the number of occupied (a, b) cells, whose expectation the estimate gives
+    rng = np.random.default_rng(0)
+    shape, T = (50, 40, 30), 2000
+    counts = []
+    for _ in range(20):
+        flat = rng.choice(np.prod(shape), size=T, replace=False)
+        a, b, c = np.unravel_index(flat, shape)
+        arr = np.zeros(shape)
+        arr[a, b, c] = 1.0
+        s = P.dense_stats(arr, "abc")
+        occupied = len(set(zip(a.tolist(), b.tolist())))
+        counts.append((occupied, P.tuple_count(s, ("a", "b"))))
+    occ = np.mean([c[0] for c in counts])
+    est = np.mean([c[1] for c in counts])
+    assert abs(est - occ) / occ < 0.03
+
+
+# ---------------------------------------------------------- Sec. 6.2
+
+def _dense(labels, bounds):
+    T = float(np.prod([bounds[l] for l in labels]))
+    return P.Stats(T * 1e3, {l: bounds[l] for l in labels})   # saturated: every tuple present
+
+
+def test_join_estimate_matches_join_of_full_relations():
+    bounds = {"J": 6, "K": 5, "j": 4}
+    sU, sV = _dense("J", bounds), _dense("JK", bounds)
+    # U keyed J (6 tuples), V keyed (J, K) (30 tuples): each U tuple meets 5 V tuples
+    actual = sum(1 for u in range(6) for (j, k) in itertools.product(range(6), range(5)) if u == j)
+    assert P.join_tuples(sU, ("J",), sV, ("J", "K")) == pytest.approx(actual)
+    # no shared promoted label: the cross product
+    assert P.join_tuples(sU, ("J",), sV, ("K",)) == pytest.approx(6 * 5)
+
+
+def test_agg_estimate_counts_groups_of_full_relations():
+    bounds = {"J": 6, "K": 5}
+    sU, sV = _dense("J", bounds), _dense("JK", bounds)
+    tj = P.join_tuples(sU, ("J",), sV, ("J", "K"))
+    groups = len({k for (j, k) in itertools.product(range(6), range(5))})
+    assert P.agg_tuples(sU, ("J",), sV, ("J", "K"), ("K",), tj) == pytest.approx(groups)
+
+
+def test_repart_cost_invariants():
+    bounds = {"a": 8, "b": 16, "c": 4}
+    v = P.Vertex("abc", 2)
+    s = P.Stats(300.0, {"a": 8, "b": 12, "c": 4})
+    cm = P.CostModel(xfer=1e-3, fixed=0.5)
+    subs = list(P.subsets("abc"))
+    for x, y in itertools.product(subs, subs):
+        cxy = P.repart_cost(cm, bounds, v, s, x, y)
+        assert cxy >= -1e-9
+        assert cxy == pytest.approx(P.repart_cost(cm, bounds, v, s, y, x))   # same intermediate both ways
+        if set(x) == set(y):
+            assert cxy == 0.0
+        if set(x) < set(y):
+            # only the decomposition step runs: T(out) − T(in) new tuples
+            per = P.tuple_bytes("abc", y, bounds, 2, 4) * cm.xfer + cm.fixed
+            assert cxy == pytest.approx((P.tuple_count(s, y) - P.tuple_count(s, x)) * per)
+
+
+# ------------------------------------------------------------ Alg. 2
+
+def test_estimate_stats_dense_product_is_exact():
+    bounds = {"i": 3, "j": 4, "k": 5}
+    sU = P.dense_stats(np.ones((3, 4)), "ij")
+    sV = P.dense_stats(np.ones((4, 5)), "jk")
+    sW = P.estimate_stats(sU, "ij", sV, "jk", "ik")
+    ref = P.dense_stats(np.ones((3, 4)) @ np.ones((4, 5)), "ik")
+    assert sW.T == ref.T and sW.V == ref.V
+
+
+# ------------------------------------------------------------ Alg. 1
+
+def _valid(graph, plan):
+    """Independent validity check of one plan: every label has one class
+    within each EinSum (inputs and output agree)."""
+    for i, v in enumerate(graph):
+        if v.left is None:
+            continue
+        upW, upU, upV = plan[i]
+        lU, lV = graph[v.left].labels, graph[v.right].labels
+        for l in set(lU) | set(lV):
+            classes = set()
+            for lab, up in ((lU, upU), (lV, upV), (v.labels, upW)):
+                if l in lab:
+                    classes.add(l in up)
+            if len(classes) != 1:
+                return False
+    return True
+
+
+def _random_tree(rng, shape):
+    bounds = {l: rng.choice([2, 4, 8, 16, 64]) for l in "abcdefg"}
+
+    def leaf(labels):
+        T = float(rng.uniform(1, np.prod([bounds[l] for l in labels])))
+        return P.Vertex(labels, int(rng.choice([2, 4])), stats=P.Stats(
+            T, {l: float(rng.integers(1, bounds[l] + 1)) for l in labels}))
+
+    if shape == "chain":      # ((X × Y) × Z), the message-passing shape
+        g = [leaf("fab"), leaf("abcd"), P.Vertex("cdf", 2, 0, 1), leaf("fg"), P.Vertex("cdg", 4, 2, 3)]
+    elif shape == "transpose":  # (X × Y)^T × Z
+        g = [leaf("ab"), leaf("bc"), P.Vertex("ca", 2, 0, 1), leaf("ad"), P.Vertex("cd", 4, 2, 3)]
+    else:                     # two products joined: (X × Y) × (Z × Q)
+        g = [leaf("ab"), leaf("bc"), P.Vertex("ac", 2, 0, 1), leaf("cd"), leaf("de"), P.Vertex("ce", 2, 3, 4),
+             P.Vertex("ae", 4, 2, 5)]
+    cm = P.CostModel(xfer=rng.uniform(0, 1e-3), flop=rng.uniform(0, 1e-4), add=rng.uniform(0, 1e-3),
+                     fixed=rng.uniform(0, 10))
+    return g, bounds, cm
+
+
+@pytest.mark.parametrize("shape", ["chain", "transpose", "bushy"])
+@pytest.mark.parametrize("seed", range(4))
+def test_dp_matches_exhaustive_search(shape, seed):
+    rng = np.random.default_rng(seed)
+    g, bounds, cm = _random_tree(rng, shape)
+    every = P.enumerate_plans(g, bounds, cm)
+    assert all(_valid(g, p) for _, p in every)
+    best = P.optimize(g, bounds, cm, k=6)
+    assert [c for c, _ in best] == pytest.approx([c for c, _ in every[:6]], rel=1e-12)
+    for c, plan in best:
+        assert _valid(g, plan)
+        assert P.plan_cost(g, bounds, cm, plan) == pytest.approx(c, rel=1e-12)
+    # the k plans are distinct
+    keys = {tuple(sorted((i, repr(x)) for i, x in p.items())) for _, p in best}
+    assert len(keys) == len(best)
+
+
+def test_plan_count_closed_form():
+    # each label takes one class per EinSum: 2^|ℓU ∪ ℓV| plans per vertex
+    rng = np.random.default_rng(1)
+    g, bounds, cm = _random_tree(rng, "chain")
+    n1 = 2 ** len(set("fab") | set("abcd"))
+    n2 = 2 ** len(set("cdf") | set("fg"))
+    assert len(P.enumerate_plans(g, bounds, cm)) == n1 * n2
+
+
+def test_planted_consistency_mistake_is_caught(monkeypatch):
+    # a planted mistake: only the output's labels constrain the inputs
+    rng = np.random.default_rng(1)
+    g, bounds, cm = _random_tree(rng, "chain")
+    orig = P.consistent
+    monkeypatch.setattr(P, "consistent", lambda lX, upX, lW, upW: True if lW != g[2].labels and lW != g[4].labels
+                        else orig(lX, upX, lW, upW))
+    every = P.enumerate_plans(g, bounds, cm)
+    assert len(every) != 2 ** 6 * 2 ** 5 or not all(_valid(g, p) for _, p in every)
+
+
+def test_tree_checks():
+    s = P.Stats(1.0, {"a": 1})
+    with pytest.raises(ValueError):
+        P.optimize([P.Vertex("a", stats=s), P.Vertex("a", 2, 0, 0)], {"a": 1}, P.CostModel())
+    with pytest.raises(ValueError):
+        P.optimize([P.Vertex("a", stats=s), P.Vertex("a", stats=s), P.Vertex("b", 2, 0, 1)], {"a": 1, "b": 1},
+                   P.CostModel())
