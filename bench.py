@@ -244,7 +244,7 @@ class Spgemm(_Binary):
 
 
 class Repart(Workload):
-    """Repartition (Sec. 5's representation change): the message-passing Y
+    """Repartition (Sec. 6's representation change): the message-passing Y
     (358136 64x64 bf16 tiles keyed (J, K)) split into 64-wide row vectors
     keyed (J, K, j), then stacked back into tiles."""
     name = "repart"
@@ -631,6 +631,98 @@ def run_ucl(args, world, rank, local):
     ctx.close()
 
 
+def run_rank_plans(args):
+    """Rank the decompositions of the message-passing tree (X x Y)^T x Z by
+    the cost model (ucl_plan, k cheapest) and time each on the GPU, as the
+    paper's Opt / 2nd / 3rd tables do.  Cost constants calibrated here: C_xfer
+    = 1 / measured HBM bandwidth, C_krnel = 1 / measured bf16 tensor
+    throughput per flop, C_fixed = device time per joined tuple of a
+    cross product of scalar tuples aggregated onto one side (the rule of thumb
+    of Sec. 7.2), C_add = 0 (the group-by sum is fused into the contraction);
+    the memory constraint of Sec. 8.2 bounds one kernel call's three tiles by
+    256 KB, about one SM's on-chip memory (227 KB shared + 256 KB TMEM).
+    Inputs are brought into each plan's split before its timing."""
+    import workloads
+    from paper_2603_08957_gb300 import Context, plan, program
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(0)
+    ctx = Context(0)
+    pk = peaks()
+
+    def timed(fn, reps):
+        fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    # C_fixed: a cross product of 4096 x 1024 scalar tuples grouped onto the 1024
+    a = ctx.relation(torch.arange(4096, dtype=torch.int32, device=dev)[:, None], (4096,),
+                     torch.ones(4096, device=dev))
+    b = ctx.relation(torch.arange(1024, dtype=torch.int32, device=dev)[:, None], (1024,),
+                     torch.ones(1024, device=dev))
+    fixed = timed(lambda: ctx.einsum("I,K->K", a, b).destroy(), 5) / 1e3 / (4096 * 1024)
+    cm = {"xfer": 1.0 / (pk["hbm_gbs"] * 1e9), "flop": 1.0 / (pk["bf16_tflops"] * 1e12), "add": 0.0, "fixed": fixed,
+          "max_call_bytes": 256e3}
+
+    n, t = args.vertices, 64
+    w = workloads.gnn_chain(seed=0, n=n, device=dev)
+    nt = -(-n // t)
+    bounds = {"f": 128, "a": nt, "b": t, "c": nt, "d": t, "g": 128}
+    verts = [{"labels": "fab"}, {"labels": "abcd"}, {"labels": "cdf", "left": 0, "right": 1, "dtype_bytes": 2},
+             {"labels": "fg"}, {"labels": "cdg", "left": 2, "right": 3, "dtype_bytes": 4}]
+    stored = {0: (ctx.relation(torch.as_tensor(w["X"][0]).to(dev), w["X"][1], w["X"][2]), "a"),
+              1: (ctx.relation(torch.as_tensor(w["Y"][0]).to(dev), w["Y"][1], w["Y"][2]), "ac"),
+              3: (ctx.relation(torch.as_tensor(w["Z"][0]).to(dev), w["Z"][1], w["Z"][2]), "")}
+    for i, (rel, up) in stored.items():
+        T, V = ctx.stats(rel)
+        lab = verts[i]["labels"]
+        order = [c for c in lab if c in up] + [c for c in lab if c not in up]
+        verts[i].update(T=T, V=dict(zip(order, V)))
+    # the k cheapest plans, and the workload's own decomposition (fJj,JjKk->Kkf
+    # then Kkf,fg->Kkg) wherever the model ranks it among the first 4096
+    ranked = plan(verts, bounds, cm, k=4096)
+    own = {2: ("c", "a", "ac"), 4: ("c", "c", "")}
+    own_rank = next((r for r, (_, ups) in enumerate(ranked)
+                     if all(tuple(ups[i]) == own[i] for i in own)), None)
+    todo = list(range(min(args.rank_plans, len(ranked))))
+    if own_rank is not None and own_rank not in todo:
+        todo.append(own_rank)
+    rows = []
+    for r in todo:
+        cost, ups = ranked[r]
+        specs = []
+        for i, v in enumerate(verts):
+            if v.get("left") is not None:
+                upW, upU, upV = ups[i]
+                specs.append(program.einsum_spec(verts[v["left"]]["labels"], upU, verts[v["right"]]["labels"], upV,
+                                                 v["labels"], upW))
+        row = {"rank": r + 1, "predicted_ms": cost * 1e3, "specs": specs}
+        try:
+            ins = program.prepare_inputs(ctx, verts, ups, stored)
+            row["ms"] = timed(lambda: program.execute(ctx, verts, ups, ins).destroy(), max(3, args.steps or 5))
+            row["input_tuples"] = {verts[i]["labels"]: r_.n for i, r_ in ins.items()}
+            for i, r_ in ins.items():
+                if r_ is not stored[i][0]:
+                    r_.destroy()
+        except Exception as e:  # noqa: BLE001 -- a plan the executor cannot run is reported, not fatal
+            row["error"] = str(e)
+        rows.append(row)
+        torch.cuda.synchronize()
+    ok = [r for r in rows if "ms" in r]
+    measured_order = [r["rank"] for r in sorted(ok, key=lambda r: r["ms"])]
+    print(json.dumps({"metric": "planner ranking vs measured step time", "workload": w["spec1"] + " ; " + w["spec2"],
+                      "vertices": n, "cost_model_s": cm, "peaks_src": pk["src"], "plans": rows,
+                      "measured_order": measured_order, "plans_ranked": len(ranked),
+                      "workload_decomposition_rank": None if own_rank is None else own_rank + 1}), flush=True)
+    ctx.close()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -649,7 +741,13 @@ def main():
     ap.add_argument("--seconds", type=float, default=3.0, help="timed seconds when --steps is not given")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-step-seconds", type=float, default=3.0)
+    ap.add_argument("--rank-plans", type=int, default=0,
+                    help="instead of the benchmark: rank the K cheapest decompositions of the message-passing "
+                         "tree by the cost model and time each")
     args = ap.parse_args()
+    if args.rank_plans:
+        run_rank_plans(args)
+        return
     world, rank, local = dist_init(args)
     if args.impl == "reference":
         if args.steps is None:

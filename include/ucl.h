@@ -182,7 +182,7 @@ ucl_status ucl_relation_download(const ucl_rel *rel, int32_t *keys_host, void *t
  * output label appears in some input; a label has one extent everywhere.
  * Labels absent from the output are summed: upper ones by the group-by, lower
  * ones inside the tile kernel.  Shared upper labels are the join attributes;
- * with none the join is a cross product (Sec. 6.2).  n_in = 1 is a unary
+ * with none the join is a cross product (Sec. 7.2).  n_in = 1 is a unary
  * EinSum (a group-by sum over one relation, e.g. with the relu epilogue).
  * n_in = 3 joins all three inputs (tuples agree on every shared upper label)
  * and multiplies the three tiles' entries, as in MTTKRP
@@ -207,7 +207,7 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec, int n_in, ucl_rel *const *
 /* ------------------------------------------------------------ repartition */
 
 /* Change a relation's upper/lower split without changing the tensor it
- * denotes (Sec. 5, the representation change between two EinSums whose
+ * denotes (Sec. 6, the representation change between two EinSums whose
  * decompositions of a tensor differ: decompose every tuple over the full
  * range of each label that becomes upper -- the ALLINTS step -- then stack
  * the labels that become lower, grouped by the new upper labels -- the STACK
@@ -235,6 +235,92 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec, int n_in, ucl_rel *const *
  * UCL_ERR_UNSUPPORTED (> 64 output key bits, a tile or count of 2^31 or
  * more), UCL_ERR_OOM, UCL_ERR_CUDA. */
 ucl_status ucl_repartition(ucl_ctx *ctx, const char *spec, const ucl_rel *in, ucl_rel **out);
+
+/* ------------------------------------------------------------ statistics */
+
+/* Statistics of the tensor a relation stores (Sec. 7.1), which the planner
+ * (ucl_plan) needs for every input tensor:
+ *   nnz       optional; receives T, the number of non-zero tile elements
+ *             (bf16/fp32 ±0 is zero; NaN counts as non-zero)
+ *   distinct  optional, int64 [u + r]; receives V for each key column (the
+ *             number of its values carried by a tuple with a non-zero
+ *             element) and then for each tile dim (the number of its indices
+ *             at which some tuple has a non-zero element)
+ * Reads every tile once.  Works on one bitmap per key column (bound / 8
+ * bytes) and per tile dim in the context's workspace.  Synchronises the
+ * stream once.
+ * Errors: UCL_ERR_ARG, UCL_ERR_OOM, UCL_ERR_CUDA. */
+ucl_status ucl_relation_stats(ucl_ctx *ctx, const ucl_rel *rel, int64_t *nnz, int64_t *distinct);
+
+/* A new relation with the tuples of `in` whose tile holds a non-zero element,
+ * in the same (key) order: the elimination of all-zero tuples that Sec. 4.2
+ * allows.  Output owned by the library (ucl_relation_destroy).  Synchronises
+ * the stream once.
+ * Errors: UCL_ERR_ARG, UCL_ERR_OOM, UCL_ERR_CUDA. */
+ucl_status ucl_drop_zero_tiles(ucl_ctx *ctx, const ucl_rel *in, ucl_rel **out);
+
+/* ---------------------------------------------------------------- planner */
+
+#define UCL_PLAN_MAX_VERTICES 64
+
+/* One vertex of a tree of binary EinSums (Sec. 8.1): an input tensor
+ * (left = right = -1) or W = sum U x V over the labels W does not keep, U
+ * and V being the tensors of vertices `left` and `right`.  Vertices come in
+ * topological order, the last is the root, and every tensor but the root is
+ * consumed exactly once. */
+typedef struct {
+    int left, right;          /* producer vertices of the two inputs, or -1, -1 */
+    const char *labels;       /* the labels of the tensor this vertex produces: one
+                                 byte each, distinct, NUL-terminated, at most 12 */
+    int dtype_bytes;          /* bytes per element of that tensor */
+    double nnz;               /* T of the tensor: required for inputs; for an EinSum
+                                 vertex, measured statistics or < 0 to estimate */
+    const double *distinct;   /* V per label in `labels` order: required for inputs;
+                                 for an EinSum vertex NULL to estimate (Alg. 2) */
+} ucl_plan_vertex;
+
+/* Per-unit costs of Sec. 7.2, in any one unit of time: per byte moved into a
+ * join or an aggregation (C_xfer), per kernel flop (C_krnel = flop x the
+ * kernel's 2 x multiply-adds), per added output-tile element (C_add = add x
+ * tile elements), per tuple (C_fixed); key_bytes = bytes per key column.
+ * max_call_bytes > 0 is the memory constraint of Sec. 8.2: a split is only
+ * considered when the three tiles of one kernel call (U's, V's and W's, at
+ * their element sizes) total at most that many bytes. */
+typedef struct {
+    double xfer, flop, add, fixed;
+    int key_bytes;
+    double max_call_bytes;
+} ucl_cost_model;
+
+/* One plan: for every vertex the promoted labels of its output (bit q = its
+ * q-th label; an input tensor's is the split its consumer reads), and for
+ * every EinSum vertex the promoted labels of its left and right input as it
+ * reads them (bits over that input's labels).  Where a producer's output split
+ * differs from its consumer's read split, the plan repartitions the tensor
+ * between them (ucl_repartition). */
+typedef struct {
+    double cost;
+    uint32_t up[UCL_PLAN_MAX_VERTICES];
+    uint32_t in_up[UCL_PLAN_MAX_VERTICES][2];
+} ucl_plan_choice;
+
+/* The k cheapest plans of an EinSum tree under the cost model of Sec. 7.2,
+ * by the dynamic programme of Alg. 1 extended to keep the k cheapest entries
+ * per vertex and output split.  Host only: no GPU work, no context.
+ *   vertices                  [n_vertices] the tree
+ *   label_names, label_bounds [n_labels] each label's extent
+ *   k                         plans wanted (>= 1)
+ *   out                       [k] receives the plans, cheapest first
+ *   n_out                     receives how many plans were written (<= k)
+ * A label takes one class within an EinSum: upper in every operand that has
+ * it, or lower in all.  Input tensors cost nothing in any split.
+ * Errors: UCL_ERR_ARG (counts, pointers, not a tree in topological order),
+ * UCL_ERR_SPEC (a label twice in a tensor, an output label in no input),
+ * UCL_ERR_SHAPE (a label without a bound), UCL_ERR_UNSUPPORTED (more than
+ * 12 labels in one tensor). */
+ucl_status ucl_plan(int n_vertices, const ucl_plan_vertex *vertices, const char *label_names,
+                    const int64_t *label_bounds, int n_labels, const ucl_cost_model *cost_model, int k,
+                    ucl_plan_choice *out, int *n_out);
 
 /* ------------------------------------------------------- no allocation */
 

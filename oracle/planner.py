@@ -5,11 +5,11 @@ use this module; it shares nothing with the executor or its planner.
 
 It restates, in plain Python and in the paper's order:
 
-* the statistics of Sec. 6.1: T(U), the number of non-zero entries of a
+* the statistics of Sec. 7.1: T(U), the number of non-zero entries of a
   tensor, and V(l, U), the number of slices along label l holding a non-zero;
 * the tuple-count estimate of Eq. eqn-count for a decomposition with
   promoted labels up(U);
-* the join, aggregation and repartition costs of Sec. 6.2;
+* the join, aggregation and repartition costs of Sec. 7.2;
 * GetStats (Alg. 2): statistics of an intermediate tensor from those of its
   inputs by textbook relational estimates over purely relational (scalar)
   versions of the tensors;
@@ -41,6 +41,10 @@ Readings where the paper is silent or inconsistent:
   exceeds the tuple count.
 * P6 Ties between plans of equal cost keep the first found, enumerating
   subsets of a label list by increasing bit mask (bit q = the q-th label).
+* P7 The memory constraint of Sec. 8.2 bounds what one kernel call touches:
+  with a positive ``max_call_bytes``, an EinSum may only read and write tiles
+  whose bytes (U's tile + V's tile + W's tile, at each tensor's element
+  size) total at most that; choices above it are left out of the search.
 """
 from __future__ import annotations
 
@@ -53,13 +57,14 @@ import numpy as np
 
 @dataclass
 class CostModel:
-    """Per-unit costs of Sec. 6.2 (seconds per byte, flop, added element and tuple)."""
+    """Per-unit costs of Sec. 7.2 (seconds per byte, flop, added element and tuple)."""
 
     xfer: float = 1.0
     flop: float = 0.0
     add: float = 0.0
     fixed: float = 0.0
     key_bytes: int = 4
+    max_call_bytes: float = 0.0     # reading P7; 0: no bound
 
 
 @dataclass
@@ -80,7 +85,7 @@ class Vertex:
     stats: Stats | None = None     # inputs: required; EinSums: estimated when None
 
 
-# ------------------------------------------------------------------ Sec. 6.1
+# ------------------------------------------------------------------ Sec. 7.1
 
 def dense_stats(arr, labels) -> Stats:
     """T(U) and V(l, U) of a dense tensor whose axes carry ``labels`` in order:
@@ -105,6 +110,32 @@ def relation_stats(keys, bounds, tiles, labels) -> Stats:
     return dense_stats(dense, labels)
 
 
+def relation_stats_direct(keys, bounds, tiles):
+    """The same statistics straight from the tuples, for relations too large
+    to form densely: (T, [V of each key column] + [V of each tile dim]).  A
+    key value counts when a tuple carrying it has a non-zero element; a tile
+    index counts when some tuple has a non-zero element at it."""
+    tiles = np.asarray(tiles)
+    n = tiles.shape[0]
+    keys = np.asarray(keys, dtype=np.int64).reshape(n, len(bounds))
+    nz = tiles != 0
+    T = int(np.count_nonzero(nz))
+    live = nz.reshape(n, -1).any(axis=1) if n else np.zeros(0, bool)
+    V = [int(len(np.unique(keys[live, c]))) for c in range(len(bounds))]
+    for q in range(1, tiles.ndim):
+        other = tuple(a for a in range(tiles.ndim) if a != q)
+        V.append(int(np.count_nonzero(nz.any(axis=other))) if n else 0)
+    return T, V
+
+
+def drop_zero_tiles(keys, tiles):
+    """The tuples whose tile holds a non-zero element, in their order (the
+    zero-tuple elimination Sec. 4.2 allows)."""
+    tiles = np.asarray(tiles)
+    keep = (tiles.reshape(len(tiles), -1) != 0).any(axis=1) if len(tiles) else np.zeros(0, bool)
+    return np.asarray(keys)[keep], tiles[keep]
+
+
 def tuple_count(s: Stats, up) -> float:
     """Eq. eqn-count: n(↑U)·(1 − exp(−T(U)/n(↑U))), n(↑U) = Π V(l, U) over ↑U."""
     n = 1.0
@@ -124,7 +155,7 @@ def tuple_bytes(labels, up, bounds, dtype_bytes, key_bytes) -> float:
     return key_bytes * len(up) + dtype_bytes * tile
 
 
-# ------------------------------------------------------------------ Sec. 6.2
+# ------------------------------------------------------------------ Sec. 7.2
 
 def join_tuples(sU, upU, sV, upV) -> float:
     """T_join: the textbook join estimate over the labels promoted on both sides."""
@@ -264,14 +295,23 @@ def _vertex_terms(graph, stats, bounds, cm, i, upW, upU, upV):
             agg_cost(cm, bounds, v, upW, sU, upU, sV, upV))
 
 
-def _input_choices(graph, i, upW):
+def tile_bytes(v, up, bounds) -> float:
+    return tuple_bytes(v.labels, up, bounds, v.dtype_bytes, 0)
+
+
+def _input_choices(graph, i, upW, bounds=None, cm=None):
     v = graph[i]
-    lU, lV = graph[v.left].labels, graph[v.right].labels
+    vU, vV = graph[v.left], graph[v.right]
+    lU, lV = vU.labels, vV.labels
     for upU in subsets(lU):
         if not consistent(lU, upU, v.labels, upW):
             continue
         for upV in subsets(lV):
             if consistent(lV, upV, v.labels, upW) and consistent(lV, upV, lU, upU):
+                if cm is not None and cm.max_call_bytes > 0 and (
+                        tile_bytes(vU, upU, bounds) + tile_bytes(vV, upV, bounds) + tile_bytes(v, upW, bounds)
+                        > cm.max_call_bytes):
+                    continue
                 yield upU, upV
 
 
@@ -290,7 +330,7 @@ def optimize(graph, bounds, cm: CostModel, k: int = 1):
         table = {}
         for upW in subsets(v.labels):
             cands = []
-            for upU, upV in _input_choices(graph, i, upW):
+            for upU, upV in _input_choices(graph, i, upW, bounds, cm):
                 here = _vertex_terms(graph, stats, bounds, cm, i, upW, upU, upV)
                 sides = []
                 for child, up_in_consumer in ((v.left, upU), (v.right, upV)):
@@ -339,7 +379,7 @@ def enumerate_plans(graph, bounds, cm: CostModel):
     for i in ein:
         opts = []
         for upW in subsets(graph[i].labels):
-            for upU, upV in _input_choices(graph, i, upW):
+            for upU, upV in _input_choices(graph, i, upW, bounds, cm):
                 opts.append((upW, upU, upV))
         per_vertex.append(opts)
     out = []
@@ -353,3 +393,18 @@ def enumerate_plans(graph, bounds, cm: CostModel):
         out.append((plan_cost(graph, bounds, cm, plan), plan))
     out.sort(key=lambda e: e[0])
     return out
+
+
+def dense_tree(graph, dense_inputs):
+    """Evaluate an EinSum tree densely in fp64 from its input tensors (each
+    a numpy array with axes in its vertex's label order): every EinSum vertex
+    is its definition, Σ over the labels absent from the output of U × V,
+    computed by numpy.einsum.  Returns every vertex's tensor."""
+    val = {}
+    for i, v in enumerate(graph):
+        if v.left is None:
+            val[i] = np.asarray(dense_inputs[i], dtype=np.float64)
+        else:
+            lU, lV = graph[v.left].labels, graph[v.right].labels
+            val[i] = np.einsum(f"{lU},{lV}->{v.labels}", val[v.left], val[v.right])
+    return val

@@ -1,7 +1,7 @@
 """Oracle for repartitioning a tensor-relation (test infrastructure only).
 
 Changing the upper/lower split of a relation between two EinSums (paper
-Sec. 5, the third step of compiling an EinSum DAG) happens in two steps:
+Sec. 6, the third step of compiling an EinSum DAG) happens in two steps:
 
   1. decompose: every tuple is split along each label that turns from lower
      to upper, one sub-tuple per index value of that label over its whole

@@ -13,7 +13,7 @@
  *   1. parse the spec and classify labels (Sec. 4.3: upper-case letters are
  *      promoted to key columns, lower-case letters index the dense tile);
  *   2. natural join of the input relations on every shared upper label
- *      (Sec. 5; with no shared label the join is a cross product, Sec. 6.2);
+ *      (Sec. 5; with no shared label the join is a cross product, Sec. 7.2);
  *      tuple at a time, with a sorted index on the inner relation;
  *   3. the kernel K: naive loops over every lower-label index combination,
  *      W[lower W] += prod_k U_k[lower U_k], accumulated in fp64, together

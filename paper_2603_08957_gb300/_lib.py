@@ -42,6 +42,9 @@ EXPORTS = [
     "ucl_relation_download",
     "ucl_einsum",
     "ucl_repartition",
+    "ucl_relation_stats",
+    "ucl_drop_zero_tiles",
+    "ucl_plan",
     "ucl_keys_check_noalloc",
     "ucl_status_str",
     "ucl_last_error",
@@ -73,6 +76,39 @@ class Stats(ctypes.Structure):
     ]
 
 
+PLAN_MAX_VERTICES = 64
+
+
+class PlanVertex(ctypes.Structure):
+    _fields_ = [
+        ("left", ctypes.c_int),
+        ("right", ctypes.c_int),
+        ("labels", ctypes.c_char_p),
+        ("dtype_bytes", ctypes.c_int),
+        ("nnz", ctypes.c_double),
+        ("distinct", ctypes.POINTER(ctypes.c_double)),
+    ]
+
+
+class CostModel(ctypes.Structure):
+    _fields_ = [
+        ("xfer", ctypes.c_double),
+        ("flop", ctypes.c_double),
+        ("add", ctypes.c_double),
+        ("fixed", ctypes.c_double),
+        ("key_bytes", ctypes.c_int),
+        ("max_call_bytes", ctypes.c_double),
+    ]
+
+
+class PlanChoice(ctypes.Structure):
+    _fields_ = [
+        ("cost", ctypes.c_double),
+        ("up", ctypes.c_uint32 * PLAN_MAX_VERTICES),
+        ("in_up", (ctypes.c_uint32 * 2) * PLAN_MAX_VERTICES),
+    ]
+
+
 _lock = threading.Lock()
 _lib = None
 
@@ -95,6 +131,10 @@ def _declare(lib):
     lib.ucl_relation_download.argtypes = [vp, vp, vp]
     lib.ucl_einsum.argtypes = [vp, c.c_char_p, i32, pp, c.POINTER(EinsumOpts), pp]
     lib.ucl_repartition.argtypes = [vp, c.c_char_p, vp, pp]
+    lib.ucl_relation_stats.argtypes = [vp, vp, c.POINTER(i64), c.POINTER(i64)]
+    lib.ucl_drop_zero_tiles.argtypes = [vp, vp, pp]
+    lib.ucl_plan.argtypes = [i32, c.POINTER(PlanVertex), c.c_char_p, c.POINTER(i64), i32, c.POINTER(CostModel), i32,
+                             c.POINTER(PlanChoice), c.POINTER(i32)]
     lib.ucl_keys_check_noalloc.argtypes = [i32, vp, i64, i32, vp, c.POINTER(i64), c.POINTER(i32)]
     lib.ucl_status_str.argtypes = [i32]
     lib.ucl_status_str.restype = c.c_char_p

@@ -456,9 +456,10 @@ ucl_status begin_timed_call(ucl_ctx *ctx) {
 // may still be writing it).
 ucl_status sync_read(ucl_ctx *ctx, const int64_t *dev, int n, int64_t *host, uint32_t *flags = nullptr) {
     cudaError_t e = cudaSuccess;
+    if (n > ucl_ctx::kPinnedRead) return fail(ctx, UCL_ERR_ARG, "too many values for one sizing sync");
     if (n > 0) e = cudaMemcpyAsync(ctx->h_pinned, dev, sizeof(int64_t) * n, cudaMemcpyDeviceToHost, ctx->stream);
     if (e == cudaSuccess)
-        e = cudaMemcpyAsync(ctx->h_pinned + 6, ctx->d_status, 4 * sizeof(uint32_t), cudaMemcpyDeviceToHost,
+        e = cudaMemcpyAsync(ctx->h_pinned + ucl_ctx::kPinnedRead, ctx->d_status, 4 * sizeof(uint32_t), cudaMemcpyDeviceToHost,
                             ctx->stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize(ctx->stream);
     if (e != cudaSuccess) return cuda_check(ctx, e, "stream sync");
@@ -466,7 +467,7 @@ ucl_status sync_read(ucl_ctx *ctx, const int64_t *dev, int n, int64_t *host, uin
     if (e != cudaSuccess) return cuda_check(ctx, e, "kernel launch");
     for (int i = 0; i < n; ++i) host[i] = ctx->h_pinned[i];
     uint32_t words[4];
-    memcpy(words, ctx->h_pinned + 6, sizeof(words));
+    memcpy(words, ctx->h_pinned + ucl_ctx::kPinnedRead, sizeof(words));
     if (flags) *flags = words[1];
     const bool on_main = ctx->stream == ctx->main;
     if (words[1]) cudaMemsetAsync(ctx->d_status + 1, 0, sizeof(uint32_t), ctx->stream);
@@ -655,7 +656,7 @@ ucl_status ucl_ctx_create(int device, void *stream, ucl_alloc_fn alloc, ucl_free
     }
     if (!st) st = cuda_check(ctx, cudaMalloc(&ctx->d_status, 256), "cudaMalloc status");
     if (!st) st = cuda_check(ctx, cudaMemset(ctx->d_status, 0, 256), "cudaMemset status");
-    if (!st) st = cuda_check(ctx, cudaMallocHost(&ctx->h_pinned, 8 * sizeof(int64_t)), "cudaMallocHost");
+    if (!st) st = cuda_check(ctx, cudaMallocHost(&ctx->h_pinned, ucl_ctx::kPinnedWords * sizeof(int64_t)), "cudaMallocHost");
     if (!st) st = cuda_check(ctx, cudaStreamCreateWithFlags(&ctx->kstream, cudaStreamNonBlocking), "cudaStreamCreate");
     if (!st) st = cuda_check(ctx, cudaEventCreateWithFlags(&ctx->ev_order, cudaEventDisableTiming), "cudaEventCreate");
     for (int i = 0; i < ucl_ctx::kArenas && !st; ++i)
@@ -1412,6 +1413,100 @@ ucl_status ucl_repartition(ucl_ctx *ctx, const char *spec_text, const ucl_rel *i
         R = nullptr;
         ctx->err.clear();
         st = UCL_OK;
+    } catch (Oom &) {
+        st = fail(ctx, UCL_ERR_OOM, "device allocation failed");
+    } catch (Fail &f) {
+        st = f.st;
+    }
+    cudaEventRecord(ctx->arena_done[arena], ctx->main);
+    if (R) ucl_relation_destroy(R);
+    return st;
+}
+
+ucl_status ucl_relation_stats(ucl_ctx *ctx, const ucl_rel *rel, int64_t *nnz, int64_t *distinct) {
+    if (!ctx || !rel) return fail(ctx, UCL_ERR_ARG, "NULL context or relation");
+    if (rel->ctx != ctx) return fail(ctx, UCL_ERR_ARG, "relation belongs to another context");
+    cudaSetDevice(ctx->device);
+    StatsGeom g;
+    stats_geometry(rel, g);
+    const int nc = rel->u + rel->r;
+    ucl_status st = UCL_OK;
+    const int arena = arena_begin(ctx);
+    try {
+        int64_t *d = (int64_t *)ws_get(ctx, sizeof(int64_t) * (1 + nc));
+        uint32_t *bits = (uint32_t *)ws_get(ctx, sizeof(uint32_t) * (size_t)std::max<int64_t>(g.words, 1));
+        check(cuda_check(ctx, cudaMemsetAsync(d, 0, sizeof(int64_t) * (1 + nc), ctx->stream), "cudaMemsetAsync"));
+        if (g.words > 0)
+            check(cuda_check(ctx, cudaMemsetAsync(bits, 0, sizeof(uint32_t) * g.words, ctx->stream),
+                             "cudaMemsetAsync"));
+        launch_relation_stats(ctx, rel, g, bits, reinterpret_cast<unsigned long long *>(d), nullptr);
+        launch_popc(ctx, bits, g, d + 1);
+        int64_t h[1 + 2 * kMaxCols];
+        check(sync_read(ctx, d, 1 + nc, h));
+        if (nnz) *nnz = h[0];
+        if (distinct)
+            for (int c = 0; c < nc; ++c) distinct[c] = h[1 + c];
+        ctx->err.clear();
+    } catch (Oom &) {
+        st = fail(ctx, UCL_ERR_OOM, "device allocation failed");
+    } catch (Fail &f) {
+        st = f.st;
+    }
+    cudaEventRecord(ctx->arena_done[arena], ctx->main);
+    return st;
+}
+
+ucl_status ucl_drop_zero_tiles(ucl_ctx *ctx, const ucl_rel *in, ucl_rel **out) {
+    if (!out) return fail(ctx, UCL_ERR_ARG, "out is NULL");
+    *out = nullptr;
+    if (!ctx || !in) return fail(ctx, UCL_ERR_ARG, "NULL context or relation");
+    if (in->ctx != ctx) return fail(ctx, UCL_ERR_ARG, "relation belongs to another context");
+    cudaSetDevice(ctx->device);
+    ucl_status st = UCL_OK;
+    ucl_rel *R = nullptr;
+    const int arena = arena_begin(ctx);
+    try {
+        const int64_t n = in->n;
+        int64_t m = 0;
+        int64_t *flag = nullptr, *excl = nullptr;
+        if (n > 0) {
+            int64_t *d_total = (int64_t *)ws_get(ctx, sizeof(int64_t));
+            flag = (int64_t *)ws_get(ctx, sizeof(int64_t) * n);
+            excl = (int64_t *)ws_get(ctx, sizeof(int64_t) * n);
+            check(cuda_check(ctx, cudaMemsetAsync(flag, 0, sizeof(int64_t) * n, ctx->stream), "cudaMemsetAsync"));
+            StatsGeom g;
+            stats_geometry(in, g);
+            g.smem_dims = 0;
+            launch_relation_stats(ctx, in, g, nullptr, nullptr, flag);
+            scan_i64(ctx, flag, excl, n, d_total);
+            check(sync_read(ctx, d_total, 1, &m));
+        }
+        R = new_rel(ctx);
+        if (!R) check(fail(ctx, UCL_ERR_OOM, "host allocation failed"));
+        R->n = m;
+        R->u = in->u;
+        R->r = in->r;
+        for (int c = 0; c < in->u; ++c) R->bounds[c] = in->bounds[c];
+        for (int q = 0; q < in->r; ++q) R->shape[q] = in->shape[q];
+        R->dtype = in->dtype;
+        R->tile = in->tile;
+        R->sorted = in->sorted;
+        R->key_bits = in->key_bits;
+        if (m > 0) {
+            const size_t tbytes = (size_t)m * in->tile * dsize(in->dtype);
+            const size_t koff = (tbytes + 255) & ~(size_t)255;
+            R->own_bytes = koff + (size_t)m * in->u * 4;
+            R->own_block = ctx_alloc(ctx, R->own_bytes);
+            if (!R->own_block) throw Oom();
+            R->tiles = R->own_block;
+            R->keys = (int32_t *)((char *)R->own_block + koff);
+            launch_compact(ctx, in, flag, excl, R->tiles, R->keys);
+        }
+        check(cuda_check(ctx, cudaGetLastError(), "kernel launch"));
+        keys_ready(ctx, R);
+        *out = R;
+        R = nullptr;
+        ctx->err.clear();
     } catch (Oom &) {
         st = fail(ctx, UCL_ERR_OOM, "device allocation failed");
     } catch (Fail &f) {

@@ -130,7 +130,10 @@ struct ucl_ctx {
     ucl::Arena *arena = &arenas[0];
     // [1] validation flags (main), [2] sticky error bits of main-stream kernels
     uint32_t *d_status = nullptr;
-    int64_t *h_pinned = nullptr;    // pinned host scratch for sizing syncs (8 words)
+    // pinned host scratch for sizing syncs: kPinnedRead int64 values, then the
+    // device status words
+    static constexpr int kPinnedRead = 36, kPinnedWords = 40;
+    int64_t *h_pinned = nullptr;
     int timing = 0;
     // CUDA events of timed calls: six per call (stage boundaries on the key
     // stream and on main), reused
@@ -246,6 +249,29 @@ void launch_out_place(ucl_ctx *ctx, const uint64_t *okey_sorted, const uint64_t 
                       const KeyUnpack &un, uint32_t *pos, int32_t *out_keys);
 void launch_repart_scatter(ucl_ctx *ctx, const void *in, ucl_dtype dt, const int32_t *keys, const uint32_t *rank,
                            const uint32_t *pos, int64_t n, const RepartCopy &pc, void *out);
+
+// ---- statistics (stats.cu)
+// Bitmap layout of one statistics pass: one bitmap per key column (bound
+// bits) then one per tile dim (extent bits), at the given word offsets.
+struct StatsGeom {
+    int u, r;
+    int64_t E;                      // elements per tile
+    int64_t ext[kMaxCols];          // tile extents
+    int64_t key_off[kMaxCols];      // word offset of key column c's bitmap
+    int64_t dim_off[kMaxCols];      // word offset of tile dim q's bitmap (dim_off[0] = end of keys if r = 0)
+    int64_t words, dim_words;       // all words; words of the tile-dim bitmaps
+    int smem_dims;                  // tile-dim bitmaps gathered in shared memory first
+};
+bool stats_geometry(const ucl_rel *R, StatsGeom &g);
+// One pass over R's tiles: count non-zeros into *nnz, mark bitmaps in bits
+// (NULL: none), set tuple_nz[t] = 1 for tuples with a non-zero (NULL: none).
+void launch_relation_stats(ucl_ctx *ctx, const ucl_rel *R, const StatsGeom &g, uint32_t *bits,
+                           unsigned long long *nnz, int64_t *tuple_nz);
+// out[c] = set bits of bitmap c (key columns, then tile dims).
+void launch_popc(ucl_ctx *ctx, const uint32_t *bits, const StatsGeom &g, int64_t *out);
+// Copy tuple t of R to position excl[t] where flag[t] is set.
+void launch_compact(ucl_ctx *ctx, const ucl_rel *R, const int64_t *flag, const int64_t *excl, void *out_tiles,
+                    int32_t *out_keys);
 
 // ---- contraction (contract_simt.cu / contract_tc.cu)
 struct ContractArgs {

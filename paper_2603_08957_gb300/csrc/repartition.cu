@@ -1,5 +1,5 @@
 // repartition.cu -- kernels that change a tensor-relation's upper/lower
-// split (paper Sec. 5: between two EinSums whose decompositions of a tensor
+// split (paper Sec. 6: between two EinSums whose decompositions of a tensor
 // differ, every tuple is decomposed along the labels that become upper, over
 // their whole range, and the pieces are stacked along the labels that become
 // lower, grouped by the new upper labels).

@@ -170,6 +170,21 @@ class Context:
         self._check(self.lib.ucl_repartition(self.handle, spec.encode(), rel.handle, ctypes.byref(h)))
         return Relation(self, h)
 
+    def stats(self, rel: "Relation"):
+        """(T, V): non-zero elements of the tensor a relation stores, and for
+        each key column then each tile dim the number of its values or indices
+        that carry a non-zero (paper Sec. 7.1)."""
+        nnz = ctypes.c_int64()
+        d = (ctypes.c_int64 * max(1, rel.u + rel.r))()
+        self._check(self.lib.ucl_relation_stats(self.handle, rel.handle, ctypes.byref(nnz), d))
+        return nnz.value, [d[i] for i in range(rel.u + rel.r)]
+
+    def drop_zero_tiles(self, rel: "Relation") -> "Relation":
+        """A relation holding the tuples of ``rel`` whose tile has a non-zero."""
+        h = ctypes.c_void_p()
+        self._check(self.lib.ucl_drop_zero_tiles(self.handle, rel.handle, ctypes.byref(h)))
+        return Relation(self, h)
+
 
 class Relation:
     """Handle of a tensor-relation living on the GPU."""
@@ -231,3 +246,63 @@ class Relation:
             self.handle, ctypes.c_void_p(keys.ctypes.data if keys.size else 0),
             ctypes.c_void_p(tiles.data_ptr() if tiles.numel() else 0)))
         return keys, tiles
+
+
+def plan(vertices, bounds: dict, cost_model: dict, k: int = 1):
+    """The k cheapest decompositions of an EinSum tree (include/ucl.h, ucl_plan).
+
+    ``vertices``: list of dicts in topological order, the last the root, each
+    with ``labels`` (str, one character per label) and either ``T`` and ``V``
+    (input tensor: non-zero count and distinct count per label) or ``left``
+    and ``right`` (producer indices; ``T``/``V`` optional measured statistics);
+    ``dtype_bytes`` defaults to 2.  ``bounds`` maps label -> extent;
+    ``cost_model`` has ``xfer``, ``flop``, ``add``, ``fixed`` (and optional
+    ``key_bytes`` and ``max_call_bytes``).  Returns [(cost, ups)], cheapest first, where ups[i] is
+    ``(up_W, up_U, up_V)`` for an EinSum vertex and ``up`` for an input, each a
+    string of the promoted labels in the tensor's label order."""
+    lib = _lib.load()
+    n = len(vertices)
+    arr = (_lib.PlanVertex * n)()
+    keep = []
+    for i, v in enumerate(vertices):
+        lab = v["labels"].encode()
+        keep.append(lab)
+        leaf = "left" not in v or v["left"] is None
+        arr[i].left = -1 if leaf else int(v["left"])
+        arr[i].right = -1 if leaf else int(v["right"])
+        arr[i].labels = lab
+        arr[i].dtype_bytes = int(v.get("dtype_bytes", 2))
+        if v.get("V") is not None:
+            dv = (ctypes.c_double * len(v["labels"]))(*[float(v["V"][c]) for c in v["labels"]])
+            keep.append(dv)
+            arr[i].distinct = dv
+            arr[i].nnz = float(v["T"])
+        else:
+            arr[i].distinct = None
+            arr[i].nnz = -1.0
+    names = "".join(bounds).encode()
+    bnd = (ctypes.c_int64 * len(bounds))(*[int(bounds[c]) for c in bounds])
+    cm = _lib.CostModel(float(cost_model.get("xfer", 0.0)), float(cost_model.get("flop", 0.0)),
+                        float(cost_model.get("add", 0.0)), float(cost_model.get("fixed", 0.0)),
+                        int(cost_model.get("key_bytes", 4)), float(cost_model.get("max_call_bytes", 0.0)))
+    out = (_lib.PlanChoice * k)()
+    n_out = ctypes.c_int()
+    st = lib.ucl_plan(n, arr, names, bnd, len(bounds), ctypes.byref(cm), k, out, ctypes.byref(n_out))
+    if st != 0:
+        raise UclError(st, "ucl_plan")
+
+    def ups(labels, mask):
+        return "".join(c for q, c in enumerate(labels) if mask >> q & 1)
+
+    res = []
+    for b in range(n_out.value):
+        pc = out[b]
+        per = []
+        for i, v in enumerate(vertices):
+            if "left" not in v or v["left"] is None:
+                per.append(ups(v["labels"], pc.up[i]))
+            else:
+                per.append((ups(v["labels"], pc.up[i]), ups(vertices[v["left"]]["labels"], pc.in_up[i][0]),
+                            ups(vertices[v["right"]]["labels"], pc.in_up[i][1])))
+        res.append((pc.cost, per))
+    return res

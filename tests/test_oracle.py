@@ -338,12 +338,12 @@ def test_relation_errors():
         oracle.einsum("Ij,Ij->I", [v, x])
 
 
-# ---------------------------------------------------- repartition (Sec. 5)
+# ---------------------------------------------------- repartition (Sec. 6)
 
 
 
 def test_repartition_row_vectors_to_column_vectors():
-    """Sec. 5's example: T stored as row vectors (upper row index) becomes T
+    """Sec. 6's example: T stored as row vectors (upper row index) becomes T
     stored as column vectors (upper column index); every column index gets a
     tuple (the decompose step ranges over the whole label)."""
     T = np.array([[1.0, 0.0, 2.0, 0.0], [0.0, 0.0, 3.0, 0.0], [4.0, 0.0, 5.0, 0.0]])

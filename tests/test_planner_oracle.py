@@ -1,5 +1,5 @@
 """Pins of the planner oracle (oracle/planner.py) against brute force, closed
-forms and invariants that the paper's definitions fix (Sec. 6.1, 6.2, Alg. 1,
+forms and invariants that the paper's definitions fix (Sec. 7.1, 7.2, Alg. 1,
 Alg. 2).  CPU only."""
 from __future__ import annotations
 
@@ -50,6 +50,31 @@ def test_relation_stats_any_decomposition():
         assert s.T == ref.T and s.V == ref.V
 
 
+def test_relation_stats_direct_matches_dense():
+    rng = np.random.default_rng(11)
+    for up in range(0, 3):
+        dense = rng.standard_normal((5, 3, 4)) * (rng.random((5, 3, 4)) < 0.15)
+        dense[1] = 0.0                                     # a key value with only zero tiles
+        dense[..., 2] = -0.0                               # a tile index holding only negative zeros
+        keys = np.array(list(itertools.product(*[range(e) for e in dense.shape[:up]])), dtype=np.int32)
+        tiles = dense.reshape((-1,) + dense.shape[up:])
+        T, V = P.relation_stats_direct(keys.reshape(len(tiles), up), dense.shape[:up], tiles)
+        ref = P.dense_stats(dense, "abc")
+        assert T == ref.T and V == [ref.V[c] for c in "abc"]
+    T, V = P.relation_stats_direct(np.zeros((0, 1), np.int32), (4,), np.zeros((0, 3)))
+    assert T == 0 and V == [0, 0]
+
+
+def test_drop_zero_tiles_keeps_the_tensor():
+    rng = np.random.default_rng(12)
+    dense = rng.standard_normal((6, 4)) * (rng.random((6, 4)) < 0.2)
+    keys = np.arange(6, dtype=np.int32)[:, None]
+    k, t = P.drop_zero_tiles(keys, dense)
+    back = np.zeros_like(dense)
+    back[k[:, 0]] = t
+    assert np.array_equal(back, dense) and all(np.any(x) for x in t)
+
+
 # ----------------------------------------------------- Eq. eqn-count
 
 def test_tuple_count_limits():
@@ -81,7 +106,7 @@ def test_tuple_count_uniform_monte_carlo():
     assert abs(est - occ) / occ < 0.03
 
 
-# ---------------------------------------------------------- Sec. 6.2
+# ---------------------------------------------------------- Sec. 7.2
 
 def _dense(labels, bounds):
     T = float(np.prod([bounds[l] for l in labels]))
@@ -192,6 +217,20 @@ def test_dp_matches_exhaustive_search(shape, seed):
     assert len(keys) == len(best)
 
 
+def test_memory_bound_exhaustive():
+    rng = np.random.default_rng(3)
+    g, bounds, cm = _random_tree(rng, "chain")
+    every = P.enumerate_plans(g, bounds, cm)
+    cm.max_call_bytes = 2048.0
+    bounded = P.enumerate_plans(g, bounds, cm)
+    ok = [(c, p) for c, p in every if all(
+        P.tile_bytes(g[v.left], p[i][1], bounds) + P.tile_bytes(g[v.right], p[i][2], bounds) +
+        P.tile_bytes(v, p[i][0], bounds) <= 2048.0 for i, v in enumerate(g) if v.left is not None)]
+    assert [c for c, _ in bounded] == [c for c, _ in ok]
+    best = P.optimize(g, bounds, cm, k=4)
+    assert [c for c, _ in best] == pytest.approx([c for c, _ in bounded[:4]], rel=1e-12)
+
+
 def test_plan_count_closed_form():
     # each label takes one class per EinSum: 2^|ℓU ∪ ℓV| plans per vertex
     rng = np.random.default_rng(1)
@@ -219,3 +258,15 @@ def test_tree_checks():
     with pytest.raises(ValueError):
         P.optimize([P.Vertex("a", stats=s), P.Vertex("a", stats=s), P.Vertex("b", 2, 0, 1)], {"a": 1, "b": 1},
                    P.CostModel())
+
+
+def test_dense_tree_brute_force():
+    from tests.ucl_testutil import brute_force
+    rng = np.random.default_rng(5)
+    X, Y, Z = rng.standard_normal((2, 3)), rng.standard_normal((3, 2, 2)), rng.standard_normal((2, 3))
+    g = [P.Vertex("ab", stats=P.Stats(1, {})), P.Vertex("bcd", stats=P.Stats(1, {})), P.Vertex("cda", 4, 0, 1),
+         P.Vertex("ae", stats=P.Stats(1, {})), P.Vertex("ce", 4, 2, 3)]
+    val = P.dense_tree(g, {0: X, 1: Y, 3: Z})
+    T = brute_force("ab,bcd->cda", [X, Y])
+    np.testing.assert_allclose(val[2], T, rtol=1e-12)
+    np.testing.assert_allclose(val[4], brute_force("cda,ae->ce", [T, Z]), rtol=1e-12)
