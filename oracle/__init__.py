@@ -41,6 +41,9 @@ STATUS = {
 }
 EPI = {"none": 0, "relu": 1}
 OUT = {"bf16": 0, "f32": 1, "f64": 2}
+AGG = {"sum": 0, "max": 1, "min": 2}
+COMB = {"mul": 0, "add": 1, "sub": 2, "div": 3}
+MAP = {"ident": 0, "relu": 1, "exp": 2, "square": 3}
 
 _MAXOPLEN = 16
 
@@ -71,6 +74,9 @@ class _Opts(ctypes.Structure):
         ("out_dtype", ctypes.c_int),
         ("sample_keys", ctypes.POINTER(ctypes.c_int32)),
         ("n_sample", ctypes.c_int64),
+        ("agg", ctypes.c_int),
+        ("comb", ctypes.c_int),
+        ("map", ctypes.c_int),
     ]
 
 
@@ -134,12 +140,16 @@ def _ptr(a: np.ndarray, ctype):
     return a.ctypes.data_as(ctypes.POINTER(ctype))
 
 
-def einsum(spec, rels, *, epi="none", scale=1.0, out_dtype="f64", sample_keys=None):
+def einsum(spec, rels, *, epi="none", scale=1.0, out_dtype="f64", sample_keys=None, agg="sum", comb="mul",
+           map="ident"):
     """Evaluate one UCL EinSum.
 
     ``rels`` is a list of ``(keys, bounds, tiles)``: keys int32 [n, u], bounds
     int [u], tiles float [n, *shape] (converted exactly to float64 here).
     ``sample_keys`` (int32 [s, uw]) restricts evaluation to those output keys.
+    ``agg`` / ``comb`` / ``map`` select the extended EinSum of Sec. 3: the
+    aggregate (sum, max, min) over the joined values of comb (mul, add, sub,
+    div) followed by map (ident, relu, exp, square).
 
     Returns a dict: keys [m, uw] int32, acc / abs / out [m, *shape] float64,
     bounds, shape, n_pairs, n_mults.
@@ -169,6 +179,9 @@ def einsum(spec, rels, *, epi="none", scale=1.0, out_dtype="f64", sample_keys=No
     opts.epi = EPI[epi]
     opts.scale = float(scale)
     opts.out_dtype = OUT[out_dtype]
+    opts.agg = AGG[agg]
+    opts.comb = COMB[comb]
+    opts.map = MAP[map]
     if sample_keys is not None:
         sk = np.ascontiguousarray(np.asarray(sample_keys, dtype=np.int32))
         arrs.append(sk)

@@ -32,7 +32,15 @@
  *     the output: a key produced by the join is kept even if its sum is 0;
  *   - tiles are row-major over the operand's lower-case letters, in the order
  *     they appear in the operand, last letter fastest;
- *   - only the (+, x) semiring is evaluated.
+ *   - the extended EinSum of Sec. 3 (Eq. Einsum's general form, an aggregate
+ *     ⊕ over the joined values of a scalar function ⊗): ⊕ is SUM, MAX or MIN,
+ *     ⊗ is the product (default), sum, difference or quotient of the two
+ *     inputs' entries, followed by an element map (identity, relu, exp or
+ *     square) -- e.g. Sec. 3's max_j (U_ij - V_ij)^2 is MAX, SUB, SQUARE; a
+ *     unary EinSum applies the map to its one input (Sec. 3's MLP example);
+ *     three inputs take the product only;
+ *   - aggregation ranges over the tuples present (SQL GROUP BY): a tuple
+ *     absent from a relation contributes nothing, also under MAX or MIN.
  */
 #include <math.h>
 #include <stdint.h>
@@ -51,6 +59,9 @@ enum {
 };
 
 enum { UO_EPI_NONE = 0, UO_EPI_RELU = 1 };
+enum { UO_AGG_SUM = 0, UO_AGG_MAX = 1, UO_AGG_MIN = 2 };
+enum { UO_COMB_MUL = 0, UO_COMB_ADD = 1, UO_COMB_SUB = 2, UO_COMB_DIV = 3 };
+enum { UO_MAP_IDENT = 0, UO_MAP_RELU = 1, UO_MAP_EXP = 2, UO_MAP_SQUARE = 3 };
 enum { UO_OUT_BF16 = 0, UO_OUT_F32 = 1, UO_OUT_F64 = 2 };
 
 #define UO_MAXIN 3
@@ -73,6 +84,7 @@ typedef struct {
     int out_dtype;
     const int32_t *sample_keys; /* optional [n_sample, uw]: only these groups are evaluated */
     int64_t n_sample;
+    int agg, comb, map;         /* extended EinSum: aggregate, combination, element map */
 } uo_opts;
 
 typedef struct {
@@ -83,7 +95,7 @@ typedef struct {
     int64_t tile;     /* prod(shape) */
     int32_t *keys;    /* [m, uw] */
     double *acc;      /* [m, tile] raw fp64 sum */
-    double *absacc;   /* [m, tile] sum of |products| */
+    double *absacc;   /* [m, tile] sum of |terms| (SUM) or largest |term| (MAX, MIN) */
     double *out;      /* [m, tile] after epilogue and cast, stored as double */
     int64_t n_pairs;  /* joined tuples (all of them, also when sampling) */
     int64_t n_mults;  /* n_pairs * prod(all lower extents) */
@@ -351,8 +363,46 @@ typedef struct {
     int err;
 } uo_ctx;
 
+/* One term of the extended EinSum: the combination of the joined entries,
+ * then the element map. */
+static double term(const uo_opts *o, int n_in, const double *x) {
+    double p;
+    if (n_in == 1) {
+        p = x[0];
+    } else if (n_in == 3 || o->comb == UO_COMB_MUL) {
+        p = 1.0;
+        for (int k = 0; k < n_in; ++k) p *= x[k];
+    } else if (o->comb == UO_COMB_ADD) {
+        p = x[0] + x[1];
+    } else if (o->comb == UO_COMB_SUB) {
+        p = x[0] - x[1];
+    } else {
+        p = x[0] / x[1];
+    }
+    switch (o->map) {
+        case UO_MAP_RELU: return p > 0 ? p : 0.0;
+        case UO_MAP_EXP: return exp(p);
+        case UO_MAP_SQUARE: return p * p;
+        default: return p;
+    }
+}
+
+/* Fold one term into the aggregate and its magnitude bound. */
+static void fold(const uo_opts *o, double *acc, double *absv, double p) {
+    if (o->agg == UO_AGG_MAX) {
+        if (p > *acc) *acc = p;
+        if (fabs(p) > *absv) *absv = fabs(p);
+    } else if (o->agg == UO_AGG_MIN) {
+        if (p < *acc) *acc = p;
+        if (fabs(p) > *absv) *absv = fabs(p);
+    } else {
+        *acc += p;
+        *absv += fabs(p);
+    }
+}
+
 /* Kernel K for one joined tuple (Sec. 5): naive loop over every lower-label
- * index combination, W[...] += prod_k U_k[...]; the last lower label is the
+ * index combination, W[...] ⊕= ⊗_k U_k[...]; the last lower label is the
  * innermost loop. */
 static void apply_kernel(uo_ctx *c, int64_t g) {
     const uo_spec *s = c->s;
@@ -362,11 +412,10 @@ static void apply_kernel(uo_ctx *c, int64_t g) {
     double *absg = c->absacc + g * c->tile_w;
     int64_t idx[UO_MAXLAB];
     for (int L = 0; L < c->nlow; ++L) idx[L] = 0;
+    double x[UO_MAXIN];
     if (c->nlow == 0) {
-        double p = 1.0;
-        for (int k = 0; k < s->n_in; ++k) p *= base[k][0];
-        accg[0] += p;
-        absg[0] += fabs(p);
+        for (int k = 0; k < s->n_in; ++k) x[k] = base[k][0];
+        fold(&c->opts, &accg[0], &absg[0], term(&c->opts, s->n_in, x));
         return;
     }
     int last = c->nlow - 1;
@@ -375,11 +424,9 @@ static void apply_kernel(uo_ctx *c, int64_t g) {
         for (int L = 0; L < last; ++L)
             for (int k = 0; k <= s->n_in; ++k) off[k] += idx[L] * c->lstr[k][L];
         for (int64_t t = 0; t < c->lext[last]; ++t) {
-            double p = 1.0;
-            for (int k = 0; k < s->n_in; ++k) p *= base[k][off[k] + t * c->lstr[k][last]];
+            for (int k = 0; k < s->n_in; ++k) x[k] = base[k][off[k] + t * c->lstr[k][last]];
             int64_t w = off[s->n_in] + t * c->lstr[s->n_in][last];
-            accg[w] += p;
-            absg[w] += fabs(p);
+            fold(&c->opts, &accg[w], &absg[w], term(&c->opts, s->n_in, x));
         }
         int L = last - 1;
         while (L >= 0) {
@@ -417,7 +464,10 @@ static void emit_joined(uo_ctx *c) {
         double *nb = (double *)realloc(c->absacc, sizeof(double) * (size_t)(ncap * c->tile_w));
         if (!nb) { c->err = UO_ERR_OOM; return; }
         c->absacc = nb;
-        memset(c->acc + c->acc_cap * c->tile_w, 0, sizeof(double) * (size_t)((ncap - c->acc_cap) * c->tile_w));
+        /* the aggregate's identity: 0, or -inf / +inf for MAX / MIN (replaced
+           by the first term, as every joined tuple reaches every entry) */
+        const double id = c->opts.agg == UO_AGG_MAX ? -INFINITY : (c->opts.agg == UO_AGG_MIN ? INFINITY : 0.0);
+        for (int64_t i = c->acc_cap * c->tile_w; i < ncap * c->tile_w; ++i) c->acc[i] = id;
         memset(c->absacc + c->acc_cap * c->tile_w, 0, sizeof(double) * (size_t)((ncap - c->acc_cap) * c->tile_w));
         c->acc_cap = ncap;
     }
@@ -501,6 +551,11 @@ int uo_einsum(const char *spec, int n_in, const uo_rel *rels, const uo_opts *opt
     if (st) return st;
     if (opts && opts->epi != UO_EPI_NONE && opts->epi != UO_EPI_RELU) return UO_ERR_ARG;
     if (opts && (opts->out_dtype < UO_OUT_BF16 || opts->out_dtype > UO_OUT_F64)) return UO_ERR_ARG;
+    if (opts && (opts->agg < UO_AGG_SUM || opts->agg > UO_AGG_MIN || opts->comb < UO_COMB_MUL ||
+                 opts->comb > UO_COMB_DIV || opts->map < UO_MAP_IDENT || opts->map > UO_MAP_SQUARE))
+        return UO_ERR_ARG;
+    if (opts && n_in == 3 && (opts->agg != UO_AGG_SUM || opts->comb != UO_COMB_MUL || opts->map != UO_MAP_IDENT))
+        return UO_ERR_UNSUPPORTED;
 
     /* arity and extents: one bound / extent per label across all operands (Sec. 3 bounds) */
     for (int k = 0; k < n_in; ++k) {

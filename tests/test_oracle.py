@@ -424,3 +424,91 @@ def test_repartition_explicit_form_with_tile_and_offset_labels():
         repartition("Jfj->fJ", rel)      # case form cannot tell J from j
     with pytest.raises(RepartitionError):
         repartition("Jfj->fj|J|", rel)
+
+
+# ------------------------------------------- extended EinSum (Sec. 3, Eq. Einsum)
+
+def _rel_from_dense(dense, labels, up):
+    keys, bounds, tiles = decompose(dense, labels, set(up), drop_zero=False)
+    return keys, bounds, tiles
+
+
+def _ext(spec, dense_ops, op_labels, ups, out_labels, out_up, **kw):
+    rels = [_rel_from_dense(d, l, u) for d, l, u in zip(dense_ops, op_labels, ups)]
+    r = oracle.einsum(spec, rels, **kw)
+    ext = {}
+    for d, l in zip(dense_ops, op_labels):
+        ext.update(zip(l, d.shape))
+    return recompose(r["keys"], r["out"], out_labels, set(out_up), ext), r
+
+
+@pytest.mark.parametrize("ups", [("ij", "ij", "i"), ("i", "i", "i"), ("", "", ""), ("j", "j", "")])
+def test_extended_max_squared_difference(ups):
+    """Sec. 3's example W_i = max_j (U_ij - V_ij)^2 under several splits."""
+    rng = np.random.default_rng(21)
+    U, V = rng.standard_normal((3, 5)), rng.standard_normal((3, 5))
+    spec = ucl_operand("ij", set(ups[0])) + "," + ucl_operand("ij", set(ups[1])) + "->" + ucl_operand("i", set(ups[2]))
+    got, r = _ext(spec, [U, V], ["ij", "ij"], ups[:2], "i", ups[2], agg="max", comb="sub", map="square")
+    np.testing.assert_allclose(got, np.max((U - V) ** 2, axis=1), rtol=1e-15)
+    # the magnitude bound of MAX is the largest |term|
+    assert np.all(r["abs"].reshape(-1) >= np.abs(r["acc"].reshape(-1)))
+
+
+@pytest.mark.parametrize("agg,np_fn", [("min", np.min), ("max", np.max), ("sum", np.sum)])
+@pytest.mark.parametrize("comb,np_op", [("mul", np.multiply), ("add", np.add), ("sub", np.subtract)])
+def test_extended_aggregates_and_combinations(agg, np_fn, comb, np_op):
+    rng = np.random.default_rng(22)
+    U, V = rng.standard_normal((4, 3)), rng.standard_normal((3, 5))
+    want = np_fn(np_op(U[:, :, None], V[None, :, :]), axis=1)
+    for ups in [("i", "k", "ik"), ("ij", "jk", "ik"), ("", "", ""), ("j", "j", "")]:
+        spec = (ucl_operand("ij", set(ups[0])) + "," + ucl_operand("jk", set(ups[1])) + "->" +
+                ucl_operand("ik", set(ups[2])))
+        got, _ = _ext(spec, [U, V], ["ij", "jk"], ups[:2], "ik", ups[2], agg=agg, comb=comb)
+        np.testing.assert_allclose(got, want, rtol=1e-13, atol=1e-15)
+
+
+def test_extended_unary_maps_and_division():
+    rng = np.random.default_rng(23)
+    U = rng.standard_normal((3, 4))
+    for m, fn in [("relu", lambda x: np.maximum(x, 0)), ("exp", np.exp), ("square", np.square), ("ident", lambda x: x)]:
+        got, _ = _ext("Ij->Ij", [U], ["ij"], ["i"], "ij", "i", map=m)
+        np.testing.assert_allclose(got, fn(U), rtol=1e-15)
+    D = rng.uniform(1, 2, 3)
+    got, _ = _ext("Ij,I->Ij", [U, D], ["ij", "i"], ["i", "i"], "ij", "i", comb="div")
+    np.testing.assert_allclose(got, U / D[:, None], rtol=1e-15)
+
+
+def test_softmax_as_extended_einsums():
+    """Row softmax as four EinSums (max; exp of the difference; sum;
+    quotient) against the textbook formula."""
+    rng = np.random.default_rng(24)
+    C = rng.standard_normal((5, 7)) * 3
+    rc = _rel_from_dense(C, "ij", {"i"})
+    M = oracle.einsum("Ij->I", [rc], agg="max")
+    rm = (M["keys"], M["bounds"], M["out"])
+    S = oracle.einsum("Ij,I->Ij", [rc, rm], comb="sub", map="exp")
+    rs = (S["keys"], S["bounds"], S["out"])
+    D = oracle.einsum("Ij->I", [rs])
+    E = oracle.einsum("Ij,I->Ij", [rs, (D["keys"], D["bounds"], D["out"])], comb="div")
+    ref = np.exp(C) / np.exp(C).sum(axis=1, keepdims=True)
+    np.testing.assert_allclose(E["out"], ref, rtol=1e-13)
+
+
+def test_extended_aggregate_ranges_over_present_tuples():
+    """MAX over a relation with absent tuples: the absent ones contribute
+    nothing (brute force over the tuples present)."""
+    rng = np.random.default_rng(25)
+    keys = np.array([[0, 1], [0, 3], [2, 0], [2, 2], [2, 3]], np.int32)
+    vals = -rng.uniform(1, 2, len(keys))               # all negative: an absent zero would win a dense max
+    r = oracle.einsum("IJ->I", [(keys, (3, 4), vals)], agg="max")
+    want = {}
+    for (i, j), v in zip(keys.tolist(), vals):
+        want[i] = max(want.get(i, -np.inf), v)
+    assert r["keys"][:, 0].tolist() == sorted(want)
+    np.testing.assert_array_equal(r["out"], [want[i] for i in sorted(want)])
+
+
+def test_extended_three_inputs_unsupported():
+    rel = (np.zeros((1, 0), np.int32), (), np.ones((1, 2)))
+    with pytest.raises(oracle.OracleError, match="UNSUPPORTED"):
+        oracle.einsum("i,i,i->i", [rel, rel, rel], agg="max")
