@@ -73,11 +73,26 @@ typedef struct ucl_rel ucl_rel;
 typedef void *(*ucl_alloc_fn)(size_t bytes, void *user);
 typedef void (*ucl_free_fn)(void *ptr, size_t bytes, void *user);
 
+/* Extended EinSum (Sec. 3, the general form of Eq. Einsum: an aggregate ⊕
+ * over the joined values of a scalar function ⊗).  The term of one joined
+ * tuple and one lower-index combination is map(comb(u, v)) -- map(u) for a
+ * unary EinSum -- and terms are folded with agg.  Sec. 3's example
+ * W_i = max_j (U_ij - V_ij)^2 is {MAX, SUB, SQUARE}; softmax is four calls
+ * ({MAX}, {SUM, SUB, EXP}, {SUM}, {SUM, DIV}).  Aggregation ranges over the
+ * tuples present, as SQL GROUP BY does: an absent tuple contributes nothing,
+ * also to MAX and MIN. */
+typedef enum { UCL_AGG_SUM = 0, UCL_AGG_MAX = 1, UCL_AGG_MIN = 2 } ucl_agg;
+typedef enum { UCL_COMB_MUL = 0, UCL_COMB_ADD = 1, UCL_COMB_SUB = 2, UCL_COMB_DIV = 3 } ucl_comb;
+typedef enum { UCL_MAP_IDENT = 0, UCL_MAP_RELU = 1, UCL_MAP_EXP = 2, UCL_MAP_SQUARE = 3 } ucl_map;
+
 typedef struct {
     ucl_dtype out_dtype;  /* dtype of the output tiles */
-    ucl_epilogue epi;     /* applied after the full group-by sum */
-    float scale;          /* out = epi(scale * sum); 1.0f for a plain sum */
+    ucl_epilogue epi;     /* applied after the full aggregate */
+    float scale;          /* out = epi(scale * aggregate); 1.0f for a plain sum */
     int path;             /* ucl_path */
+    int agg;              /* ucl_agg; UCL_AGG_SUM for the plain EinSum */
+    int comb;             /* ucl_comb; UCL_COMB_MUL for the plain EinSum */
+    int map;              /* ucl_map; UCL_MAP_IDENT for the plain EinSum */
 } ucl_einsum_opts;
 
 #define UCL_NSTAGES 4
@@ -193,6 +208,13 @@ ucl_status ucl_relation_download(const ucl_rel *rel, int32_t *keys_host, void *t
  * ucl_relation_destroy), one tuple per distinct output key produced by at
  * least one joined pair -- also when its sum is zero -- in ascending
  * lexicographic key order; tiles row-major over the output's lower labels.
+ *
+ * opts (NULL: fp32 output, plain sum of products, automatic path) selects the
+ * extended EinSum (ucl_agg / ucl_comb / ucl_map).  Anything but {SUM, MUL,
+ * IDENT} runs on the FFMA path (UCL_PATH_TC gives UCL_ERR_UNSUPPORTED) and,
+ * with three inputs, is UCL_ERR_UNSUPPORTED.  MAX / MIN fold in any order,
+ * exactly; exp is CUDA's expf; DIV is IEEE division (a zero divisor gives
+ * inf or NaN, as in IEEE arithmetic).
  *
  * Synchronises the stream twice (after the join count and after the segment
  * count: both sizes depend on the data; three inputs add one sync after the

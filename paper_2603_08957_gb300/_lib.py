@@ -60,6 +60,9 @@ class EinsumOpts(ctypes.Structure):
         ("epi", ctypes.c_int),
         ("scale", ctypes.c_float),
         ("path", ctypes.c_int),
+        ("agg", ctypes.c_int),
+        ("comb", ctypes.c_int),
+        ("map", ctypes.c_int),
     ]
 
 

@@ -883,11 +883,17 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
     if (!out) return fail(ctx, UCL_ERR_ARG, "out is NULL");
     *out = nullptr;
     if (!ctx || !in) return fail(ctx, UCL_ERR_ARG, "NULL context or inputs");
-    ucl_einsum_opts o{UCL_F32, UCL_EPI_NONE, 1.0f, UCL_PATH_AUTO};
+    ucl_einsum_opts o{UCL_F32, UCL_EPI_NONE, 1.0f, UCL_PATH_AUTO, UCL_AGG_SUM, UCL_COMB_MUL, UCL_MAP_IDENT};
     if (opts) o = *opts;
     if ((o.out_dtype != UCL_BF16 && o.out_dtype != UCL_F32) || (o.epi != UCL_EPI_NONE && o.epi != UCL_EPI_RELU) ||
-        o.path < UCL_PATH_AUTO || o.path > UCL_PATH_TC)
+        o.path < UCL_PATH_AUTO || o.path > UCL_PATH_TC || o.agg < UCL_AGG_SUM || o.agg > UCL_AGG_MIN ||
+        o.comb < UCL_COMB_MUL || o.comb > UCL_COMB_DIV || o.map < UCL_MAP_IDENT || o.map > UCL_MAP_SQUARE)
         return fail(ctx, UCL_ERR_ARG, "bad options");
+    // the extended EinSum (anything but a sum of products) runs on the FFMA path
+    const bool extended = o.agg != UCL_AGG_SUM || o.map != UCL_MAP_IDENT || (n_in > 1 && o.comb != UCL_COMB_MUL);
+    if (extended && n_in == 3) return fail(ctx, UCL_ERR_UNSUPPORTED, "three inputs take the sum of products only");
+    if (extended && o.path == UCL_PATH_TC)
+        return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: the sum of products only");
     Spec s;
     ucl_status st = parse_spec(ctx, spec_text, n_in, s);
     if (st) return st;
@@ -899,7 +905,7 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
     TcPlan tp;
     Tc3Plan tp3;
     std::string why;
-    const bool tc_ok = n_in == 3 ? plan_tc3(s, in, kp, tp3, &why) : plan_tc(s, in, tp, &why);
+    const bool tc_ok = !extended && (n_in == 3 ? plan_tc3(s, in, kp, tp3, &why) : plan_tc(s, in, tp, &why));
     if (o.path == UCL_PATH_TC && !tc_ok) return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why);
     cudaSetDevice(ctx->device);
 
@@ -1112,6 +1118,9 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             a.dout = o.out_dtype;
             a.epi = o.epi;
             a.scale = o.scale;
+            a.agg = o.agg;
+            a.comb = o.comb;
+            a.map = o.map;
             a.tile_w = lp.tile_w;
             bool use_tc = tc_ok && o.path != UCL_PATH_SIMT;
             if (use_tc && n_in < 3) {

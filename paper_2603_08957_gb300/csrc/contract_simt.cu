@@ -13,7 +13,11 @@
 //
 // This kernel is the general path: any label classes (batch labels, labels
 // summed inside one operand, rank-0 tiles, unary EinSums, fp32 or bf16
-// operands).  Accumulation is fp32 FFMA -- never TF32.
+// operands).  Accumulation is fp32 FFMA -- never TF32.  It also evaluates the
+// extended EinSum of Sec. 3 (aggregate MAX / MIN / SUM of map(comb(u, v))),
+// in a separate instantiation so that the plain sum of products keeps its
+// FFMA inner loop; partials of split segments are folded with the same
+// aggregate.
 #include "internal.cuh"
 
 namespace ucl {
@@ -36,6 +40,39 @@ __device__ __forceinline__ float epilogue(float x, int epi, float scale) {
     return x;
 }
 
+// ---- extended EinSum: term = map(comb(u, v)) (map(u) when unary), folded by agg
+__device__ __forceinline__ float sem_map(int map, float p) {
+    switch (map) {
+        case UCL_MAP_RELU: return fmaxf(p, 0.0f);
+        case UCL_MAP_EXP: return expf(p);
+        case UCL_MAP_SQUARE: return p * p;
+        default: return p;
+    }
+}
+
+__device__ __forceinline__ float sem_term(int comb, int map, float u, float v) {
+    float p;
+    switch (comb) {
+        case UCL_COMB_ADD: p = u + v; break;
+        case UCL_COMB_SUB: p = u - v; break;
+        case UCL_COMB_DIV: p = u / v; break;
+        default: p = u * v; break;
+    }
+    return sem_map(map, p);
+}
+
+__device__ __forceinline__ float sem_fold(int agg, float acc, float p) {
+    switch (agg) {
+        case UCL_AGG_MAX: return fmaxf(acc, p);
+        case UCL_AGG_MIN: return fminf(acc, p);
+        default: return acc + p;
+    }
+}
+
+__device__ __forceinline__ float sem_identity(int agg) {
+    return agg == UCL_AGG_MAX ? -INFINITY : (agg == UCL_AGG_MIN ? INFINITY : 0.0f);
+}
+
 __device__ __forceinline__ void store_out(void *out, ucl_dtype dt, int64_t idx, float x) {
     if (dt == UCL_BF16)
         reinterpret_cast<__nv_bfloat16 *>(out)[idx] = __float2bfloat16_rn(x);
@@ -53,9 +90,11 @@ __device__ __forceinline__ int64_t find_seg(const int64_t *seg_start, int64_t S,
     return a - 1;
 }
 
-template <typename TU, typename TV>
-__global__ void __launch_bounds__(kSimtThreads) simt_contract_kernel(ContractArgs a, LowerPlan lp,
-                                                                     uint32_t *status) {
+// Wide tiles with a real contraction: the whole CTA takes one segment at a
+// time, threads over output elements, pairs and contracted indices in order.
+template <typename TU, typename TV, bool EXT>
+__global__ void __launch_bounds__(kSimtThreads, 4) simt_wide_kernel(ContractArgs a, LowerPlan lp,
+                                                                   uint32_t *status) {
     __shared__ int s_cu[kMaxTab];
     __shared__ int s_cv[kMaxTab];
     const bool tab = lp.n_c <= kMaxTab;
@@ -94,7 +133,7 @@ __global__ void __launch_bounds__(kSimtThreads) simt_contract_kernel(ContractArg
                 ou += idx * lp.w_su[q];
                 ov += idx * lp.w_sv[q];
             }
-            float acc = 0.0f;
+            float acc = EXT ? sem_identity(a.agg) : 0.0f;
             for (int64_t p = p0; p < p1; ++p) {
                 const uint32_t iu = a.pu[p], iv = a.pv[p];
                 if (iu >= a.nU || (V && iv >= a.nV)) {
@@ -104,7 +143,10 @@ __global__ void __launch_bounds__(kSimtThreads) simt_contract_kernel(ContractArg
                 const TU *up = U + (int64_t)iu * lp.tile_u + ou;
                 if (V) {
                     const TV *vp = V + (int64_t)iv * lp.tile_v + ov;
-                    if (tab) {
+                    if (EXT && tab) {
+                        for (int64_t c = 0; c < lp.n_c; ++c)
+                            acc = sem_fold(a.agg, acc, sem_term(a.comb, a.map, ld<TU>(up + s_cu[c]), ld<TV>(vp + s_cv[c])));
+                    } else if (tab) {
                         for (int64_t c = 0; c < lp.n_c; ++c) acc = fmaf(ld<TU>(up + s_cu[c]), ld<TV>(vp + s_cv[c]), acc);
                     } else {
                         for (int64_t c = 0; c < lp.n_c; ++c) {
@@ -116,12 +158,16 @@ __global__ void __launch_bounds__(kSimtThreads) simt_contract_kernel(ContractArg
                                 cu += idx * lp.c_su[q];
                                 cv += idx * lp.c_sv[q];
                             }
-                            acc = fmaf(ld<TU>(up + cu), ld<TV>(vp + cv), acc);
+                            acc = EXT ? sem_fold(a.agg, acc, sem_term(a.comb, a.map, ld<TU>(up + cu), ld<TV>(vp + cv)))
+                                      : fmaf(ld<TU>(up + cu), ld<TV>(vp + cv), acc);
                         }
                     }
                 } else {
                     if (tab) {
-                        for (int64_t c = 0; c < lp.n_c; ++c) acc += ld<TU>(up + s_cu[c]);
+                        for (int64_t c = 0; c < lp.n_c; ++c) {
+                            const float x = ld<TU>(up + s_cu[c]);
+                            acc = EXT ? sem_fold(a.agg, acc, sem_map(a.map, x)) : acc + x;
+                        }
                     } else {
                         for (int64_t c = 0; c < lp.n_c; ++c) {
                             int64_t rem2 = c;
@@ -131,7 +177,8 @@ __global__ void __launch_bounds__(kSimtThreads) simt_contract_kernel(ContractArg
                                 rem2 /= lp.c_ext[q];
                                 cu += idx * lp.c_su[q];
                             }
-                            acc += ld<TU>(up + cu);
+                            const float x = ld<TU>(up + cu);
+                            acc = EXT ? sem_fold(a.agg, acc, sem_map(a.map, x)) : acc + x;
                         }
                     }
                 }
@@ -145,6 +192,148 @@ __global__ void __launch_bounds__(kSimtThreads) simt_contract_kernel(ContractArg
     if (bad) atomicOr(status, bad);
 }
 
+// Fold of one joined pair's terms for output element (ou, ov) over this
+// lane's share of the contracted index range (c = c0, c0 + R, ...).
+template <typename TU, typename TV, bool EXT>
+__device__ __forceinline__ float pair_terms(const ContractArgs &a, const LowerPlan &lp, const int *s_cu,
+                                            const int *s_cv, bool tab, const TU *up, const TV *vp, int64_t c0,
+                                            int R, float acc) {
+    for (int64_t c = c0; c < lp.n_c; c += R) {
+        int cu, cv = 0;
+        if (tab) {
+            cu = s_cu[c];
+            if (vp) cv = s_cv[c];
+        } else {
+            int64_t rem2 = c;
+            cu = 0;
+            for (int q = lp.nc - 1; q >= 0; --q) {
+                int idx = (int)(rem2 % lp.c_ext[q]);
+                rem2 /= lp.c_ext[q];
+                cu += idx * lp.c_su[q];
+                cv += idx * lp.c_sv[q];
+            }
+        }
+        const float u = ld<TU>(up + cu);
+        if (vp) {
+            const float v = ld<TV>(vp + cv);
+            acc = EXT ? sem_fold(a.agg, acc, sem_term(a.comb, a.map, u, v)) : fmaf(u, v, acc);
+        } else {
+            acc = EXT ? sem_fold(a.agg, acc, sem_map(a.map, u)) : acc + u;
+        }
+    }
+    return acc;
+}
+
+// Narrow tiles, or one term per pair: teams of T warps (T = 1, 2, 4 or 8,
+// from the tile width) take the unit's segments in turn, so that every warp
+// stays busy.  Within a team, lanes_w lanes (a power of two, at most the tile
+// width) take output elements w; when the tile is narrower than a warp the
+// R = 32 / lanes_w lanes sharing an element split the contracted index range
+// and their terms are folded by a fixed shuffle tree.  Pairs are visited in
+// order, four index pairs loaded ahead.
+template <typename TU, typename TV, bool EXT>
+__global__ void __launch_bounds__(kSimtThreads, 3) simt_team_kernel(ContractArgs a, LowerPlan lp, int team_warps,
+                                                                   uint32_t *status) {
+    __shared__ int s_cu[kMaxTab];
+    __shared__ int s_cv[kMaxTab];
+    const bool tab = lp.n_c <= kMaxTab;
+    if (tab) {
+        for (int64_t c = threadIdx.x; c < lp.n_c; c += blockDim.x) {
+            int64_t rem = c;
+            int ou = 0, ov = 0;
+            for (int q = lp.nc - 1; q >= 0; --q) {
+                int idx = (int)(rem % lp.c_ext[q]);
+                rem /= lp.c_ext[q];
+                ou += idx * lp.c_su[q];
+                ov += idx * lp.c_sv[q];
+            }
+            s_cu[c] = ou;
+            s_cv[c] = ov;
+        }
+    }
+    __syncthreads();
+
+    const TU *U = reinterpret_cast<const TU *>(a.U);
+    const TV *V = reinterpret_cast<const TV *>(a.V);
+    const int T = team_warps;
+    const int nteams = (int)(blockDim.x >> 5) / T;
+    const int team = (int)(threadIdx.x >> 5) / T;
+    const int tsize = 32 * T;
+    const int tl = (int)threadIdx.x - team * tsize;
+    int lanes_w = tsize;
+    while (lanes_w > 1 && lanes_w > a.tile_w) lanes_w >>= 1;
+    const int R = tsize / lanes_w;            // > 1 only when T = 1
+    const int wl = tl % lanes_w, rl = tl / lanes_w;
+    const float ident = EXT ? sem_identity(a.agg) : 0.0f;
+    const int unit = blockIdx.x;
+    const int64_t pb = a.units.begin(unit), pe = a.units.begin(unit + 1);
+    uint32_t bad = 0;
+    for (int64_t s = find_seg(a.seg_start, a.S, pb) + team; s < a.S; s += nteams) {
+        const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
+        if (ss >= pe) break;
+        const int64_t p0 = ss > pb ? ss : pb, p1 = se < pe ? se : pe;
+        const int kind = (ss >= pb && se <= pe) ? 0 : (ss < pb ? 1 : 2);
+        for (int64_t w0 = 0; w0 < a.tile_w; w0 += lanes_w) {
+            const int64_t w = w0 + wl;
+            const bool act = w < a.tile_w;
+            int ou = 0, ov = 0;
+            if (act) {
+                int64_t rem = w;
+                for (int q = lp.nw - 1; q >= 0; --q) {
+                    int idx = (int)(rem % lp.w_ext[q]);
+                    rem /= lp.w_ext[q];
+                    ou += idx * lp.w_su[q];
+                    ov += idx * lp.w_sv[q];
+                }
+            }
+            float acc = ident;
+            if (act) {
+                int64_t p = p0;
+                for (; p + 4 <= p1; p += 4) {
+                    uint32_t iu[4], iv[4];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        iu[j] = a.pu[p + j];
+                        iv[j] = V ? a.pv[p + j] : 0u;
+                    }
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        if (iu[j] >= a.nU || (V && iv[j] >= a.nV)) {
+                            bad = kStBadIndex;
+                            continue;
+                        }
+                        acc = pair_terms<TU, TV, EXT>(a, lp, s_cu, s_cv, tab, U + (int64_t)iu[j] * lp.tile_u + ou,
+                                                      V ? V + (int64_t)iv[j] * lp.tile_v + ov : nullptr, rl, R, acc);
+                    }
+                }
+                for (; p < p1; ++p) {
+                    const uint32_t iu = a.pu[p], iv = V ? a.pv[p] : 0u;
+                    if (iu >= a.nU || (V && iv >= a.nV)) {
+                        bad = kStBadIndex;
+                        continue;
+                    }
+                    acc = pair_terms<TU, TV, EXT>(a, lp, s_cu, s_cv, tab, U + (int64_t)iu * lp.tile_u + ou,
+                                                  V ? V + (int64_t)iv * lp.tile_v + ov : nullptr, rl, R, acc);
+                }
+            }
+            if (R > 1) {
+                // lanes sharing w differ in the bits at and above lanes_w (T = 1: one warp)
+                for (int o = lanes_w; o < 32; o <<= 1) {
+                    const float x = __shfl_xor_sync(0xffffffffu, acc, o);
+                    acc = EXT ? sem_fold(a.agg, acc, x) : acc + x;
+                }
+            }
+            if (act && rl == 0) {
+                if (kind == 0)
+                    store_out(a.out, a.dout, s * a.tile_w + w, epilogue(acc, a.epi, a.scale));
+                else
+                    a.partials[((int64_t)unit * 2 + (kind == 1 ? 0 : 1)) * a.tile_w + w] = acc;
+            }
+        }
+    }
+    if (bad) atomicOr(status, bad);
+}
+
 __device__ __forceinline__ float ld_any(const void *base, int64_t i, bool bf16) {
     return bf16 ? __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(base)[i])
                 : __ldg(reinterpret_cast<const float *>(base) + i);
@@ -153,7 +342,7 @@ __device__ __forceinline__ float ld_any(const void *base, int64_t i, bool bf16) 
 // Three-way EinSum (a star join such as MTTKRP): the product of the three
 // tiles' entries summed over the contracted lower labels.  Operand dtypes are
 // read at run time; the partial/fixup protocol is the binary kernel's.
-__global__ void __launch_bounds__(kSimtThreads) simt_contract3_kernel(ContractArgs a, LowerPlan lp,
+__global__ void __launch_bounds__(kSimtThreads, 1) simt_contract3_kernel(ContractArgs a, LowerPlan lp,
                                                                       uint32_t *status) {
     __shared__ int s_c[3][kMaxTab];
     const bool tab = lp.n_c <= kMaxTab;
@@ -247,7 +436,7 @@ __global__ void __launch_bounds__(kSimtThreads) fixup_kernel(ContractArgs a) {
     const float *first = a.partials + ((int64_t)(c - 1) * 2 + 1) * a.tile_w;
     for (int64_t w = threadIdx.x; w < a.tile_w; w += blockDim.x) {
         float acc = first[w];
-        for (int u = c; u < u_end; ++u) acc += a.partials[((int64_t)u * 2) * a.tile_w + w];
+        for (int u = c; u < u_end; ++u) acc = sem_fold(a.agg, acc, a.partials[((int64_t)u * 2) * a.tile_w + w]);
         store_out(a.out, a.dout, s * a.tile_w + w, epilogue(acc, a.epi, a.scale));
     }
 }
@@ -262,14 +451,28 @@ void launch_contract_simt(ucl_ctx *ctx, const ContractArgs &a, const LowerPlan &
         ctx->launches++;
         return;
     }
+    const bool ext = a.agg != UCL_AGG_SUM || a.map != UCL_MAP_IDENT || (a.V && a.comb != UCL_COMB_MUL);
+    // wide tiles with a real contraction: one segment per CTA at a time;
+    // otherwise warp teams (one warp per 32 output elements, up to the CTA)
+    const bool wide = a.tile_w >= kSimtThreads && lp.n_c >= 8;
+    int team = 1;
+    while (team < kSimtThreads / 32 && (int64_t)team * 64 <= a.tile_w) team <<= 1;
+#define UCL_SIMT(TU, TV)                                                                                         \
+    (wide ? (ext ? simt_wide_kernel<TU, TV, true><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status + 2)   \
+                 : simt_wide_kernel<TU, TV, false><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status + 2)) \
+          : (ext ? simt_team_kernel<TU, TV, true><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, team,                \
+                                                                                      ctx->d_status + 2)           \
+                 : simt_team_kernel<TU, TV, false><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, team,               \
+                                                                                       ctx->d_status + 2)))
     if (a.du == UCL_F32 && (!a.V || a.dv == UCL_F32))
-        simt_contract_kernel<float, float><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status + 2);
+        UCL_SIMT(float, float);
     else if (a.du == UCL_F32)
-        simt_contract_kernel<float, __nv_bfloat16><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status + 2);
+        UCL_SIMT(float, __nv_bfloat16);
     else if (!a.V || a.dv == UCL_BF16)
-        simt_contract_kernel<__nv_bfloat16, __nv_bfloat16><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status + 2);
+        UCL_SIMT(__nv_bfloat16, __nv_bfloat16);
     else
-        simt_contract_kernel<__nv_bfloat16, float><<<G, kSimtThreads, 0, ctx->stream>>>(a, lp, ctx->d_status + 2);
+        UCL_SIMT(__nv_bfloat16, float);
+#undef UCL_SIMT
     ctx->launches++;
 }
 

@@ -292,6 +292,7 @@ struct ContractArgs {
     ucl_dtype dout;
     int epi;
     float scale;
+    int agg, comb, map;    // extended EinSum (ucl_agg / ucl_comb / ucl_map); 0, 0, 0 = sum of products
     float *partials;       // [G, 2, tile_w]
     int64_t tile_w;
 };

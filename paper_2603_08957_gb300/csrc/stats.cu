@@ -38,7 +38,7 @@ struct Vec {
 };
 
 template <typename W, int V>
-__global__ void __launch_bounds__(kThreads) stats_kernel(const Vec<W, V> *__restrict__ tiles,
+__global__ void __launch_bounds__(kThreads, 1) stats_kernel(const Vec<W, V> *__restrict__ tiles,
                                                          const int32_t *__restrict__ keys, int64_t n, StatsGeom g,
                                                          uint32_t *bits, unsigned long long *nnz, int64_t *tuple_nz) {
     extern __shared__ uint32_t sbits[];

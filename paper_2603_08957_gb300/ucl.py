@@ -19,6 +19,9 @@ _DTYPES = {torch.bfloat16: BF16, torch.float32: F32}
 _TORCH = {BF16: torch.bfloat16, F32: torch.float32}
 EPI = {"none": 0, "relu": 1}
 PATH = {"auto": 0, "simt": 1, "tc": 2}
+AGG = {"sum": 0, "max": 1, "min": 2}
+COMB = {"mul": 0, "add": 1, "sub": 2, "div": 3}
+MAP = {"ident": 0, "relu": 1, "exp": 2, "square": 3}
 OUT = {"bf16": BF16, "f32": F32, torch.bfloat16: BF16, torch.float32: F32}
 MEM_BORROW, MEM_DEVICE_COPY, MEM_HOST_COPY = 0, 1, 2
 
@@ -155,9 +158,11 @@ class Context:
         return rel
 
     def einsum(self, spec: str, *rels: "Relation", out_dtype="f32", epi="none", scale: float = 1.0,
-               path="auto") -> "Relation":
-        """Evaluate one UCL EinSum (see include/ucl.h for the grammar)."""
-        opts = _lib.EinsumOpts(OUT[out_dtype], EPI[epi], float(scale), PATH[path])
+               path="auto", agg="sum", comb="mul", map="ident") -> "Relation":
+        """Evaluate one UCL EinSum (see include/ucl.h for the grammar); agg /
+        comb / map select the extended EinSum (sum|max|min, mul|add|sub|div,
+        ident|relu|exp|square)."""
+        opts = _lib.EinsumOpts(OUT[out_dtype], EPI[epi], float(scale), PATH[path], AGG[agg], COMB[comb], MAP[map])
         arr = (ctypes.c_void_p * len(rels))(*[r.handle for r in rels])
         h = ctypes.c_void_p()
         self._check(self.lib.ucl_einsum(self.handle, spec.encode(), len(rels), arr, ctypes.byref(opts),

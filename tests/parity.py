@@ -24,10 +24,11 @@ def gpu_rel(ctx, rel, copy=False):
     return ctx.relation(torch.as_tensor(keys).to(dev), bounds, tiles.to(dev), copy=copy)
 
 
-def oracle_ref(spec, rels, *, epi="none", scale=1.0, sample_keys=None):
-    """Oracle result with the epilogue applied in fp64 (no output cast)."""
+def oracle_ref(spec, rels, *, epi="none", scale=1.0, sample_keys=None, **ext):
+    """Oracle result with the epilogue applied in fp64 (no output cast);
+    ``ext`` passes the extended EinSum's agg / comb / map."""
     ins = [(k, b, t.detach().to("cpu", torch.float64).numpy() if torch.is_tensor(t) else t) for k, b, t in rels]
-    return oracle.einsum(spec, ins, epi=epi, scale=scale, out_dtype="f64", sample_keys=sample_keys)
+    return oracle.einsum(spec, ins, epi=epi, scale=scale, out_dtype="f64", sample_keys=sample_keys, **ext)
 
 
 def assert_parity(out_rel, ref, in_dtype, *, scale=1.0, select=None):

@@ -309,6 +309,59 @@ def mttkrp(seed=0, n=100_000, nnz=10_000_000, t=16, rank=64, s=1.1, device="cpu"
     }
 
 
+def graph_attention(seed=0, n=3327, feat=3703, feat_nnz=32, edges=9104, dk=1024, device="cpu"):
+    """Sparse attention of a graph transformer, shaped like the paper's
+    Planetoid.CiteSeer experiment (3327 nodes, 3703 bag-of-words features,
+    9104 directed edge entries, 1024-wide projections).
+
+    X: 0/1 bag-of-words, ``feat_nnz`` distinct features per node drawn
+    uniformly, as scalar tuples keyed (node, feature); WQ, WK: feat x dk bf16
+    N(0, 1/feat), one dk-vector per feature; A: ``edges`` / 2 distinct
+    undirected node pairs (no self-loops) drawn uniformly, both directions,
+    value 1, keyed (node, node).
+
+    The chain (the schema of the paper's table of UCL EinSums, then row
+    softmax over the neighbours present as four extended EinSums):
+      T0 = IM,Mk->Ik   T1 = JN,Nk->Jk   T2 = Ik,IJ->IJk   T3 = IJk,Jk->IJ
+      Attn = IJ->IJ scaled by 1/sqrt(dk)
+      M = max_J Attn; S = exp(Attn - M); D = sum_J S; P = S / D."""
+    rng = np.random.default_rng(seed)
+    rows = np.repeat(np.arange(n), feat_nnz)
+    cols = np.concatenate([rng.choice(feat, size=feat_nnz, replace=False) for _ in range(n)])
+    xk = np.stack([rows, cols], axis=1).astype(np.int32)
+    xk = xk[np.lexsort((xk[:, 1], xk[:, 0]))]
+    X = (xk, (n, feat), torch.ones(len(xk), dtype=torch.bfloat16, device=device))
+    g = torch.Generator().manual_seed(seed)
+
+    def proj():
+        w = (torch.randn((feat, dk), generator=g) / math.sqrt(feat)).to(torch.bfloat16)
+        return (np.arange(feat, dtype=np.int32)[:, None], (feat,), w.to(device))
+
+    want = edges // 2
+    pairs = set()
+    while len(pairs) < want:
+        a, b = rng.integers(0, n, size=2 * (want - len(pairs)) + 16).reshape(-1, 2).T
+        for x, y in zip(a.tolist(), b.tolist()):
+            if x != y and len(pairs) < want:
+                pairs.add((min(x, y), max(x, y)))
+    e = np.array(sorted(pairs), dtype=np.int64)
+    ak = np.concatenate([e, e[:, ::-1]]).astype(np.int32)
+    ak = ak[np.lexsort((ak[:, 1], ak[:, 0]))]
+    A = (ak, (n, n), torch.ones(len(ak), dtype=torch.bfloat16, device=device))
+    chain = [
+        ("T0", "IM,Mk->Ik", ["XQ", "WQ"], {"out_dtype": "bf16"}),
+        ("T1", "JN,Nk->Jk", ["XK", "WK"], {"out_dtype": "bf16"}),
+        ("T2", "Ik,IJ->IJk", ["T0", "A"], {"out_dtype": "bf16"}),
+        ("T3", "IJk,Jk->IJ", ["T2", "T1"], {"out_dtype": "f32"}),
+        ("Attn", "IJ->IJ", ["T3"], {"out_dtype": "f32", "scale": 1.0 / math.sqrt(dk)}),
+        ("M", "IJ->I", ["Attn"], {"out_dtype": "f32", "agg": "max"}),
+        ("S", "IJ,I->IJ", ["Attn", "M"], {"out_dtype": "f32", "comb": "sub", "map": "exp"}),
+        ("D", "IJ->I", ["S"], {"out_dtype": "f32"}),
+        ("P", "IJ,I->IJ", ["S", "D"], {"out_dtype": "f32", "comb": "div"}),
+    ]
+    return {"X": X, "XQ": X, "XK": X, "WQ": proj(), "WK": proj(), "A": A, "chain": chain, "n": n, "dk": dk}
+
+
 def to_oracle(rel):
     """(keys, bounds, tiles) with tiles converted exactly to float64 numpy."""
     keys, bounds, tiles = rel
