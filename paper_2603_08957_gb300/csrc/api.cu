@@ -659,6 +659,9 @@ ucl_status ucl_ctx_create(int device, void *stream, ucl_alloc_fn alloc, ucl_free
     if (!st) st = cuda_check(ctx, cudaMallocHost(&ctx->h_pinned, ucl_ctx::kPinnedWords * sizeof(int64_t)), "cudaMallocHost");
     if (!st) st = cuda_check(ctx, cudaStreamCreateWithFlags(&ctx->kstream, cudaStreamNonBlocking), "cudaStreamCreate");
     if (!st) st = cuda_check(ctx, cudaEventCreateWithFlags(&ctx->ev_order, cudaEventDisableTiming), "cudaEventCreate");
+    if (!st) st = cuda_check(ctx, cudaStreamCreateWithFlags(&ctx->cstream, cudaStreamNonBlocking), "cudaStreamCreate");
+    if (!st) st = cuda_check(ctx, cudaEventCreateWithFlags(&ctx->ev_copy0, cudaEventDisableTiming), "cudaEventCreate");
+    if (!st) st = cuda_check(ctx, cudaEventCreateWithFlags(&ctx->ev_copy1, cudaEventDisableTiming), "cudaEventCreate");
     for (int i = 0; i < ucl_ctx::kArenas && !st; ++i)
         st = cuda_check(ctx, cudaEventCreateWithFlags(&ctx->arena_done[i], cudaEventDisableTiming), "cudaEventCreate");
     if (st) {
@@ -666,6 +669,9 @@ ucl_status ucl_ctx_create(int device, void *stream, ucl_alloc_fn alloc, ucl_free
         if (ctx->h_pinned) cudaFreeHost(ctx->h_pinned);
         if (ctx->kstream) cudaStreamDestroy(ctx->kstream);
         if (ctx->ev_order) cudaEventDestroy(ctx->ev_order);
+        if (ctx->cstream) cudaStreamDestroy(ctx->cstream);
+        if (ctx->ev_copy0) cudaEventDestroy(ctx->ev_copy0);
+        if (ctx->ev_copy1) cudaEventDestroy(ctx->ev_copy1);
         for (cudaEvent_t e : ctx->arena_done)
             if (e) cudaEventDestroy(e);
         delete ctx;
@@ -687,7 +693,11 @@ ucl_status ucl_ctx_destroy(ucl_ctx *ctx) {
     cudaFree(ctx->d_status);
     cudaFreeHost(ctx->h_pinned);
     cudaStreamDestroy(ctx->kstream);
+    cudaStreamSynchronize(ctx->cstream);
+    cudaStreamDestroy(ctx->cstream);
     cudaEventDestroy(ctx->ev_order);
+    cudaEventDestroy(ctx->ev_copy0);
+    cudaEventDestroy(ctx->ev_copy1);
     for (cudaEvent_t e : ctx->arena_done) cudaEventDestroy(e);
     for (cudaEvent_t e : ctx->ev_pool) cudaEventDestroy(e);
     delete ctx;
@@ -778,6 +788,7 @@ ucl_status ucl_relation_create(ucl_ctx *ctx, int64_t n, int u, const int32_t *ke
 
     size_t kbytes = (size_t)n * u * sizeof(int32_t), tbytes = (size_t)n * tmp.tile * dsize(dtype);
     size_t koff = (tbytes + 255) & ~(size_t)255;
+    bool copying = false;   // a tile copy is in flight on the copy stream
     if (mem == UCL_MEM_DEVICE_BORROW) {
         tmp.keys = const_cast<int32_t *>(keys);
         tmp.tiles = const_cast<void *>(tiles);
@@ -788,15 +799,25 @@ ucl_status ucl_relation_create(ucl_ctx *ctx, int64_t n, int u, const int32_t *ke
         tmp.tiles = tmp.own_block;
         tmp.keys = (int32_t *)((char *)tmp.own_block + koff);
         cudaMemcpyKind kind = mem == UCL_MEM_HOST_COPY ? cudaMemcpyHostToDevice : cudaMemcpyDeviceToDevice;
-        cudaError_t e = cudaMemcpyAsync(tmp.tiles, tiles, tbytes, kind, ctx->stream);
+        // The tile copy goes on the copy stream, ordered after main's earlier
+        // work (the block may be one main freed a moment ago), so that the key
+        // copy and validation below run on main while it is in flight.  Main
+        // is ordered after the copy before this call returns.
+        cudaError_t e = cudaEventRecord(ctx->ev_copy0, ctx->stream);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(ctx->cstream, ctx->ev_copy0, 0);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(tmp.tiles, tiles, tbytes, kind, ctx->cstream);
+        if (e == cudaSuccess) e = cudaEventRecord(ctx->ev_copy1, ctx->cstream);
+        if (e == cudaSuccess) copying = true;
         if (e == cudaSuccess && kbytes) e = cudaMemcpyAsync(tmp.keys, keys, kbytes, kind, ctx->stream);
         if (e != cudaSuccess) {
+            if (copying) cudaStreamWaitEvent(ctx->stream, ctx->ev_copy1, 0);
             ctx_free(ctx, tmp.own_block, tmp.own_bytes);
             return cuda_check(ctx, e, "copy of relation storage");
         }
     }
     tmp.sorted = 1;
     ucl_status st = UCL_OK;
+    ucl_rel *R = nullptr;
     if (n > 0 && u > 0) {
         const int arena = arena_begin(ctx);
         try {
@@ -818,17 +839,27 @@ ucl_status ucl_relation_create(ucl_ctx *ctx, int64_t n, int u, const int32_t *ke
         }
         cudaEventRecord(ctx->arena_done[arena], ctx->main);
     }
+    if (!st && !(R = new_rel(ctx))) st = fail(ctx, UCL_ERR_OOM, "host allocation failed");
     if (st) {
+        if (copying) cudaStreamWaitEvent(ctx->stream, ctx->ev_copy1, 0);
         if (tmp.own_block) ctx_free(ctx, tmp.own_block, tmp.own_bytes);
         return st;
     }
-    ucl_rel *R = new_rel(ctx);
-    if (!R) {
-        if (tmp.own_block) ctx_free(ctx, tmp.own_block, tmp.own_bytes);
-        return fail(ctx, UCL_ERR_OOM, "host allocation failed");
-    }
     *R = tmp;
+    // keys are valid here: the key stream may start on them while the tile
+    // copy is still in flight; main (contractions, frees) waits for the copy
     keys_ready(ctx, R);
+    if (copying) {
+        cudaStreamWaitEvent(ctx->stream, ctx->ev_copy1, 0);
+        // host memory may be reused as soon as this call returns
+        if (mem == UCL_MEM_HOST_COPY) {
+            cudaError_t e = cudaEventSynchronize(ctx->ev_copy1);
+            if (e != cudaSuccess) {
+                ucl_relation_destroy(R);
+                return cuda_check(ctx, e, "copy of relation storage");
+            }
+        }
+    }
     *out = R;
     ctx->err.clear();
     return UCL_OK;

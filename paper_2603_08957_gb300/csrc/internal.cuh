@@ -117,6 +117,12 @@ struct ucl_ctx {
     cudaStream_t main = nullptr;
     cudaStream_t kstream = nullptr;
     cudaEvent_t ev_order = nullptr;   // scratch event for one-off stream ordering
+    // Tile copies of ucl_relation_create run on `cstream`, so that the key
+    // validation on main (and the next call's key stage) overlaps them;
+    // ev_copy0 orders the copy after main's earlier work, ev_copy1 orders
+    // main after the copy.
+    cudaStream_t cstream = nullptr;
+    cudaEvent_t ev_copy0 = nullptr, ev_copy1 = nullptr;
     ucl_alloc_fn alloc = nullptr;
     ucl_free_fn free_fn = nullptr;
     void *user = nullptr;

@@ -243,10 +243,30 @@ class Relation:
             tiles = tiles.view(torch.bfloat16)
         return keys, tiles
 
-    def download(self):
-        """Copy to the host through the C ABI: (keys np.int32 [n, u], tiles torch CPU [n, *shape])."""
-        keys = np.zeros((self.n, self.u), dtype=np.int32)
-        tiles = torch.empty((self.n,) + self.shape, dtype=self.dtype)
+    def download(self, keys_out=None, tiles_out=None):
+        """Copy to the host through the C ABI: (keys np.int32 [n, u], tiles torch CPU [n, *shape]).
+
+        keys_out / tiles_out: optional host buffers to copy into (e.g. pinned
+        torch tensors reused across calls); they must hold at least n * u
+        int32 and n * prod(shape) elements of the relation's dtype, and the
+        returned arrays are views of their leading elements."""
+        if keys_out is None:
+            keys = np.zeros((self.n, self.u), dtype=np.int32)
+        else:
+            kt = torch.as_tensor(keys_out)
+            if kt.device.type != "cpu" or kt.dtype != torch.int32 or not kt.is_contiguous() \
+                    or kt.numel() < self.n * self.u:
+                raise ValueError("keys_out must be a contiguous host int32 buffer of at least n * u elements")
+            keys = kt.reshape(-1)[: self.n * self.u].numpy().reshape(self.n, self.u)
+        if tiles_out is None:
+            tiles = torch.empty((self.n,) + self.shape, dtype=self.dtype)
+        else:
+            per = int(np.prod(self.shape)) if self.shape else 1
+            if tiles_out.device.type != "cpu" or tiles_out.dtype != self.dtype or not tiles_out.is_contiguous() \
+                    or tiles_out.numel() < self.n * per:
+                raise ValueError("tiles_out must be a contiguous host buffer of the relation's dtype, "
+                                 "at least n * prod(shape) elements")
+            tiles = tiles_out.reshape(-1)[: self.n * per].view((self.n,) + self.shape)
         self.ctx._check(self.ctx.lib.ucl_relation_download(
             self.handle, ctypes.c_void_p(keys.ctypes.data if keys.size else 0),
             ctypes.c_void_p(tiles.data_ptr() if tiles.numel() else 0)))

@@ -294,6 +294,24 @@ def test_host_copy_and_download(ctx):
     B = ctx.relation(torch.from_numpy(w["B"][0]), w["B"][1], w["B"][2])
     out = ctx.einsum(w["spec"], A, B)
     assert_parity(out, oracle_ref(w["spec"], [w["A"], w["B"]]), torch.float32)
+    # the same result downloaded into reused pinned buffers (larger than needed)
+    k0, t0 = out.download()
+    kb = torch.full((out.n * out.u + 7,), -1, dtype=torch.int32).pin_memory()
+    tb = torch.full((t0.numel() + 5,), float("nan"), dtype=torch.float32).pin_memory()
+    for _ in range(2):
+        k1, t1 = out.download(kb, tb)
+        assert np.array_equal(k1, k0) and torch.equal(t1, t0)
+    assert np.all(kb[out.n * out.u:].numpy() == -1) and torch.isnan(tb[t0.numel():]).all()
+    # copied relations from pinned host memory and from device memory
+    ta_p = ta.pin_memory()
+    A2 = ctx.relation(torch.from_numpy(ka), ba, ta_p)
+    A3 = ctx.relation(torch.from_numpy(ka).cuda(), ba, ta.cuda(), copy=True)
+    for R in (A2, A3):
+        o = ctx.einsum(w["spec"], R, B)
+        k2, t2 = o.download()
+        assert np.array_equal(k2, k0) and torch.equal(t2, t0)
+    with pytest.raises(ValueError):
+        out.download(kb[:1], tb)
 
 
 def test_deterministic(ctx):
