@@ -452,6 +452,53 @@ def cpu_baseline(W, seconds=12.0):
                       f"{dt:.1f} s single-threaded fp64 C); FLOPs of those tuples / time"}
 
 
+def _oracle_proc(sample, ready, start, out):
+    """One host core of the all-cores baseline: load the oracle, report
+    ready, wait for the common start, time the oracle on its own sample."""
+    import oracle
+    oracle.build()
+    spec, rels, sk, _ = sample
+    ready.put(os.getpid())
+    start.wait()
+    t0 = time.perf_counter()
+    r = oracle.einsum(spec, rels, sample_keys=sk)
+    out.put((time.perf_counter() - t0, int(r["keys"].shape[0])))
+
+
+def cpu_baseline_all_cores(W, seconds=6.0, cores=None):
+    """The oracle as it stands, one process per host core, each on its own
+    bounded sample of the workload (independent output keys), all started
+    together; value = all samples' FLOPs / the slowest process's time."""
+    import multiprocessing as mpc
+    if hasattr(W, "oracle_time"):   # a workload timed its own way (repartition)
+        return None
+    cores = cores or os.cpu_count() or 1
+    target = max(16, int(oracle_rate(W) * seconds))
+    samples = [W.sample(target, seed=2000 + i) for i in range(cores)]
+    mp = mpc.get_context("spawn")   # never fork a process that holds a CUDA context
+    ready, out, start = mp.Queue(), mp.Queue(), mp.Event()
+    procs = [mp.Process(target=_oracle_proc, args=(smp, ready, start, out), daemon=True) for smp in samples]
+    for p in procs:
+        p.start()
+    try:
+        for _ in procs:
+            ready.get(timeout=600)
+        start.set()
+        res = [out.get(timeout=1200) for _ in procs]
+    finally:
+        for p in procs:
+            p.join(60)
+    wall = max(t for t, _ in res)
+    tuples = sum(smp[3] for smp in samples)
+    assert sorted(k for _, k in res) == sorted(len(smp[2]) for smp in samples)
+    spec = W.chain[0][1]
+    return {"value": W.flops_per_tuple * tuples / wall / W.scale, "unit": W.unit or UNIT, "cores": cores,
+            "kind": "oracle",
+            "sample": f"first EinSum {spec}, {cores} processes at once, each on a random sample of output keys "
+                      f"(~{target} joined tuples each, {tuples} in all, slowest {wall:.1f} s, single-threaded fp64 C "
+                      f"per process); FLOPs of all samples / slowest time"}
+
+
 def run_reference(args, world, rank):
     """The oracle as the reference arm: each step a bounded sample of the workload."""
     if rank != 0:
@@ -650,9 +697,10 @@ def run_ucl(args, world, rank, local):
                "d2h_bytes_per_step": int(d2h), "ms_per_step": te * 1e3}
         del host
 
-    cpu = None
+    cpu = cpu_all = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(W, seconds=args.cpu_seconds)
+        cpu_all = cpu_baseline_all_cores(W, seconds=args.cpu_seconds / 4)
 
     if rank == 0:
         line = {"metric": W.metric or METRIC, "value": value, "unit": W.unit or UNIT, "n_gpus": world, "steps": steps,
@@ -663,6 +711,7 @@ def run_ucl(args, world, rank, local):
                            "l2": W.l2, "path": [s["path"] for s in stats],
                            "parallelism": f"replicas x{world}", "alloc": args.alloc},
                 "roofline": roof, "stage_ms": stages, "stage_roofline": per_einsum, "cpu_baseline": cpu,
+                "cpu_baseline_all_cores": cpu_all,
                 "e2e": e2e if e2e is not None else (None if W.hostable else
                                                     {"value": None, "unit": UNIT,
                                                      "skipped": "inputs too large to stage through host memory"}),
