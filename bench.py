@@ -162,13 +162,13 @@ class Mttkrp(Workload):
     def __init__(self, dev, args):
         super().__init__(dev, args)
         import workloads
-        self.w = w = workloads.mttkrp(seed=0, nnz=args.nnz, device=dev)
+        self.w = w = workloads.mttkrp(seed=0, nnz=args.nnz, device=dev, layout=args.t_layout)
         self.inputs = {k: w[k] for k in ("T", "B", "C")}
         self.chain = [("M", w["spec"], ["T", "B", "C"], {"out_dtype": "f32"})]
         self.flops_per_tuple = 2.0 * 16 * 16 * 16 * 64
         nt = len(w["T"][0])
         self.desc = (f"MTTKRP M[i,r]=sum T[i,j,k] B[j,r] C[k,r]: T 100000^3 with {args.nnz:.0e} Zipf(1.1) nonzeros in {nt} "
-                     f"nonempty 16^3 bf16 tiles, B, C 100000x64 bf16; spec IJKijk,Jjr,Kkr->Iir")
+                     f"nonempty 16^3 bf16 tiles, B, C 100000x64 bf16; spec {w['spec']}")
         self.l2 = f"inputs larger than L2 (T {nt * 8192 / 1e9:.1f} GB); no flush"
 
     def sample(self, target, seed):
@@ -829,6 +829,8 @@ def main():
                          "allocator hooks) or the library's cudaMallocAsync pool")
     ap.add_argument("--vertices", type=int, default=100_000, help="gnn graph size (reduced sizes for profiling)")
     ap.add_argument("--nnz", type=int, default=10_000_000, help="mttkrp nonzeros (reduced sizes for profiling)")
+    ap.add_argument("--t-layout", choices=["ijk", "kij"], default="ijk",
+                    help="mttkrp: storage order of each T tile (the same EinSum either way)")
     ap.add_argument("--seconds", type=float, default=3.0, help="timed seconds when --steps is not given")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-step-seconds", type=float, default=3.0)

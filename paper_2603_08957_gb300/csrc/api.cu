@@ -336,8 +336,8 @@ bool plan_tc(const Spec &s, ucl_rel *const *in, TcPlan &tp, std::string *why) {
     return true;
 }
 
-// Three inputs of the MTTKRP shape: T with lower labels (i, e, f) in that
-// tile order, factor E with e and r, factor F with f and r laid out [f][r],
+// Three inputs of the MTTKRP shape: T with lower labels (i, e, f) or
+// (f, i, e) in that tile order, factor E with e and r, factor F with f and r laid out [f][r],
 // output with i and r; no other lower label; extents i = e = f = 16,
 // r = 64; all bf16.  E is the factor of the first join when T is in it (its
 // tuple changes least often along the pair list).
@@ -358,7 +358,12 @@ bool plan_tc3(const Spec &s, ucl_rel *const *in, const KeyPlan &kp, Tc3Plan &tp,
     int lab[3] = {-1, -1, -1};
     for (size_t i = 0; i < s.labs.size(); ++i)
         if (!s.labs[i].upper && s.labs[i].pos[t] >= 0) lab[s.labs[i].pos[t]] = (int)i;
-    const Label &Li = s.labs[lab[0]], &Le = s.labs[lab[1]], &Lf = s.labs[lab[2]];
+    // T laid out [i][e][f] (f fastest: a K-major MMA operand with 32-byte
+    // rows) or [f][i][e] ((i, e) contiguous: an MN-major operand with
+    // 128-byte rows); i is the output label
+    tp.t_mn = s.labs[lab[0]].pos[3] < 0 && s.labs[lab[1]].pos[3] >= 0;
+    const int li = tp.t_mn ? lab[1] : lab[0], le = tp.t_mn ? lab[2] : lab[1], lf = tp.t_mn ? lab[0] : lab[2];
+    const Label &Li = s.labs[li], &Le = s.labs[le], &Lf = s.labs[lf];
     int fe = -1, ff = -1;
     for (int k = 0; k < 3; ++k) {
         if (k == t) continue;

@@ -86,6 +86,7 @@ struct Tc3Args {
     int64_t tile_w, sWi, sWr;
     uint32_t idesc;
     uint64_t a_desc0, b_desc0;      // start address field 0
+    int t_mn;                       // T tiles [k][(i, j)]: four 64-column boxes of 16 rows (else one box of 256 rows)
     uint32_t *status;
 };
 
@@ -156,11 +157,11 @@ __device__ __forceinline__ void arrive(uint32_t bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 
-__device__ __forceinline__ void tma3d(uint32_t dst, const CUtensorMap *map, int z, uint32_t bar) {
+__device__ __forceinline__ void tma3d(uint32_t dst, const CUtensorMap *map, int z, uint32_t bar, int x = 0) {
     asm volatile(
         "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
         "[%5];" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(0), "r"(z), "r"(bar)
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(0), "r"(z), "r"(bar)
         : "memory");
 }
 
@@ -338,7 +339,15 @@ __global__ void __launch_bounds__(kThreads3, 1)
             if (!__shfl_sync(0xffffffffu, okw, 0)) break;
             if (lane < np) {
                 const uint32_t fb = full0 + 8u * st, s0 = sbase + st * kStageBytes;
-                tma3d(s0 + (uint32_t)lane * kTBytes, &tmT, (int)it, fb);
+                if (a.t_mn) {
+                    // [k][(i, j)]: 16 rows of 512 bytes as four 128-byte-wide
+                    // boxes, each its own 2 KB 128B-swizzled sub-tile
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        tma3d(s0 + (uint32_t)lane * kTBytes + (uint32_t)q * (kTBytes / 4), &tmT, (int)it, fb, 64 * q);
+                } else {
+                    tma3d(s0 + (uint32_t)lane * kTBytes, &tmT, (int)it, fb);
+                }
                 tma3d(s0 + kPps3 * kTBytes + (2u * lane + 1u) * kFBytes, &tmF, (int)iff, fb);
             }
             __syncwarp();
@@ -526,7 +535,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode3() {
 }
 
 // 3-D map over an array of [rows][cols] bf16 tiles, one box per tile.
-bool map3(CUtensorMap *m, const void *base, int64_t n, int cols, int rows, CUtensorMapSwizzle swz, std::string *why) {
+bool map3(CUtensorMap *m, const void *base, int64_t n, int cols, int rows, CUtensorMapSwizzle swz, std::string *why,
+          int box_cols = 0) {
     auto enc = encode3();
     if (!enc) {
         *why = "cuTensorMapEncodeTiled unavailable";
@@ -534,7 +544,7 @@ bool map3(CUtensorMap *m, const void *base, int64_t n, int cols, int rows, CUten
     }
     cuuint64_t dims[3] = {(cuuint64_t)cols, (cuuint64_t)rows, (cuuint64_t)n};
     cuuint64_t strides[2] = {(cuuint64_t)cols * 2, (cuuint64_t)rows * cols * 2};
-    cuuint32_t box[3] = {(cuuint32_t)cols, (cuuint32_t)rows, 1};
+    cuuint32_t box[3] = {(cuuint32_t)(box_cols ? box_cols : cols), (cuuint32_t)rows, 1};
     cuuint32_t estr[3] = {1, 1, 1};
     CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, estr,
                      CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -560,7 +570,9 @@ ucl_status launch_contract_tc3(ucl_ctx *ctx, const ContractArgs &a, const Tc3Pla
         return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: tile arrays not 16-byte aligned");
     CUtensorMap mT, mF, mE;
     // E is copied as stored (no swizzle): [shape0][shape1]
-    if (!map3(&mT, T->tiles, T->n, 16, 256, CU_TENSOR_MAP_SWIZZLE_32B, &why) ||
+    const bool tmn = tp.t_mn;
+    if (!(tmn ? map3(&mT, T->tiles, T->n, 256, 16, CU_TENSOR_MAP_SWIZZLE_128B, &why, 64)
+              : map3(&mT, T->tiles, T->n, 16, 256, CU_TENSOR_MAP_SWIZZLE_32B, &why)) ||
         !map3(&mF, F->tiles, F->n, 64, 16, CU_TENSOR_MAP_SWIZZLE_128B, &why) ||
         !map3(&mE, E->tiles, E->n, (int)E->shape[1], (int)E->shape[0], CU_TENSOR_MAP_SWIZZLE_NONE, &why))
         return fail(ctx, UCL_ERR_CUDA, "tcgen05 path: " + why);
@@ -585,13 +597,21 @@ ucl_status launch_contract_tc3(ucl_ctx *ctx, const ContractArgs &a, const Tc3Pla
     k.sWi = tp.sWi;
     k.sWr = tp.sWr;
     // kind::f16, D fp32, A and B bf16, A MN-major (F tile rows run over k,
-    // r contiguous), B K-major (T rows (i, j), k contiguous), N = 128, M = 128
-    k.idesc = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
+    // r contiguous), B K-major (T rows (i, j), k contiguous) or, for T laid out
+    // [k][(i, j)], MN-major; N = 128, M = 128
+    k.t_mn = tmn ? 1 : 0;
+    k.idesc = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | ((tmn ? 1u : 0u) << 16) | ((128u >> 3) << 17) |
+              ((128u >> 4) << 24);
     // A: 128B swizzle, next 64-row M atom one F block further (LBO), next 8
-    // k rows 1024 bytes further (SBO).  B: 32B swizzle, 8 rows of 32 bytes per
-    // core matrix group (SBO 256).
+    // k rows 1024 bytes further (SBO).  B, K-major: 32B swizzle, 8 rows of
+    // 32 bytes per core matrix group (SBO 256).  B, MN-major: 128B swizzle,
+    // next 64-column N atom one 2 KB box further (LBO), next 8 k rows 1024
+    // bytes further (SBO); the second half of (i, j) starts two boxes (4 KB)
+    // in, the same offset as the K-major layout's row 128.
     k.a_desc0 = ((uint64_t)(kFBytes >> 4) << 16) | ((uint64_t)(1024 >> 4) << 32) | (1ull << 46) | (2ull << 61);
-    k.b_desc0 = ((uint64_t)(16 >> 4) << 16) | ((uint64_t)(256 >> 4) << 32) | (1ull << 46) | (6ull << 61);
+    k.b_desc0 = tmn ? (((uint64_t)((kTBytes / 4) >> 4) << 16) | ((uint64_t)(1024 >> 4) << 32) | (1ull << 46) |
+                       (2ull << 61))
+                    : (((uint64_t)(16 >> 4) << 16) | ((uint64_t)(256 >> 4) << 32) | (1ull << 46) | (6ull << 61));
     k.status = ctx->d_status + 2;
     ucl_status st = cuda_check(
         ctx, cudaFuncSetAttribute(tc3_contract_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem3),

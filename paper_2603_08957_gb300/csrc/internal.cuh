@@ -79,6 +79,7 @@ struct TcPlan {
 // tile laid out [i][j][k] and the F tile [k][r]; i = j = k = 16, r = 64.
 struct Tc3Plan {
     int t, e, f;             // spec positions of T, the epilogue factor E, the MMA factor F
+    bool t_mn;               // T tiles laid out [f][i][e] (else [i][e][f])
     int64_t sEj, sEr;        // E tile strides of j and r
     int64_t sWi, sWr;        // output tile strides of i and r
 };

@@ -436,6 +436,10 @@ def test_mttkrp_small(ctx, path):
     # operands in another order: the join order is chosen from the keys
     out2 = ctx.einsum("Jjr,IJKijk,Kkr->Iir", *(gpu_rel(ctx, w[k]) for k in ("B", "T", "C")), path=path)
     assert_parity(out2, ref, torch.bfloat16)
+    # T tiles stored [k][i][j]: the same EinSum, the same output
+    wk = workloads.mttkrp(seed=0, n=1000, nnz=5000, layout="kij")
+    out3 = ctx.einsum(wk["spec"], *(gpu_rel(ctx, wk[k]) for k in ("T", "B", "C")), path=path)
+    assert_parity(out3, ref, torch.bfloat16)
 
 
 def test_mttkrp_full_size_sampled(ctx):
@@ -478,6 +482,9 @@ TC3_CASES = [
     ("IJKijk,Kkr,Jjr->Iir", (0, 1, 2), "CB", "jr"),   # first join on K: E changes every triple
     ("IJKikj,Kkr,Jjr->Iir", (0, 2, 1), "CB", "jr"),   # T laid out [i][k][j]: E = C, F = B
     ("IJKijk,Jrj,Kkr->Iir", (0, 1, 2), "BC", "rj"),   # E stored [r][j]
+    ("IJKkij,Jjr,Kkr->Iir", (2, 0, 1), "BC", "jr"),   # T laid out [k][i][j]: MN-major T, 128-byte TMA rows
+    ("IJKkij,Jjr,Kkr->rIi", (2, 0, 1), "BC", "jr"),   # ... with a transposed output tile
+    ("IJKjik,Kkr,Jjr->Iir", (1, 0, 2), "CB", "jr"),   # T laid out [j][i][k]: E = C, F = B
 ]
 
 

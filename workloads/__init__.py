@@ -276,12 +276,16 @@ def zipf_coords(n: int, nnz: int, order=3, s=1.1, seed=0, device="cpu", batch=1 
     return torch.sort(uniq[keep]).values
 
 
-def mttkrp(seed=0, n=100_000, nnz=10_000_000, t=16, rank=64, s=1.1, device="cpu"):
+def mttkrp(seed=0, n=100_000, nnz=10_000_000, t=16, rank=64, s=1.1, device="cpu", layout="ijk"):
     """MTTKRP M[i,r] = sum_{j,k} T[i,j,k] B[j,r] C[k,r]: T sparse n^3 with nnz
     Zipf(s) coordinates (zipf_coords), values U[-1,1), grouped into only-
     nonempty t^3 bf16 tiles keyed (I, J, K); B and C dense n x rank bf16
     U[-1,1) as per-tile-row relations keyed J (resp. K) with [t x rank] tiles
-    (rows past n zero).  Spec "IJKijk,Jjr,Kkr->Iir"."""
+    (rows past n zero).  Spec "IJKijk,Jjr,Kkr->Iir"; layout="kij" stores each
+    T tile as [k][i][j] instead (spec "IJKkij,Jjr,Kkr->Iir", the same EinSum
+    and the same values)."""
+    if layout not in ("ijk", "kij"):
+        raise ValueError("layout must be 'ijk' or 'kij'")
     codes = zipf_coords(n, nnz, 3, s, seed, device)
     g = torch.Generator(device=device).manual_seed(seed + 1)
     vals = torch.rand(codes.numel(), generator=g, device=device) * 2 - 1
@@ -298,8 +302,10 @@ def mttkrp(seed=0, n=100_000, nnz=10_000_000, t=16, rank=64, s=1.1, device="cpu"
         f[:n] = torch.rand((n, rank), generator=g, device=device) * 2 - 1
         return (np.arange(nt, dtype=np.int32)[:, None], (nt,), f.view(nt, t, rank).to(torch.bfloat16))
 
+    if layout == "kij":
+        tiles = tiles.permute(0, 3, 1, 2).contiguous()
     return {
-        "spec": "IJKijk,Jjr,Kkr->Iir",
+        "spec": "IJKijk,Jjr,Kkr->Iir" if layout == "ijk" else "IJKkij,Jjr,Kkr->Iir",
         "T": (keys, (nt, nt, nt), tiles),
         "B": factor(),
         "C": factor(),
