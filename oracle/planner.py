@@ -16,6 +16,10 @@ It restates, in plain Python and in the paper's order:
 * ComputeMinCostForTree (Alg. 1): the dynamic programme over a tree of binary
   EinSums, keeping for every vertex and output decomposition the cheapest way
   to produce it;
+* the heuristic of Sec. 8.2 for programs whose results are consumed more than
+  once: split the DAG into trees in which no result is used twice, optimise
+  them one after another with Alg. 1, each treating the decompositions already
+  chosen as fixed;
 * an exhaustive enumeration of every plan, which the tests use to pin the
   dynamic programme (and its k-best extension) independently of its recursion.
 
@@ -45,6 +49,18 @@ Readings where the paper is silent or inconsistent:
   with a positive ``max_call_bytes``, an EinSum may only read and write tiles
   whose bytes (U's tile + V's tile + W's tile, at each tensor's element
   size) total at most that; choices above it are left out of the search.
+* P8 The trees of Sec. 8.2's multi-use heuristic are cut at every EinSum
+  result used more than once (and at every result no EinSum uses, an
+  output): such a result roots its own tree, and every other EinSum vertex
+  joins the tree of its one consumer.  Trees are optimised in increasing
+  order of their root, so every result a tree reads from another tree is
+  already decided.  Its consumers read it as an input whose decomposition is
+  fixed: reading it in another split costs C_repart (an input tensor of the
+  program stays free in any split, P4).  The paper asks for maximal trees; a
+  result used twice could also join one of its consumers' trees, but that
+  choice can make the order between trees cyclic (two trees each reading a
+  result the other decides), so it is not taken.  A result that one EinSum
+  reads as both operands counts as used twice.
 """
 from __future__ import annotations
 
@@ -83,6 +99,8 @@ class Vertex:
     left: int | None = None
     right: int | None = None
     stats: Stats | None = None     # inputs: required; EinSums: estimated when None
+    fixed_up: tuple | None = None  # inputs only: the split the tensor is already stored in
+                                   # (reading P8); None = free in any split (reading P4)
 
 
 # ------------------------------------------------------------------ Sec. 7.1
@@ -325,7 +343,7 @@ def optimize(graph, bounds, cm: CostModel, k: int = 1):
     C = []   # C[i][↑W] = sorted list of (cost, plan)
     for i, v in enumerate(graph):
         if v.left is None:
-            C.append({up: [(0.0, {i: up})] for up in subsets(v.labels)})
+            C.append({up: [(_leaf_cost(v, stats[i], bounds, cm, up), {i: up})] for up in subsets(v.labels)})
             continue
         table = {}
         for upW in subsets(v.labels):
@@ -356,6 +374,14 @@ def optimize(graph, bounds, cm: CostModel, k: int = 1):
     return best[:k]
 
 
+def _leaf_cost(v, s, bounds, cm, up) -> float:
+    """Reading an input tensor in split ``up``: free (P4), or a repartition
+    from the split it is already stored in (P8)."""
+    if v.fixed_up is None:
+        return 0.0
+    return repart_cost(cm, bounds, v, s, tuple(v.fixed_up), tuple(up))
+
+
 def plan_cost(graph, bounds, cm: CostModel, plan) -> float:
     """Cost of one complete plan, term by term."""
     stats = all_stats(graph)
@@ -368,6 +394,8 @@ def plan_cost(graph, bounds, cm: CostModel, plan) -> float:
         for child, up_in in ((v.left, upU), (v.right, upV)):
             if graph[child].left is not None:
                 total += repart_cost(cm, bounds, graph[child], stats[child], plan[child][0], up_in)
+            else:
+                total += _leaf_cost(graph[child], stats[child], bounds, cm, up_in)
     return total
 
 
@@ -408,3 +436,102 @@ def dense_tree(graph, dense_inputs):
             lU, lV = graph[v.left].labels, graph[v.right].labels
             val[i] = np.einsum(f"{lU},{lV}->{v.labels}", val[v.left], val[v.right])
     return val
+
+
+# ------------------------------------------------- Sec. 8.2, results used twice
+
+def check_dag(graph):
+    """Topological order, two producers per EinSum, output labels present."""
+    for i, v in enumerate(graph):
+        if (v.left is None) != (v.right is None):
+            raise ValueError("a vertex has one input")
+        if v.left is not None:
+            for p in (v.left, v.right):
+                if not 0 <= p < i:
+                    raise ValueError("vertices must be in topological order")
+            lU, lV = graph[v.left].labels, graph[v.right].labels
+            if any(l not in lU and l not in lV for l in v.labels):
+                raise ValueError("an output label appears in no input")
+        elif v.stats is None:
+            raise ValueError("an input tensor needs statistics")
+
+
+def dag_trees(graph):
+    """Reading P8: the tree (its root vertex) of every EinSum vertex, and the
+    consuming edges (consumer, side) of every vertex."""
+    uses = {i: [] for i in range(len(graph))}
+    for i, v in enumerate(graph):
+        if v.left is not None:
+            uses[v.left].append((i, 0))
+            uses[v.right].append((i, 1))
+    tree = {}
+    for i in reversed(range(len(graph))):
+        if graph[i].left is None:
+            continue
+        tree[i] = tree[uses[i][0][0]] if len(uses[i]) == 1 else i
+    return tree, uses
+
+
+def optimize_dag(graph, bounds, cm: CostModel):
+    """Sec. 8.2: optimise the trees of ``dag_trees`` one after another with
+    Alg. 1 (k = 1).  Returns (cost, plan, tree) with plan[i] = (↑W, ↑U, ↑V) for
+    every EinSum vertex (how it writes its result and reads its inputs)."""
+    check_dag(graph)
+    tree, _ = dag_trees(graph)
+    stats = all_stats(graph)
+    plan = {}
+    total = 0.0
+    for r in sorted(set(tree.values())):
+        members = sorted(i for i in tree if tree[i] == r)
+        sub, where = [], {}
+
+        def leaf(p):
+            # one leaf per consuming edge; a result decided by an earlier tree
+            # keeps the split that tree chose
+            v = graph[p]
+            fixed = plan[p][0] if v.left is not None else None
+            sub.append(Vertex(v.labels, v.dtype_bytes, stats=stats[p], fixed_up=fixed))
+            return len(sub) - 1
+
+        for i in members:
+            v = graph[i]
+            a = where[v.left] if v.left in where else leaf(v.left)
+            b = where[v.right] if v.right in where else leaf(v.right)
+            sub.append(Vertex(v.labels, v.dtype_bytes, a, b, stats=stats[i]))
+            where[i] = len(sub) - 1
+        cost, sp = optimize(sub, bounds, cm, k=1)[0]
+        total += cost
+        for i in members:
+            plan[i] = sp[where[i]]
+    return total, plan, tree
+
+
+def dag_plan_cost(graph, bounds, cm: CostModel, plan) -> float:
+    """Cost of a DAG plan term by term: every EinSum's join and aggregation,
+    plus a repartition on every edge whose producer (an EinSum) wrote another
+    split than its consumer reads.  Inputs of the program are free (P4)."""
+    stats = all_stats(graph)
+    total = 0.0
+    for i, v in enumerate(graph):
+        if v.left is None:
+            continue
+        upW, upU, upV = plan[i]
+        total += _vertex_terms(graph, stats, bounds, cm, i, upW, upU, upV)
+        for child, up_in in ((v.left, upU), (v.right, upV)):
+            if graph[child].left is not None:
+                total += repart_cost(cm, bounds, graph[child], stats[child], plan[child][0], up_in)
+    return total
+
+
+def enumerate_dag_plans(graph, bounds, cm: CostModel):
+    """Every plan of a DAG with its cost, by exhaustive search (tests only)."""
+    check_dag(graph)
+    ein = [i for i, v in enumerate(graph) if v.left is not None]
+    per_vertex = [[(upW, upU, upV) for upW in subsets(graph[i].labels)
+                   for upU, upV in _input_choices(graph, i, upW, bounds, cm)] for i in ein]
+    out = []
+    for combo in itertools.product(*per_vertex):
+        plan = dict(zip(ein, combo))
+        out.append((dag_plan_cost(graph, bounds, cm, plan), plan))
+    out.sort(key=lambda e: e[0])
+    return out

@@ -270,3 +270,177 @@ def test_dense_tree_brute_force():
     T = brute_force("ab,bcd->cda", [X, Y])
     np.testing.assert_allclose(val[2], T, rtol=1e-12)
     np.testing.assert_allclose(val[4], brute_force("cda,ae->ce", [T, Z]), rtol=1e-12)
+
+
+# ------------------------------------------- Sec. 8.2: results used twice
+
+def _rand_dag(rng, n_ein, bounds_choice=(2, 3, 4, 8), labels="abcde", max_lab=3, reuse=True):
+    """A random EinSum DAG: three or four inputs, then n_ein binary EinSums on
+    earlier vertices; with ``reuse`` some intermediate is consumed twice."""
+    bounds = {l: int(rng.choice(bounds_choice)) for l in labels}
+
+    def stats_for(lab):
+        T = float(rng.uniform(1, np.prod([float(bounds[l]) for l in lab])))
+        return P.Stats(T, {l: float(rng.integers(1, bounds[l] + 1)) for l in lab})
+
+    g = []
+    for _ in range(int(rng.integers(3, 5))):
+        lab = "".join(rng.choice(list(labels), size=int(rng.integers(1, max_lab + 1)), replace=False))
+        g.append(P.Vertex(lab, int(rng.choice([2, 4])), stats=stats_for(lab)))
+    n_in = len(g)
+    for j in range(n_ein):
+        i = len(g)
+        if reuse and j == n_ein - 1 and n_ein >= 2:
+            a, b = n_in, i - 1          # the first intermediate is read again
+        else:
+            a, b = (int(x) for x in rng.choice(i, size=2, replace=False))
+            if j > 0 and rng.random() < 0.6:
+                a = i - 1
+        pool = sorted(set(g[a].labels) | set(g[b].labels))
+        k = int(rng.integers(1, min(max_lab, len(pool)) + 1))
+        lab = "".join(rng.choice(pool, size=k, replace=False))
+        g.append(P.Vertex(lab, int(rng.choice([2, 4])), a, b))
+    return g, bounds
+
+
+def _cm(rng, repart=True):
+    return P.CostModel(xfer=float(rng.uniform(1e-9, 1e-6)) if repart else 0.0,
+                       flop=float(rng.uniform(1e-12, 1e-9)), add=float(rng.uniform(0, 1e-9)),
+                       fixed=float(rng.uniform(0, 1e-6)) if repart else 0.0)
+
+
+def _rand_tree(rng, bushy):
+    """A tree: a chain ((A B) C) D, or a bushy (A B) (C D), random labels."""
+    bounds = {l: int(rng.choice([2, 3, 4, 8])) for l in "abcde"}
+
+    def leaf(lab):
+        T = float(rng.uniform(1, np.prod([float(bounds[l]) for l in lab])))
+        return P.Vertex(lab, int(rng.choice([2, 4])), stats=P.Stats(
+            T, {l: float(rng.integers(1, bounds[l] + 1)) for l in lab}))
+
+    def lab():
+        return "".join(rng.choice(list("abcde"), size=int(rng.integers(1, 4)), replace=False))
+
+    def ein(g, a, b):
+        pool = sorted(set(g[a].labels) | set(g[b].labels))
+        out = "".join(rng.choice(pool, size=int(rng.integers(1, min(3, len(pool)) + 1)), replace=False))
+        g.append(P.Vertex(out, int(rng.choice([2, 4])), a, b))
+
+    g = [leaf(lab()), leaf(lab())]
+    ein(g, 0, 1)                               # 2
+    g.append(leaf(lab()))                      # 3
+    if bushy:
+        g.append(leaf(lab()))                  # 4
+        ein(g, 3, 4)                           # 5
+        ein(g, 2, 5)                           # 6
+    else:
+        ein(g, 2, 3)                           # 4
+        g.append(leaf(lab()))                  # 5
+        ein(g, 4, 5)                           # 6
+    return g, bounds
+
+
+@pytest.mark.parametrize("seed", range(6))
+@pytest.mark.parametrize("bushy", [False, True])
+def test_dag_on_a_tree_is_alg1(seed, bushy):
+    """Without a result used twice the heuristic is Alg. 1 itself: one tree,
+    the same cost and the same plan."""
+    rng = np.random.default_rng(500 + seed)
+    g, bounds = _rand_tree(rng, bushy)
+    cm = _cm(rng)
+    cost, plan, tree = P.optimize_dag(g, bounds, cm)
+    c1, p1 = P.optimize(g, bounds, cm, k=1)[0]
+    assert cost == pytest.approx(c1, rel=1e-12)
+    assert plan == {i: p1[i] for i in p1 if g[i].left is not None}
+    assert set(tree.values()) == {6}
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_dag_trees_cut_at_results_used_twice(seed):
+    rng = np.random.default_rng(600 + seed)
+    g, _ = _rand_dag(rng, int(rng.integers(3, 7)))
+    tree, uses = P.dag_trees(g)
+    ein = [i for i, v in enumerate(g) if v.left is not None]
+    assert sorted(tree) == ein
+    for i in ein:
+        n_use = len(uses[i])
+        if n_use != 1:
+            assert tree[i] == i                         # an output or a result used twice roots a tree
+        else:
+            assert tree[i] == tree[uses[i][0][0]]      # else it joins its consumer's tree
+    for r in set(tree.values()):
+        members = [i for i in ein if tree[i] == r]
+        assert max(members) == r
+        # inside a tree no result is read twice
+        reads = [p for i in members for p in (g[i].left, g[i].right) if p in members]
+        assert len(reads) == len(set(reads)) == len(members) - 1
+        # what a tree reads from other trees are roots decided before it
+        for i in members:
+            for p in (g[i].left, g[i].right):
+                if g[p].left is not None and tree[p] != r:
+                    assert tree[p] == p < r
+
+
+@pytest.mark.parametrize("seed", range(10))
+def test_dag_plan_cost_and_local_optimality(seed):
+    """The reported cost is the plan's cost term by term, and each tree's
+    choices are the cheapest for that tree with the earlier trees' splits
+    held fixed (exhaustive over the tree's own vertices)."""
+    rng = np.random.default_rng(700 + seed)
+    g, bounds = _rand_dag(rng, int(rng.integers(2, 5)))
+    cm = _cm(rng)
+    cost, plan, tree = P.optimize_dag(g, bounds, cm)
+    assert cost == pytest.approx(P.dag_plan_cost(g, bounds, cm, plan), rel=1e-12)
+    stats = P.all_stats(g)
+    for r in set(tree.values()):
+        members = sorted(i for i in tree if tree[i] == r)
+
+        def tree_cost(choice):
+            tot = 0.0
+            for i in members:
+                upW, upU, upV = choice[i]
+                tot += P._vertex_terms(g, stats, bounds, cm, i, upW, upU, upV)
+                for p, up_in in ((g[i].left, upU), (g[i].right, upV)):
+                    if g[p].left is not None:
+                        up_p = choice[p][0] if p in choice else plan[p][0]
+                        tot += P.repart_cost(cm, bounds, g[p], stats[p], up_p, up_in)
+            return tot
+
+        opts = [[(upW, upU, upV) for upW in P.subsets(g[i].labels)
+                 for upU, upV in P._input_choices(g, i, upW, bounds, cm)] for i in members]
+        best = min(tree_cost(dict(zip(members, c))) for c in itertools.product(*opts))
+        assert tree_cost({i: plan[i] for i in members}) == pytest.approx(best, rel=1e-12)
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_dag_heuristic_against_exhaustive(seed):
+    """Exhaustive search over the whole DAG: the heuristic never beats the
+    optimum, and with free repartition (no C_xfer, no C_fixed) the trees are
+    independent, so it finds the optimum."""
+    rng = np.random.default_rng(800 + seed)
+    g, bounds = _rand_dag(rng, 3, labels="abcd", max_lab=3)
+    every = P.enumerate_dag_plans(g, bounds, _cm(np.random.default_rng(seed)))
+    cm = _cm(np.random.default_rng(seed))
+    cost, plan, _ = P.optimize_dag(g, bounds, cm)
+    assert cost >= every[0][0] * (1 - 1e-12)
+    cm0 = _cm(np.random.default_rng(seed), repart=False)
+    cost0, plan0, _ = P.optimize_dag(g, bounds, cm0)
+    best0 = P.enumerate_dag_plans(g, bounds, cm0)[0][0]
+    assert cost0 == pytest.approx(best0, rel=1e-12)
+
+
+def test_dag_fixed_split_costs_a_repartition():
+    """A result decided by an earlier tree is read for free in its own split
+    and for C_repart in another (reading P8); a planted mistake that reads it
+    for free in every split is caught by the exhaustive check above."""
+    rng = np.random.default_rng(9)
+    s = P.Stats(50.0, {"a": 8.0, "b": 6.0})
+    bounds = {"a": 8, "b": 8}
+    cm = _cm(rng)
+    leaf = P.Vertex("ab", 2, stats=s, fixed_up=("a",))
+    assert P._leaf_cost(leaf, s, bounds, cm, ("a",)) == 0.0
+    for up in (("b",), (), ("a", "b")):
+        assert P._leaf_cost(leaf, s, bounds, cm, up) == pytest.approx(
+            P.repart_cost(cm, bounds, leaf, s, ("a",), up), rel=0) and P._leaf_cost(leaf, s, bounds, cm, up) > 0
+    free = P.Vertex("ab", 2, stats=s)
+    assert all(P._leaf_cost(free, s, bounds, cm, up) == 0.0 for up in P.subsets("ab"))
