@@ -350,6 +350,32 @@ ucl_status ucl_plan(int n_vertices, const ucl_plan_vertex *vertices, const char 
                     const int64_t *label_bounds, int n_labels, const ucl_cost_model *cost_model, int k,
                     ucl_plan_choice *out, int *n_out);
 
+/* One plan for an EinSum program whose tensors may be consumed more than once
+ * (a DAG), by the heuristic of Sec. 8.2 ("when results are consumed more than
+ * once").  The DAG is cut into trees at every EinSum result used more than
+ * once and at every result no EinSum uses (an output): such a result roots a
+ * tree, every other EinSum vertex joins the tree of its one consumer.  Trees
+ * are optimised one after another in increasing order of their root, each by
+ * the dynamic programme of Alg. 1; a result an earlier tree decided is read as
+ * an input whose split is fixed (reading it in another split costs C_repart),
+ * and the program's input tensors stay free in any split.  Not globally
+ * optimal: a result used twice is decided for its own tree alone.  Host only.
+ *   vertices   [n_vertices] in topological order, as for ucl_plan, except that
+ *              any tensor may be consumed any number of times (an EinSum may
+ *              read one tensor as both operands) and several vertices may be
+ *              outputs
+ *   out        receives the plan: cost = the sum of the trees' costs; up[i]
+ *              an EinSum's output split, or for an input tensor the split its
+ *              first consumer (lowest index, left operand first) reads; in_up
+ *              every EinSum's read splits
+ *   tree_root  optional [n_vertices]; receives the root of each EinSum
+ *              vertex's tree, -1 for inputs
+ * Errors: as ucl_plan (no tree condition), and UCL_ERR_UNSUPPORTED when no
+ * split of some tree satisfies the memory bound. */
+ucl_status ucl_plan_dag(int n_vertices, const ucl_plan_vertex *vertices, const char *label_names,
+                        const int64_t *label_bounds, int n_labels, const ucl_cost_model *cost_model,
+                        ucl_plan_choice *out, int *tree_root);
+
 /* ------------------------------------------------------- no allocation */
 
 /* Largest key array ucl_keys_check_noalloc accepts (tuples). */

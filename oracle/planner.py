@@ -499,7 +499,10 @@ def optimize_dag(graph, bounds, cm: CostModel):
             b = where[v.right] if v.right in where else leaf(v.right)
             sub.append(Vertex(v.labels, v.dtype_bytes, a, b, stats=stats[i]))
             where[i] = len(sub) - 1
-        cost, sp = optimize(sub, bounds, cm, k=1)[0]
+        best = optimize(sub, bounds, cm, k=1)
+        if not best:
+            raise ValueError("no decomposition of a tree satisfies the memory bound")
+        cost, sp = best[0]
         total += cost
         for i in members:
             plan[i] = sp[where[i]]

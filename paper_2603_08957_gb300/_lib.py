@@ -45,6 +45,7 @@ EXPORTS = [
     "ucl_relation_stats",
     "ucl_drop_zero_tiles",
     "ucl_plan",
+    "ucl_plan_dag",
     "ucl_keys_check_noalloc",
     "ucl_status_str",
     "ucl_last_error",
@@ -138,6 +139,8 @@ def _declare(lib):
     lib.ucl_drop_zero_tiles.argtypes = [vp, vp, pp]
     lib.ucl_plan.argtypes = [i32, c.POINTER(PlanVertex), c.c_char_p, c.POINTER(i64), i32, c.POINTER(CostModel), i32,
                              c.POINTER(PlanChoice), c.POINTER(i32)]
+    lib.ucl_plan_dag.argtypes = [i32, c.POINTER(PlanVertex), c.c_char_p, c.POINTER(i64), i32, c.POINTER(CostModel),
+                                 c.POINTER(PlanChoice), c.POINTER(i32)]
     lib.ucl_keys_check_noalloc.argtypes = [i32, vp, i64, i32, vp, c.POINTER(i64), c.POINTER(i32)]
     lib.ucl_status_str.argtypes = [i32]
     lib.ucl_status_str.restype = c.c_char_p

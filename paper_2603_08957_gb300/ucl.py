@@ -273,19 +273,8 @@ class Relation:
         return keys, tiles
 
 
-def plan(vertices, bounds: dict, cost_model: dict, k: int = 1):
-    """The k cheapest decompositions of an EinSum tree (include/ucl.h, ucl_plan).
-
-    ``vertices``: list of dicts in topological order, the last the root, each
-    with ``labels`` (str, one character per label) and either ``T`` and ``V``
-    (input tensor: non-zero count and distinct count per label) or ``left``
-    and ``right`` (producer indices; ``T``/``V`` optional measured statistics);
-    ``dtype_bytes`` defaults to 2.  ``bounds`` maps label -> extent;
-    ``cost_model`` has ``xfer``, ``flop``, ``add``, ``fixed`` (and optional
-    ``key_bytes`` and ``max_call_bytes``).  Returns [(cost, ups)], cheapest first, where ups[i] is
-    ``(up_W, up_U, up_V)`` for an EinSum vertex and ``up`` for an input, each a
-    string of the promoted labels in the tensor's label order."""
-    lib = _lib.load()
+def _plan_args(vertices, bounds, cost_model):
+    """ctypes arguments of ucl_plan / ucl_plan_dag (plus buffers to keep alive)."""
     n = len(vertices)
     arr = (_lib.PlanVertex * n)()
     keep = []
@@ -310,24 +299,58 @@ def plan(vertices, bounds: dict, cost_model: dict, k: int = 1):
     cm = _lib.CostModel(float(cost_model.get("xfer", 0.0)), float(cost_model.get("flop", 0.0)),
                         float(cost_model.get("add", 0.0)), float(cost_model.get("fixed", 0.0)),
                         int(cost_model.get("key_bytes", 4)), float(cost_model.get("max_call_bytes", 0.0)))
+    return n, arr, names, bnd, cm, keep
+
+
+def _ups(labels, mask):
+    return "".join(c for q, c in enumerate(labels) if mask >> q & 1)
+
+
+def _per_vertex(vertices, pc):
+    per = []
+    for i, v in enumerate(vertices):
+        if "left" not in v or v["left"] is None:
+            per.append(_ups(v["labels"], pc.up[i]))
+        else:
+            per.append((_ups(v["labels"], pc.up[i]), _ups(vertices[v["left"]]["labels"], pc.in_up[i][0]),
+                        _ups(vertices[v["right"]]["labels"], pc.in_up[i][1])))
+    return per
+
+
+def plan(vertices, bounds: dict, cost_model: dict, k: int = 1):
+    """The k cheapest decompositions of an EinSum tree (include/ucl.h, ucl_plan).
+
+    ``vertices``: list of dicts in topological order, the last the root, each
+    with ``labels`` (str, one character per label) and either ``T`` and ``V``
+    (input tensor: non-zero count and distinct count per label) or ``left``
+    and ``right`` (producer indices; ``T``/``V`` optional measured statistics);
+    ``dtype_bytes`` defaults to 2.  ``bounds`` maps label -> extent;
+    ``cost_model`` has ``xfer``, ``flop``, ``add``, ``fixed`` (and optional
+    ``key_bytes`` and ``max_call_bytes``).  Returns [(cost, ups)], cheapest first, where ups[i] is
+    ``(up_W, up_U, up_V)`` for an EinSum vertex and ``up`` for an input, each a
+    string of the promoted labels in the tensor's label order."""
+    lib = _lib.load()
+    n, arr, names, bnd, cm, keep = _plan_args(vertices, bounds, cost_model)
     out = (_lib.PlanChoice * k)()
     n_out = ctypes.c_int()
     st = lib.ucl_plan(n, arr, names, bnd, len(bounds), ctypes.byref(cm), k, out, ctypes.byref(n_out))
     if st != 0:
         raise UclError(st, "ucl_plan")
+    return [(out[b].cost, _per_vertex(vertices, out[b])) for b in range(n_out.value)]
 
-    def ups(labels, mask):
-        return "".join(c for q, c in enumerate(labels) if mask >> q & 1)
 
-    res = []
-    for b in range(n_out.value):
-        pc = out[b]
-        per = []
-        for i, v in enumerate(vertices):
-            if "left" not in v or v["left"] is None:
-                per.append(ups(v["labels"], pc.up[i]))
-            else:
-                per.append((ups(v["labels"], pc.up[i]), ups(vertices[v["left"]]["labels"], pc.in_up[i][0]),
-                            ups(vertices[v["right"]]["labels"], pc.in_up[i][1])))
-        res.append((pc.cost, per))
-    return res
+def plan_dag(vertices, bounds: dict, cost_model: dict):
+    """One decomposition of an EinSum DAG whose tensors may be consumed more
+    than once, by Sec. 8.2's tree-by-tree heuristic (include/ucl.h,
+    ucl_plan_dag).  Arguments as for ``plan``.  Returns (cost, ups, tree_root):
+    ups[i] as for ``plan`` (an input's entry is the split its first consumer
+    reads) and tree_root[i] the root of the tree EinSum vertex i was optimised
+    in (-1 for inputs)."""
+    lib = _lib.load()
+    n, arr, names, bnd, cm, keep = _plan_args(vertices, bounds, cost_model)
+    out = _lib.PlanChoice()
+    roots = (ctypes.c_int * n)()
+    st = lib.ucl_plan_dag(n, arr, names, bnd, len(bounds), ctypes.byref(cm), ctypes.byref(out), roots)
+    if st != 0:
+        raise UclError(st, "ucl_plan_dag")
+    return out.cost, _per_vertex(vertices, out), list(roots)
