@@ -1,6 +1,7 @@
-"""Run a tree of binary EinSums under a plan chosen by ``plan`` (ucl_plan).
+"""Run a tree of binary EinSums under a plan chosen by ``plan`` (ucl_plan),
+or a DAG under a plan chosen by ``plan_dag`` (ucl_plan_dag).
 
-The tree is the one handed to the planner: vertices in topological order, each
+The program is the one handed to the planner: vertices in topological order, each
 an input tensor or W = Σ U × V, every label one lower-case letter.  A plan
 gives every tensor's split (its promoted labels).  In the executor's spec
 grammar a promoted label is written upper case, so the plan alone fixes every
@@ -64,6 +65,45 @@ def prepare_inputs(ctx, vertices, ups, stored):
             rel, up = stored[i]
             out[i] = resplit(ctx, rel, v["labels"], up, ups[i])
     return out
+
+
+def execute_dag(ctx, vertices, ups, inputs, *, path="auto", keep=False):
+    """Evaluate a program whose tensors may be consumed more than once under
+    one plan (``ups`` as ``plan`` or ``plan_dag`` return it; ``inputs`` maps
+    each input vertex to its relation in ``ups[i]``).  Every consuming edge
+    reads its tensor in the split its consumer wants, repartitioning a copy
+    when the tensor has another split.  An intermediate is destroyed after
+    its last consumer ran, unless ``keep``.  Returns {vertex: relation} for
+    every EinSum vertex no EinSum consumes (the program's outputs)."""
+    uses = [0] * len(vertices)
+    for v in vertices:
+        if v.get("left") is not None:
+            uses[v["left"]] += 1
+            uses[v["right"]] += 1
+    pending = list(uses)
+    rel = dict(inputs)
+    for i, v in enumerate(vertices):
+        if v.get("left") is None:
+            continue
+        upW, upU, upV = ups[i]
+        operands, copies = [], []
+        for child, up_read in ((v["left"], upU), (v["right"], upV)):
+            cv = vertices[child]
+            up_have = ups[child] if cv.get("left") is None else ups[child][0]
+            r = resplit(ctx, rel[child], cv["labels"], up_have, up_read)
+            if r is not rel[child]:
+                copies.append(r)
+            operands.append(r)
+        spec = einsum_spec(vertices[v["left"]]["labels"], upU, vertices[v["right"]]["labels"], upV, v["labels"], upW)
+        out_dtype = "bf16" if v.get("dtype_bytes", 2) == 2 else "f32"
+        rel[i] = ctx.einsum(spec, *operands, out_dtype=out_dtype, path=path)
+        for r in copies:
+            r.destroy()
+        for child in (v["left"], v["right"]):
+            pending[child] -= 1
+            if pending[child] == 0 and not keep and vertices[child].get("left") is not None:
+                rel.pop(child).destroy()
+    return {i: rel[i] for i, v in enumerate(vertices) if v.get("left") is not None and uses[i] == 0}
 
 
 def execute(ctx, vertices, ups, inputs, *, path="auto", keep=False):

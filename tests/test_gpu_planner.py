@@ -7,7 +7,7 @@ import torch
 
 import workloads
 from oracle import planner as P
-from paper_2603_08957_gb300 import Context, plan, program
+from paper_2603_08957_gb300 import Context, plan, plan_dag, program
 from tests.parity import gpu_rel
 from tests.ucl_testutil import decompose, random_sparse, recompose
 
@@ -155,3 +155,48 @@ def test_cheapest_plans_compute_the_same_tensor(ctx):
             if r is not stored[i][0]:
                 r.destroy()
         out.destroy()
+
+
+def test_dag_plan_with_a_result_read_twice(ctx):
+    """Two heads read the message-passing result T: O1 = T Z, O2 = T W.
+    ucl_plan_dag decides T in its own tree, each head reads it in the split it
+    chose (repartitioned where they differ); both outputs match the dense
+    definition."""
+    n, t = 4096, 64
+    w = workloads.gnn_chain(seed=4, n=n, degree=8, device="cpu")
+    nt = -(-n // t)
+    bounds = {"f": 128, "a": nt, "b": t, "c": nt, "d": t, "g": 128, "h": 16}
+    gen = torch.Generator().manual_seed(11)
+    Wt = (torch.randn((1, 128, 16), generator=gen) * 0.1).to(torch.bfloat16)
+    Wrel = (np.zeros((1, 0), dtype=np.int32), (), Wt)
+    verts = _chain_tree(w) + [{"labels": "fh"}, {"labels": "cdh", "left": 2, "right": 5, "dtype_bytes": 4}]
+    stored = {0: (gpu_rel(ctx, w["X"]), "a"), 1: (gpu_rel(ctx, w["Y"]), "ac"), 3: (gpu_rel(ctx, w["Z"]), ""),
+              5: (gpu_rel(ctx, Wrel), "")}
+    for i, (rel, up) in stored.items():
+        T, V = ctx.stats(rel)
+        lab = verts[i]["labels"]
+        order = [c for c in lab if c in up] + [c for c in lab if c not in up]
+        verts[i].update(T=T, V=dict(zip(order, V)))
+    cm = {"xfer": 1 / 6.7e12, "flop": 1 / 1.0e15, "add": 0.0, "fixed": 2e-9, "max_call_bytes": 256e3}
+    cost, ups, roots = plan_dag(verts, bounds, cm)
+    assert roots == [-1, -1, 2, -1, 4, -1, 6] and cost > 0
+    X = recompose(w["X"][0], w["X"][2].to(torch.float64).numpy(), "fab", {"a"}, bounds)
+    Y = recompose(w["Y"][0], w["Y"][2].to(torch.float64).numpy(), "abcd", {"a", "c"}, bounds)
+    Z = w["Z"][2][0].to(torch.float64).numpy()
+    Wd = Wt[0].to(torch.float64).numpy()
+    Td, Ta = np.einsum("fab,abcd->cdf", X, Y), np.einsum("fab,abcd->cdf", np.abs(X), np.abs(Y))
+    ref = {4: (np.einsum("cdf,fg->cdg", Td, Z), np.einsum("cdf,fg->cdg", Ta, np.abs(Z))),
+           6: (np.einsum("cdf,fh->cdh", Td, Wd), np.einsum("cdf,fh->cdh", Ta, np.abs(Wd)))}
+    ins = program.prepare_inputs(ctx, verts, ups, stored)
+    outs = program.execute_dag(ctx, verts, ups, ins)
+    assert sorted(outs) == [4, 6]
+    for i, r in outs.items():
+        k, tl = r.download()
+        got = recompose(k, tl.to(torch.float64).numpy(), verts[i]["labels"], set(ups[i][0]), bounds)
+        want, mag = ref[i]
+        err = np.abs(got - want)
+        assert np.all(err <= 3e-5 * mag + 1e-30), (i, ups, float(err.max()))
+        r.destroy()
+    for i, r in ins.items():
+        if r is not stored[i][0]:
+            r.destroy()
