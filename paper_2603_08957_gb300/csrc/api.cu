@@ -983,7 +983,7 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             if (radix_sort(ctx, jk, vals, ka, va, cnt, bits)) { jk = ka; perm = va; } else perm = vals;
         };
         auto sync_count = [&](int64_t *dev) {
-            int64_t h;
+            int64_t h = 0;
             check(sync_read(ctx, dev, 1, &h));
             if (h >= (1ll << 31)) check(fail(ctx, UCL_ERR_UNSUPPORTED, "more than 2^31-1 joined pairs"));
             return h;
