@@ -396,10 +396,13 @@ ucl_status ucl_plan_dag(int n_vertices, const ucl_plan_vertex *vertices, const c
  *   sorted          optional; receives 1 if the keys are strictly ascending
  * Returns UCL_ERR_UNSUPPORTED for n > UCL_NOALLOC_MAX_TUPLES or more than 64
  * key bits.  Synchronises `stream` (once, or twice for unsorted keys).  The
+ * calling thread's current device is the same on return as on entry.  The
  * first call on a device looks up the scratch array's device address for
- * that device; make that first call before any stream capture.  Every call
- * shares the one scratch array: calls whose GPU work overlaps (e.g. on two
- * streams) race on it and must be serialised by the caller. */
+ * that device and keeps it for the life of the process; make that first
+ * call before any stream capture, and do not use this call on a device after
+ * cudaDeviceReset (the kept address would be stale).  Every call shares the
+ * one scratch array: calls whose GPU work overlaps (e.g. on two streams) race
+ * on it and must be serialised by the caller. */
 ucl_status ucl_keys_check_noalloc(int device, void *stream, int64_t n, int u, const int32_t *keys,
                                   const int64_t *key_bounds, int *sorted);
 

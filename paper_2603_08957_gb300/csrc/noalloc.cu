@@ -151,10 +151,22 @@ cudaError_t scratch_for(int device, void **out) {
     return cudaSuccess;
 }
 
-}  // namespace
+// Restores the calling thread's current device on every return path.
+struct DeviceGuard {
+    int prev = -1;
+    DeviceGuard() {
+        if (cudaGetDevice(&prev) != cudaSuccess) {
+            cudaGetLastError();
+            prev = -1;
+        }
+    }
+    ~DeviceGuard() {
+        if (prev >= 0) cudaSetDevice(prev);
+    }
+};
 
-extern "C" ucl_status ucl_keys_check_noalloc(int device, void *stream, int64_t n, int u, const int32_t *keys,
-                                             const int64_t *key_bounds, int *sorted) {
+ucl_status check_keys(int device, void *stream, int64_t n, int u, const int32_t *keys, const int64_t *key_bounds,
+                      int *sorted) {
     if (sorted) *sorted = 0;
     if (n < 0 || u < 0 || u > ucl::kMaxCols || (n > 0 && u > 0 && !keys) || (u > 0 && !key_bounds))
         return UCL_ERR_ARG;
@@ -180,6 +192,7 @@ extern "C" ucl_status ucl_keys_check_noalloc(int device, void *stream, int64_t n
         if (sorted) *sorted = 1;
         return UCL_OK;
     }
+    DeviceGuard guard;
     cudaError_t e = cudaSetDevice(device);
     if (e != cudaSuccess) return UCL_ERR_CUDA;
     void *base = nullptr;
@@ -194,8 +207,10 @@ extern "C" ucl_status ucl_keys_check_noalloc(int device, void *stream, int64_t n
     e = cudaMemsetAsync(flags, 0, sizeof(uint32_t), s);
     if (e == cudaSuccess) {
         nk_check<<<grid, kThreads, 0, s>>>(keys, u, n, bd, k0, flags);
-        e = cudaMemcpyAsync(&host_flags, flags, sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
+        // a launch that failed leaves the flags at 0: never read them then
+        e = cudaGetLastError();
     }
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&host_flags, flags, sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return UCL_ERR_CUDA;
     if (host_flags & kRange) return UCL_ERR_KEY_RANGE;
@@ -206,18 +221,28 @@ extern "C" ucl_status ucl_keys_check_noalloc(int device, void *stream, int64_t n
     // unsorted: LSD radix sort of the packed keys, then an adjacent-equal check
     const int nblocks = (int)((n + kItems - 1) / kItems);
     uint64_t *src = k0, *dst = k1;
-    for (int sh = 0; sh < total; sh += 8) {
+    for (int sh = 0; sh < total && e == cudaSuccess; sh += 8) {
         nk_hist<<<nblocks, kThreads, 0, s>>>(src, n, sh, hist, nblocks);
         nk_scan<<<1, kThreads, 0, s>>>(hist, kBuckets * nblocks);
         nk_scatter<<<nblocks, kThreads, 0, s>>>(src, dst, n, sh, hist, nblocks);
+        e = cudaGetLastError();
         uint64_t *t = src;
         src = dst;
         dst = t;
     }
-    nk_dups<<<grid, kThreads, 0, s>>>(src, n, flags);
-    e = cudaGetLastError();
+    if (e == cudaSuccess) {
+        nk_dups<<<grid, kThreads, 0, s>>>(src, n, flags);
+        e = cudaGetLastError();
+    }
     if (e == cudaSuccess) e = cudaMemcpyAsync(&host_flags, flags, sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return UCL_ERR_CUDA;
     return (host_flags & kDup) ? UCL_ERR_DUP_KEY : UCL_OK;
+}
+
+}  // namespace
+
+extern "C" ucl_status ucl_keys_check_noalloc(int device, void *stream, int64_t n, int u, const int32_t *keys,
+                                             const int64_t *key_bounds, int *sorted) {
+    return check_keys(device, stream, n, u, keys, key_bounds, sorted);
 }

@@ -38,6 +38,16 @@ def _cases():
     # a large random unique set near the size limit, three columns (54 bits)
     big = np.unique(rng.integers(0, 2**18, size=(900_000, 3)), axis=0)
     out.append(("large", big[rng.permutation(len(big))].astype(np.int32), (2**18,) * 3))
+    # sorted except for one adjacent duplicate: flagged unsorted, then sorted and caught
+    a = k.copy()
+    a[41] = a[40]
+    out.append(("adjacent duplicate", a, (300, 7)))
+    # exactly the size limit, shuffled (the scan runs over the full histogram)
+    m = 1 << 20
+    full = np.stack([np.arange(m) // 1024, np.arange(m) % 1024], 1).astype(np.int32)
+    out.append(("at the limit", full[rng.permutation(m)], (1024, 1024)))
+    # every bound 1: zero key bits, so two tuples are the same key
+    out.append(("zero bits", np.zeros((2, 3), np.int32), (1, 1, 1)))
     return out
 
 
@@ -65,6 +75,7 @@ def _ascending(keys):
 def test_matches_relation_create_twice():
     ctx = Context(0)
     lib = _lib.load()
+    cases = []
     for name, keys, bounds in _cases():
         n, u = keys.shape
         kd = torch.from_numpy(keys).cuda()
@@ -74,12 +85,32 @@ def test_matches_relation_create_twice():
             want = 0
         except UclError as e:
             want = e.status
-        for _ in range(2):
-            st, srt = _noalloc(lib, kd, n, u, bounds)
-            assert st == want, (name, st, want)
-            if want == 0:
-                assert bool(srt) == _ascending(keys), name
+        cases.append((name, keys, kd, bounds, want))
+    expect = {"duplicate": 4, "adjacent duplicate": 4, "zero bits": 4, "range": 5}   # DUP_KEY, KEY_RANGE
+    for name, _, _, _, want in cases:
+        assert want == expect.get(name, 0), (name, want)
     ctx.close()
+
+    def run_all():
+        for name, keys, kd, bounds, want in cases:
+            n, u = keys.shape
+            for _ in range(2):
+                st, srt = _noalloc(lib, kd, n, u, bounds)
+                assert st == want, (name, st, want)
+                if want == 0:
+                    assert bool(srt) == _ascending(keys), name
+
+    run_all()   # the first calls look up the scratch address and load the kernels
+    torch.cuda.synchronize()
+    torch_before = torch.cuda.memory_stats().get("allocation.all.allocated", 0)
+    free_before, _ = torch.cuda.mem_get_info()
+    dev = torch.cuda.current_device()
+    run_all()
+    torch.cuda.synchronize()
+    assert torch.cuda.current_device() == dev
+    assert torch.cuda.memory_stats().get("allocation.all.allocated", 0) == torch_before
+    free_after, _ = torch.cuda.mem_get_info()
+    assert free_after == free_before, (free_before, free_after)
 
 
 def test_rejects_oversize_without_gpu_work():
