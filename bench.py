@@ -81,6 +81,11 @@ class Workload:
     def sample(self, target, seed):
         raise NotImplementedError
 
+    def release(self):
+        """Drop the device tensors of the inputs (description and chain stay)."""
+        self.inputs = {}
+        self.w = None
+
 
 def _pick_keys(counts, target, seed):
     """Random output keys (indices into counts) whose tuple counts total
@@ -531,13 +536,20 @@ def run_reference(args, world, rank):
 # ---------------------------------------------------------------- GPU leg
 
 
-def stage_roofline(W, arity, stats, tim, pk):
+def stage_roofline(W, arity, stats, tim, iso, fixup, pk):
     """Per EinSum of the chain: mean stage times and the achieved fraction of
-    the HBM roofline for the key/join stages (algorithmic bytes: read every
-    input key once, write and read back the 16-byte pair records once, write
-    the index arrays and output keys) and for the contraction (its
-    algorithmic bytes: every input tile once, the output once, the indices),
-    with the tensor-pipe fraction of the contraction's FLOPs."""
+    the HBM roofline for
+      sort_join -- the key stages (algorithmic bytes: read every input key
+                   once, write and read back the 16-byte pair records once,
+                   write the index arrays and output keys); timed both in the
+                   back-to-back loop (overlapping the previous contraction)
+                   and alone after a device sync ("isolated");
+      contract  -- the contraction with its fused group-by sum (every input
+                   tile once, the output once, the indices), with the tensor
+                   fraction of its FLOPs;
+      reduce    -- the fixup that adds the partials of output keys split
+                   across work units (bytes counted by the fixup kernels:
+                   partials read once, output tiles written once)."""
     out = []
     L = len(W.chain)
     for c, (name, spec, ins, _) in enumerate(W.chain):
@@ -548,32 +560,58 @@ def stage_roofline(W, arity, stats, tim, pk):
         uw = len(rhs.split("|")[0]) if "|" in rhs else sum(ch.isupper() for ch in rhs)
         sort_bytes = key_bytes + 32.0 * P + 4.0 * len(ins) * P + 4.0 * uw * S
         ms = tim[c::L].mean(axis=0) if len(tim) else np.full(4, np.nan)
-        sj = float(ms[0] + ms[1])
-        ct = float(ms[2])
+        mi = iso[c::L].mean(axis=0) if len(iso) else np.full(4, np.nan)
+        sj, sj_iso, ct, fx = float(ms[0] + ms[1]), float(mi[0] + mi[1]), float(ms[2]), float(ms[3])
         gbs_sj = sort_bytes / (sj / 1e3) / 1e9
+        gbs_sji = sort_bytes / (sj_iso / 1e3) / 1e9
         gbs_c = s["bytes_contract"] / (ct / 1e3) / 1e9
         tf_c = s["flops"] / (ct / 1e3) / 1e12
-        out.append({"spec": spec, "path": s["path"], "tuples": P, "segments": S,
-                    "sort_join": {"ms": sj, "alg_bytes": sort_bytes, "GB/s": gbs_sj, "frac": gbs_sj / pk["hbm_gbs"]},
+        fb = float(fixup[c])
+        gbs_f = fb / (fx / 1e3) / 1e9 if fx > 0 else 0.0
+        out.append({"spec": spec, "path": s["path"], "tuples": P, "segments": S, "units": s["n_units"],
+                    "sort_join": {"ms": sj, "alg_bytes": sort_bytes, "GB/s": gbs_sj, "frac": gbs_sj / pk["hbm_gbs"],
+                                  "isolated_ms": sj_iso, "isolated_frac": gbs_sji / pk["hbm_gbs"]},
                     "contract": {"ms": ct, "alg_bytes": s["bytes_contract"], "GB/s": gbs_c,
                                  "frac": gbs_c / pk["hbm_gbs"], "TFLOP/s": tf_c,
                                  "tensor_frac": tf_c / pk["bf16_tflops"]},
-                    "fixup": {"ms": float(ms[3])}})
+                    "reduce": {"ms": fx, "alg_bytes": fb, "GB/s": gbs_f, "frac": gbs_f / pk["hbm_gbs"]}})
     return out
 
 
-def run_ucl(args, world, rank, local):
-    from paper_2603_08957_gb300 import Context
+def host_memory_bytes():
+    """Bytes of host memory this process may still use: the smaller of
+    MemAvailable and the cgroup's remaining limit."""
+    avail = None
+    try:
+        for line in open("/proc/meminfo"):
+            if line.startswith("MemAvailable:"):
+                avail = int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    for path, used in (("/sys/fs/cgroup/memory.max", "/sys/fs/cgroup/memory.current"),
+                       ("/sys/fs/cgroup/memory/memory.limit_in_bytes", "/sys/fs/cgroup/memory/memory.usage_in_bytes")):
+        try:
+            lim = open(path).read().strip()
+            if lim != "max" and int(lim) < (1 << 60):
+                rest = int(lim) - int(open(used).read().strip())
+                avail = rest if avail is None else min(avail, rest)
+            break
+        except (OSError, ValueError):
+            continue
+    return avail
 
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    W = WORKLOADS[args.workload](dev, args)
-    ctx = Context(local, torch_allocator=(args.alloc == "torch"))
+
+def measure(W, ctx, args, dev, world, *, steps, warmup, cpu_seconds, all_cores, e2e_on):
+    """Time one workload: its chain of EinSums back to back (inputs larger
+    than L2) or with an L2 flush before each step, then one isolated chain
+    (latency), the end-to-end run from host buffers, and the oracle's CPU
+    baseline.  Returns the measurement as a dict."""
     rels = {k: ctx.relation(torch.as_tensor(r[0]).to(dev), r[1], r[2].to(dev)) for k, r in W.inputs.items()}
     path = args.path
     flush = None if W.big else torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    arity = {k: (r.n, r.u) for k, r in rels.items()}
 
-    def run_chain(env, collect=None):
+    def run_chain(env, collect=None, fixup=None):
         made = []
         for name, spec, ins, opts in W.chain:
             if opts.get("op") == "repartition":
@@ -583,6 +621,8 @@ def run_ucl(args, world, rank, local):
             if collect is not None:
                 collect.append(ctx.last_stats())
                 arity[name] = (r.n, r.u)
+            if fixup is not None:
+                fixup.append(ctx.fixup_bytes(reset=True))
             env[name] = r
             made.append(r)
         return made
@@ -591,11 +631,11 @@ def run_ucl(args, world, rank, local):
         for r in run_chain(dict(rels)):
             r.destroy()
 
-    stats = []
-    arity = {k: (r.n, r.u) for k, r in rels.items()}
-    for r in run_chain(dict(rels), stats):
+    stats, fixup = [], []
+    ctx.fixup_bytes(reset=True)
+    for r in run_chain(dict(rels), stats, fixup):
         r.destroy()
-    for _ in range(max(0, args.warmup - 1)):
+    for _ in range(max(0, warmup - 1)):
         step()
     torch.cuda.synchronize()
     flops_step = sum(s["flops"] for s in stats)
@@ -603,7 +643,6 @@ def run_ucl(args, world, rank, local):
         flops_step = sum(s["bytes_contract"] for s in stats)
     launches_step = sum(s["launches"] for s in stats)
 
-    steps = args.steps
     if steps is None:
         t0 = time.perf_counter()
         for _ in range(3):
@@ -612,7 +651,7 @@ def run_ucl(args, world, rank, local):
         per = (time.perf_counter() - t0) / 3
         steps = int(min(2000, max(10, args.seconds / max(per, 1e-6))))
 
-    clocks = Clocks(local)
+    clocks = Clocks(dev.index)
     ctx.set_timing(True)
     ctx.timings(reset=True)
     barrier(world)
@@ -641,12 +680,31 @@ def run_ucl(args, world, rank, local):
     L = len(W.chain)
     tim = ctx.timings(reset=True, max_calls=steps * L + L)
     tim = tim[: (len(tim) // L) * L]
+
+    # latency: one chain alone after a device sync (the key stages then
+    # overlap nothing), three times
+    lat, iso = [], []
+    for _ in range(3):
+        if flush is not None:
+            flush.fill_(1)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        made = run_chain(dict(rels))
+        b.record()
+        torch.cuda.synchronize()
+        lat.append(a.elapsed_time(b))
+        for r in made:
+            r.destroy()
+        t = ctx.timings(reset=True, max_calls=L)
+        iso.append(t[:L])
+    iso = np.concatenate(iso) if iso else np.zeros((0, 4))
     ctx.set_timing(False)
     ms_max = allreduce_max(ms, world, dev)
     value = flops_step * steps * world / (ms_max / 1e3) / W.scale
 
     pk = peaks()
-    per_einsum = stage_roofline(W, arity, stats, tim, pk)
+    per_einsum = stage_roofline(W, arity, stats, tim, iso, fixup, pk)
     # dominant kernel: the contraction with the largest total time
     dom = max(range(len(per_einsum)), key=lambda c: per_einsum[c]["contract"]["ms"])
     d, s = per_einsum[dom], stats[dom]
@@ -659,16 +717,23 @@ def run_ucl(args, world, rank, local):
             "kernel": f"{kfile} ({d['spec']})", "avg_launch_ms": d["contract"]["ms"],
             "alg_bytes_per_launch": s["bytes_contract"], "peak_src": pk["src"],
             "tensor_frac": d["contract"]["tensor_frac"]}
-    stages = {name: float(tim[:, i].reshape(-1, len(W.chain)).sum(axis=1).mean()) if len(tim) else None
+    stages = {name: float(tim[:, i].reshape(-1, L).sum(axis=1).mean()) if len(tim) else None
               for i, name in enumerate(STAGES)}
 
     # end to end through the C ABI with host buffers
     e2e = None
-    if not args.no_e2e and W.hostable:
+    in_bytes = sum(int(np.asarray(r[0]).size) * 4 + r[2].numel() * r[2].element_size() for r in W.inputs.values())
+    host_avail = host_memory_bytes()
+    if not e2e_on:
+        e2e = {"value": None, "unit": W.unit or UNIT, "skipped": "disabled (--no-e2e)"}
+    elif host_avail is not None and in_bytes > 0.4 * host_avail:
+        e2e = {"value": None, "unit": W.unit or UNIT,
+               "skipped": f"inputs ({in_bytes / 1e9:.1f} GB) exceed 40% of the host memory this process may use "
+                          f"({host_avail / 1e9:.1f} GB): they cannot be staged in pinned host memory"}
+    else:
         host = {k: (torch.as_tensor(r[0]).pin_memory(), r[1], r[2].cpu().pin_memory()) for k, r in W.inputs.items()}
         h2d = sum(t[0].numel() * 4 + t[2].numel() * t[2].element_size() for t in host.values())
         last = W.chain[-1][0]
-
         outbuf = {}
 
         def e2e_step():
@@ -694,31 +759,77 @@ def run_ucl(args, world, rank, local):
         te = (time.perf_counter() - t0) / ne
         te = allreduce_max(te, world, dev)
         e2e = {"value": flops_step * world / te / W.scale, "unit": W.unit or UNIT, "h2d_bytes_per_step": int(h2d),
-               "d2h_bytes_per_step": int(d2h), "ms_per_step": te * 1e3}
-        del host
+               "d2h_bytes_per_step": int(d2h), "ms_per_step": te * 1e3, "steps": ne}
+        del host, outbuf
 
     cpu = cpu_all = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(W, seconds=args.cpu_seconds)
-        cpu_all = cpu_baseline_all_cores(W, seconds=args.cpu_seconds / 4)
-
-    if rank == 0:
-        line = {"metric": W.metric or METRIC, "value": value, "unit": W.unit or UNIT, "n_gpus": world, "steps": steps,
-                "warmup": args.warmup, "ms_per_step": ms_max / steps, "higher_is_better": True, "scaling": "weak",
-                "vs_baseline": None, "dtype": W.dtype, "data": "synthetic",
-                "config": {"workload": W.desc, "pairs": [s["n_pairs"] for s in stats],
-                           "segments": [s["n_segments"] for s in stats], "flops_per_step": flops_step,
-                           "l2": W.l2, "path": [s["path"] for s in stats],
-                           "parallelism": f"replicas x{world}", "alloc": args.alloc},
-                "roofline": roof, "stage_ms": stages, "stage_roofline": per_einsum, "cpu_baseline": cpu,
-                "cpu_baseline_all_cores": cpu_all,
-                "e2e": e2e if e2e is not None else (None if W.hostable else
-                                                    {"value": None, "unit": UNIT,
-                                                     "skipped": "inputs too large to stage through host memory"}),
-                "gpu_launches": int(launches_step * steps), "clocks": ck}
-        print(json.dumps(line), flush=True)
+    if cpu_seconds > 0:
+        cpu = cpu_baseline(W, seconds=cpu_seconds)
+        if all_cores:
+            cpu_all = cpu_baseline_all_cores(W, seconds=cpu_seconds / 4)
     for r in rels.values():
         r.destroy()
+    ctx.synchronize()
+    W.release()
+    del rels, flush
+    torch.cuda.empty_cache()
+    return {"W": W, "value": value, "steps": steps, "ms_per_step": ms_max / steps, "stats": stats,
+            "flops_step": flops_step, "roofline": roof, "stage_ms": stages, "stage_roofline": per_einsum,
+            "latency_ms": float(np.median(lat)), "e2e": e2e, "cpu_baseline": cpu, "cpu_baseline_all_cores": cpu_all,
+            "gpu_launches": int(launches_step * steps), "clocks": ck, "host_memory_bytes": host_avail,
+            "input_bytes": in_bytes}
+
+
+PER_CONFIG = ["blocksparse", "gnn", "mttkrp", "spgemm"]
+
+
+def config_of(m, world, args):
+    W = m["W"]
+    return {"workload": W.desc, "pairs": [s["n_pairs"] for s in m["stats"]],
+            "segments": [s["n_segments"] for s in m["stats"]], "flops_per_step": m["flops_step"], "l2": W.l2,
+            "path": [s["path"] for s in m["stats"]], "parallelism": f"replicas x{world}", "alloc": args.alloc}
+
+
+def run_ucl(args, world, rank, local):
+    from paper_2603_08957_gb300 import Context
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    ctx = Context(local, torch_allocator=(args.alloc == "torch"))
+    solo = rank == 0 and world == 1
+    W = WORKLOADS[args.workload](dev, args)
+    m = measure(W, ctx, args, dev, world, steps=args.steps, warmup=args.warmup,
+                cpu_seconds=args.cpu_seconds if solo and not args.no_cpu_baseline else 0.0,
+                all_cores=True, e2e_on=not args.no_e2e)
+    del W
+    per_config = None
+    todo = PER_CONFIG if (args.per_config == "all" and world == 1 and args.workload == "gnn2") else []
+    if todo:
+        per_config = {}
+        for name in todo:
+            torch.cuda.empty_cache()
+            Wc = WORKLOADS[name](dev, args)
+            mc = measure(Wc, ctx, args, dev, world, steps=None, warmup=args.warmup,
+                         cpu_seconds=0.0 if args.no_cpu_baseline else args.sub_cpu_seconds, all_cores=False,
+                         e2e_on=not args.no_e2e)
+            per_config[name] = {"metric": Wc.metric or METRIC, "value": mc["value"], "unit": Wc.unit or UNIT,
+                                "steps": mc["steps"], "ms_per_step": mc["ms_per_step"],
+                                "latency_ms": mc["latency_ms"], "dtype": Wc.dtype,
+                                "config": config_of(mc, world, args), "roofline": mc["roofline"],
+                                "stage_roofline": mc["stage_roofline"], "cpu_baseline": mc["cpu_baseline"],
+                                "e2e": mc["e2e"], "gpu_launches": mc["gpu_launches"], "clocks": mc["clocks"]}
+            del Wc, mc
+    if rank == 0:
+        Wm = m["W"]
+        line = {"metric": Wm.metric or METRIC, "value": m["value"], "unit": Wm.unit or UNIT, "n_gpus": world,
+                "steps": m["steps"], "warmup": args.warmup, "ms_per_step": m["ms_per_step"],
+                "latency_ms": m["latency_ms"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": Wm.dtype, "data": "synthetic", "config": config_of(m, world, args),
+                "roofline": m["roofline"], "stage_ms": m["stage_ms"], "stage_roofline": m["stage_roofline"],
+                "cpu_baseline": m["cpu_baseline"], "cpu_baseline_all_cores": m["cpu_baseline_all_cores"],
+                "e2e": m["e2e"], "gpu_launches": m["gpu_launches"], "clocks": m["clocks"],
+                "host_memory_bytes": m["host_memory_bytes"], "per_config": per_config}
+        print(json.dumps(line), flush=True)
     ctx.close()
 
 
@@ -820,7 +931,9 @@ def main():
     ap.add_argument("--steps", type=int, default=None)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ucl", "reference"], default="ucl")
-    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="gnn")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="gnn2")
+    ap.add_argument("--per-config", choices=["all", "none"], default="all",
+                    help="with the default two-layer GNN: also measure the other four workloads into per_config")
     ap.add_argument("--path", choices=["auto", "simt", "tc"], default="auto")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -833,6 +946,7 @@ def main():
                     help="mttkrp: storage order of each T tile (the same EinSum either way)")
     ap.add_argument("--seconds", type=float, default=3.0, help="timed seconds when --steps is not given")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--sub-cpu-seconds", type=float, default=5.0, help="oracle seconds for each per_config entry")
     ap.add_argument("--ref-step-seconds", type=float, default=3.0)
     ap.add_argument("--rank-plans", type=int, default=0,
                     help="instead of the benchmark: rank the K cheapest decompositions of the message-passing "

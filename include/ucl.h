@@ -106,6 +106,7 @@ typedef struct {
     int path;              /* ucl_path actually used (SIMT or TC) */
     int launches;          /* GPU kernels launched by the call */
     int timed;             /* 1 if stage_ms is valid (timing enabled) */
+    int n_units;           /* work units (CTAs) the pair list was cut into for the contraction */
     /* stage_ms: [0] key pack/sort/join count, [1] pair expansion, pair sort,
      * segments, [2] tile contraction + fused group-by, [3] split-segment fixup
      * and output key compaction.  CUDA-event times on the context stream. */
@@ -145,6 +146,14 @@ ucl_status ucl_get_last_stats(ucl_ctx *ctx, ucl_stats *out);
  * calls recorded.  Synchronises on the last recorded event.  reset != 0
  * forgets the recorded calls and recycles their events. */
 ucl_status ucl_ctx_timings(ucl_ctx *ctx, float *ms, int max_calls, int *n_calls, int reset);
+
+/* Bytes moved by the fixup kernels of every ucl_einsum on this context since
+ * the last reset: the fp32 partials of output keys whose pairs straddle work
+ * units, read once, plus those keys' output tiles, written once -- the
+ * algorithmic bytes of the cross-unit part of the group-by sum (Sec. 5's
+ * SUM ... GROUP BY).  Counted on the device by the fixup kernels themselves.
+ * Synchronises the context's stream.  reset != 0 zeroes the counter. */
+ucl_status ucl_ctx_fixup_bytes(ucl_ctx *ctx, int64_t *bytes, int reset);
 
 /* ------------------------------------------------------------- relations */
 

@@ -35,6 +35,7 @@ EXPORTS = [
     "ucl_ctx_set_timing",
     "ucl_get_last_stats",
     "ucl_ctx_timings",
+    "ucl_ctx_fixup_bytes",
     "ucl_relation_create",
     "ucl_relation_destroy",
     "ucl_relation_info",
@@ -76,6 +77,7 @@ class Stats(ctypes.Structure):
         ("path", ctypes.c_int),
         ("launches", ctypes.c_int),
         ("timed", ctypes.c_int),
+        ("n_units", ctypes.c_int),
         ("stage_ms", ctypes.c_float * UCL_NSTAGES),
     ]
 
@@ -127,6 +129,7 @@ def _declare(lib):
     lib.ucl_ctx_set_timing.argtypes = [vp, i32]
     lib.ucl_get_last_stats.argtypes = [vp, c.POINTER(Stats)]
     lib.ucl_ctx_timings.argtypes = [vp, c.POINTER(c.c_float), i32, c.POINTER(i32), i32]
+    lib.ucl_ctx_fixup_bytes.argtypes = [vp, c.POINTER(i64), i32]
     lib.ucl_relation_create.argtypes = [vp, i64, i32, vp, c.POINTER(i64), i32, c.POINTER(i64), i32, vp, i32, pp]
     lib.ucl_relation_destroy.argtypes = [vp]
     lib.ucl_relation_info.argtypes = [vp, c.POINTER(i64), c.POINTER(i32), c.POINTER(i32), c.POINTER(i64),

@@ -756,6 +756,19 @@ ucl_status ucl_ctx_timings(ucl_ctx *ctx, float *ms, int max_calls, int *n_calls,
     return UCL_OK;
 }
 
+ucl_status ucl_ctx_fixup_bytes(ucl_ctx *ctx, int64_t *bytes, int reset) {
+    if (!ctx || !bytes) return fail(ctx, UCL_ERR_ARG, "NULL context or output");
+    cudaSetDevice(ctx->device);
+    unsigned long long *d = reinterpret_cast<unsigned long long *>(ctx->d_status + ucl_ctx::kFixupCounterWord);
+    unsigned long long h = 0;
+    cudaError_t e = cudaMemcpyAsync(&h, d, sizeof(h), cudaMemcpyDeviceToHost, ctx->main);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(ctx->main);
+    if (e == cudaSuccess && reset) e = cudaMemsetAsync(d, 0, sizeof(h), ctx->main);
+    if (e != cudaSuccess) return cuda_check(ctx, e, "fixup byte counter");
+    *bytes = (int64_t)h;
+    return UCL_OK;
+}
+
 ucl_status ucl_relation_create(ucl_ctx *ctx, int64_t n, int u, const int32_t *keys, const int64_t *key_bounds,
                                int r, const int64_t *tile_shape, ucl_dtype dtype, const void *tiles, ucl_mem mem,
                                ucl_rel **out) {
@@ -1158,6 +1171,7 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             a.comb = o.comb;
             a.map = o.map;
             a.tile_w = lp.tile_w;
+            a.fixup_bytes = reinterpret_cast<unsigned long long *>(ctx->d_status + ucl_ctx::kFixupCounterWord);
             bool use_tc = tc_ok && o.path != UCL_PATH_SIMT;
             if (use_tc && n_in < 3) {
                 std::string why2;
@@ -1170,6 +1184,7 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
                            : (int)std::min<int64_t>(P, (int64_t)ctx->sm_count * 4);
             a.units.P = P;
             a.units.G = G;
+            stats.n_units = G;
             a.partials = (float *)ws_get(ctx, sizeof(float) * 2 * (size_t)G * lp.tile_w);
             if (use_tc && n_in == 3) {
                 check(launch_contract_tc3(ctx, a, tp3, in));

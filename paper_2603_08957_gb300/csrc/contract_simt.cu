@@ -433,6 +433,11 @@ __global__ void __launch_bounds__(kSimtThreads) fixup_kernel(ContractArgs a) {
     // units c .. u_end - 1 hold the segment's continuation partials (slot 0)
     int u_end = c;
     while (u_end < a.units.G && a.units.begin(u_end) < se) ++u_end;
+    if (a.fixup_bytes && threadIdx.x == 0) {
+        // partials of units c - 1 .. u_end - 1 read, one output tile written
+        const int osz = a.dout == UCL_BF16 ? 2 : 4;
+        atomicAdd(a.fixup_bytes, (unsigned long long)(a.tile_w * (4 * (u_end - c + 1) + osz)));
+    }
     // kU elements per thread per round, all loads of a partial issued before
     // any is used, so a round costs one memory latency per partial rather
     // than one per element; the fold order (units in order) is unchanged

@@ -135,8 +135,10 @@ struct ucl_ctx {
     cudaEvent_t arena_done[kArenas] = {};
     int arena_next = 0;
     ucl::Arena *arena = &arenas[0];
-    // [1] validation flags (main), [2] sticky error bits of main-stream kernels
+    // [1] validation flags (main), [2] sticky error bits of main-stream kernels,
+    // words [16, 18): the fixup kernels' byte counter (64-bit)
     uint32_t *d_status = nullptr;
+    static constexpr int kFixupCounterWord = 16;
     // pinned host scratch for sizing syncs: kPinnedRead int64 values, then the
     // device status words
     static constexpr int kPinnedRead = 36, kPinnedWords = 40;
@@ -302,6 +304,7 @@ struct ContractArgs {
     int agg, comb, map;    // extended EinSum (ucl_agg / ucl_comb / ucl_map); 0, 0, 0 = sum of products
     float *partials;       // [G, 2, tile_w]
     int64_t tile_w;
+    unsigned long long *fixup_bytes;   // device counter the fixup kernel adds its bytes to (may be NULL)
 };
 void launch_contract_simt(ucl_ctx *ctx, const ContractArgs &a, const LowerPlan &lp);
 void launch_fixup(ucl_ctx *ctx, const ContractArgs &a);

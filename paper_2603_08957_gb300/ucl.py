@@ -123,8 +123,15 @@ class Context:
             "bytes_contract": st.bytes_contract,
             "path": {1: "simt", 2: "tc"}.get(st.path, "none"),
             "launches": st.launches,
+            "n_units": st.n_units,
             "stage_ms": list(st.stage_ms) if st.timed else None,
         }
+
+    def fixup_bytes(self, reset: bool = True) -> int:
+        """Bytes the fixup kernels moved since the last reset (device counter)."""
+        v = ctypes.c_int64()
+        self._check(self.lib.ucl_ctx_fixup_bytes(self.handle, ctypes.byref(v), 1 if reset else 0))
+        return v.value
 
     # ---------------------------------------------------------- relations
     def relation(self, keys, bounds, tiles, *, copy: bool = False) -> "Relation":
