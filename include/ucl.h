@@ -107,6 +107,8 @@ typedef struct {
     int launches;          /* GPU kernels launched by the call */
     int timed;             /* 1 if stage_ms is valid (timing enabled) */
     int n_units;           /* work units (CTAs) the pair list was cut into for the contraction */
+    int n_bands;           /* bands of the contracted label (1: not banded; see ucl_einsum) */
+    int64_t n_band_segments; /* (band, output key) groups of a banded EinSum, else n_segments */
     /* stage_ms: [0] key pack/sort/join count, [1] pair expansion, pair sort,
      * segments, [2] tile contraction + fused group-by, [3] split-segment fixup
      * and output key compaction.  CUDA-event times on the context stream. */

@@ -78,6 +78,8 @@ class Stats(ctypes.Structure):
         ("launches", ctypes.c_int),
         ("timed", ctypes.c_int),
         ("n_units", ctypes.c_int),
+        ("n_bands", ctypes.c_int),
+        ("n_band_segments", ctypes.c_int64),
         ("stage_ms", ctypes.c_float * UCL_NSTAGES),
     ]
 

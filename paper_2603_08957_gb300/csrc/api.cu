@@ -11,6 +11,7 @@
 //      contraction with the group-by sum fused into its epilogue
 //   3  fixup of segments split across work units
 #include <algorithm>
+#include <cstdlib>
 #include <cstdio>
 #include <new>
 
@@ -406,6 +407,51 @@ bool plan_tc3(const Spec &s, ucl_rel *const *in, const KeyPlan &kp, Tc3Plan &tp,
 
 size_t dsize(ucl_dtype d) { return d == UCL_BF16 ? 2 : 4; }
 
+// Banding of the contracted label.  When U (the operand whose tuples each
+// join many V tuples) is larger than L2, the contraction re-reads U's tiles
+// from HBM: the pairs of one output key visit the whole range of the join
+// label, and all CTAs together sweep all of U at every moment.  Cutting the
+// leading join label into B ranges (bands) whose share of U fits L2, and
+// contracting band after band, keeps U's working set in L2.  Each band sums
+// into fp32 partials keyed (band, output key), and a band sum adds them in
+// band order.  The EinSum computed is unchanged: the band is an extra upper
+// label of the partial output, derived from the join label and summed out
+// again (the Sec. 5 template applied twice, with part of the contracted label
+// promoted in between).  The band field is packed above the output key, from
+// the top bits of U's join label.
+struct BandPlan {
+    int B = 1, bits = 0;
+};
+
+constexpr int kMaxBands = 16;   // 2 (B + 1) band ranges are read in one sizing sync
+
+BandPlan plan_bands(ucl_ctx *ctx, const Spec &s, ucl_rel *const *in, KeyPlan &kp, bool tc_ok) {
+    BandPlan bp;
+    if (s.n_in != 2 || !tc_ok || kp.join.empty() || ctx->tune_bands == 0 || ctx->tune_bands == 1) return bp;
+    const Label &L = s.labs[kp.join[0]];
+    const int ku = kp.ord[0];
+    if (L.pos[3] >= 0 || kp.out_k[ku].nf >= kMaxCols) return bp;   // the join label is kept in the output
+    const ucl_rel *U = in[ku], *V = in[kp.ord[1]];
+    const double ubytes = (double)U->n * (double)U->tile * (double)dsize(U->dtype);
+    const int jb = bit_width(L.ext);
+    int B = 1;
+    if (ctx->tune_bands > 1) {
+        B = std::min(ctx->tune_bands, kMaxBands);
+    } else {
+        const double l2 = ctx->l2_bytes > 0 ? (double)ctx->l2_bytes : 126e6;
+        if (!(ubytes > l2 && V->n >= 4 * U->n)) return bp;
+        while (B < kMaxBands && ubytes / B > l2) B *= 2;
+    }
+    int bits = 0;
+    while ((1 << bits) < B) ++bits;
+    if (bits > jb) bits = jb;
+    if (bits == 0 || kp.out_bits + bits > 64) return bp;
+    bp.B = 1 << bits;
+    bp.bits = bits;
+    kp.out_k[ku].f[kp.out_k[ku].nf++] = KeyField{L.pos[ku], kp.out_bits, bits, jb - bits};
+    return bp;
+}
+
 // Take the next workspace arena in turn.  The stream in use first waits until
 // main has finished the call that used it last; a grown arena is merged into
 // one block.
@@ -659,6 +705,12 @@ ucl_status ucl_ctx_create(int device, void *stream, ucl_alloc_fn alloc, ucl_free
         if (!st) st = cuda_check(ctx, cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep),
                                  "cudaMemPoolSetAttribute");
     }
+    if (!st && cudaDeviceGetAttribute(&ctx->l2_bytes, cudaDevAttrL2CacheSize, device) != cudaSuccess) {
+        cudaGetLastError();
+        ctx->l2_bytes = 0;
+    }
+    if (const char *e = getenv("UCL_BANDS")) ctx->tune_bands = atoi(e);
+    if (const char *e = getenv("UCL_L2_HINTS")) ctx->tune_hints = atoi(e);
     if (!st) st = cuda_check(ctx, cudaMalloc(&ctx->d_status, 256), "cudaMalloc status");
     if (!st) st = cuda_check(ctx, cudaMemset(ctx->d_status, 0, 256), "cudaMemset status");
     if (!st) st = cuda_check(ctx, cudaMallocHost(&ctx->h_pinned, ucl_ctx::kPinnedWords * sizeof(int64_t)), "cudaMallocHost");
@@ -956,6 +1008,9 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
     std::string why;
     const bool tc_ok = !extended && (n_in == 3 ? plan_tc3(s, in, kp, tp3, &why) : plan_tc(s, in, tp, &why));
     if (o.path == UCL_PATH_TC && !tc_ok) return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why);
+    const BandPlan bp = plan_bands(ctx, s, in, kp, tc_ok && o.path != UCL_PATH_SIMT);
+    const bool banded = bp.B > 1;
+    const int sort_bits = kp.out_bits + bp.bits;
     cudaSetDevice(ctx->device);
 
     const ucl_rel *U = in[0];
@@ -978,7 +1033,10 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
     for (int k = 0; k < n_in; ++k) wait_keys(ctx, in[k]);
     try {
         record(ctx, 0);
-        int64_t *d_scal = (int64_t *)ws_get(ctx, 8 * sizeof(int64_t));
+        // [0] pair count, [1] segment count, [2] triple count or, banded,
+        // [2, 2 + B] band starts and [3 + B, 3 + 2B] their segment indices,
+        // [39] banded: output key count
+        int64_t *d_scal = (int64_t *)ws_get(ctx, 40 * sizeof(int64_t));
         // ---------------------------------------------------------- stage 0
         // pack keys; sort each side of a join by its join key unless it is
         // already grouped; count the joined pairs (for three inputs: the
@@ -1064,6 +1122,7 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
 
         // ---------------------------------------------------------- stage 1
         int64_t S = 0;
+        int64_t band_start[kMaxBands + 1] = {}, band_seg[kMaxBands + 1] = {};
         uint64_t *pk = nullptr, *pv = nullptr;
         int64_t *seg_excl = nullptr;
         if (P > 0) {
@@ -1081,18 +1140,24 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             // and alone supplies the output key, as its leading key columns,
             // the pairs are already in output-key order: the stable sort
             // would leave them as they are, so it is skipped.
-            bool presorted = A->sorted && permA == nullptr;
+            bool presorted = A->sorted && permA == nullptr && !banded;
             for (int k = 1; k < n_in && presorted; ++k) presorted = kp.out_k[kp.ord[k]].nf == 0;
             for (int q = 0; q < kp.out_k[kp.ord[0]].nf && presorted; ++q)
                 presorted = kp.out_k[kp.ord[0]].f[q].col == q;
-            if (!presorted && radix_sort(ctx, pk, pv, pk2, pv2, P, kp.out_bits)) { pk = pk2; pv = pv2; }
+            if (!presorted && radix_sort(ctx, pk, pv, pk2, pv2, P, sort_bits)) { pk = pk2; pv = pv2; }
             int64_t *flag = (int64_t *)ws_get(ctx, 8 * P);
             seg_excl = (int64_t *)ws_get(ctx, 8 * P);
             launch_heads(ctx, pk, P, flag);
             scan_i64(ctx, flag, seg_excl, P, d_scal + 1);
-            int64_t h;
-            check(sync_read(ctx, d_scal + 1, 1, &h));
-            S = h;
+            if (banded)
+                launch_band_ranges(ctx, pk, P, seg_excl, d_scal + 1, kp.out_bits, bp.B, d_scal + 2, d_scal + 3 + bp.B);
+            int64_t h[1 + 2 * (kMaxBands + 1)];
+            check(sync_read(ctx, d_scal + 1, banded ? 1 + 2 * (bp.B + 1) : 1, h));
+            S = h[0];
+            for (int b = 0; banded && b <= bp.B; ++b) {
+                band_start[b] = h[1 + b];
+                band_seg[b] = h[2 + bp.B + b];
+            }
         }
 
         // ------------------------------------------------------ segments
@@ -1114,6 +1179,30 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             } else {
                 launch_segments(ctx, pk, pv, seg_excl, P, S, kp.unpack, okeys, seg_start, pu, pvi);
             }
+        }
+        // banded: the S (band, output key) segments hold fp32 partials; sort
+        // them by (output key, band) and find the output keys
+        const int64_t Sp = S;
+        uint64_t *band_order = nullptr;
+        int64_t *fstart = nullptr;
+        if (banded && P > 0) {
+            uint64_t *sk = (uint64_t *)ws_get(ctx, 8 * Sp), *sv = (uint64_t *)ws_get(ctx, 8 * Sp),
+                     *sk2 = (uint64_t *)ws_get(ctx, 8 * Sp), *sv2 = (uint64_t *)ws_get(ctx, 8 * Sp);
+            launch_band_keys(ctx, pk, seg_start, Sp, kp.out_bits, bp.bits, sk, sv);
+            if (radix_sort(ctx, sk, sv, sk2, sv2, Sp, sort_bits)) {
+                sk = sk2;
+                sv = sv2;
+            }
+            int64_t *flag2 = (int64_t *)ws_get(ctx, 8 * Sp), *excl2 = (int64_t *)ws_get(ctx, 8 * Sp);
+            launch_heads(ctx, sk, Sp, flag2, bp.bits);
+            scan_i64(ctx, flag2, excl2, Sp, d_scal + 39);
+            int64_t hs = 0;
+            check(sync_read(ctx, d_scal + 39, 1, &hs));
+            S = hs;
+            okeys = (int32_t *)ws_get(ctx, 4 * (size_t)S * kp.uw);
+            fstart = (int64_t *)ws_get(ctx, 8 * (S + 1));
+            launch_band_outputs(ctx, sk, excl2, Sp, S, bp.bits, kp.unpack, okeys, fstart);
+            band_order = sv;
         }
         record(ctx, 2);
         to_main(ctx);
@@ -1184,21 +1273,56 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
                            : (int)std::min<int64_t>(P, (int64_t)ctx->sm_count * 4);
             a.units.P = P;
             a.units.G = G;
+            a.units.base = 0;
+            a.bands = bp.B;
+            a.l2_hints = ctx->tune_hints;
             stats.n_units = G;
             a.partials = (float *)ws_get(ctx, sizeof(float) * 2 * (size_t)G * lp.tile_w);
-            if (use_tc && n_in == 3) {
-                check(launch_contract_tc3(ctx, a, tp3, in));
-                path = UCL_PATH_TC;
-            } else if (use_tc) {
-                const ucl_rel *ra = tp.a_is_u ? U : V, *rb = tp.a_is_u ? V : U;
-                check(launch_contract_tc(ctx, a, tp, ra, rb));
-                path = UCL_PATH_TC;
+            auto contract = [&](const ContractArgs &c) {
+                if (use_tc && n_in == 3) {
+                    check(launch_contract_tc3(ctx, c, tp3, in));
+                    path = UCL_PATH_TC;
+                } else if (use_tc) {
+                    const ucl_rel *ra = tp.a_is_u ? U : V, *rb = tp.a_is_u ? V : U;
+                    check(launch_contract_tc(ctx, c, tp, ra, rb));
+                    path = UCL_PATH_TC;
+                } else {
+                    launch_contract_simt(ctx, c, lp);
+                }
+            };
+            if (!banded) {
+                contract(a);
+                record(ctx, 4);
+                launch_fixup(ctx, a);
+                record(ctx, 5);
             } else {
-                launch_contract_simt(ctx, a, lp);
+                // band after band into fp32 partials keyed (band, output
+                // key), each band cut into its own G units; then the band sum
+                const size_t pbytes = sizeof(float) * (size_t)Sp * lp.tile_w;
+                float *part = (float *)ctx_alloc(ctx, pbytes);
+                if (!part) throw Oom();
+                for (int b = 0; b < bp.B; ++b) {
+                    const int64_t Pb = band_start[b + 1] - band_start[b];
+                    if (Pb <= 0) continue;
+                    ContractArgs c = a;
+                    c.seg_start = seg_start + band_seg[b];
+                    c.S = band_seg[b + 1] - band_seg[b];
+                    c.units.P = Pb;
+                    c.units.G = use_tc ? tc_units(ctx, tp, Pb) : (int)std::min<int64_t>(Pb, (int64_t)ctx->sm_count * 4);
+                    c.units.base = band_start[b];
+                    c.out = part + (size_t)band_seg[b] * lp.tile_w;
+                    c.dout = UCL_F32;
+                    c.epi = UCL_EPI_NONE;
+                    c.scale = 1.0f;
+                    contract(c);
+                    launch_fixup(ctx, c);
+                }
+                record(ctx, 4);
+                launch_band_sum(ctx, part, band_order, fstart, S, lp.tile_w, R->tiles, o.out_dtype, o.epi, o.scale,
+                                a.fixup_bytes);
+                record(ctx, 5);
+                ctx_free(ctx, part, pbytes);
             }
-            record(ctx, 4);
-            launch_fixup(ctx, a);
-            record(ctx, 5);
         } else {
             record(ctx, 4);
             record(ctx, 5);
@@ -1207,6 +1331,8 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
 
         stats.n_pairs = P;
         stats.n_segments = S;
+        stats.n_bands = bp.B;
+        stats.n_band_segments = Sp;
         stats.flops = 2.0 * (double)P * (double)lp.tile_w * (double)lp.n_c;
         stats.bytes_contract = (double)nU * U->tile * dsize(U->dtype) +
                                (V ? (double)nV * V->tile * dsize(V->dtype) : 0.0) +

@@ -18,6 +18,8 @@
 // in a separate instantiation so that the plain sum of products keeps its
 // FFMA inner loop; partials of split segments are folded with the same
 // aggregate.
+#include <algorithm>
+
 #include "internal.cuh"
 
 namespace ucl {
@@ -426,7 +428,7 @@ __global__ void __launch_bounds__(kSimtThreads, 1) simt_contract3_kernel(Contrac
 __global__ void __launch_bounds__(kSimtThreads) fixup_kernel(ContractArgs a) {
     const int c = blockIdx.x + 1;
     const int64_t p = a.units.begin(c);
-    if (p >= a.units.P) return;
+    if (p >= a.units.base + a.units.P) return;
     const int64_t s = find_seg(a.seg_start, a.S, p);
     const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
     if (ss >= p || ss < a.units.begin(c - 1)) return;
@@ -470,7 +472,70 @@ __global__ void __launch_bounds__(kSimtThreads) fixup_kernel(ContractArgs a) {
     }
 }
 
+// Band sum: output key f is the sum, in band order, of its band partials
+// part[order[r]] for r in [fstart[f], fstart[f + 1]) (fp32 tiles), then the
+// epilogue and the output cast.  One CTA per output tile at a time; two
+// 16-byte loads per thread and row in flight.
+__global__ void __launch_bounds__(kSimtThreads) band_sum_kernel(const float *__restrict__ part,
+                                                                const uint64_t *__restrict__ order,
+                                                                const int64_t *__restrict__ fstart, int64_t S,
+                                                                int64_t tile_w, void *out, int dout, int epi,
+                                                                float scale, unsigned long long *bytes) {
+    const bool vec = (tile_w & 3) == 0;
+    const int osz = dout == UCL_BF16 ? 2 : 4;
+    for (int64_t f = blockIdx.x; f < S; f += gridDim.x) {
+        const int64_t r0 = fstart[f], r1 = fstart[f + 1];
+        if (bytes && threadIdx.x == 0) atomicAdd(bytes, (unsigned long long)(tile_w * (4 * (r1 - r0) + osz)));
+        if (vec) {
+            const int64_t step = (int64_t)blockDim.x * 4;
+            for (int64_t e0 = (int64_t)threadIdx.x * 4; e0 < tile_w; e0 += 2 * step) {
+                const int64_t e1 = e0 + step;
+                const bool two = e1 < tile_w;
+                float4 a0 = make_float4(0.f, 0.f, 0.f, 0.f), a1 = a0;
+                for (int64_t r = r0; r < r1; ++r) {
+                    const float *row = part + (int64_t)order[r] * tile_w;
+                    const float4 v0 = __ldg(reinterpret_cast<const float4 *>(row + e0));
+                    const float4 v1 = two ? __ldg(reinterpret_cast<const float4 *>(row + e1)) : a1;
+                    a0.x += v0.x; a0.y += v0.y; a0.z += v0.z; a0.w += v0.w;
+                    if (two) { a1.x += v1.x; a1.y += v1.y; a1.z += v1.z; a1.w += v1.w; }
+                }
+                for (int h = 0; h < (two ? 2 : 1); ++h) {
+                    const float4 a = h ? a1 : a0;
+                    const int64_t e = h ? e1 : e0;
+                    const float x0 = epilogue(a.x, epi, scale), x1 = epilogue(a.y, epi, scale),
+                                x2 = epilogue(a.z, epi, scale), x3 = epilogue(a.w, epi, scale);
+                    if (dout == UCL_BF16) {
+                        __nv_bfloat162 lo = __floats2bfloat162_rn(x0, x1), hi = __floats2bfloat162_rn(x2, x3);
+                        uint2 w;
+                        w.x = *reinterpret_cast<uint32_t *>(&lo);
+                        w.y = *reinterpret_cast<uint32_t *>(&hi);
+                        *reinterpret_cast<uint2 *>(reinterpret_cast<__nv_bfloat16 *>(out) + f * tile_w + e) = w;
+                    } else {
+                        *reinterpret_cast<float4 *>(reinterpret_cast<float *>(out) + f * tile_w + e) =
+                            make_float4(x0, x1, x2, x3);
+                    }
+                }
+            }
+        } else {
+            for (int64_t e = threadIdx.x; e < tile_w; e += blockDim.x) {
+                float acc = 0.0f;
+                for (int64_t r = r0; r < r1; ++r) acc += __ldg(part + (int64_t)order[r] * tile_w + e);
+                store_out(out, (ucl_dtype)dout, f * tile_w + e, epilogue(acc, epi, scale));
+            }
+        }
+    }
+}
+
 }  // namespace
+
+void launch_band_sum(ucl_ctx *ctx, const float *part, const uint64_t *order, const int64_t *fstart, int64_t S,
+                     int64_t tile_w, void *out, ucl_dtype dout, int epi, float scale, unsigned long long *bytes) {
+    if (S <= 0) return;
+    const int64_t grid = std::min<int64_t>(S, (int64_t)ctx->sm_count * 8);
+    band_sum_kernel<<<(int)grid, kSimtThreads, 0, ctx->stream>>>(part, order, fstart, S, tile_w, out, (int)dout, epi,
+                                                                  scale, bytes);
+    ctx->launches++;
+}
 
 void launch_contract_simt(ucl_ctx *ctx, const ContractArgs &a, const LowerPlan &lp) {
     const int G = a.units.G;

@@ -75,6 +75,7 @@ struct TcArgs {
     int ns, nacc, nmma;
     int pf_a, pf_b;              // prefetch the A / B tiles into L2 ahead of their TMA loads
     int pf_dist;                 // how many of its own fills ahead a producer prefetches
+    int hint_a, hint_b;          // L2 policy of the A / B tile loads: 0 none, 1 evict first, 2 evict last
     uint32_t tmem_cols;
     uint32_t idesc;
     // descriptor templates (stage 0, slot 0, k step 0) and per-step offsets in
@@ -177,6 +178,27 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map
         "[%5];" ::"r"(dst),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar)
         : "memory");
+}
+
+// The same copy with an L2 eviction policy (from createpolicy).
+__device__ __forceinline__ void tma_load_3d_hint(uint32_t dst, const CUtensorMap *map, int x, int y, int z,
+                                                 uint32_t bar, uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1, "
+        "{%2, %3, %4}], [%5], %6;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar), "l"(policy)
+        : "memory");
+}
+
+// L2 policies: lines a copy brings in are evicted before (first) or after
+// (last) lines of normal priority.
+__device__ __forceinline__ uint64_t policy_of(int hint) {
+    uint64_t p = 0;
+    if (hint == 1)
+        asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    else
+        asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
 }
 
 // Hint that a box of the tensor will be loaded soon: fetched into L2 only,
@@ -310,6 +332,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int nfills = (n + pps - 1) / pps;
         const int kmask = (1 << a.kc_lg) - 1;
         uint32_t mine = 0;
+        const uint64_t pol_a = a.hint_a ? policy_of(a.hint_a) : 0ull, pol_b = a.hint_b ? policy_of(a.hint_b) : 0ull;
         // raw index loads two own fills ahead, checked only when used, so a
         // fill never waits on the latency of its own index loads
         auto load_idx = [&](int f, uint32_t &ia, uint32_t &ib) {
@@ -369,10 +392,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 const uint32_t sa = sbase + st * a.stage_bytes + (uint32_t)lane * a.a_pair;
                 const uint32_t sb = sbase + st * a.stage_bytes + (uint32_t)a.pps * a.a_pair + (uint32_t)lane * a.b_pair;
                 const int c = (f * pps + lane) & kmask;   // K chunk
-                for (int q = 0; q < a.na_sub; ++q)
-                    tma_load_3d(sa + q * a.a_sub, &tmA, q * a.wa + c * a.a_cx, c * a.a_cy, (int)ia, fb);
-                for (int q = 0; q < a.nb_sub; ++q)
-                    tma_load_3d(sb + q * a.b_sub, &tmB, q * a.wb + c * a.b_cx, c * a.b_cy, (int)ib, fb);
+                for (int q = 0; q < a.na_sub; ++q) {
+                    if (a.hint_a)
+                        tma_load_3d_hint(sa + q * a.a_sub, &tmA, q * a.wa + c * a.a_cx, c * a.a_cy, (int)ia, fb, pol_a);
+                    else
+                        tma_load_3d(sa + q * a.a_sub, &tmA, q * a.wa + c * a.a_cx, c * a.a_cy, (int)ia, fb);
+                }
+                for (int q = 0; q < a.nb_sub; ++q) {
+                    if (a.hint_b)
+                        tma_load_3d_hint(sb + q * a.b_sub, &tmB, q * a.wb + c * a.b_cx, c * a.b_cy, (int)ib, fb, pol_b);
+                    else
+                        tma_load_3d(sb + q * a.b_sub, &tmB, q * a.wb + c * a.b_cx, c * a.b_cy, (int)ib, fb);
+                }
             }
             __syncwarp();
             ++mine;
@@ -904,11 +935,29 @@ ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan 
             l2 = 0;
         }
         const double big = l2 > 0 ? l2 / 4.0 : 32.0 * (1 << 20);
-        const double bytes_a = (double)ra->n * tp.M * tp.K * 2, bytes_b = (double)rb->n * tp.N * tp.K * 2;
-        const int64_t P = a.units.P;
-        k.pf_a = g.kc == 1 && bytes_a > big && 2 * ra->n >= P && bytes_b <= big;
-        k.pf_b = g.kc == 1 && bytes_b > big && 2 * rb->n >= P && bytes_a <= big;
+        // a banded launch covers one band: about 1 / bands of each input's tuples
+        const double band = a.bands > 1 ? (double)a.bands : 1.0;
+        const double na = ra->n / band, nb = rb->n / band;
+        const double bytes_a = na * tp.M * tp.K * 2, bytes_b = nb * tp.N * tp.K * 2;
+        const double P = (double)a.units.P;
+        k.pf_a = g.kc == 1 && bytes_a > big && 2 * na >= P && bytes_b <= big;
+        k.pf_b = g.kc == 1 && bytes_b > big && 2 * nb >= P && bytes_a <= big;
         k.pf_dist = 2;
+        // L2 eviction hints: a streamed operand (each tuple joined about once,
+        // larger than a quarter of L2) is evicted first, so that the reused
+        // operand (joined at least four times per tuple) stays; that one is
+        // evicted last
+        k.hint_a = k.hint_b = 0;
+        if (a.l2_hints) {
+            const bool stream_a = bytes_a > big && 2 * na >= P, stream_b = bytes_b > big && 2 * nb >= P;
+            if (stream_a && !stream_b) {
+                k.hint_a = 1;
+                if (P >= 4 * nb) k.hint_b = 2;
+            } else if (stream_b && !stream_a) {
+                k.hint_b = 1;
+                if (P >= 4 * na) k.hint_a = 2;
+            }
+        }
     }
     k.tmem_cols = g.tmem_cols;
     // instruction descriptor, kind::f16: D fp32 (bits 4-5), A and B bf16 (7-9, 10-12),

@@ -30,6 +30,7 @@ struct KeyField {
     int col;
     int shift;
     int bits;
+    int rshift;   // the field holds the column's value >> rshift (0: the whole value)
 };
 
 // How to build one packed key from a relation's key row.
@@ -84,11 +85,13 @@ struct Tc3Plan {
     int64_t sWi, sWr;        // output tile strides of i and r
 };
 
-// Partition of the pair list into G contiguous units (one CTA each).
+// Partition of the pair list into G contiguous units (one CTA each): unit u
+// covers pairs [begin(u), begin(u + 1)) of the P pairs that start at `base`.
 struct Units {
     int64_t P;
     int G;
-    __host__ __device__ int64_t begin(int u) const { return P * u / G; }
+    int64_t base;
+    __host__ __device__ int64_t begin(int u) const { return base + P * u / G; }
 };
 
 // Stream-ordered bump allocator over blocks obtained from the context hooks.
@@ -154,6 +157,12 @@ struct ucl_ctx {
     ucl_stats last{};
     std::string err;
     int live_rels = 0;
+    // Overrides read from the environment at creation, for measurement:
+    // UCL_BANDS (unset: automatic; 0 or 1: no banding; 2..16: that many
+    // bands where banding applies) and UCL_L2_HINTS (0: no L2 eviction hints).
+    int tune_bands = -1;
+    int tune_hints = 1;
+    int l2_bytes = 0;
 };
 
 struct ucl_rel {
@@ -212,8 +221,19 @@ void launch_expand(ucl_ctx *ctx, const int64_t *off, int64_t nu, const uint32_t 
                    uint64_t *pv);
 // Unary: pairs = tuples of U.
 void launch_unary_pairs(ucl_ctx *ctx, const uint64_t *ko_u, int64_t n, uint64_t *pk, uint64_t *pv);
-// Segment heads (flag[p] = 1 where the key changes), as int64 for the scan.
-void launch_heads(ucl_ctx *ctx, const uint64_t *pk, int64_t P, int64_t *flag);
+// Segment heads (flag[p] = 1 where key >> shift changes), as int64 for the scan.
+void launch_heads(ucl_ctx *ctx, const uint64_t *pk, int64_t P, int64_t *flag, int shift = 0);
+// Banded pair lists, sorted by (band << out_bits | output key): band_start[b]
+// = first pair of band b, band_seg[b] = its segment index (b = 0..B; B <= 63).
+void launch_band_ranges(ucl_ctx *ctx, const uint64_t *pk, int64_t P, const int64_t *seg_excl, const int64_t *n_seg,
+                        int out_bits, int B, int64_t *band_start, int64_t *band_seg);
+// sk[s] = (output key << band_bits) | band of band segment s, sv[s] = s.
+void launch_band_keys(ucl_ctx *ctx, const uint64_t *pk, const int64_t *seg_start, int64_t Sp, int out_bits,
+                      int band_bits, uint64_t *sk, uint64_t *sv);
+// After sorting sk: the S output keys and fstart[f] = first sorted band
+// segment of output key f (fstart[S] = Sp).
+void launch_band_outputs(ucl_ctx *ctx, const uint64_t *sk, const int64_t *excl, int64_t Sp, int64_t S, int band_bits,
+                         KeyUnpack un, int32_t *out_keys, int64_t *fstart);
 // Segment starts, output keys, pair index arrays.
 void launch_segments(ucl_ctx *ctx, const uint64_t *pk, const uint64_t *pv, const int64_t *seg_excl, int64_t P,
                      int64_t S, KeyUnpack un, int32_t *out_keys, int64_t *seg_start, uint32_t *pu, uint32_t *pvi);
@@ -305,9 +325,16 @@ struct ContractArgs {
     float *partials;       // [G, 2, tile_w]
     int64_t tile_w;
     unsigned long long *fixup_bytes;   // device counter the fixup kernel adds its bytes to (may be NULL)
+    int bands;             // > 1: U's tuples are split into this many bands of its join label (one launch each)
+    int l2_hints;          // TMA loads carry L2 eviction hints (streamed operand first, reused operand last)
 };
 void launch_contract_simt(ucl_ctx *ctx, const ContractArgs &a, const LowerPlan &lp);
 void launch_fixup(ucl_ctx *ctx, const ContractArgs &a);
+// Band sum of a banded EinSum (see launch_band_outputs): out[f] = epilogue(sum
+// over r in [fstart[f], fstart[f + 1]) of part[order[r]]), cast to dout; adds
+// its bytes (partials read, outputs written) to *bytes if not NULL.
+void launch_band_sum(ucl_ctx *ctx, const float *part, const uint64_t *order, const int64_t *fstart, int64_t S,
+                     int64_t tile_w, void *out, ucl_dtype dout, int epi, float scale, unsigned long long *bytes);
 // tcgen05 path; returns false (nothing launched) if the shapes do not fit.
 bool tc_supported(const TcPlan &tp, const ContractArgs &a, std::string *why);
 ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan &tp, const ucl_rel *ra,

@@ -23,7 +23,7 @@ int grid_for(ucl_ctx *ctx, int64_t n, int per_thread = 1) {
 __device__ __forceinline__ uint64_t pack_row(const int32_t *row, const KeyPack &kp) {
     uint64_t k = 0;
     for (int i = 0; i < kp.nf; ++i) {
-        uint64_t v = (uint32_t)row[kp.f[i].col];
+        uint64_t v = (uint32_t)row[kp.f[i].col] >> kp.f[i].rshift;
         k |= v << kp.f[i].shift;
     }
     return k;
@@ -286,9 +286,54 @@ __global__ void unary_pairs_kernel(const uint64_t *__restrict__ ko_u, int64_t n,
     }
 }
 
-__global__ void heads_kernel(const uint64_t *__restrict__ pk, int64_t P, int64_t *flag) {
+__global__ void heads_kernel(const uint64_t *__restrict__ pk, int64_t P, int shift, int64_t *flag) {
     for (int64_t p = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; p < P; p += (int64_t)gridDim.x * blockDim.x)
-        flag[p] = (p == 0 || pk[p] != pk[p - 1]) ? 1 : 0;
+        flag[p] = (p == 0 || (pk[p] >> shift) != (pk[p - 1] >> shift)) ? 1 : 0;
+}
+
+// Banded pair lists (pairs sorted by (band, output key)): thread b finds the
+// first pair of band b (b = B: P) and the index of its segment.
+__global__ void band_ranges_kernel(const uint64_t *__restrict__ pk, int64_t P, const int64_t *__restrict__ seg_excl,
+                                   const int64_t *__restrict__ n_seg, int out_bits, int B, int64_t *band_start,
+                                   int64_t *band_seg) {
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b > B) return;
+    int64_t lo = 0, hi = P;
+    while (lo < hi) {
+        const int64_t mid = (lo + hi) >> 1;
+        if ((int64_t)(pk[mid] >> out_bits) < b) lo = mid + 1; else hi = mid;
+    }
+    band_start[b] = lo;
+    band_seg[b] = lo < P ? seg_excl[lo] : *n_seg;
+}
+
+// Key of each band segment for the band sum: (output key, band), so that a
+// sort groups every output key's band partials in band order.
+__global__ void band_keys_kernel(const uint64_t *__restrict__ pk, const int64_t *__restrict__ seg_start, int64_t Sp,
+                                 int out_bits, int band_bits, uint64_t *sk, uint64_t *sv) {
+    const uint64_t omask = out_bits ? (~0ull >> (64 - out_bits)) : 0ull;
+    for (int64_t s = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; s < Sp; s += (int64_t)gridDim.x * blockDim.x) {
+        const uint64_t k = pk[seg_start[s]];
+        sk[s] = ((k & omask) << band_bits) | (k >> out_bits);
+        sv[s] = (uint64_t)s;
+    }
+}
+
+// Output keys and the first sorted band segment of each output key.
+__global__ void band_outputs_kernel(const uint64_t *__restrict__ sk, const int64_t *__restrict__ excl, int64_t Sp,
+                                    int64_t S, int band_bits, KeyUnpack un, int32_t *out_keys, int64_t *fstart) {
+    for (int64_t p = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; p < Sp; p += (int64_t)gridDim.x * blockDim.x) {
+        const uint64_t k = sk[p] >> band_bits;
+        if (p == 0 || k != (sk[p - 1] >> band_bits)) {
+            const int64_t f = excl[p];
+            fstart[f] = p;
+            for (int c = 0; c < un.uw; ++c) {
+                uint64_t mask = un.bits[c] ? ((~0ull) >> (64 - un.bits[c])) : 0ull;
+                out_keys[f * un.uw + c] = (int32_t)((k >> un.shift[c]) & mask);
+            }
+        }
+        if (p == 0) fstart[S] = Sp;
+    }
 }
 
 __global__ void segments_kernel(const uint64_t *__restrict__ pk, const uint64_t *__restrict__ pv,
@@ -447,9 +492,30 @@ void launch_unary_pairs(ucl_ctx *ctx, const uint64_t *ko_u, int64_t n, uint64_t 
     ctx->launches++;
 }
 
-void launch_heads(ucl_ctx *ctx, const uint64_t *pk, int64_t P, int64_t *flag) {
+void launch_heads(ucl_ctx *ctx, const uint64_t *pk, int64_t P, int64_t *flag, int shift) {
     if (P <= 0) return;
-    heads_kernel<<<grid_for(ctx, P), kThreads, 0, ctx->stream>>>(pk, P, flag);
+    heads_kernel<<<grid_for(ctx, P), kThreads, 0, ctx->stream>>>(pk, P, shift, flag);
+    ctx->launches++;
+}
+
+void launch_band_ranges(ucl_ctx *ctx, const uint64_t *pk, int64_t P, const int64_t *seg_excl, const int64_t *n_seg,
+                        int out_bits, int B, int64_t *band_start, int64_t *band_seg) {
+    band_ranges_kernel<<<1, 64, 0, ctx->stream>>>(pk, P, seg_excl, n_seg, out_bits, B, band_start, band_seg);
+    ctx->launches++;
+}
+
+void launch_band_keys(ucl_ctx *ctx, const uint64_t *pk, const int64_t *seg_start, int64_t Sp, int out_bits,
+                      int band_bits, uint64_t *sk, uint64_t *sv) {
+    if (Sp <= 0) return;
+    band_keys_kernel<<<grid_for(ctx, Sp), kThreads, 0, ctx->stream>>>(pk, seg_start, Sp, out_bits, band_bits, sk, sv);
+    ctx->launches++;
+}
+
+void launch_band_outputs(ucl_ctx *ctx, const uint64_t *sk, const int64_t *excl, int64_t Sp, int64_t S, int band_bits,
+                         KeyUnpack un, int32_t *out_keys, int64_t *fstart) {
+    if (Sp <= 0) return;
+    band_outputs_kernel<<<grid_for(ctx, Sp), kThreads, 0, ctx->stream>>>(sk, excl, Sp, S, band_bits, un, out_keys,
+                                                                         fstart);
     ctx->launches++;
 }
 

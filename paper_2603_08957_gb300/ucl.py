@@ -124,6 +124,8 @@ class Context:
             "path": {1: "simt", 2: "tc"}.get(st.path, "none"),
             "launches": st.launches,
             "n_units": st.n_units,
+            "n_bands": st.n_bands,
+            "n_band_segments": st.n_band_segments,
             "stage_ms": list(st.stage_ms) if st.timed else None,
         }
 

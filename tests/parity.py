@@ -41,6 +41,29 @@ def oracle_ref(spec, rels, *, epi="none", scale=1.0, sample_keys=None, **ext):
     return oracle.einsum(spec, ins, epi=epi, scale=scale, out_dtype="f64", sample_keys=sample_keys, **ext)
 
 
+def _oracle_task(task):
+    spec, rels, kw = task
+    return oracle.einsum(spec, rels, out_dtype="f64", **kw)
+
+
+def oracle_parallel(tasks):
+    """oracle_ref for several independent (spec, rels, kwargs) tasks at once,
+    one spawned process each (never a fork of a process holding a CUDA
+    context).  Tiles are passed as float32 arrays (bf16 and fp32 inputs are
+    exact in float32); results come back in task order."""
+    import multiprocessing as mpc
+    import os
+    conv = []
+    for spec, rels, kw in tasks:
+        ins = [(np.asarray(k), tuple(int(x) for x in b),
+                t.detach().to("cpu", torch.float32).numpy() if torch.is_tensor(t) else np.asarray(t, np.float32))
+               for k, b, t in rels]
+        conv.append((spec, ins, kw))
+    n = max(1, min(len(conv), os.cpu_count() or 1))
+    with mpc.get_context("spawn").Pool(n) as pool:
+        return pool.map(_oracle_task, conv, chunksize=1)
+
+
 def check_values(g, want, mag, in_dtype, out_bf16, scale=1.0):
     """Element-wise value bar on arrays: g (GPU, float64), want and mag (the
     oracle's value and Sigma|a*b|).  Raises AssertionError on the first

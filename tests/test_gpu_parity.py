@@ -10,7 +10,7 @@ import torch
 import oracle
 import workloads
 from paper_2603_08957_gb300 import Context, UclError
-from tests.parity import TOL, assert_parity, gpu_rel, oracle_ref
+from tests.parity import assert_parity, gpu_rel, oracle_parallel, oracle_ref
 from tests.ucl_testutil import decompose, golden, random_sparse, ucl_operand
 
 pytestmark = pytest.mark.gpu
@@ -181,6 +181,51 @@ def test_gnn_chain_small(ctx, path):
     assert_parity(out, ref2, torch.bfloat16)
 
 
+@pytest.mark.parametrize("bands", [2, 4, 16])
+def test_banded_message_passing(monkeypatch, bands):
+    """Banding of the contracted label (forced): the message passing of a
+    4096-vertex R-MAT graph with 128-wide embeddings, its pairs contracted
+    band after band into fp32 (band, K) partials and summed per K in band
+    order.  Both layers' EinSums against the oracle, every output key."""
+    monkeypatch.setenv("UCL_BANDS", str(bands))
+    c = Context(0)
+    monkeypatch.delenv("UCL_BANDS")
+    w = workloads.gnn_two_layer(seed=4, n=4096, n_edges=20_000, feat=128, device="cuda")
+    X, Y = gpu_rel(c, w["X"]), gpu_rel(c, w["Y"])
+    T1 = c.einsum(w["spec1"], X, Y, out_dtype="bf16")
+    st = c.last_stats()
+    assert st["n_bands"] == bands and st["path"] == "tc"
+    assert st["n_band_segments"] > st["n_segments"]
+    host = {k: (w[k][0], w[k][1], w[k][2].cpu()) for k in ("X", "Y")}
+    assert_parity(T1, oracle_ref(w["spec1"], [host["X"], host["Y"]]), torch.bfloat16)
+    # the second message passing reads T1 keyed by the source block
+    k1, t1 = T1.download()
+    T2 = c.einsum(w["spec3"], T1, Y, out_dtype="f32")
+    assert c.last_stats()["n_bands"] == bands
+    assert_parity(T2, oracle_ref(w["spec3"], [(k1, T1.bounds, t1), host["Y"]]), torch.bfloat16)
+    for r in (X, Y, T1, T2):
+        r.destroy()
+    c.close()
+
+
+def test_l2_hints_do_not_change_results(monkeypatch):
+    """L2 eviction hints on the TMA loads change where lines live, never the
+    arithmetic: results with and without them are bit-identical."""
+    w = workloads.gnn_chain(seed=5, n=30000, degree=16)
+    outs = []
+    for hints in ("1", "0"):
+        monkeypatch.setenv("UCL_L2_HINTS", hints)
+        c = Context(0)
+        X, Y = gpu_rel(c, w["X"]), gpu_rel(c, w["Y"])
+        T = c.einsum(w["spec1"], X, Y, out_dtype="bf16")
+        outs.append(T.download())
+        for r in (X, Y, T):
+            r.destroy()
+        c.close()
+    assert np.array_equal(outs[0][0], outs[1][0])
+    assert torch.equal(outs[0][1], outs[1][1])
+
+
 def test_spgemm_small(ctx):
     """Block-sparse x block-sparse, 128 x 128 bf16 tiles, band + uniform, fp32 out."""
     w = workloads.spgemm(seed=2, n=8192, density=0.05)
@@ -349,12 +394,40 @@ def test_errors(ctx):
     ctx.synchronize()
 
 
+def _band_crossings(ky, jext, bands, G):
+    """Work-unit boundaries inside each output key's pairs for a message
+    passing whose pairs are one per Y tuple (J, K) and are ordered by
+    (band of J, K): per band b, G_b = min(P_b, G) units of equal pair count.
+    Returns the crossing count of every K (summed over bands)."""
+    jb = int(np.ceil(np.log2(jext))) if jext > 1 else 0
+    bits = int(np.log2(bands))
+    band = ky[:, 0].astype(np.int64) >> (jb - bits) if bits else np.zeros(len(ky), np.int64)
+    nk = int(ky[:, 1].max()) + 1
+    cross = np.zeros(nk, np.int64)
+    base = 0
+    for b in range(bands):
+        kb = ky[band == b, 1]
+        Pb = len(kb)
+        if Pb == 0:
+            continue
+        cnt = np.bincount(kb, minlength=nk)
+        pre = base + np.concatenate([[0], np.cumsum(cnt)])[:-1]
+        Gb = min(Pb, G)
+        starts = [base + Pb * u // Gb for u in range(1, Gb)]
+        cross += np.where(cnt > 0, _crossings(pre, pre + cnt, starts), 0)
+        base += Pb
+    return cross
+
+
 def test_two_layer_gnn_full_size_sampled(ctx):
     """Two-layer GNN at scale: R-MAT with 2M vertices / 40M drawn edges as
     64x64 0/1 tiles (~16.6M tiles, ~136 GB), 256-wide embeddings, chained
     T1=(XY)^T, H1=relu(T1 W1), T2=(H1 Y)^T, O=T2 W2.  Every step's key set
-    is checked in full; values stage-locally on sampled output keys (the
-    oracle gets exactly the tiles those keys join with)."""
+    is checked in full; values stage-locally on sampled output keys drawn
+    over the whole size distribution, always including one whose pairs span
+    at least three work units (carried across CTAs by partials and the
+    fixup).  The oracle gets exactly the tiles each sampled key joins with,
+    one spawned process per key."""
     w = workloads.gnn_two_layer(seed=0)
     dev = torch.device("cuda", 0)
     X, Y, W1, W2 = (gpu_rel(ctx, w[k]) for k in ("X", "Y", "W1", "W2"))
@@ -363,15 +436,12 @@ def test_two_layer_gnn_full_size_sampled(ctx):
     src, dst = w["edges"]
     t, n = w["t"], w["n"]
     cnt = np.bincount(ky[:, 1], minlength=want_k.max() + 1)
-    rng = np.random.default_rng(3)
-    small = np.nonzero((cnt > 0) & (cnt <= np.median(cnt[cnt > 0])))[0]
-    sk = np.sort(rng.choice(small, size=3, replace=False)).astype(np.int32)
 
     def y_subset(kset):
         m = torch.isin(dst // t, torch.as_tensor(kset, device=dst.device, dtype=torch.int64))
-        s, d = src[m].cpu().numpy(), dst[m].cpu().numpy()
+        s_, d_ = src[m].cpu().numpy(), dst[m].cpu().numpy()
         yk = ky[np.isin(ky[:, 1], kset)]
-        return yk, workloads.adjacency_tiles_subset(s, d, n, t, yk)
+        return yk, workloads.adjacency_tiles_subset(s_, d_, n, t, yk)
 
     def rows(rel, keys_sel):
         k, tl = rel.device_tensors()
@@ -380,16 +450,31 @@ def test_two_layer_gnn_full_size_sampled(ctx):
         assert np.array_equal(kk[idx], keys_sel)
         return keys_sel[:, None].astype(np.int32), tl[torch.as_tensor(idx, device=tl.device)].cpu()
 
-    yk, yt = y_subset(sk)
     # step 1: T1 = (X Y)^T
     T1 = ctx.einsum(w["spec1"], X, Y, out_dtype="bf16")
+    st = ctx.last_stats()
     kt1, _ = T1.device_tensors()
     assert np.array_equal(kt1.cpu().numpy(), want_k)
-    jneed = np.unique(yk[:, 0])
-    xrel = (jneed[:, None].astype(np.int32), w["X"][1], w["X"][2][torch.as_tensor(jneed, device=dev)].cpu())
-    ref = oracle_ref(w["spec1"], [xrel, (yk, w["Y"][1], yt)], sample_keys=sk[:, None])
-    sel = np.searchsorted(kt1[:, 0].cpu().numpy(), sk)
-    assert_parity(T1, ref, torch.bfloat16, select=sel)
+    cross = _band_crossings(ky, w["X"][1][0], st["n_bands"], st["n_units"])
+    rng = np.random.default_rng(3)
+    present = np.nonzero(cnt > 0)[0]
+    picks = set(rng.choice(present, size=3, replace=False).tolist())
+    big = np.nonzero(cross >= 2)[0]
+    assert len(big) > 0
+    kbig = int(big[np.argmin(cnt[big])])
+    picks.add(kbig)
+    sk = np.array(sorted(picks), dtype=np.int32)
+    subsets = {int(k): y_subset(np.array([k])) for k in sk}
+    tasks = []
+    for k in sk:
+        yk, yt = subsets[int(k)]
+        jneed = np.unique(yk[:, 0])
+        xrel = (jneed[:, None].astype(np.int32), w["X"][1], w["X"][2][torch.as_tensor(jneed, device=dev)].cpu())
+        tasks.append((w["spec1"], [xrel, (yk, w["Y"][1], yt)], {"sample_keys": np.array([[k]], np.int32)}))
+    kt1h = kt1[:, 0].cpu().numpy()
+    for k, ref in zip(sk, oracle_parallel(tasks)):
+        assert_parity(T1, ref, torch.bfloat16, select=np.searchsorted(kt1h, [k]))
+    sel = np.searchsorted(kt1h, sk)
     # step 2: H1 = relu(T1 W1), stage-local
     H1 = ctx.einsum(w["spec2"], T1, W1, out_dtype="bf16", epi="relu")
     t1k, t1t = rows(T1, sk)
@@ -402,13 +487,18 @@ def test_two_layer_gnn_full_size_sampled(ctx):
     want_k2 = np.unique(ky[np.isin(ky[:, 0], want_k[:, 0]), 1]).astype(np.int32)[:, None]
     assert np.array_equal(kt2, want_k2)
     sk2 = sk[np.isin(sk, kt2[:, 0])]
-    assert len(sk2) > 0
-    yk2 = yk[np.isin(yk[:, 1], sk2) & np.isin(yk[:, 0], want_k[:, 0])]
-    yt2 = yt[np.isin(yk[:, 1], sk2) & np.isin(yk[:, 0], want_k[:, 0])]
-    hk, ht = rows(H1, np.unique(yk2[:, 0]))
-    ref = oracle_ref(w["spec3"], [(hk, H1.bounds, ht), (yk2, w["Y"][1], yt2)], sample_keys=sk2[:, None])
+    assert len(sk2) > 0 and kbig in sk2
+    tasks = []
+    for k in sk2:
+        yk, yt = subsets[int(k)]
+        keep = np.isin(yk[:, 0], want_k[:, 0])
+        yk2, yt2 = yk[keep], yt[keep]
+        hk, ht = rows(H1, np.unique(yk2[:, 0]))
+        tasks.append((w["spec3"], [(hk, H1.bounds, ht), (yk2, w["Y"][1], yt2)],
+                      {"sample_keys": np.array([[k]], np.int32)}))
+    for k, ref in zip(sk2, oracle_parallel(tasks)):
+        assert_parity(T2, ref, torch.bfloat16, select=np.searchsorted(kt2[:, 0], [k]))
     sel2 = np.searchsorted(kt2[:, 0], sk2)
-    assert_parity(T2, ref, torch.bfloat16, select=sel2)
     # step 4: O = T2 W2
     O = ctx.einsum(w["spec4"], T2, W2)
     t2k, t2t = rows(T2, sk2)
@@ -442,33 +532,58 @@ def test_mttkrp_small(ctx, path):
     assert_parity(out3, ref, torch.bfloat16)
 
 
+def _crossings(seg_lo, seg_hi, starts):
+    """Unit boundaries strictly inside each pair range [seg_lo, seg_hi)."""
+    starts = np.asarray(starts)
+    return np.searchsorted(starts, seg_hi, side="left") - np.searchsorted(starts, seg_lo, side="right")
+
+
 def test_mttkrp_full_size_sampled(ctx):
     """MTTKRP at full size: a 100000^3 tensor with 1e7 Zipf(1.1) nonzeros in
     16^3 tiles (~3.9M tiles, ~32 GB bf16), rank-64 factors.  The whole output
-    key set is checked, values on sampled output keys (the oracle gets the T
-    tiles of those keys and the factor tiles they join with)."""
+    key set is checked; values on sampled output keys drawn over the whole
+    size distribution, always including a key whose triples span at least
+    three work units (its sum is carried across CTAs by the partial / fixup
+    path).  The oracle gets the T tiles of those keys and the factor tiles
+    they join with, one spawned process per key."""
     w = workloads.mttkrp(seed=0, device="cuda")
     dev = torch.device("cuda", 0)
     rels = [gpu_rel(ctx, w[k]) for k in ("T", "B", "C")]
     out = ctx.einsum(w["spec"], *rels)
+    st = ctx.last_stats()
     kt = w["T"][0]
     got = out.device_tensors()[0].cpu().numpy()
     assert np.array_equal(got, np.unique(kt[:, 0]).astype(np.int32)[:, None])
-    assert ctx.last_stats()["n_pairs"] == len(kt)
+    P, G = st["n_pairs"], st["n_units"]
+    assert P == len(kt)
     cnt = np.bincount(kt[:, 0])
+    # triples are ordered by output key I: key i holds [pre[i], pre[i] + cnt[i])
+    pre = np.concatenate([[0], np.cumsum(cnt)])[:-1]
+    units = np.array([P * u // G for u in range(1, G)])
+    cross = _crossings(pre, pre + cnt, units)
     rng = np.random.default_rng(5)
-    small = np.nonzero((cnt > 0) & (cnt <= np.median(cnt[cnt > 0])))[0]
-    sk = np.sort(rng.choice(small, size=3, replace=False)).astype(np.int32)
-    m = np.nonzero(np.isin(kt[:, 0], sk))[0]
-    tsub = (kt[m], w["T"][1], w["T"][2][torch.as_tensor(m, device=dev)].cpu())
+    present = np.nonzero(cnt > 0)[0]
+    picks = set(rng.choice(present, size=4, replace=False).tolist())
+    # the smallest key spanning at least three units (oracle time ~ its triples)
+    big = np.nonzero(cross >= 2)[0]
+    assert len(big) > 0
+    kbig = int(big[np.argmin(cnt[big])])
+    picks.add(kbig)
+    tasks, order = [], sorted(picks)
 
     def factor_rows(f, rows):
         rows = np.unique(rows)
         return (rows[:, None].astype(np.int32), f[1], f[2][torch.as_tensor(rows, device=dev)].cpu())
 
-    ref = oracle_ref(w["spec"], [tsub, factor_rows(w["B"], kt[m, 1]), factor_rows(w["C"], kt[m, 2])],
-                     sample_keys=sk[:, None])
-    assert_parity(out, ref, torch.bfloat16, select=np.searchsorted(got[:, 0], sk))
+    for key in order:
+        m = np.nonzero(kt[:, 0] == key)[0]
+        tsub = (kt[m], w["T"][1], w["T"][2][torch.as_tensor(m, device=dev)].cpu())
+        tasks.append((w["spec"], [tsub, factor_rows(w["B"], kt[m, 1]), factor_rows(w["C"], kt[m, 2])],
+                      {"sample_keys": np.array([[key]], np.int32)}))
+    refs = oracle_parallel(tasks)
+    for key, ref in zip(order, refs):
+        assert_parity(out, ref, torch.bfloat16, select=np.searchsorted(got[:, 0], [key]))
+    assert cross[kbig] >= 2 and cnt[kbig] >= 2 * P // G
     for r in rels + [out]:
         r.destroy()
     del w
