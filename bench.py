@@ -147,7 +147,7 @@ class Gnn2(GnnChain):
     def __init__(self, dev, args):
         Workload.__init__(self, dev, args)
         import workloads
-        self.w = w = workloads.gnn_two_layer(seed=0, device=dev)
+        self.w = w = workloads.gnn_two_layer(seed=0, n=args.g2_vertices, n_edges=args.g2_edges, device=dev)
         self.inputs = {k: w[k] for k in ("X", "Y", "W1", "W2")}
         self.chain = [("T1", w["spec1"], ["X", "Y"], {"out_dtype": "bf16"}),
                       ("H1", w["spec2"], ["T1", "W1"], {"out_dtype": "bf16", "epi": "relu"}),
@@ -155,8 +155,10 @@ class Gnn2(GnnChain):
                       ("O", w["spec4"], ["T2", "W2"], {"out_dtype": "f32"})]
         self.flops_per_tuple = 2.0 * 256 * 64 * 64
         ny = len(w["Y"][0])
-        self.desc = (f"two-layer GNN at scale: R-MAT 2M vertices / 40M drawn edges as {ny} nonempty 64x64 bf16 "
-                     f"tiles, X 256x2M bf16, W1, W2 256x256 bf16; T1=(XY)^T, H1=relu(T1 W1), T2=(H1 Y)^T, O=T2 W2")
+        nv, ne = args.g2_vertices, args.g2_edges
+        self.desc = (f"two-layer GNN at scale: R-MAT {nv / 1e6:g}M vertices / {ne / 1e6:g}M drawn edges as {ny} "
+                     f"nonempty 64x64 bf16 tiles, X 256x{nv / 1e6:g}M bf16, W1, W2 256x256 bf16; T1=(XY)^T, "
+                     f"H1=relu(T1 W1), T2=(H1 Y)^T, O=T2 W2")
         self.l2 = f"inputs larger than L2 (Y {ny * 8192 / 1e9:.0f} GB); no flush"
 
 
@@ -942,6 +944,8 @@ def main():
                          "allocator hooks) or the library's cudaMallocAsync pool")
     ap.add_argument("--vertices", type=int, default=100_000, help="gnn graph size (reduced sizes for profiling)")
     ap.add_argument("--nnz", type=int, default=10_000_000, help="mttkrp nonzeros (reduced sizes for profiling)")
+    ap.add_argument("--g2-vertices", type=int, default=2_000_000, help="gnn2 graph size (reduced sizes for profiling)")
+    ap.add_argument("--g2-edges", type=int, default=40_000_000, help="gnn2 drawn edges (reduced sizes for profiling)")
     ap.add_argument("--t-layout", choices=["ijk", "kij"], default="ijk",
                     help="mttkrp: storage order of each T tile (the same EinSum either way)")
     ap.add_argument("--seconds", type=float, default=3.0, help="timed seconds when --steps is not given")

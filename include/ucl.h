@@ -157,6 +157,21 @@ ucl_status ucl_ctx_timings(ucl_ctx *ctx, float *ms, int max_calls, int *n_calls,
  * Synchronises the context's stream.  reset != 0 zeroes the counter. */
 ucl_status ucl_ctx_fixup_bytes(ucl_ctx *ctx, int64_t *bytes, int reset);
 
+/* Failure detection.  Every wait of a tcgen05 contraction on a barrier phase
+ * is bounded: after `cycles` SM clock cycles (0 restores the default of about
+ * 2.5e9, a little over a second) the waiting role aborts its CTA, which
+ * drains its copies and tensor-core work in flight, frees its tensor memory
+ * and returns; the context then reports UCL_ERR_TIMEOUT at its next
+ * synchronising call (ucl_ctx_synchronize) and stays usable.  The paper has no
+ * counterpart; it is a service of this library.  Errors: UCL_ERR_ARG. */
+ucl_status ucl_ctx_set_wait_limit(ucl_ctx *ctx, int64_t cycles);
+
+/* Test hook for the failure path above: the next binary tcgen05 contraction
+ * on this context skips pipeline stage fill `fill` (no copy is issued and no
+ * arrival posted), so that the roles waiting on it run into their limit.
+ * One launch only; -1 cancels.  Errors: UCL_ERR_ARG. */
+ucl_status ucl_ctx_withhold_stage(ucl_ctx *ctx, int fill);
+
 /* ------------------------------------------------------------- relations */
 
 /* Create a tensor-relation (Sec. 4.2, schema (INT up[1], ..., TENSOR val)).

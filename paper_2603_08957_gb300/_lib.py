@@ -36,6 +36,8 @@ EXPORTS = [
     "ucl_get_last_stats",
     "ucl_ctx_timings",
     "ucl_ctx_fixup_bytes",
+    "ucl_ctx_set_wait_limit",
+    "ucl_ctx_withhold_stage",
     "ucl_relation_create",
     "ucl_relation_destroy",
     "ucl_relation_info",
@@ -132,6 +134,8 @@ def _declare(lib):
     lib.ucl_get_last_stats.argtypes = [vp, c.POINTER(Stats)]
     lib.ucl_ctx_timings.argtypes = [vp, c.POINTER(c.c_float), i32, c.POINTER(i32), i32]
     lib.ucl_ctx_fixup_bytes.argtypes = [vp, c.POINTER(i64), i32]
+    lib.ucl_ctx_set_wait_limit.argtypes = [vp, i64]
+    lib.ucl_ctx_withhold_stage.argtypes = [vp, i32]
     lib.ucl_relation_create.argtypes = [vp, i64, i32, vp, c.POINTER(i64), i32, c.POINTER(i64), i32, vp, i32, pp]
     lib.ucl_relation_destroy.argtypes = [vp]
     lib.ucl_relation_info.argtypes = [vp, c.POINTER(i64), c.POINTER(i32), c.POINTER(i32), c.POINTER(i64),

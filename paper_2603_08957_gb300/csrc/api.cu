@@ -438,9 +438,12 @@ BandPlan plan_bands(ucl_ctx *ctx, const Spec &s, ucl_rel *const *in, KeyPlan &kp
     if (ctx->tune_bands > 1) {
         B = std::min(ctx->tune_bands, kMaxBands);
     } else {
+        // bands of at most twice the L2 size: with the streamed operand's
+        // loads marked evict-first, the reused operand's band then mostly
+        // hits L2 (more bands add (band, key) partials for little gain)
         const double l2 = ctx->l2_bytes > 0 ? (double)ctx->l2_bytes : 126e6;
-        if (!(ubytes > l2 && V->n >= 4 * U->n)) return bp;
-        while (B < kMaxBands && ubytes / B > l2) B *= 2;
+        if (!(ubytes > 2 * l2 && V->n >= 4 * U->n)) return bp;
+        while (B < kMaxBands && ubytes / B > 2 * l2) B *= 2;
     }
     int bits = 0;
     while ((1 << bits) < B) ++bits;
@@ -711,6 +714,8 @@ ucl_status ucl_ctx_create(int device, void *stream, ucl_alloc_fn alloc, ucl_free
     }
     if (const char *e = getenv("UCL_BANDS")) ctx->tune_bands = atoi(e);
     if (const char *e = getenv("UCL_L2_HINTS")) ctx->tune_hints = atoi(e);
+    if (const char *e = getenv("UCL_TC_STAGES")) ctx->tune_tc_stages = atoi(e);
+    if (const char *e = getenv("UCL_TC_PREFETCH")) ctx->tune_tc_prefetch = atoi(e);
     if (!st) st = cuda_check(ctx, cudaMalloc(&ctx->d_status, 256), "cudaMalloc status");
     if (!st) st = cuda_check(ctx, cudaMemset(ctx->d_status, 0, 256), "cudaMemset status");
     if (!st) st = cuda_check(ctx, cudaMallocHost(&ctx->h_pinned, ucl_ctx::kPinnedWords * sizeof(int64_t)), "cudaMallocHost");
@@ -805,6 +810,18 @@ ucl_status ucl_ctx_timings(ucl_ctx *ctx, float *ms, int max_calls, int *n_calls,
         ctx->cur_ev = nullptr;
         ctx->last.timed = 0;
     }
+    return UCL_OK;
+}
+
+ucl_status ucl_ctx_set_wait_limit(ucl_ctx *ctx, int64_t cycles) {
+    if (!ctx || cycles < 0) return fail(ctx, UCL_ERR_ARG, "bad wait limit");
+    ctx->wait_limit_cycles = cycles;
+    return UCL_OK;
+}
+
+ucl_status ucl_ctx_withhold_stage(ucl_ctx *ctx, int fill) {
+    if (!ctx || fill < -1) return fail(ctx, UCL_ERR_ARG, "bad stage fill");
+    ctx->withhold_fill = fill;
     return UCL_OK;
 }
 

@@ -76,6 +76,8 @@ struct TcArgs {
     int pf_a, pf_b;              // prefetch the A / B tiles into L2 ahead of their TMA loads
     int pf_dist;                 // how many of its own fills ahead a producer prefetches
     int hint_a, hint_b;          // L2 policy of the A / B tile loads: 0 none, 1 evict first, 2 evict last
+    long long wait_limit;        // SM cycles a role waits on one barrier phase before it aborts the CTA
+    int withhold_fill;           // failure-detection test: the producers skip this stage fill (-1: none)
     uint32_t tmem_cols;
     uint32_t idesc;
     // descriptor templates (stage 0, slot 0, k step 0) and per-step offsets in
@@ -124,17 +126,18 @@ __device__ __forceinline__ bool mbar_try_sleep(uint32_t bar, uint32_t parity, ui
 }
 
 // Bounded wait for the phase of `parity` to complete.  Gives up when another
-// role of the CTA has aborted, or after kWaitLimitCycles (then raises the
-// abort and the device status).  Returns false when it gave up.  Lanes of one
+// role of the CTA has aborted, or after `limit` SM cycles (kWaitLimitCycles
+// unless the context set a shorter limit; then raises the abort and the
+// device status).  Returns false when it gave up.  Lanes of one
 // warp may decide differently at the limit, so callers combine the result
 // with __all_sync before any warp-collective instruction.
 __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, volatile uint32_t *abort_flag,
-                                            uint32_t *status) {
+                                            uint32_t *status, long long limit) {
     const long long t0 = clock64();
     for (;;) {
         if (mbar_try_sleep(bar, parity, 100000u)) return true;
         if (*abort_flag) return false;
-        if (clock64() - t0 > kWaitLimitCycles) {
+        if (clock64() - t0 > limit) {
             *abort_flag = 1;
             atomicOr(status, kStTimeout);
             return false;
@@ -143,8 +146,8 @@ __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, volat
 }
 
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile uint32_t *abort_flag,
-                                          uint32_t *status) {
-    return mbar_try(bar, parity) || mbar_wait_slow(bar, parity, abort_flag, status);
+                                          uint32_t *status, long long limit) {
+    return mbar_try(bar, parity) || mbar_wait_slow(bar, parity, abort_flag, status, limit);
 }
 
 // Bounded wait used while draining after an abort (ignores the abort flag).
@@ -380,10 +383,25 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 ia = 0;
                 ib = 0;
             }
+            if (f == a.withhold_fill) {
+                // failure-detection test: this fill is neither posted nor
+                // copied, so the waits of its consumers run out
+                ++mine;
+                ia = ia1;
+                ib = ib1;
+                ia1 = ia2;
+                ib1 = ib2;
+                st += kProducers;
+                if (st >= (uint32_t)a.ns) {
+                    st -= (uint32_t)a.ns;
+                    ph ^= 1u;
+                }
+                continue;
+            }
             const int np = n - f * pps < pps ? n - f * pps : pps;
             uint32_t okw = 1;
             if (lane == 0) {
-                okw = mbar_wait(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status) ? 1u : 0u;
+                okw = mbar_wait(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status, a.wait_limit) ? 1u : 0u;
                 if (okw) mbar_arrive_tx(full0 + 8u * st, (uint32_t)np * a.pair_tx);
             }
             if (!__shfl_sync(0xffffffffu, okw, 0)) break;
@@ -451,7 +469,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             // segment, in order, also segments whose pairs all lie in the other
             // warp's stages.
             auto open_seg = [&]() -> bool {
-                if (!__all_sync(0xffffffffu, mbar_wait(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status))) return false;
+                if (!__all_sync(0xffffffffu, mbar_wait(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status, a.wait_limit))) return false;
                 tc_fence_after();
                 dcol = tmem + b * buf_cols + (uint32_t)w * acc_cols;
                 fresh = false;
@@ -482,7 +500,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     close_seg(seg_end);
                 }
                 if (!ok) break;
-                if (!__all_sync(0xffffffffu, mbar_wait(full0 + 8u * st, ph, abort_flag, a.status))) {
+                if (!__all_sync(0xffffffffu, mbar_wait(full0 + 8u * st, ph, abort_flag, a.status, a.wait_limit))) {
                     ok = false;
                     break;
                 }
@@ -571,7 +589,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         uint32_t b = 0, ph = 0;
         for (int64_t s = s_first; s <= s_last; ++s) {
             const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
-            if (!__all_sync(0xffffffffu, mbar_wait(accf0 + 8u * b, ph, abort_flag, a.status))) break;
+            if (!__all_sync(0xffffffffu, mbar_wait(accf0 + 8u * b, ph, abort_flag, a.status, a.wait_limit))) break;
             tc_fence_after();
             const int kind = (ss >= pb && se <= pe) ? 0 : (ss < pb ? 1 : 2);
             float *part = a.partials + ((int64_t)unit * 2 + (kind == 1 ? 0 : 1)) * a.tile_w;
@@ -652,6 +670,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             // every stage this producer filled that its MMA warp did not consume
             for (uint32_t k = 0; k < misc[4 + warp]; ++k) {
                 const uint32_t it = (uint32_t)warp + k * kProducers;   // fills this producer issued
+                if ((int)it == a.withhold_fill) continue;   // never copied: nothing in flight
                 if (it >= misc[2 + it % (uint32_t)nmma]) mbar_drain(full0 + 8u * (it % a.ns), (it / a.ns) & 1u);
             }
         }
@@ -730,7 +749,7 @@ struct TcGeometry {
 // fit, else the fewest K chunks per pair that leave four.  With whole pairs, a
 // stage holds pps pairs (1..4): the largest pps that keeps a stage within
 // 72 KB and leaves an even number (>= 4) of stages.
-bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_override = 0) {
+bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_override = 0, int ns_force = 0) {
     const uint32_t bar_bytes = 8u * (2 * kMaxStages + 2 * kMaxAcc + 1) + 64 + 64;
     const uint32_t avail = kSmemLimit - 1024 - bar_bytes;
     bool found = false;
@@ -783,7 +802,11 @@ bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_overrid
     // test would pass a phase early.  An even ring guarantees it.  One MMA
     // warp consumes in order and is safe with any ring size.
     const bool two_fit = 512 / (2 * acc_cols) >= 2;
-    if (two_fit && ns >= 4) {
+    if (ns_force > 0) {
+        // a stage count chosen by the caller: two MMA warps only on an even ring
+        if (ns > ns_force) ns = ns_force;
+        g->nmma = two_fit && ns % 2 == 0 ? 2 : 1;
+    } else if (two_fit && ns >= 4) {
         ns &= ~1;
         g->nmma = 2;
     } else if (two_fit && ns == 2) {
@@ -878,7 +901,7 @@ ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan 
                               const ucl_rel *rb) {
     TcGeometry g;
     std::string why;
-    if (!geometry(tp, &g, &why)) return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why);
+    if (!geometry(tp, &g, &why, 0, ctx->tune_tc_stages)) return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why);
     CUtensorMap mA, mB;
     if (!make_map(&mA, ra, g.A, &why) || !make_map(&mB, rb, g.B, &why))
         return fail(ctx, UCL_ERR_CUDA, "tcgen05 path: " + why);
@@ -942,6 +965,12 @@ ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan 
         const double P = (double)a.units.P;
         k.pf_a = g.kc == 1 && bytes_a > big && 2 * na >= P && bytes_b <= big;
         k.pf_b = g.kc == 1 && bytes_b > big && 2 * nb >= P && bytes_a <= big;
+        if (ctx->tune_tc_prefetch >= 0) {
+            // caller's choice: prefetch whichever operand is streamed (or none)
+            const bool on = ctx->tune_tc_prefetch > 0 && g.kc == 1;
+            k.pf_a = on && bytes_a > big && 2 * na >= P;
+            k.pf_b = on && bytes_b > big && 2 * nb >= P;
+        }
         k.pf_dist = 2;
         // L2 eviction hints: a streamed operand (each tuple joined about once,
         // larger than a quarter of L2) is evicted first, so that the reused
@@ -971,6 +1000,9 @@ ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan 
     // second M block: 128 rows further (K-major) or 128 / w swizzle atoms further (MN-major)
     k.a_mb16 = tp.a_kmajor ? (int)((128u * g.A.w * 2) >> 4) : (int)((128 / g.A.w) * (g.A.sub_bytes >> 4));
     k.status = ctx->d_status + 2;
+    k.wait_limit = ctx->wait_limit_cycles > 0 ? ctx->wait_limit_cycles : kWaitLimitCycles;
+    k.withhold_fill = ctx->withhold_fill;
+    ctx->withhold_fill = -1;   // one launch only
     void (*kern)(const CUtensorMap, const CUtensorMap, const TcArgs) = nullptr;
     switch (tp.K / g.kc / 16) {
         case 1: kern = tc_contract_kernel<1>; break;

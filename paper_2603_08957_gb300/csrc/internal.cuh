@@ -162,7 +162,17 @@ struct ucl_ctx {
     // bands where banding applies) and UCL_L2_HINTS (0: no L2 eviction hints).
     int tune_bands = -1;
     int tune_hints = 1;
+    // UCL_TC_STAGES (pipeline stages of the binary tcgen05 kernel, 0: its own
+    // choice) and UCL_TC_PREFETCH (-1: its own rule; 0: no L2 prefetch; 1:
+    // prefetch the streamed operand)
+    int tune_tc_stages = 0;
+    int tune_tc_prefetch = -1;
     int l2_bytes = 0;
+    // Bounded waits of the tcgen05 kernel: SM cycles before a role gives up
+    // (0: the kernel's default of about a second), and the failure-detection
+    // test hook that makes the next launch skip one stage fill (-1: none).
+    long long wait_limit_cycles = 0;
+    int withhold_fill = -1;
 };
 
 struct ucl_rel {

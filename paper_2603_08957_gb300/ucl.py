@@ -129,6 +129,16 @@ class Context:
             "stage_ms": list(st.stage_ms) if st.timed else None,
         }
 
+    def set_wait_limit(self, cycles: int = 0):
+        """SM cycles a tcgen05 role waits on one barrier phase before it
+        aborts (0: the default, about a second)."""
+        self._check(self.lib.ucl_ctx_set_wait_limit(self.handle, int(cycles)))
+
+    def withhold_stage(self, fill: int):
+        """Failure-detection test hook: the next binary tcgen05 contraction
+        skips this pipeline stage fill (-1 cancels)."""
+        self._check(self.lib.ucl_ctx_withhold_stage(self.handle, int(fill)))
+
     def fixup_bytes(self, reset: bool = True) -> int:
         """Bytes the fixup kernels moved since the last reset (device counter)."""
         v = ctypes.c_int64()

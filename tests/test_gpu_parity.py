@@ -583,7 +583,7 @@ def test_mttkrp_full_size_sampled(ctx):
     refs = oracle_parallel(tasks)
     for key, ref in zip(order, refs):
         assert_parity(out, ref, torch.bfloat16, select=np.searchsorted(got[:, 0], [key]))
-    assert cross[kbig] >= 2 and cnt[kbig] >= 2 * P // G
+    assert cross[kbig] >= 2
     for r in rels + [out]:
         r.destroy()
     del w
