@@ -455,6 +455,34 @@ BandPlan plan_bands(ucl_ctx *ctx, const Spec &s, ucl_rel *const *in, KeyPlan &kp
     return bp;
 }
 
+// Windows of output keys for the windowed tcgen05 kernel: the pairs of 2^wb
+// consecutive output keys accumulate in one TMEM buffer of 2^wb slots, so
+// that the pairs of one A tuple within a window load its tile once.  It pays
+// when A's tuples are each joined many times and A's tile is at least B's;
+// windows of as many keys as two buffers hold.  Returns wb (0: none) and the
+// kernel's run cap.
+int plan_windows(ucl_ctx *ctx, const Spec &s, ucl_rel *const *in, const KeyPlan &kp, const TcPlan &tp, bool tc_ok,
+                 int *cap) {
+    *cap = 0;
+    if (s.n_in != 2 || !tc_ok || ctx->tune_window == 0) return 0;
+    const ucl_rel *RA = tp.a_is_u ? in[0] : in[1], *RB = tp.a_is_u ? in[1] : in[0];
+    if ((reinterpret_cast<uintptr_t>(RA->tiles) | reinterpret_cast<uintptr_t>(RB->tiles)) & 15) return 0;
+    int wb = 0;
+    if (ctx->tune_window > 0) {
+        wb = ctx->tune_window;
+    } else {
+        // not chosen automatically: measured slower than the plain kernel
+        // on the message-passing shapes (see the design notes)
+        (void)RB;
+        return 0;
+    }
+    if (wb < 1 || wb > 5 || wb > kp.out_bits) return 0;
+    const int c = tc_window_cap(tp, wb);
+    if (c < 1) return 0;
+    *cap = c;
+    return wb;
+}
+
 // Take the next workspace arena in turn.  The stream in use first waits until
 // main has finished the call that used it last; a grown arena is merged into
 // one block.
@@ -716,6 +744,7 @@ ucl_status ucl_ctx_create(int device, void *stream, ucl_alloc_fn alloc, ucl_free
     if (const char *e = getenv("UCL_L2_HINTS")) ctx->tune_hints = atoi(e);
     if (const char *e = getenv("UCL_TC_STAGES")) ctx->tune_tc_stages = atoi(e);
     if (const char *e = getenv("UCL_TC_PREFETCH")) ctx->tune_tc_prefetch = atoi(e);
+    if (const char *e = getenv("UCL_WINDOW")) ctx->tune_window = atoi(e);
     if (!st) st = cuda_check(ctx, cudaMalloc(&ctx->d_status, 256), "cudaMalloc status");
     if (!st) st = cuda_check(ctx, cudaMemset(ctx->d_status, 0, 256), "cudaMemset status");
     if (!st) st = cuda_check(ctx, cudaMallocHost(&ctx->h_pinned, ucl_ctx::kPinnedWords * sizeof(int64_t)), "cudaMallocHost");
@@ -1026,6 +1055,8 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
     const bool tc_ok = !extended && (n_in == 3 ? plan_tc3(s, in, kp, tp3, &why) : plan_tc(s, in, tp, &why));
     if (o.path == UCL_PATH_TC && !tc_ok) return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why);
     const BandPlan bp = plan_bands(ctx, s, in, kp, tc_ok && o.path != UCL_PATH_SIMT);
+    int win_cap = 0;
+    const int wb = n_in == 2 ? plan_windows(ctx, s, in, kp, tp, tc_ok && o.path != UCL_PATH_SIMT, &win_cap) : 0;
     const bool banded = bp.B > 1;
     const int sort_bits = kp.out_bits + bp.bits;
     cudaSetDevice(ctx->device);
@@ -1140,6 +1171,7 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
         // ---------------------------------------------------------- stage 1
         int64_t S = 0;
         int64_t band_start[kMaxBands + 1] = {}, band_seg[kMaxBands + 1] = {};
+        int64_t *flag = nullptr;
         uint64_t *pk = nullptr, *pv = nullptr;
         int64_t *seg_excl = nullptr;
         if (P > 0) {
@@ -1157,14 +1189,18 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             // and alone supplies the output key, as its leading key columns,
             // the pairs are already in output-key order: the stable sort
             // would leave them as they are, so it is skipped.
+            // (pairs in output-key order are also in window order; sharing
+            // of A tiles only needs equal A tuples to be adjacent to pay)
             bool presorted = A->sorted && permA == nullptr && !banded;
             for (int k = 1; k < n_in && presorted; ++k) presorted = kp.out_k[kp.ord[k]].nf == 0;
             for (int q = 0; q < kp.out_k[kp.ord[0]].nf && presorted; ++q)
                 presorted = kp.out_k[kp.ord[0]].f[q].col == q;
-            if (!presorted && radix_sort(ctx, pk, pv, pk2, pv2, P, sort_bits)) { pk = pk2; pv = pv2; }
-            int64_t *flag = (int64_t *)ws_get(ctx, 8 * P);
+            // windows: sort by (band, output key >> wb) only, keeping the
+            // expansion order (A tuple order) inside a window
+            if (!presorted && radix_sort(ctx, pk, pv, pk2, pv2, P, sort_bits - wb, wb)) { pk = pk2; pv = pv2; }
+            flag = (int64_t *)ws_get(ctx, 8 * P);
             seg_excl = (int64_t *)ws_get(ctx, 8 * P);
-            launch_heads(ctx, pk, P, flag);
+            launch_heads(ctx, pk, P, flag, wb);
             scan_i64(ctx, flag, seg_excl, P, d_scal + 1);
             if (banded)
                 launch_band_ranges(ctx, pk, P, seg_excl, d_scal + 1, kp.out_bits, bp.B, d_scal + 2, d_scal + 3 + bp.B);
@@ -1194,18 +1230,50 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
                 uint32_t *const idx[3] = {pu, pvi, pxi};
                 launch_segments3(ctx, pk, pv, pv1, seg_excl, P, S, kp.unpack, kp.ord, okeys, seg_start, idx);
             } else {
-                launch_segments(ctx, pk, pv, seg_excl, P, S, kp.unpack, okeys, seg_start, pu, pvi);
+                launch_segments(ctx, pk, pv, seg_excl, P, S, kp.unpack, okeys, seg_start, pu, pvi, wb);
             }
         }
         // banded: the S (band, output key) segments hold fp32 partials; sort
         // them by (output key, band) and find the output keys
-        const int64_t Sp = S;
+        // windows: per pair its slot and A-tile run, per window segment its
+        // present slots and first row; rows are the (band and) output keys
+        // present, in key order
+        const int64_t Sseg = S;   // pair segments (windows when wb > 0)
+        uint8_t *wslot = nullptr, *warun = nullptr;
+        uint32_t *wmask = nullptr;
+        int64_t *wbase = nullptr;
+        uint64_t *rowkey = nullptr;
+        int64_t rows = S;
+        if (wb > 0 && P > 0) {
+            wslot = (uint8_t *)ws_get(ctx, (size_t)P);
+            warun = (uint8_t *)ws_get(ctx, (size_t)P);
+            wmask = (uint32_t *)ws_get(ctx, 4 * (size_t)Sseg);
+            int64_t *wcnt = (int64_t *)ws_get(ctx, 8 * (size_t)Sseg);
+            wbase = (int64_t *)ws_get(ctx, 8 * (size_t)Sseg);
+            check(cuda_check(ctx, cudaMemsetAsync(wmask, 0, 4 * (size_t)Sseg, ctx->stream), "memset"));
+            launch_win_slots(ctx, pk, P, wb, flag, seg_excl, wslot, wmask);
+            launch_win_count(ctx, wmask, Sseg, wcnt);
+            scan_i64(ctx, wcnt, wbase, Sseg, d_scal + 38);
+            launch_arun(ctx, tp.a_is_u ? pu : pvi, P, win_cap, warun);
+            check(sync_read(ctx, d_scal + 38, 1, &rows));
+            rowkey = (uint64_t *)ws_get(ctx, 8 * (size_t)rows);
+            launch_win_rows(ctx, pk, seg_start, Sseg, wmask, wbase, wb, rowkey);
+            if (!banded) {
+                S = rows;
+                okeys = (int32_t *)ws_get(ctx, 4 * (size_t)S * kp.uw);
+                launch_unpack_keys(ctx, rowkey, S, kp.unpack, okeys);
+            }
+        }
+        const int64_t Sp = rows;   // rows the contraction writes (band partials when banded)
         uint64_t *band_order = nullptr;
         int64_t *fstart = nullptr;
         if (banded && P > 0) {
             uint64_t *sk = (uint64_t *)ws_get(ctx, 8 * Sp), *sv = (uint64_t *)ws_get(ctx, 8 * Sp),
                      *sk2 = (uint64_t *)ws_get(ctx, 8 * Sp), *sv2 = (uint64_t *)ws_get(ctx, 8 * Sp);
-            launch_band_keys(ctx, pk, seg_start, Sp, kp.out_bits, bp.bits, sk, sv);
+            if (wb > 0)
+                launch_band_keys(ctx, rowkey, nullptr, Sp, kp.out_bits, bp.bits, sk, sv);
+            else
+                launch_band_keys(ctx, pk, seg_start, Sp, kp.out_bits, bp.bits, sk, sv);
             if (radix_sort(ctx, sk, sv, sk2, sv2, Sp, sort_bits)) {
                 sk = sk2;
                 sv = sv2;
@@ -1268,7 +1336,7 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             a.pv = pvi;
             a.px = pxi;
             a.seg_start = seg_start;
-            a.S = S;
+            a.S = Sseg;
             a.out = R->tiles;
             a.dout = o.out_dtype;
             a.epi = o.epi;
@@ -1286,6 +1354,7 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
                     use_tc = false;
                 }
             }
+            if (wb > 0 && !use_tc) check(fail(ctx, UCL_ERR_UNSUPPORTED, "windowed pair list without the tcgen05 path"));
             int G = use_tc ? (n_in == 3 ? tc3_units(ctx, P) : tc_units(ctx, tp, P))
                            : (int)std::min<int64_t>(P, (int64_t)ctx->sm_count * 4);
             a.units.P = P;
@@ -1294,7 +1363,13 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             a.bands = bp.B;
             a.l2_hints = ctx->tune_hints;
             stats.n_units = G;
-            a.partials = (float *)ws_get(ctx, sizeof(float) * 2 * (size_t)G * lp.tile_w);
+            a.win_bits = wb;
+            a.slot = wslot;
+            a.arun = warun;
+            a.wmask = wmask;
+            a.wbase = wbase;
+            a.share_cap = win_cap;
+            a.partials = (float *)ws_get(ctx, sizeof(float) * 2 * (size_t)G * ((size_t)1 << wb) * lp.tile_w);
             auto contract = [&](const ContractArgs &c) {
                 if (use_tc && n_in == 3) {
                     check(launch_contract_tc3(ctx, c, tp3, in));
@@ -1310,7 +1385,7 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             if (!banded) {
                 contract(a);
                 record(ctx, 4);
-                launch_fixup(ctx, a);
+                if (wb > 0) launch_fixup_window(ctx, a); else launch_fixup(ctx, a);
                 record(ctx, 5);
             } else {
                 // band after band into fp32 partials keyed (band, output
@@ -1327,12 +1402,16 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
                     c.units.P = Pb;
                     c.units.G = use_tc ? tc_units(ctx, tp, Pb) : (int)std::min<int64_t>(Pb, (int64_t)ctx->sm_count * 4);
                     c.units.base = band_start[b];
-                    c.out = part + (size_t)band_seg[b] * lp.tile_w;
+                    c.out = wb > 0 ? part : part + (size_t)band_seg[b] * lp.tile_w;
+                    if (wb > 0) {
+                        c.wmask = wmask + band_seg[b];
+                        c.wbase = wbase + band_seg[b];
+                    }
                     c.dout = UCL_F32;
                     c.epi = UCL_EPI_NONE;
                     c.scale = 1.0f;
                     contract(c);
-                    launch_fixup(ctx, c);
+                    if (wb > 0) launch_fixup_window(ctx, c); else launch_fixup(ctx, c);
                 }
                 record(ctx, 4);
                 launch_band_sum(ctx, part, band_order, fstart, S, lp.tile_w, R->tiles, o.out_dtype, o.epi, o.scale,

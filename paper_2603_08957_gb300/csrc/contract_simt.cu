@@ -472,6 +472,39 @@ __global__ void __launch_bounds__(kSimtThreads) fixup_kernel(ContractArgs a) {
     }
 }
 
+// Windowed fixup (the windowed tcgen05 kernel's partials): boundary c owns
+// the window segment that crosses it if that segment starts inside unit
+// c - 1; for each present slot it sums the slot's partials in unit order and
+// writes the slot's output row.  Partials: [unit][2][2^win_bits][tile_w].
+__global__ void __launch_bounds__(kSimtThreads) fixup_window_kernel(ContractArgs a) {
+    const int c = blockIdx.x + 1;
+    const int64_t p = a.units.begin(c);
+    if (p >= a.units.base + a.units.P) return;
+    const int64_t s = find_seg(a.seg_start, a.S, p);
+    const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
+    if (ss >= p || ss < a.units.begin(c - 1)) return;
+    int u_end = c;
+    while (u_end < a.units.G && a.units.begin(u_end) < se) ++u_end;
+    const int W = 1 << a.win_bits;
+    const uint32_t mask = a.wmask[s];
+    const int64_t base = a.wbase[s];
+    if (a.fixup_bytes && threadIdx.x == 0) {
+        const int osz = a.dout == UCL_BF16 ? 2 : 4;
+        atomicAdd(a.fixup_bytes,
+                  (unsigned long long)(__popc(mask) * a.tile_w * (4 * (u_end - c + 1) + osz)));
+    }
+    for (int q = 0; q < W; ++q) {
+        if (!((mask >> q) & 1u)) continue;
+        const int64_t row = base + __popc(mask & ((1u << q) - 1u));
+        const float *__restrict__ first = a.partials + (((int64_t)(c - 1) * 2 + 1) * W + q) * a.tile_w;
+        for (int64_t w = threadIdx.x; w < a.tile_w; w += blockDim.x) {
+            float acc = __ldg(first + w);
+            for (int u = c; u < u_end; ++u) acc += __ldg(a.partials + (((int64_t)u * 2) * W + q) * a.tile_w + w);
+            store_out(a.out, a.dout, row * a.tile_w + w, epilogue(acc, a.epi, a.scale));
+        }
+    }
+}
+
 // Band sum: output key f is the sum, in band order, of its band partials
 // part[order[r]] for r in [fstart[f], fstart[f + 1]) (fp32 tiles), then the
 // epilogue and the output cast.  One CTA per output tile at a time; two
@@ -567,6 +600,12 @@ void launch_contract_simt(ucl_ctx *ctx, const ContractArgs &a, const LowerPlan &
     else
         UCL_SIMT(__nv_bfloat16, float);
 #undef UCL_SIMT
+    ctx->launches++;
+}
+
+void launch_fixup_window(ucl_ctx *ctx, const ContractArgs &a) {
+    if (a.units.G <= 1) return;
+    fixup_window_kernel<<<a.units.G - 1, kSimtThreads, 0, ctx->stream>>>(a);
     ctx->launches++;
 }
 

@@ -33,6 +33,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <cstdlib>
 #include <mutex>
 
 #include "internal.cuh"
@@ -48,6 +49,9 @@ constexpr long long kWaitLimitCycles = 2500000000ll;   // ~1.2 s at 2.07 GHz
 constexpr int kMaxStages = 8;
 constexpr int kMaxAcc = 4;
 constexpr uint32_t kSmemLimit = 227 * 1024;
+// barriers, then 16 misc words, then (windowed kernel) 4 pair words and a
+// release word per stage, with room to spare
+constexpr uint32_t kBarBytes = 8u * (2 * kMaxStages + 2 * kMaxAcc + 1) + 64 + 64 + 256;
 
 struct TcArgs {
     const uint32_t *pa;   // [P] A tuple of each pair
@@ -78,6 +82,16 @@ struct TcArgs {
     int hint_a, hint_b;          // L2 policy of the A / B tile loads: 0 none, 1 evict first, 2 evict last
     long long wait_limit;        // SM cycles a role waits on one barrier phase before it aborts the CTA
     int withhold_fill;           // failure-detection test: the producers skip this stage fill (-1: none)
+    // windows (tc_window_kernel): the pairs of 2^wb consecutive output keys
+    // accumulate into one buffer of 2^wb slots; consecutive pairs with the
+    // same A tuple load its tile once
+    int win_bits;
+    const uint8_t *slot;         // [P] slot of each pair in its window
+    const uint8_t *arun;         // [P] low nibble: pairs back to the one that loads this pair's A tile;
+                                 //     high nibble (for that loader): pairs after it sharing the tile
+    const uint32_t *wmask;       // [S] slots present in each window segment
+    const int64_t *wbase;        // [S] output row of each window segment's first present slot
+    int share_cap;               // a loaded A tile serves at most this many consecutive pairs
     uint32_t tmem_cols;
     uint32_t idesc;
     // descriptor templates (stage 0, slot 0, k step 0) and per-step offsets in
@@ -688,6 +702,394 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
 }
 
+// Windowed variant.  The pair list is ordered by (output key >> wb, A tuple
+// order), so the pairs of a window of 2^wb consecutive output keys are
+// contiguous and those of one A tuple within it consecutive.  A window's
+// accumulator buffer holds 2^wb slots (slot q at columns q * acc_cols); a
+// pair accumulates into its own key's slot.  A run of consecutive pairs with
+// the same A tuple loads the A tile once (into the stage of its first pair,
+// the loader) and its other pairs read it from there; that stage is released
+// only after the run's last pair.  Runs are cut every share_cap pairs (in
+// pair-list position) and at unit starts, so that no stage is held longer
+// than the ring allows.  One MMA warp; segments are window segments; the
+// epilogue writes each present slot to its output row (wbase + rank of the
+// slot in the window's mask), or all slots to the unit's partials.
+template <int KSTEPS>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    tc_window_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                     const TcArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    const uint32_t sbase = smem_u32(smem);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)a.ns * a.stage_bytes);
+    const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8u * a.ns, accf0 = empty0 + 8u * a.ns,
+                   acce0 = accf0 + 8u * a.nacc, done_bar = acce0 + 8u * a.nacc;
+    uint32_t *misc = reinterpret_cast<uint32_t *>(bars + 2 * a.ns + 2 * a.nacc + 1);
+    // misc[0] TMEM base, [1] abort flag, [2] stage fills the MMA warp has
+    // walked past, [4 + w] stages filled by producer w; then per stage four
+    // pair words (slot | A source stage << 8 | A source pair << 16) and the
+    // fill after which the stage is released
+    volatile uint32_t *abort_flag = misc + 1;
+    volatile uint32_t *pinfo = misc + 16;
+    volatile int32_t *prel = reinterpret_cast<volatile int32_t *>(misc + 16 + 4 * kMaxStages);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int W = 1 << a.win_bits;
+    const uint32_t acc_cols = (uint32_t)(a.N * a.m_blocks), buf_cols = acc_cols * (uint32_t)W;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < a.ns; ++i) {
+            mbar_init(full0 + 8u * i, 1);
+            mbar_init(empty0 + 8u * i, 1);
+        }
+        for (int i = 0; i < a.nacc; ++i) {
+            mbar_init(accf0 + 8u * i, 1);
+            mbar_init(acce0 + 8u * i, 4);
+        }
+        mbar_init(done_bar, 1);
+        for (int i = 1; i < 16; ++i) misc[i] = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == kProducers) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(misc)),
+                     "r"(a.tmem_cols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = misc[0];
+    if (warp >= kProducers + kMmaWarps) {
+        const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+        for (uint32_t c = 0; c < a.tmem_cols; c += 16) tmem_st16_zero(tmem + lane_base + c);
+        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+
+    const int unit = blockIdx.x;
+    const int64_t pb = a.units.begin(unit), pe = a.units.begin(unit + 1);
+    const int64_t s_first = pe > pb ? find_seg(a.seg_start, a.S, pb) : 0;
+    const int64_t s_last = pe > pb ? find_seg(a.seg_start, a.S, pe - 1) : -1;
+    const uint32_t a_tx = a.pair_tx - (uint32_t)(a.N * a.K * 2), b_tx = (uint32_t)(a.N * a.K * 2);
+
+    if (warp < kProducers) {
+        // ------------------------------------------------------ producers
+        // Producer w fills stages w, w + 2, ...; lane j takes pair j of the
+        // fill.  Each pair's A source comes from arun: its loader is the pair
+        // arun's low nibble back, or the unit's first pair if that is later.
+        const int n = (int)(pe - pb), pps = a.pps;
+        const int nfills = (n + pps - 1) / pps;
+        const uint64_t pol_a = a.hint_a ? policy_of(a.hint_a) : 0ull, pol_b = a.hint_b ? policy_of(a.hint_b) : 0ull;
+        uint32_t mine = 0;
+        uint32_t st = (uint32_t)(warp % a.ns), ph = (uint32_t)((warp / a.ns) & 1);
+        // per-pair words loaded two own fills ahead (as in the plain kernel),
+        // so that a fill never waits on the latency of its own index loads
+        struct PairWords {
+            uint32_t ia, ib, q, r;
+        };
+        auto load_words = [&](int f2) {
+            PairWords w{0u, 0u, 0u, 0u};
+            const int v = f2 * pps + lane;
+            if (f2 < nfills && lane < pps && v < n) {
+                const int64_t p = pb + v;
+                w.ia = a.pa[p];
+                w.ib = a.pb[p];
+                w.q = a.slot[p];
+                w.r = a.arun[p];
+            }
+            return w;
+        };
+        PairWords w0 = load_words(warp), w1 = load_words(warp + kProducers);
+        for (int f = warp; f < nfills; f += kProducers) {
+            const PairWords w2 = load_words(f + 2 * kProducers);
+            const PairWords cur = w0;
+            w0 = w1;
+            w1 = w2;
+            if (f == a.withhold_fill) {
+                // failure-detection test: this fill is neither posted nor copied
+                ++mine;
+                st += kProducers;
+                if (st >= (uint32_t)a.ns) {
+                    st -= (uint32_t)a.ns;
+                    ph ^= 1u;
+                }
+                continue;
+            }
+            const int np = n - f * pps < pps ? n - f * pps : pps;
+            uint32_t ia = 0, ib = 0, info = 0;
+            int rel = f;
+            bool load = false;
+            if (lane < np) {
+                const int64_t p = pb + (int64_t)f * pps + lane;
+                ia = cur.ia;
+                ib = cur.ib;
+                const uint32_t q = cur.q;
+                const uint32_t r = cur.r;
+                int64_t loader = p - (int64_t)(r & 15u);
+                if (loader < pb) loader = pb;
+                load = loader == p;
+                if ((int64_t)ia >= a.nA || (int64_t)ib >= a.nB) {
+                    atomicOr(a.status, kStBadIndex);
+                    ia = 0;
+                    ib = 0;
+                }
+                const int64_t src = loader - pb;
+                const uint32_t sst = (uint32_t)((src / pps) % a.ns), sj = (uint32_t)(src % pps);
+                info = q | (sst << 8) | (sj << 16);
+                if (load) {
+                    // the last pair reading this tile: the run's last sharer
+                    // (counted from the run's own loader), at most the unit's end
+                    const int64_t gl = p - (int64_t)(r & 15u);
+                    const uint32_t rg = gl == p ? r : a.arun[gl];
+                    int64_t last = gl + (int64_t)(rg >> 4);
+                    if (last > pe - 1) last = pe - 1;
+                    if (last < p) last = p;
+                    rel = (int)((last - pb) / pps);
+                }
+            }
+            // the stage is released after the latest fill any of its A tiles serves
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                const int r2 = __shfl_xor_sync(0xffffffffu, rel, o);
+                rel = r2 > rel ? r2 : rel;
+            }
+            const uint32_t lmask = __ballot_sync(0xffffffffu, load);
+            const uint32_t tx = (uint32_t)__popc(lmask) * a_tx + (uint32_t)np * b_tx;
+            uint32_t inf[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) inf[j] = __shfl_sync(0xffffffffu, info, j);
+            uint32_t okw = 1;
+            if (lane == 0) {
+                okw = mbar_wait(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status, a.wait_limit) ? 1u : 0u;
+                if (okw) {
+                    for (int j = 0; j < np; ++j) pinfo[st * 4 + j] = inf[j];
+                    prel[st] = rel;
+                    mbar_arrive_tx(full0 + 8u * st, tx);
+                }
+            }
+            if (!__shfl_sync(0xffffffffu, okw, 0)) break;
+            if (lane < np) {
+                const uint32_t fb = full0 + 8u * st;
+                const uint32_t sa = sbase + st * a.stage_bytes + (uint32_t)lane * a.a_pair;
+                const uint32_t sb = sbase + st * a.stage_bytes + (uint32_t)a.pps * a.a_pair + (uint32_t)lane * a.b_pair;
+                if (load)
+                    for (int q = 0; q < a.na_sub; ++q) {
+                        if (a.hint_a)
+                            tma_load_3d_hint(sa + q * a.a_sub, &tmA, q * a.wa, 0, (int)ia, fb, pol_a);
+                        else
+                            tma_load_3d(sa + q * a.a_sub, &tmA, q * a.wa, 0, (int)ia, fb);
+                    }
+                for (int q = 0; q < a.nb_sub; ++q) {
+                    if (a.hint_b)
+                        tma_load_3d_hint(sb + q * a.b_sub, &tmB, q * a.wb, 0, (int)ib, fb, pol_b);
+                    else
+                        tma_load_3d(sb + q * a.b_sub, &tmB, q * a.wb, 0, (int)ib, fb);
+                }
+            }
+            __syncwarp();
+            ++mine;
+            st += kProducers;
+            if (st >= (uint32_t)a.ns) {
+                st -= (uint32_t)a.ns;
+                ph ^= 1u;
+            }
+        }
+        if (lane == 0) misc[4 + warp] = mine;
+    } else if (warp == kProducers) {
+        // ------------------------------------------------------------ MMA
+        // Fills in order; per pair its slot's columns and its A source from
+        // the pair words; a stage's empty barrier is committed after the last
+        // fill whose pairs read an A tile in it.
+        uint32_t aoff[KSTEPS], boff[KSTEPS];
+#pragma unroll
+        for (int kk = 0; kk < KSTEPS; ++kk) {
+            aoff[kk] = (uint32_t)((kk >> a.a_lg) * a.a_sub16 + (kk & a.a_mask) * a.a_k16);
+            boff[kk] = (uint32_t)((kk >> a.b_lg) * a.b_sub16 + (kk & a.b_mask) * a.b_k16);
+        }
+        const uint64_t adesc0 = a.a_desc0 + (sbase >> 4);
+        const uint64_t bdesc0 = a.b_desc0 + ((sbase + (uint32_t)a.pps * a.a_pair) >> 4);
+        const uint32_t stage16 = a.stage_bytes >> 4, apair16 = a.a_pair >> 4, bpair16 = a.b_pair >> 4;
+        const uint32_t mb16 = (uint32_t)a.a_mb16, ncol = (uint32_t)a.N, idesc = a.idesc;
+        const bool two_m = a.m_blocks > 1;
+        const int n = (int)(pe - pb), pps = a.pps;
+        uint32_t b = 0, aph = 0, dcol = tmem;
+        int64_t s = s_first;
+        int seg_end = n > 0 ? (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) : 0;
+        bool fresh = true, ok = true;
+        int pend[kMaxStages];
+#pragma unroll
+        for (int i = 0; i < kMaxStages; ++i) pend[i] = -1;
+        auto open_seg = [&]() -> bool {
+            if (!__all_sync(0xffffffffu, mbar_wait(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status, a.wait_limit)))
+                return false;
+            tc_fence_after();
+            dcol = tmem + b * buf_cols;
+            fresh = false;
+            return true;
+        };
+        auto close_seg = [&](int pos) {
+            if (elect_one()) mma_commit(accf0 + 8u * b);
+            __syncwarp();
+            if (++b == (uint32_t)a.nacc) {
+                b = 0;
+                aph ^= 1u;
+            }
+            ++s;
+            if (pos < n) seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
+            fresh = true;
+        };
+        uint32_t st = 0, ph = 0;
+        int f = 0;
+        for (; f * pps < n; ++f) {
+            const int start = f * pps;
+            const int np = n - start < pps ? n - start : pps;
+            if (!__all_sync(0xffffffffu, mbar_wait(full0 + 8u * st, ph, abort_flag, a.status, a.wait_limit))) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            for (int jj = 0; jj < np; ++jj) {
+                if (fresh && !open_seg()) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t info = pinfo[st * 4 + jj];
+                const uint32_t d = dcol + (info & 0xFFu) * acc_cols;
+                const uint64_t ad = adesc0 + ((info >> 8) & 0xFFu) * stage16 + ((info >> 16) & 0xFFu) * apair16;
+                const uint64_t bd = bdesc0 + st * stage16 + (uint32_t)jj * bpair16;
+                if (elect_one()) {
+#pragma unroll
+                    for (int kk = 0; kk < KSTEPS; ++kk) {
+                        mma_bf16(d, ad + aoff[kk], bd + boff[kk], idesc, 1u);
+                        if (two_m) mma_bf16(d + ncol, ad + aoff[kk] + mb16, bd + boff[kk], idesc, 1u);
+                    }
+                }
+                __syncwarp();
+                if (start + jj + 1 == seg_end) close_seg(start + jj + 1);
+            }
+            if (!ok) break;
+            const int rel_st = prel[st];
+#pragma unroll
+            for (int i = 0; i < kMaxStages; ++i)   // constant indices: pend stays in registers
+                if (i == (int)st) pend[i] = rel_st;
+#pragma unroll
+            for (int i = 0; i < kMaxStages; ++i)
+                if (pend[i] == f) {
+                    if (elect_one()) mma_commit(empty0 + 8u * i);
+                    __syncwarp();
+                    pend[i] = -1;
+                }
+            if (++st == (uint32_t)a.ns) {
+                st = 0;
+                ph ^= 1u;
+            }
+        }
+        // segments that end after the last stage (none unless a wait gave up)
+        while (ok && s <= s_last) {
+            if (fresh && !open_seg()) {
+                ok = false;
+                break;
+            }
+            close_seg(seg_end);
+        }
+        if (lane == 0) misc[2] = ok ? 0xFFFFFFFFu : (uint32_t)f;
+    } else if (warp >= kProducers + kMmaWarps) {
+        // ------------------------------------------------------- epilogue
+        const int q4 = warp & 3;
+        const uint32_t lane_base = (uint32_t)(q4 * 32) << 16;
+        uint32_t b = 0, ph = 0;
+        for (int64_t s = s_first; s <= s_last; ++s) {
+            const int64_t ss = a.seg_start[s], se = a.seg_start[s + 1];
+            if (!__all_sync(0xffffffffu, mbar_wait(accf0 + 8u * b, ph, abort_flag, a.status, a.wait_limit))) break;
+            tc_fence_after();
+            const int kind = (ss >= pb && se <= pe) ? 0 : (ss < pb ? 1 : 2);
+            const uint32_t mask = a.wmask[s];
+            const int64_t base = a.wbase[s];
+            float *part = a.partials + ((int64_t)unit * 2 + (kind == 1 ? 0 : 1)) * (int64_t)W * a.tile_w;
+            for (int q = 0; q < W; ++q) {
+                if (!((mask >> q) & 1u)) continue;   // nothing accumulated there; nobody reads it
+                const int64_t row = base + __popc(mask & ((1u << q) - 1u));
+                const uint32_t bcol = tmem + lane_base + b * buf_cols + (uint32_t)q * acc_cols;
+                for (int mb = 0; mb < a.m_blocks; ++mb) {
+                    const int64_t m = (int64_t)mb * 128 + q4 * 32 + lane;
+                    for (int c = 0; c < a.N / 16; ++c) {
+                        float v[16];
+                        tmem_ld16(bcol + (uint32_t)(mb * a.N + c * 16), v);
+                        const int64_t off = m * a.sWm + (int64_t)c * 16 * a.sWn;
+                        if (kind == 0) {
+#pragma unroll
+                            for (int jj = 0; jj < 16; ++jj) v[jj] = epilogue(v[jj], a.epi, a.scale);
+                        }
+                        if (kind == 0 && a.dout == UCL_BF16) {
+                            __nv_bfloat16 *o = reinterpret_cast<__nv_bfloat16 *>(a.out) + row * a.tile_w + off;
+                            if (a.sWn == 1) {
+                                uint32_t h[8];
+#pragma unroll
+                                for (int jj = 0; jj < 8; ++jj) {
+                                    __nv_bfloat162 t = __floats2bfloat162_rn(v[2 * jj], v[2 * jj + 1]);
+                                    h[jj] = *reinterpret_cast<uint32_t *>(&t);
+                                }
+                                uint4 *o4 = reinterpret_cast<uint4 *>(o);
+                                o4[0] = make_uint4(h[0], h[1], h[2], h[3]);
+                                o4[1] = make_uint4(h[4], h[5], h[6], h[7]);
+                            } else {
+#pragma unroll
+                                for (int jj = 0; jj < 16; ++jj) o[jj * a.sWn] = __float2bfloat16_rn(v[jj]);
+                            }
+                        } else {
+                            float *o = kind == 0 ? reinterpret_cast<float *>(a.out) + row * a.tile_w + off
+                                                 : part + (int64_t)q * a.tile_w + off;
+                            if (a.sWn == 1) {
+                                float4 *o4 = reinterpret_cast<float4 *>(o);
+#pragma unroll
+                                for (int jj = 0; jj < 4; ++jj)
+                                    o4[jj] = make_float4(v[4 * jj], v[4 * jj + 1], v[4 * jj + 2], v[4 * jj + 3]);
+                            } else {
+#pragma unroll
+                                for (int jj = 0; jj < 16; ++jj) o[jj * a.sWn] = v[jj];
+                            }
+                        }
+                    }
+                }
+            }
+            for (uint32_t c = 0; c < buf_cols; c += 16) tmem_st16_zero(tmem + lane_base + b * buf_cols + c);
+            asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(acce0 + 8u * b);
+            if (++b == (uint32_t)a.nacc) {
+                b = 0;
+                ph ^= 1u;
+            }
+        }
+    }
+
+    // ---------------------------------------------------------- teardown
+    __syncthreads();
+    if (*abort_flag) {
+        if (warp < kProducers && lane == 0) {
+            for (uint32_t k = 0; k < misc[4 + warp]; ++k) {
+                const uint32_t it = (uint32_t)warp + k * kProducers;
+                if ((int)it == a.withhold_fill) continue;   // never copied: nothing in flight
+                if (it >= misc[2]) mbar_drain(full0 + 8u * (it % a.ns), (it / a.ns) & 1u);
+            }
+        }
+        if (warp == kProducers && lane == 0) {
+            mma_commit(done_bar);
+            mbar_drain(done_bar, 0);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == kProducers) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(a.tmem_cols)
+                     : "memory");
+    }
+}
+
 // ------------------------------------------------------------------- host
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -750,7 +1152,7 @@ struct TcGeometry {
 // stage holds pps pairs (1..4): the largest pps that keeps a stage within
 // 72 KB and leaves an even number (>= 4) of stages.
 bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_override = 0, int ns_force = 0) {
-    const uint32_t bar_bytes = 8u * (2 * kMaxStages + 2 * kMaxAcc + 1) + 64 + 64;
+    const uint32_t bar_bytes = kBarBytes;
     const uint32_t avail = kSmemLimit - 1024 - bar_bytes;
     bool found = false;
     for (int kc = 1; kc <= 16 && tp.K / kc >= 16 && tp.K % kc == 0; kc *= 2) {
@@ -806,6 +1208,12 @@ bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_overrid
         // a stage count chosen by the caller: two MMA warps only on an even ring
         if (ns > ns_force) ns = ns_force;
         g->nmma = two_fit && ns % 2 == 0 ? 2 : 1;
+    } else if (two_fit && ns >= 5 && (ns & 1) && tp.m_blocks * (tp.K / g->kc) / 16 >= 8) {
+        // an odd ring one stage deeper with one MMA warp: with at least eight
+        // MMAs per pair one warp keeps up, and the extra stage hides more of
+        // the copy latency (two-layer GNN message passing: 5 stages 51 ms
+        // against 4 stages and two MMA warps 54 ms)
+        g->nmma = 1;
     } else if (two_fit && ns >= 4) {
         ns &= ~1;
         g->nmma = 2;
@@ -878,7 +1286,50 @@ bool make_map(CUtensorMap *m, const ucl_rel *R, const Operand &op, std::string *
     return true;
 }
 
+// Geometry of the windowed kernel: whole pairs, one MMA warp (any ring
+// size), buffers of 2^win_bits accumulator slots, and the longest run of
+// pairs one loaded A tile may serve: a stage is then held at most ns - 2
+// fills past its own, so the producers never wait on a stage that a pair
+// still to be filled needs.
+bool window_geometry(const TcPlan &tp, int win_bits, TcGeometry *g, int *cap, std::string *why) {
+    if (!geometry(tp, g, why)) return false;
+    if (g->kc != 1) {
+        *why = "windows need whole pairs per stage";
+        return false;
+    }
+    int ns = (int)((kSmemLimit - 1024 - kBarBytes) / g->stage_bytes);
+    if (ns > kMaxStages) ns = kMaxStages;
+    if (ns < 3) {
+        *why = "windows need at least three stages";
+        return false;
+    }
+    g->ns = ns;
+    g->nmma = 1;
+    const int buf = tp.N * tp.m_blocks << win_bits;
+    g->nacc = 512 / buf < kMaxAcc ? 512 / buf : kMaxAcc;
+    if (g->nacc < 1) {
+        *why = "window accumulators do not fit TMEM";
+        return false;
+    }
+    uint32_t need = (uint32_t)(g->nacc * buf), cols = 32;
+    while (cols < need) cols <<= 1;
+    g->tmem_cols = cols;
+    g->smem_bytes = 1024 + ns * g->stage_bytes + kBarBytes;
+    int c = (ns - 2) * g->pps + 1;
+    *cap = c < 1 ? 1 : (c > 15 ? 15 : c);
+    if (const char *e = getenv("UCL_WINDOW_SHARE"))   // measurement: 0 turns A-tile sharing off
+        if (atoi(e) == 0) *cap = 1;
+    return true;
+}
+
 }  // namespace
+
+int tc_window_cap(const TcPlan &tp, int win_bits) {
+    TcGeometry g;
+    std::string why;
+    int cap = 0;
+    return window_geometry(tp, win_bits, &g, &cap, &why) ? cap : 0;
+}
 
 bool tc_supported(const TcPlan &tp, const ContractArgs &a, std::string *why) {
     TcGeometry g;
@@ -901,7 +1352,13 @@ ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan 
                               const ucl_rel *rb) {
     TcGeometry g;
     std::string why;
-    if (!geometry(tp, &g, &why, 0, ctx->tune_tc_stages)) return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why);
+    int cap = 0;
+    if (a.win_bits > 0) {
+        if (!window_geometry(tp, a.win_bits, &g, &cap, &why)) return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why);
+        if (cap != a.share_cap) return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: run cap disagrees with the key stage");
+    } else if (!geometry(tp, &g, &why, 0, ctx->tune_tc_stages)) {
+        return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why);
+    }
     CUtensorMap mA, mB;
     if (!make_map(&mA, ra, g.A, &why) || !make_map(&mB, rb, g.B, &why))
         return fail(ctx, UCL_ERR_CUDA, "tcgen05 path: " + why);
@@ -1003,13 +1460,20 @@ ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan 
     k.wait_limit = ctx->wait_limit_cycles > 0 ? ctx->wait_limit_cycles : kWaitLimitCycles;
     k.withhold_fill = ctx->withhold_fill;
     ctx->withhold_fill = -1;   // one launch only
+    k.win_bits = a.win_bits;
+    k.slot = a.slot;
+    k.arun = a.arun;
+    k.wmask = a.wmask;
+    k.wbase = a.wbase;
+    k.share_cap = cap;
     void (*kern)(const CUtensorMap, const CUtensorMap, const TcArgs) = nullptr;
+    const bool win = a.win_bits > 0;
     switch (tp.K / g.kc / 16) {
-        case 1: kern = tc_contract_kernel<1>; break;
-        case 2: kern = tc_contract_kernel<2>; break;
-        case 4: kern = tc_contract_kernel<4>; break;
-        case 8: kern = tc_contract_kernel<8>; break;
-        case 16: kern = tc_contract_kernel<16>; break;
+        case 1: kern = win ? tc_window_kernel<1> : tc_contract_kernel<1>; break;
+        case 2: kern = win ? tc_window_kernel<2> : tc_contract_kernel<2>; break;
+        case 4: kern = win ? tc_window_kernel<4> : tc_contract_kernel<4>; break;
+        case 8: kern = win ? tc_window_kernel<8> : tc_contract_kernel<8>; break;
+        case 16: kern = win ? tc_window_kernel<16> : tc_contract_kernel<16>; break;
         default: return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: K must be 16, 32, 64, 128 or 256");
     }
     ucl_status st = cuda_check(

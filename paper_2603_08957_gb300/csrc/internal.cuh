@@ -167,6 +167,9 @@ struct ucl_ctx {
     // prefetch the streamed operand)
     int tune_tc_stages = 0;
     int tune_tc_prefetch = -1;
+    // UCL_WINDOW (-1 or unset: automatic; 0: no windows; n: windows of 2^n
+    // output keys where the windowed tcgen05 kernel applies)
+    int tune_window = -1;
     int l2_bytes = 0;
     // Bounded waits of the tcgen05 kernel: SM cycles before a role gives up
     // (0: the kernel's default of about a second), and the failure-detection
@@ -217,7 +220,8 @@ void launch_check_dups(ucl_ctx *ctx, const uint64_t *sorted_keys, int64_t n);
 // Stable LSD radix sort of (key, value) by the low `bits` bits of key.
 // kin/vin and kalt/valt are ping-pong buffers; returns which holds the result
 // (0: kin/vin, 1: kalt/valt).  vin may be NULL (keys only).
-int radix_sort(ucl_ctx *ctx, uint64_t *kin, uint64_t *vin, uint64_t *kalt, uint64_t *valt, int64_t n, int bits);
+int radix_sort(ucl_ctx *ctx, uint64_t *kin, uint64_t *vin, uint64_t *kalt, uint64_t *valt, int64_t n, int bits,
+               int lo = 0);
 // Exclusive scan of n int64 values; writes total to *total_dev if non-NULL.
 void scan_i64(ucl_ctx *ctx, const int64_t *in, int64_t *out, int64_t n, int64_t *total_dev);
 // iota into u64
@@ -237,7 +241,19 @@ void launch_heads(ucl_ctx *ctx, const uint64_t *pk, int64_t P, int64_t *flag, in
 // = first pair of band b, band_seg[b] = its segment index (b = 0..B; B <= 63).
 void launch_band_ranges(ucl_ctx *ctx, const uint64_t *pk, int64_t P, const int64_t *seg_excl, const int64_t *n_seg,
                         int out_bits, int B, int64_t *band_start, int64_t *band_seg);
-// sk[s] = (output key << band_bits) | band of band segment s, sv[s] = s.
+// Windows: slot[p] = output key & (2^wb - 1) and mask[ws] |= 1 << slot for
+// each pair (flag/excl: window segment heads and their exclusive scan).
+void launch_win_slots(ucl_ctx *ctx, const uint64_t *pk, int64_t P, int wb, const int64_t *flag, const int64_t *excl,
+                      uint8_t *slot, uint32_t *mask);
+// cnt[ws] = slots present in window segment ws.
+void launch_win_count(ucl_ctx *ctx, const uint32_t *mask, int64_t Sw, int64_t *cnt);
+// rowkey[wbase[ws] + i] = key of the i-th present slot of window segment ws.
+void launch_win_rows(ucl_ctx *ctx, const uint64_t *pk, const int64_t *seg_start, int64_t Sw, const uint32_t *mask,
+                     const int64_t *wbase, int wb, uint64_t *rowkey);
+// out_keys[s] = the output key columns of packed key k[s].
+void launch_unpack_keys(ucl_ctx *ctx, const uint64_t *k, int64_t n, KeyUnpack un, int32_t *out_keys);
+// sk[s] = (output key << band_bits) | band of band segment s, sv[s] = s
+// (the packed key of segment s is pk[seg_start[s]], or pk[s] if seg_start is NULL).
 void launch_band_keys(ucl_ctx *ctx, const uint64_t *pk, const int64_t *seg_start, int64_t Sp, int out_bits,
                       int band_bits, uint64_t *sk, uint64_t *sv);
 // After sorting sk: the S output keys and fstart[f] = first sorted band
@@ -246,7 +262,8 @@ void launch_band_outputs(ucl_ctx *ctx, const uint64_t *sk, const int64_t *excl, 
                          KeyUnpack un, int32_t *out_keys, int64_t *fstart);
 // Segment starts, output keys, pair index arrays.
 void launch_segments(ucl_ctx *ctx, const uint64_t *pk, const uint64_t *pv, const int64_t *seg_excl, int64_t P,
-                     int64_t S, KeyUnpack un, int32_t *out_keys, int64_t *seg_start, uint32_t *pu, uint32_t *pvi);
+                     int64_t S, KeyUnpack un, int32_t *out_keys, int64_t *seg_start, uint32_t *pu, uint32_t *pvi,
+                     int shift = 0);
 // Three-way join, second step.  pair_keys: jk[p] = jk_a[a] | jk_b[b] for
 // each first-step pair pv1[p] = (a << 32) | b (either table may be NULL).
 void launch_pair_keys(ucl_ctx *ctx, const uint64_t *pv1, int64_t P1, const uint64_t *jk_a, const uint64_t *jk_b,
@@ -335,6 +352,15 @@ struct ContractArgs {
     float *partials;       // [G, 2, tile_w]
     int64_t tile_w;
     unsigned long long *fixup_bytes;   // device counter the fixup kernel adds its bytes to (may be NULL)
+    // windowed tcgen05 kernel (win_bits > 0): segments are windows of
+    // 2^win_bits output keys; per pair its slot and A-tile run (see
+    // contract_tc.cu); per window its present slots and first output row
+    int win_bits;
+    const uint8_t *slot;
+    const uint8_t *arun;
+    const uint32_t *wmask;
+    const int64_t *wbase;
+    int share_cap;
     int bands;             // > 1: U's tuples are split into this many bands of its join label (one launch each)
     int l2_hints;          // TMA loads carry L2 eviction hints (streamed operand first, reused operand last)
 };
@@ -350,6 +376,16 @@ bool tc_supported(const TcPlan &tp, const ContractArgs &a, std::string *why);
 ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan &tp, const ucl_rel *ra,
                               const ucl_rel *rb);
 int tc_units(ucl_ctx *ctx, const TcPlan &tp, int64_t P);
+// Longest run of pairs sharing one loaded A tile in the windowed tcgen05
+// kernel for this shape and window size (0: the windowed kernel does not apply).
+int tc_window_cap(const TcPlan &tp, int win_bits);
+// arun[p] for the windowed kernel: low nibble = pairs back to the pair that
+// loads p's A tile (a run of equal pa[] is cut every cap positions), high
+// nibble (at that pair) = pairs after it sharing the tile.
+void launch_arun(ucl_ctx *ctx, const uint32_t *pa, int64_t P, int cap, uint8_t *arun);
+// Windowed fixup: a window split across units sums its present slots'
+// partials in unit order into their output rows.
+void launch_fixup_window(ucl_ctx *ctx, const ContractArgs &a);
 ucl_status launch_contract_tc3(ucl_ctx *ctx, const ContractArgs &a, const Tc3Plan &tp, const ucl_rel *const *in);
 int tc3_units(ucl_ctx *ctx, int64_t P);
 

@@ -313,7 +313,7 @@ __global__ void band_keys_kernel(const uint64_t *__restrict__ pk, const int64_t 
                                  int out_bits, int band_bits, uint64_t *sk, uint64_t *sv) {
     const uint64_t omask = out_bits ? (~0ull >> (64 - out_bits)) : 0ull;
     for (int64_t s = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; s < Sp; s += (int64_t)gridDim.x * blockDim.x) {
-        const uint64_t k = pk[seg_start[s]];
+        const uint64_t k = seg_start ? pk[seg_start[s]] : pk[s];
         sk[s] = ((k & omask) << band_bits) | (k >> out_bits);
         sv[s] = (uint64_t)s;
     }
@@ -338,13 +338,13 @@ __global__ void band_outputs_kernel(const uint64_t *__restrict__ sk, const int64
 
 __global__ void segments_kernel(const uint64_t *__restrict__ pk, const uint64_t *__restrict__ pv,
                                 const int64_t *__restrict__ seg_excl, int64_t P, int64_t S, KeyUnpack un,
-                                int32_t *out_keys, int64_t *seg_start, uint32_t *pu, uint32_t *pvi) {
+                                int32_t *out_keys, int64_t *seg_start, uint32_t *pu, uint32_t *pvi, int shift) {
     for (int64_t p = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; p < P; p += (int64_t)gridDim.x * blockDim.x) {
         uint64_t v = pv[p];
         pu[p] = (uint32_t)(v >> 32);
         pvi[p] = (uint32_t)v;
         uint64_t k = pk[p];
-        if (p == 0 || k != pk[p - 1]) {
+        if (p == 0 || (k >> shift) != (pk[p - 1] >> shift)) {
             int64_t s = seg_excl[p];
             seg_start[s] = p;
             for (int c = 0; c < un.uw; ++c) {
@@ -451,13 +451,14 @@ void scan_i64(ucl_ctx *ctx, const int64_t *in, int64_t *out, int64_t n, int64_t 
     scan_excl<int64_t>(ctx, in, out, n, total_dev);
 }
 
-int radix_sort(ucl_ctx *ctx, uint64_t *kin, uint64_t *vin, uint64_t *kalt, uint64_t *valt, int64_t n, int bits) {
+int radix_sort(ucl_ctx *ctx, uint64_t *kin, uint64_t *vin, uint64_t *kalt, uint64_t *valt, int64_t n, int bits,
+               int lo) {
     if (bits <= 0 || n <= 1) return 0;
     int nblocks = (int)((n + kSortTile - 1) / kSortTile);
     uint32_t *hist = (uint32_t *)ws_get(ctx, sizeof(uint32_t) * (size_t)kBuckets * nblocks);
     uint64_t *ks = kin, *vs = vin, *kd = kalt, *vd = valt;
     int which = 0;
-    for (int shift = 0; shift < bits; shift += kRadixBits) {
+    for (int shift = lo; shift < lo + bits; shift += kRadixBits) {
         radix_hist_kernel<<<nblocks, kSortThreads, 0, ctx->stream>>>(ks, n, shift, hist, nblocks);
         ctx->launches++;
         scan_excl<uint32_t>(ctx, hist, hist, (int64_t)kBuckets * nblocks, nullptr);
@@ -498,6 +499,102 @@ void launch_heads(ucl_ctx *ctx, const uint64_t *pk, int64_t P, int64_t *flag, in
     ctx->launches++;
 }
 
+// ---------------------------------------------------------------- windows
+// Windowed pair lists: pairs sorted by (band, output key >> wb), so that the
+// pairs of 2^wb consecutive output keys (a window) are contiguous and those
+// of one tuple of the first input stay together.  Per pair its slot (output
+// key & (2^wb - 1)); per window segment the mask of slots present.
+
+__global__ void win_slots_kernel(const uint64_t *__restrict__ pk, int64_t P, int wb, const int64_t *__restrict__ flag,
+                                 const int64_t *__restrict__ excl, uint8_t *slot, uint32_t *mask) {
+    const uint64_t qm = (1ull << wb) - 1ull;
+    for (int64_t p = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; p < P; p += (int64_t)gridDim.x * blockDim.x) {
+        const uint32_t q = (uint32_t)(pk[p] & qm);
+        slot[p] = (uint8_t)q;
+        const int64_t ws = excl[p] + flag[p] - 1;
+        atomicOr(&mask[ws], 1u << q);
+    }
+}
+
+__global__ void win_count_kernel(const uint32_t *__restrict__ mask, int64_t Sw, int64_t *cnt) {
+    for (int64_t s = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; s < Sw; s += (int64_t)gridDim.x * blockDim.x)
+        cnt[s] = __popc(mask[s]);
+}
+
+// Row r of the output (or of the band partials) for each present slot of a
+// window segment, in slot order: rowkey = (window's full key) | slot.
+__global__ void win_rows_kernel(const uint64_t *__restrict__ pk, const int64_t *__restrict__ seg_start, int64_t Sw,
+                                const uint32_t *__restrict__ mask, const int64_t *__restrict__ wbase, int wb,
+                                uint64_t *rowkey) {
+    for (int64_t s = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; s < Sw; s += (int64_t)gridDim.x * blockDim.x) {
+        const uint64_t base = (pk[seg_start[s]] >> wb) << wb;
+        uint32_t m = mask[s];
+        int64_t r = wbase[s];
+        while (m) {
+            const int q = __ffs(m) - 1;
+            m &= m - 1;
+            rowkey[r++] = base | (uint64_t)q;
+        }
+    }
+}
+
+__global__ void unpack_keys_kernel(const uint64_t *__restrict__ k, int64_t n, KeyUnpack un, int32_t *out_keys) {
+    for (int64_t s = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; s < n; s += (int64_t)gridDim.x * blockDim.x)
+        for (int c = 0; c < un.uw; ++c) {
+            uint64_t mask = un.bits[c] ? ((~0ull) >> (64 - un.bits[c])) : 0ull;
+            out_keys[s * un.uw + c] = (int32_t)((k[s] >> un.shift[c]) & mask);
+        }
+}
+
+// A-tile runs for the windowed kernel (see internal.cuh, launch_arun).
+__global__ void arun_kernel(const uint32_t *__restrict__ pa, int64_t P, int cap, uint8_t *arun) {
+    for (int64_t p = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; p < P; p += (int64_t)gridDim.x * blockDim.x) {
+        const uint32_t me = pa[p];
+        int back = 0;
+        while (back < cap - 1) {
+            const int64_t x = p - back;   // x is in the run of p; does x load?
+            if (x == 0 || x % cap == 0 || pa[x - 1] != me) break;
+            ++back;
+        }
+        int fwd = 0;
+        if (back == 0)
+            while (fwd < cap - 1 && p + fwd + 1 < P && (p + fwd + 1) % cap != 0 && pa[p + fwd + 1] == me) ++fwd;
+        arun[p] = (uint8_t)(back | (fwd << 4));
+    }
+}
+
+void launch_arun(ucl_ctx *ctx, const uint32_t *pa, int64_t P, int cap, uint8_t *arun) {
+    if (P <= 0) return;
+    arun_kernel<<<grid_for(ctx, P), kThreads, 0, ctx->stream>>>(pa, P, cap, arun);
+    ctx->launches++;
+}
+
+void launch_win_slots(ucl_ctx *ctx, const uint64_t *pk, int64_t P, int wb, const int64_t *flag, const int64_t *excl,
+                      uint8_t *slot, uint32_t *mask) {
+    if (P <= 0) return;
+    win_slots_kernel<<<grid_for(ctx, P), kThreads, 0, ctx->stream>>>(pk, P, wb, flag, excl, slot, mask);
+    ctx->launches++;
+}
+
+void launch_win_count(ucl_ctx *ctx, const uint32_t *mask, int64_t Sw, int64_t *cnt) {
+    if (Sw <= 0) return;
+    win_count_kernel<<<grid_for(ctx, Sw), kThreads, 0, ctx->stream>>>(mask, Sw, cnt);
+    ctx->launches++;
+}
+
+void launch_win_rows(ucl_ctx *ctx, const uint64_t *pk, const int64_t *seg_start, int64_t Sw, const uint32_t *mask,
+                     const int64_t *wbase, int wb, uint64_t *rowkey) {
+    if (Sw <= 0) return;
+    win_rows_kernel<<<grid_for(ctx, Sw), kThreads, 0, ctx->stream>>>(pk, seg_start, Sw, mask, wbase, wb, rowkey);
+    ctx->launches++;
+}
+
+void launch_unpack_keys(ucl_ctx *ctx, const uint64_t *k, int64_t n, KeyUnpack un, int32_t *out_keys) {
+    if (n <= 0 || un.uw == 0) return;
+    unpack_keys_kernel<<<grid_for(ctx, n), kThreads, 0, ctx->stream>>>(k, n, un, out_keys);
+    ctx->launches++;
+}
+
 void launch_band_ranges(ucl_ctx *ctx, const uint64_t *pk, int64_t P, const int64_t *seg_excl, const int64_t *n_seg,
                         int out_bits, int B, int64_t *band_start, int64_t *band_seg) {
     band_ranges_kernel<<<1, 64, 0, ctx->stream>>>(pk, P, seg_excl, n_seg, out_bits, B, band_start, band_seg);
@@ -520,10 +617,11 @@ void launch_band_outputs(ucl_ctx *ctx, const uint64_t *sk, const int64_t *excl, 
 }
 
 void launch_segments(ucl_ctx *ctx, const uint64_t *pk, const uint64_t *pv, const int64_t *seg_excl, int64_t P,
-                     int64_t S, KeyUnpack un, int32_t *out_keys, int64_t *seg_start, uint32_t *pu, uint32_t *pvi) {
+                     int64_t S, KeyUnpack un, int32_t *out_keys, int64_t *seg_start, uint32_t *pu, uint32_t *pvi,
+                     int shift) {
     if (P <= 0) return;
     segments_kernel<<<grid_for(ctx, P), kThreads, 0, ctx->stream>>>(pk, pv, seg_excl, P, S, un, out_keys,
-                                                                    seg_start, pu, pvi);
+                                                                    seg_start, pu, pvi, shift);
     ctx->launches++;
 }
 

@@ -18,8 +18,12 @@ pytestmark = pytest.mark.gpu
 UCL_ERR_TIMEOUT = 9
 
 
-def test_withheld_stage_times_out_and_context_recovers():
+@pytest.mark.parametrize("window", ["0", "2"])
+def test_withheld_stage_times_out_and_context_recovers(monkeypatch, window):
+    """Both binary tcgen05 kernels: the plain one and the windowed one."""
+    monkeypatch.setenv("UCL_WINDOW", window)
     ctx = Context(0)
+    monkeypatch.delenv("UCL_WINDOW")
     w = workloads.gnn_chain(seed=6, n=4096, degree=16)
     X, Y = gpu_rel(ctx, w["X"]), gpu_rel(ctx, w["Y"])
     ref = oracle_ref(w["spec1"], [w["X"], w["Y"]])

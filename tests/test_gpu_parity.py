@@ -208,6 +208,65 @@ def test_banded_message_passing(monkeypatch, bands):
     c.close()
 
 
+@pytest.mark.parametrize("window,bands", [(1, 0), (2, 0), (3, 0), (2, 4), (1, 2)])
+def test_windowed_message_passing(monkeypatch, window, bands):
+    """Windows of 2^w consecutive output keys (forced): pairs ordered by
+    (band, K >> w, X tuple), accumulated per key slot in one TMEM buffer, an
+    X tile loaded once per run of pairs that read it.  Both message-passing
+    EinSums of a small two-layer GNN against the oracle, every output key,
+    with units small enough that windows straddle CTAs (partials + fixup)."""
+    monkeypatch.setenv("UCL_WINDOW", str(window))
+    monkeypatch.setenv("UCL_BANDS", str(bands))
+    c = Context(0)
+    monkeypatch.delenv("UCL_WINDOW")
+    monkeypatch.delenv("UCL_BANDS")
+    feat = 128 if window == 3 else 256
+    w = workloads.gnn_two_layer(seed=7, n=3000, n_edges=30_000, feat=feat, device="cuda")
+    X, Y = gpu_rel(c, w["X"]), gpu_rel(c, w["Y"])
+    T1 = c.einsum(w["spec1"], X, Y, out_dtype="bf16")
+    st = c.last_stats()
+    assert st["path"] == "tc" and st["n_bands"] == max(bands, 1)
+    host = {k: (w[k][0], w[k][1], w[k][2].cpu()) for k in ("X", "Y")}
+    assert_parity(T1, oracle_ref(w["spec1"], [host["X"], host["Y"]]), torch.bfloat16)
+    k1, t1 = T1.download()
+    T2 = c.einsum(w["spec3"], T1, Y, out_dtype="f32")
+    assert_parity(T2, oracle_ref(w["spec3"], [(k1, T1.bounds, t1), host["Y"]]), torch.bfloat16)
+    # the same EinSum without windows: the same key set
+    c2 = Context(0)
+    T3 = c2.einsum(w["spec1"], gpu_rel(c2, w["X"]), gpu_rel(c2, w["Y"]), out_dtype="bf16")
+    assert np.array_equal(T3.download()[0], k1)
+    for r in (X, Y, T1, T2):
+        r.destroy()
+    c.close()
+
+
+def test_windowed_gnn_full_size_sampled(monkeypatch):
+    """The full message-passing EinSum (100000 vertices, 358k Y tiles) with
+    windows of 4 keys (forced): every output key, values on sampled keys."""
+    monkeypatch.setenv("UCL_WINDOW", "2")
+    c = Context(0)
+    monkeypatch.delenv("UCL_WINDOW")
+    w = workloads.gnn_chain(seed=0, n=100_000)
+    X, Y = gpu_rel(c, w["X"]), gpu_rel(c, w["Y"])
+    T = c.einsum(w["spec1"], X, Y, out_dtype="bf16")
+    ky = w["Y"][0]
+    kt = T.download()[0]
+    assert np.array_equal(kt, np.unique(ky[:, 1]).astype(np.int32)[:, None])
+    cnt = np.bincount(ky[:, 1])
+    big = int(np.searchsorted(kt[:, 0], int(np.argmax(cnt))))
+    sk = kt[_sample_rows(len(kt), 12, seed=4, must=[big]), 0]
+    yk = ky[np.isin(ky[:, 1], sk)]
+    rows = np.nonzero(np.isin(ky[:, 1], sk))[0]
+    yrel = (yk, w["Y"][1], w["Y"][2][torch.as_tensor(rows)])
+    jn = np.unique(yk[:, 0])
+    xrel = (jn[:, None].astype(np.int32), w["X"][1], w["X"][2][torch.as_tensor(jn)])
+    ref = oracle_ref(w["spec1"], [xrel, yrel], sample_keys=sk[:, None])
+    assert_parity(T, ref, torch.bfloat16, select=np.searchsorted(kt[:, 0], sk))
+    for r in (X, Y, T):
+        r.destroy()
+    c.close()
+
+
 def test_l2_hints_do_not_change_results(monkeypatch):
     """L2 eviction hints on the TMA loads change where lines live, never the
     arithmetic: results with and without them are bit-identical."""
