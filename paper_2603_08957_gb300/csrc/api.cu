@@ -1090,6 +1090,29 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
         // already grouped; count the joined pairs (for three inputs: the
         // pairs of the first join, then the triples)
         int64_t P = 0, P1 = 0;
+        // small binary EinSums: the whole key stage in one CTA and one sync;
+        // more pairs than it holds fall through to the general path
+        bool small = false;
+        int64_t *sm_seg = nullptr;
+        int32_t *sm_keys = nullptr;
+        uint32_t *sm_pu = nullptr, *sm_pv = nullptr;
+        int64_t sm_S = 0;
+        if (n_in == 2 && !banded && wb == 0 && small_join_fits(nA, nB)) {
+            sm_seg = (int64_t *)ws_get(ctx, 8 * (kSmallPairs + 1));
+            sm_keys = (int32_t *)ws_get(ctx, 4 * (size_t)kSmallPairs * (kp.uw > 0 ? kp.uw : 1));
+            sm_pu = (uint32_t *)ws_get(ctx, 4 * kSmallPairs);
+            sm_pv = (uint32_t *)ws_get(ctx, 4 * kSmallPairs);
+            launch_small_join(ctx, A->keys, A->u, nA, B->keys, B->u, nB, kp.join_u, kp.join_v, kp.out_k[kp.ord[0]],
+                              kp.out_k[kp.ord[1]], kp.unpack, !kp.join.empty(), d_scal, sm_seg, sm_keys, sm_pu,
+                              sm_pv);
+            int64_t h[2] = {0, 0};
+            check(sync_read(ctx, d_scal, 2, h));
+            if (h[0] <= kSmallPairs) {
+                small = true;
+                P = h[0];
+                sm_S = h[1];
+            }
+        }
         uint64_t *koA = nullptr, *koB = nullptr, *koC = nullptr;
         uint64_t *permA = nullptr, *permB = nullptr, *permC = nullptr;
         int64_t *off = nullptr, *off2 = nullptr;
@@ -1107,7 +1130,9 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             if (h >= (1ll << 31)) check(fail(ctx, UCL_ERR_UNSUPPORTED, "more than 2^31-1 joined pairs"));
             return h;
         };
-        if (nA > 0 && nB > 0 && nC > 0) {
+        if (small) {
+            record(ctx, 1);
+        } else if (nA > 0 && nB > 0 && nC > 0) {
             koA = (uint64_t *)ws_get(ctx, 8 * nA);
             uint64_t *jkA = B ? (uint64_t *)ws_get(ctx, 8 * nA) : nullptr;
             launch_pack(ctx, A->keys, A->u, nA, kp.join_u, jkA, kp.out_k[kp.ord[0]], koA);
@@ -1174,7 +1199,7 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
         int64_t *flag = nullptr;
         uint64_t *pk = nullptr, *pv = nullptr;
         int64_t *seg_excl = nullptr;
-        if (P > 0) {
+        if (P > 0 && !small) {
             pk = (uint64_t *)ws_get(ctx, 8 * P);
             pv = (uint64_t *)ws_get(ctx, 8 * P);
             uint64_t *pk2 = (uint64_t *)ws_get(ctx, 8 * P), *pv2 = (uint64_t *)ws_get(ctx, 8 * P);
@@ -1220,7 +1245,13 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
         int64_t *seg_start = nullptr;
         uint32_t *pu = nullptr, *pvi = nullptr, *pxi = nullptr;
         int32_t *okeys = nullptr;
-        if (P > 0) {
+        if (small) {
+            S = sm_S;
+            seg_start = sm_seg;
+            pu = sm_pu;
+            pvi = sm_pv;
+            okeys = sm_keys;
+        } else if (P > 0) {
             seg_start = (int64_t *)ws_get(ctx, 8 * (S + 1));
             pu = (uint32_t *)ws_get(ctx, 4 * P);
             pvi = (uint32_t *)ws_get(ctx, 4 * P);

@@ -28,19 +28,24 @@
 //   warp 0      TMA producer: T tile (16 x 256 rows, 32B swizzle) and F tile
 //               (64 x 16 rows, 128B swizzle) of each triple into a ring of
 //               stages of `pps` triples;
+//   warp 6      group warp: per stage, which triples open a group, close one
+//               or end an output key; for each group opening there it waits
+//               until the epilogue has released the group's accumulator
+//               buffer and requests the group's E tile by TMA into that
+//               buffer's E slot; then it posts the stage's plan;
 //   warp 1      MMA issuer (owns TMEM): one thread issues two tcgen05.mma per
-//               triple into the group's accumulator buffer, following a group
-//               plan the producer posts with each stage;
+//               triple into the group's accumulator buffer, following the
+//               plan, and commits a group's buffer after its last triple;
 //   warps 2-5   epilogue: per group, load E's 16 values for its r, drain the
 //               group's accumulator and fold it into 8 fp32 registers; at the
 //               end of an output key, store the output tile (or a partial for
 //               the fixup kernel when the key straddles two work units).
 //
-// When the MMA warp opens a group it also requests the group's E tile by TMA
-// into the buffer's E slot; when it closes the group it posts whether the
-// group ends its output key.  The epilogue thus never searches the pair list
-// nor waits on a global load.
-//
+// Keeping the group bookkeeping (buffer waits, E requests) out of both the
+// producer and the issuing thread lets the copies run a full ring ahead and
+// leaves the issuing thread only stage waits, MMAs and commits.  The
+// epilogue never searches the pair list nor waits on a global load.
+
 // Every mbarrier wait is bounded; on expiry the CTA raises kStTimeout, all
 // roles leave their loops, in-flight copies and MMAs are drained (bounded),
 // TMEM is freed and the kernel returns.
@@ -55,7 +60,7 @@ namespace ucl {
 
 namespace {
 
-constexpr int kThreads3 = 32 * 6;
+constexpr int kThreads3 = 32 * 7;            // producer, MMA, 4 epilogue warps, group warp
 constexpr long long kWait3 = 2500000000ll;   // ~1.2 s at 2.07 GHz
 constexpr int kPps3 = 4;                     // triples per stage
 constexpr int kStages3 = 4;
@@ -67,7 +72,8 @@ constexpr uint32_t kFRegion = (2 * kPps3 + 1) * kFBytes;
 constexpr uint32_t kStageBytes = kPps3 * kTBytes + kFRegion;
 constexpr uint32_t kEBytes = 16 * 64 * 2;    // E tile: 16 j x 64 r, bf16, one slot per accumulator buffer
 // barriers: full, empty (per stage); accf, acce, ef, infoc (per buffer); done
-constexpr uint32_t kBarBytes = 8 * (2 * kStages3 + 4 * kAcc3 + 1) + 64 + 8 * kAcc3 + 4 * kStages3 * (kPps3 + 1);
+constexpr uint32_t kBarBytes =
+    8 * (3 * kStages3 + 4 * kAcc3 + 1) + 64 + 8 * kAcc3 + 4 * kStages3 * (kPps3 + 1);
 constexpr uint32_t kSmem3 = 1024 + kStages3 * kStageBytes + kAcc3 * kEBytes + kBarBytes;
 static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
 static_assert(kSmem3 <= 227 * 1024, "shared memory budget");
@@ -214,15 +220,15 @@ __global__ void __launch_bounds__(kThreads3, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     const uint32_t sbase = smem_u32(smem);
-    // E slot of buffer b: the group's E tile, fetched by TMA when the MMA warp
-    // opens the group (ef[b]), read by the epilogue before it frees the buffer
+    // E slot of buffer b: the group's E tile, fetched by TMA when the group
+    // warp opens the group (ef[b]), read by the epilogue before it frees the buffer
     const __nv_bfloat16 *eslots = reinterpret_cast<const __nv_bfloat16 *>(smem + (size_t)kStages3 * kStageBytes);
     const uint32_t eslot0 = sbase + kStages3 * kStageBytes;
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)kStages3 * kStageBytes + kAcc3 * kEBytes);
     const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8u * kStages3, accf0 = empty0 + 8u * kStages3,
                    acce0 = accf0 + 8u * kAcc3, done_bar = acce0 + 8u * kAcc3, ef0 = done_bar + 8u,
-                   infoc0 = ef0 + 8u * kAcc3;
-    uint32_t *misc = reinterpret_cast<uint32_t *>(bars + 2 * kStages3 + 4 * kAcc3 + 1);
+                   infoc0 = ef0 + 8u * kAcc3, planned0 = infoc0 + 8u * kAcc3;
+    uint32_t *misc = reinterpret_cast<uint32_t *>(bars + 3 * kStages3 + 4 * kAcc3 + 1);
     // misc[0] TMEM base, [1] abort flag, [2] stage fills the MMA warp consumed,
     // [3] stage fills the producer issued, [4] E tiles requested, [5] E tiles
     // the epilogue received
@@ -230,9 +236,9 @@ __global__ void __launch_bounds__(kThreads3, 1)
     // per accumulator buffer: [2b + 1] 1 if the group ends its output key
     // (posted at close through infoc[b])
     volatile uint32_t *info = misc + 16;
-    // per stage: the E tuple of each triple, then a word whose bit j marks
-    // triple j as opening a group and bit 8 + j marks the group before it as
-    // ending its output key (written by the producer before its arrive)
+    // per stage: a word whose bit j marks triple j as opening a group, bit
+    // 8 + j its group as ending the output key and bit 16 + j its group as
+    // closing after it (written by the group warp before planned[st])
     volatile uint32_t *plan = info + 2 * kAcc3;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -257,6 +263,7 @@ __global__ void __launch_bounds__(kThreads3, 1)
             mbar_init(ef0 + 8u * i, 1);
             mbar_init(infoc0 + 8u * i, 1);
         }
+        for (int i = 0; i < kStages3; ++i) mbar_init(planned0 + 8u * i, 1);
         for (int i = 1; i < 16; ++i) misc[i] = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -278,22 +285,17 @@ __global__ void __launch_bounds__(kThreads3, 1)
 
     if (warp == 0) {
         // ------------------------------------------------------- producer
-        // Lane j < pps handles triple j of each stage: its tuple indices are
-        // loaded one stage ahead; lane 0 posts the stage's group plan (each
-        // triple's E tuple, which triples open a group, which groups end their
-        // output key) in shared memory before its arrive, so the plan is
-        // visible to whoever observes the stage full; then lane j issues the
-        // two copies of triple j.
+        // Copies only: lane j < pps handles triple j of each stage (indices
+        // loaded one stage ahead) and issues its T and F copies.  The group
+        // plan of a stage is posted separately by the group warp.
         const int nfills = (n + kPps3 - 1) / kPps3;
-        auto load_idx = [&](int f, uint32_t &it, uint32_t &iff, uint32_t &ie) {
+        auto load_idx = [&](int f, uint32_t &it, uint32_t &iff) {
             it = 0;
             iff = 0;
-            ie = 0;
             const int64_t p = pb + (int64_t)f * kPps3 + lane;
             if (f < nfills && lane < kPps3 && p < pe) {
                 it = a.idx_t[p];
                 iff = a.idx_f[p];
-                ie = a.idx_e[p];
                 if ((int64_t)it >= a.nT || (int64_t)iff >= a.nF) {
                     atomicOr(a.status, kStBadIndex);
                     it = 0;
@@ -301,40 +303,18 @@ __global__ void __launch_bounds__(kThreads3, 1)
                 }
             }
         };
-        uint32_t it, iff, ie;
-        load_idx(0, it, iff, ie);
-        uint32_t st = 0, ph = 0, mine = 0, e_last = 0;
-        int64_t s = s_first;
-        int seg_end = n > 0 ? (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) : 0;
+        uint32_t it, iff;
+        load_idx(0, it, iff);
+        uint32_t st = 0, ph = 0, mine = 0;
         for (int f = 0; f < nfills; ++f) {
-            uint32_t nit, niff, nie;
-            load_idx(f + 1, nit, niff, nie);
+            uint32_t nit, niff;
+            load_idx(f + 1, nit, niff);
             const int start = f * kPps3;
             const int np = n - start < kPps3 ? n - start : kPps3;
-            // segment starts inside this stage (uniform; rare)
-            uint32_t brk = 0;
-            while (seg_end < start + np) {
-                brk |= 1u << (seg_end - start);
-                ++s;
-                seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
-            }
-            const uint32_t eup = __shfl_up_sync(0xffffffffu, ie, 1);
-            const uint32_t eprev = lane == 0 ? e_last : eup;
-            const bool newg = lane < np && (start + lane == 0 || ie != eprev || ((brk >> lane) & 1u));
-            const uint32_t gmask = __ballot_sync(0xffffffffu, newg) & 0xFu;
-            e_last = __shfl_sync(0xffffffffu, ie, np - 1);
-            uint32_t e4[kPps3];
-#pragma unroll
-            for (int j = 0; j < kPps3; ++j) e4[j] = __shfl_sync(0xffffffffu, ie, j);
             uint32_t okw = 1;
             if (lane == 0) {
                 okw = wait3f(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status) ? 1u : 0u;
-                if (okw) {
-#pragma unroll
-                    for (int j = 0; j < kPps3; ++j) plan[st * (kPps3 + 1) + j] = e4[j];
-                    plan[st * (kPps3 + 1) + kPps3] = gmask | (brk << 8);
-                    arrive_tx(full0 + 8u * st, (uint32_t)np * (kTBytes + kFBytes));
-                }
+                if (okw) arrive_tx(full0 + 8u * st, (uint32_t)np * (kTBytes + kFBytes));
             }
             if (!__shfl_sync(0xffffffffu, okw, 0)) break;
             if (lane < np) {
@@ -354,37 +334,111 @@ __global__ void __launch_bounds__(kThreads3, 1)
             ++mine;
             it = nit;
             iff = niff;
-            ie = nie;
             if (++st == (uint32_t)kStages3) {
                 st = 0;
                 ph ^= 1u;
             }
         }
         if (lane == 0) misc[3] = mine;
+    } else if (warp == 6) {
+        // ---------------------------------------------------- group warp
+        // For each stage, in order: which triples open a group (the E tuple
+        // changes, or a segment starts), close one, end an output key; for
+        // each group opening there, wait until the epilogue has released the
+        // group's accumulator buffer and request its E tile; then post the
+        // plan (planned[st]).  It waits for the stage's previous fill to be
+        // consumed (empty) so that the plan word is free.  No wait here can
+        // deadlock: a stage holds at most four triples, so the group whose
+        // buffer a new group reuses (four groups back) closed in an earlier,
+        // already planned stage.
+        const int nfills = (n + kPps3 - 1) / kPps3;
+        auto load_e = [&](int f) -> uint32_t {
+            const int64_t p = pb + (int64_t)f * kPps3 + lane;
+            return (f < nfills && lane < kPps3 && p < pe) ? a.idx_e[p] : 0u;
+        };
+        uint32_t ie = load_e(0);
+        uint32_t st = 0, ph = 0, e_last = 0, gb = 0, gph = 0, opened = 0;
+        int64_t s = s_first;
+        int seg_end = n > 0 ? (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) : 0;
+        for (int f = 0; f < nfills; ++f) {
+            const uint32_t nie = load_e(f + 1);
+            const int start = f * kPps3;
+            const int np = n - start < kPps3 ? n - start : kPps3;
+            // segment starts inside this stage (uniform; rare)
+            uint32_t brk = 0;
+            while (seg_end < start + np) {
+                brk |= 1u << (seg_end - start);
+                ++s;
+                seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
+            }
+            // a segment (or the unit) ends right after this stage's last triple
+            const bool ends_after = seg_end == start + np;
+            const uint32_t eup = __shfl_up_sync(0xffffffffu, ie, 1);
+            const uint32_t eprev = lane == 0 ? e_last : eup;
+            const bool newg = lane < np && (start + lane == 0 || ie != eprev || ((brk >> lane) & 1u));
+            const uint32_t gmask = __ballot_sync(0xffffffffu, newg) & 0xFu;
+            e_last = __shfl_sync(0xffffffffu, ie, np - 1);
+            const uint32_t e_next = __shfl_sync(0xffffffffu, nie, 0);
+            // close flags: triple j ends its group when triple j + 1 opens one;
+            // the last triple when the next stage's first does (or the unit ends)
+            const uint32_t below = (1u << (np - 1)) - 1u;
+            const bool last_unit = start + np == n;
+            const bool next_new = last_unit || ends_after || e_next != e_last;
+            const uint32_t cmask = ((gmask >> 1) & below) | ((next_new ? 1u : 0u) << (np - 1));
+            const uint32_t emask = ((brk >> 1) & below) | ((last_unit || ends_after ? 1u : 0u) << (np - 1));
+            uint32_t e4[kPps3];
+#pragma unroll
+            for (int j = 0; j < kPps3; ++j) e4[j] = __shfl_sync(0xffffffffu, ie, j);
+            uint32_t okw = 1;
+            if (lane == 0) {
+                okw = wait3f(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status) ? 1u : 0u;
+                for (int j = 0; j < np && okw; ++j) {
+                    if (!((gmask >> j) & 1u)) continue;
+                    if (!wait3f(acce0 + 8u * gb, gph ^ 1u, abort_flag, a.status)) {
+                        okw = 0;
+                        break;
+                    }
+                    uint32_t ei = e4[j];
+                    if ((int64_t)ei >= a.nE) {
+                        atomicOr(a.status, kStBadIndex);
+                        ei = 0;
+                    }
+                    arrive_tx(ef0 + 8u * gb, kEBytes);
+                    tma3d(eslot0 + gb * kEBytes, &tmE, (int)ei, ef0 + 8u * gb);
+                    ++opened;
+                    if (++gb == (uint32_t)kAcc3) {
+                        gb = 0;
+                        gph ^= 1u;
+                    }
+                }
+                if (okw) {
+                    plan[st * (kPps3 + 1) + kPps3] = gmask | (emask << 8) | (cmask << 16);
+                    arrive(planned0 + 8u * st);
+                }
+            }
+            if (!__shfl_sync(0xffffffffu, okw, 0)) break;
+            ie = nie;
+            if (++st == (uint32_t)kStages3) {
+                st = 0;
+                ph ^= 1u;
+            }
+        }
+        if (lane == 0) misc[4] = opened;
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA
-        // One thread issues everything, following the producer's group plan.
-        // A group (a run of triples of one output key with the same E tuple)
-        // accumulates into one TMEM buffer; its first MMA overwrites.
+        // One thread issues everything, following the group warp's plan: a
+        // group accumulates into one TMEM buffer (its first MMA overwrites);
+        // after its last triple the thread posts whether the group ends its
+        // output key and commits the buffer to the epilogue.
         if (lane == 0) {
             const uint64_t adesc = a.a_desc0, bdesc = a.b_desc0;
             const uint32_t idesc = a.idesc;
-            uint32_t b = 0, aph = 0, dcol = tmem, st = 0, ph = 0, consumed = 0, opened = 0;
-            bool open = false, ok = true;
-            // group close: post whether it ends its output key, then hand the
-            // buffer to the epilogue once its MMAs complete
-            auto close_grp = [&](uint32_t ends) {
-                info[2 * b + 1] = ends;
-                arrive(infoc0 + 8u * b);
-                commit(accf0 + 8u * b);
-                if (++b == (uint32_t)kAcc3) {
-                    b = 0;
-                    aph ^= 1u;
-                }
-            };
+            uint32_t b = 0, dcol = tmem, st = 0, ph = 0, consumed = 0;
+            bool ok = true;
             for (int start = 0; start < n; start += kPps3) {
                 const int np = n - start < kPps3 ? n - start : kPps3;
-                if (!wait3f(full0 + 8u * st, ph, abort_flag, a.status)) {
+                if (!wait3f(full0 + 8u * st, ph, abort_flag, a.status) ||
+                    !wait3f(planned0 + 8u * st, ph, abort_flag, a.status)) {
                     ok = false;
                     break;
                 }
@@ -394,25 +448,7 @@ __global__ void __launch_bounds__(kThreads3, 1)
                 const uint64_t bd0 = bdesc + (s0 >> 4), ad0 = adesc + ((s0 + kPps3 * kTBytes + kFBytes) >> 4);
                 for (int jj = 0; jj < np; ++jj) {
                     const bool newgrp = (flags >> jj) & 1u;
-                    if (newgrp) {
-                        if (open) close_grp((flags >> (8 + jj)) & 1u);
-                        if (!wait3f(acce0 + 8u * b, aph ^ 1u, abort_flag, a.status)) {
-                            ok = false;
-                            open = false;
-                            break;
-                        }
-                        fence_after();
-                        uint32_t ei = plan[st * (kPps3 + 1) + jj];
-                        if ((int64_t)ei >= a.nE) {
-                            atomicOr(a.status, kStBadIndex);
-                            ei = 0;
-                        }
-                        arrive_tx(ef0 + 8u * b, kEBytes);
-                        tma3d(eslot0 + b * kEBytes, &tmE, (int)ei, ef0 + 8u * b);
-                        ++opened;
-                        dcol = tmem + b * 128u;
-                        open = true;
-                    }
+                    if (newgrp) dcol = tmem + b * 128u;
                     // F slot jj at (2 jj + 1) blocks; T slot jj at jj tiles
                     const uint64_t ad = ad0 + (uint64_t)(jj * (2 * kFBytes >> 4));
                     const uint64_t bd = bd0 + (uint64_t)(jj * (kTBytes >> 4));
@@ -420,8 +456,13 @@ __global__ void __launch_bounds__(kThreads3, 1)
                     mma(dcol, ad, bd, idesc, newgrp ? 0u : 1u);
                     // x = 1: F^T in M rows 64-127 (zeros above), i in 8..15
                     mma(dcol, ad - (kFBytes >> 4), bd + ((kTBytes / 2) >> 4), idesc, 1u);
+                    if ((flags >> (16 + jj)) & 1u) {
+                        info[2 * b + 1] = (flags >> (8 + jj)) & 1u;
+                        arrive(infoc0 + 8u * b);
+                        commit(accf0 + 8u * b);
+                        if (++b == (uint32_t)kAcc3) b = 0;
+                    }
                 }
-                if (!ok) break;
                 commit(empty0 + 8u * st);
                 ++consumed;
                 if (++st == (uint32_t)kStages3) {
@@ -429,9 +470,7 @@ __global__ void __launch_bounds__(kThreads3, 1)
                     ph ^= 1u;
                 }
             }
-            if (open) close_grp(1u);
             misc[2] = ok ? 0xFFFFFFFFu : consumed;
-            misc[4] = opened;
         }
         __syncwarp();
     } else {
@@ -446,7 +485,7 @@ __global__ void __launch_bounds__(kThreads3, 1)
         int64_t s = s_first;
         const int64_t s_last = n > 0 ? seg_of(a.seg_start, a.S, pe - 1) : s_first - 1;
         while (s <= s_last) {
-            // the group's E tile was requested when the MMA warp opened it
+            // the group's E tile was requested by the group warp when it opened the group
             if (!__all_sync(0xffffffffu, wait3f(ef0 + 8u * b, ph, abort_flag, a.status))) break;
             ++got_e;
             float ef[16];

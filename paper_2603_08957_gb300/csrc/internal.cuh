@@ -241,6 +241,17 @@ void launch_heads(ucl_ctx *ctx, const uint64_t *pk, int64_t P, int64_t *flag, in
 // = first pair of band b, band_seg[b] = its segment index (b = 0..B; B <= 63).
 void launch_band_ranges(ucl_ctx *ctx, const uint64_t *pk, int64_t P, const int64_t *seg_excl, const int64_t *n_seg,
                         int out_bits, int B, int64_t *band_start, int64_t *band_seg);
+// Small binary EinSums: the whole key stage in one CTA (shared memory) with
+// one result read: res[0] = pairs P, res[1] = segments S.  Applies when both
+// inputs have at most kSmallTuples tuples (small_join_fits); when P exceeds
+// kSmallPairs nothing but res[0] is written and the general path runs.
+constexpr int kSmallTuples = 2048;
+constexpr int kSmallPairs = 4096;
+bool small_join_fits(int64_t na, int64_t nb);
+void launch_small_join(ucl_ctx *ctx, const int32_t *keys_a, int ua, int64_t na, const int32_t *keys_b, int ub,
+                       int64_t nb, const KeyPack &join_a, const KeyPack &join_b, const KeyPack &out_a,
+                       const KeyPack &out_b, const KeyUnpack &un, bool has_join, int64_t *res, int64_t *seg_start,
+                       int32_t *out_keys, uint32_t *pu, uint32_t *pvi);
 // Windows: slot[p] = output key & (2^wb - 1) and mask[ws] |= 1 << slot for
 // each pair (flag/excl: window segment heads and their exclusive scan).
 void launch_win_slots(ucl_ctx *ctx, const uint64_t *pk, int64_t P, int wb, const int64_t *flag, const int64_t *excl,

@@ -546,6 +546,204 @@ __global__ void unpack_keys_kernel(const uint64_t *__restrict__ k, int64_t n, Ke
         }
 }
 
+// ------------------------------------------------------------ small join
+// The whole key stage of a small binary EinSum in one CTA of 1024 threads,
+// in shared memory: pack both inputs' keys, join by comparing every A tuple
+// with every B tuple (A in row order, B in row order), expand the pairs,
+// sort them by output key (stable: bitonic on (key, expansion index)), find
+// the segments and write seg_start, the output keys and each pair's rows.
+// res[0] = P (pair count; when above kSmallPairs nothing else is written and
+// the caller runs the general key stage), res[1] = S.
+constexpr int kSmallThreads = 1024;
+
+__device__ __forceinline__ uint64_t pack_col(const int32_t *row, const KeyPack &kp) { return pack_row(row, kp); }
+
+__global__ void __launch_bounds__(kSmallThreads) small_join_kernel(
+    const int32_t *__restrict__ keys_a, int ua, int na, const int32_t *__restrict__ keys_b, int ub, int nb,
+    KeyPack join_a, KeyPack join_b, KeyPack out_a, KeyPack out_b, KeyUnpack un, int has_join, int64_t *res,
+    int64_t *seg_start, int32_t *out_keys, uint32_t *pu, uint32_t *pvi) {
+    extern __shared__ uint64_t sm[];
+    uint64_t *ja = sm, *oa = ja + kSmallTuples, *jb = oa + kSmallTuples, *ob = jb + kSmallTuples;
+    uint64_t *pk = ob + kSmallTuples, *pv = pk + kSmallPairs;
+    uint32_t *ord = reinterpret_cast<uint32_t *>(pv + kSmallPairs);   // expansion index, then scan scratch
+    __shared__ int32_t cnt[kSmallTuples];
+    __shared__ int32_t wsum[kSmallThreads / 32];
+    __shared__ int32_t total;
+    const int tid = threadIdx.x;
+    for (int i = tid; i < na; i += kSmallThreads) {
+        ja[i] = has_join ? pack_col(keys_a + (int64_t)i * ua, join_a) : 0ull;
+        oa[i] = pack_col(keys_a + (int64_t)i * ua, out_a);
+    }
+    for (int i = tid; i < nb; i += kSmallThreads) {
+        jb[i] = has_join ? pack_col(keys_b + (int64_t)i * ub, join_b) : 0ull;
+        ob[i] = pack_col(keys_b + (int64_t)i * ub, out_b);
+    }
+    __syncthreads();
+    // matches per A tuple
+    for (int i = tid; i < na; i += kSmallThreads) {
+        int c = 0;
+        const uint64_t k = ja[i];
+        for (int j = 0; j < nb; ++j) c += jb[j] == k;
+        cnt[i] = c;
+    }
+    __syncthreads();
+    // exclusive scan of cnt[0, na) (na <= 4096: four per thread)
+    {
+        int v[4], run = 0;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int i = tid * 4 + q;
+            v[q] = i < na ? cnt[i] : 0;
+            run += v[q];
+        }
+        int x = run;
+        const int lane = tid & 31, w = tid >> 5;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        if (lane == 31) wsum[w] = x;
+        __syncthreads();
+        if (tid == 0) {
+            int r = 0;
+            for (int q = 0; q < kSmallThreads / 32; ++q) {
+                const int t = wsum[q];
+                wsum[q] = r;
+                r += t;
+            }
+            total = r;
+        }
+        __syncthreads();
+        int base = wsum[w] + x - run;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int i = tid * 4 + q;
+            if (i < na) cnt[i] = base;
+            base += v[q];
+        }
+    }
+    __syncthreads();
+    const int P = total;
+    if (tid == 0) res[0] = P;
+    if (P > kSmallPairs || P == 0) {
+        if (tid == 0) res[1] = 0;
+        return;
+    }
+    // expand: A row order, then B row order
+    for (int i = tid; i < na; i += kSmallThreads) {
+        int o = cnt[i];
+        const uint64_t k = ja[i];
+        for (int j = 0; j < nb; ++j)
+            if (jb[j] == k) {
+                pk[o] = oa[i] | ob[j];
+                pv[o] = ((uint64_t)i << 32) | (uint32_t)j;
+                ord[o] = (uint32_t)o;
+                ++o;
+            }
+    }
+    int n2 = 1;
+    while (n2 < P) n2 <<= 1;
+    for (int i = P + tid; i < n2; i += kSmallThreads) {
+        pk[i] = ~0ull;
+        pv[i] = 0;
+        ord[i] = 0xFFFFFFFFu;
+    }
+    __syncthreads();
+    // bitonic sort by (output key, expansion index): unique, so stable
+    for (int k = 2; k <= n2; k <<= 1)
+        for (int j = k >> 1; j > 0; j >>= 1) {
+            for (int i = tid; i < n2; i += kSmallThreads) {
+                const int l = i ^ j;
+                if (l > i) {
+                    const bool up = (i & k) == 0;
+                    const bool gt = pk[i] > pk[l] || (pk[i] == pk[l] && ord[i] > ord[l]);
+                    if (gt == up) {
+                        uint64_t t = pk[i]; pk[i] = pk[l]; pk[l] = t;
+                        t = pv[i]; pv[i] = pv[l]; pv[l] = t;
+                        const uint32_t u = ord[i]; ord[i] = ord[l]; ord[l] = u;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+    // segment heads and their exclusive scan (reusing ord as scratch)
+    {
+        int v[4], run = 0;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int p = tid * 4 + q;
+            v[q] = p < P && (p == 0 || pk[p] != pk[p - 1]) ? 1 : 0;
+            run += v[q];
+        }
+        int x = run;
+        const int lane = tid & 31, w = tid >> 5;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        __syncthreads();
+        if (lane == 31) wsum[w] = x;
+        __syncthreads();
+        if (tid == 0) {
+            int r = 0;
+            for (int q = 0; q < kSmallThreads / 32; ++q) {
+                const int t = wsum[q];
+                wsum[q] = r;
+                r += t;
+            }
+            total = r;
+        }
+        __syncthreads();
+        int base = wsum[w] + x - run;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int p = tid * 4 + q;
+            if (p < P) {
+                if (v[q]) {
+                    seg_start[base] = p;
+                    const uint64_t key = pk[p];
+                    for (int c = 0; c < un.uw; ++c) {
+                        const uint64_t m = un.bits[c] ? ((~0ull) >> (64 - un.bits[c])) : 0ull;
+                        out_keys[(int64_t)base * un.uw + c] = (int32_t)((key >> un.shift[c]) & m);
+                    }
+                }
+                pu[p] = (uint32_t)(pv[p] >> 32);
+                pvi[p] = (uint32_t)pv[p];
+            }
+            base += v[q];
+        }
+    }
+    __syncthreads();
+    if (tid == 0) {
+        seg_start[total] = P;
+        res[1] = total;
+    }
+}
+
+bool small_join_fits(int64_t na, int64_t nb) {
+    return na >= 1 && nb >= 1 && na <= kSmallTuples && nb <= kSmallTuples && na * nb <= (int64_t)1 << 22;
+}
+
+void launch_small_join(ucl_ctx *ctx, const int32_t *keys_a, int ua, int64_t na, const int32_t *keys_b, int ub,
+                       int64_t nb, const KeyPack &join_a, const KeyPack &join_b, const KeyPack &out_a,
+                       const KeyPack &out_b, const KeyUnpack &un, bool has_join, int64_t *res, int64_t *seg_start,
+                       int32_t *out_keys, uint32_t *pu, uint32_t *pvi) {
+    const size_t smem = sizeof(uint64_t) * (4 * (size_t)kSmallTuples + 2 * (size_t)kSmallPairs) +
+                        sizeof(uint32_t) * (size_t)kSmallPairs;
+    static bool attr[64] = {};   // the attribute is set once per device
+    const int d = ctx->device >= 0 && ctx->device < 64 ? ctx->device : 0;
+    if (!attr[d]) {
+        cudaFuncSetAttribute(small_join_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        attr[d] = true;
+    }
+    small_join_kernel<<<1, kSmallThreads, smem, ctx->stream>>>(keys_a, ua, (int)na, keys_b, ub, (int)nb, join_a,
+                                                                join_b, out_a, out_b, un, has_join ? 1 : 0, res,
+                                                                seg_start, out_keys, pu, pvi);
+    ctx->launches++;
+}
+
 // A-tile runs for the windowed kernel (see internal.cuh, launch_arun).
 __global__ void arun_kernel(const uint32_t *__restrict__ pa, int64_t P, int cap, uint8_t *arun) {
     for (int64_t p = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; p < P; p += (int64_t)gridDim.x * blockDim.x) {

@@ -285,6 +285,30 @@ def test_l2_hints_do_not_change_results(monkeypatch):
     assert torch.equal(outs[0][1], outs[1][1])
 
 
+@pytest.mark.parametrize("na,nb", [(64, 64), (65, 64), (100, 100), (2048, 2), (2049, 2)])
+def test_small_key_stage_and_fallback(ctx, na, nb):
+    """Small binary EinSums run their whole key stage in one CTA (at most
+    2048 tuples per input, 4096 pairs); a cross product just past 4096 pairs,
+    or an input past 2048 tuples, takes the general path.  Both against the
+    oracle; the small path launches far fewer kernels."""
+    rng = np.random.default_rng(na * 7 + nb)
+    a = (np.arange(na, dtype=np.int32)[:, None], (na,), torch.from_numpy(rng.standard_normal((na, 4))).float())
+    b = (np.arange(nb, dtype=np.int32)[:, None], (nb,), torch.from_numpy(rng.standard_normal((nb, 4))).float())
+    out = ctx.einsum("Ii,Ki->IK", gpu_rel(ctx, a), gpu_rel(ctx, b))
+    st = ctx.last_stats()
+    assert_parity(out, oracle_ref("Ii,Ki->IK", [a, b]), torch.float32)
+    small = na * nb <= 4096 and na <= 2048 and nb <= 2048
+    assert (st["launches"] <= 4) == small, st
+    # a join on a shared label, inputs shuffled
+    pa, pb = rng.permutation(na), rng.permutation(nb)
+    ka = np.stack([np.arange(na) % 7, np.arange(na)], 1).astype(np.int32)[pa]
+    kb = np.stack([np.arange(nb) % 7, np.arange(nb)], 1).astype(np.int32)[pb]
+    ra = (ka, (7, na), torch.from_numpy(rng.standard_normal((na, 3, 2))).float())
+    rb = (kb, (7, nb), torch.from_numpy(rng.standard_normal((nb, 3))).float())
+    out = ctx.einsum("JIij,JKi->IKj", gpu_rel(ctx, ra), gpu_rel(ctx, rb))
+    assert_parity(out, oracle_ref("JIij,JKi->IKj", [ra, rb]), torch.float32)
+
+
 def test_spgemm_small(ctx):
     """Block-sparse x block-sparse, 128 x 128 bf16 tiles, band + uniform, fp32 out."""
     w = workloads.spgemm(seed=2, n=8192, density=0.05)
