@@ -241,12 +241,14 @@ void launch_heads(ucl_ctx *ctx, const uint64_t *pk, int64_t P, int64_t *flag, in
 // = first pair of band b, band_seg[b] = its segment index (b = 0..B; B <= 63).
 void launch_band_ranges(ucl_ctx *ctx, const uint64_t *pk, int64_t P, const int64_t *seg_excl, const int64_t *n_seg,
                         int out_bits, int B, int64_t *band_start, int64_t *band_seg);
-// Small binary EinSums: the whole key stage in one CTA (shared memory) with
-// one result read: res[0] = pairs P, res[1] = segments S.  Applies when both
-// inputs have at most kSmallTuples tuples (small_join_fits); when P exceeds
-// kSmallPairs nothing but res[0] is written and the general path runs.
-constexpr int kSmallTuples = 2048;
-constexpr int kSmallPairs = 4096;
+// Small binary EinSums: the whole key stage in one CTA (28 KB of shared
+// memory, so that it still fits beside a running contraction) with one
+// result read: res[0] = pairs P, res[1] = segments S.  Applies when both
+// inputs have at most kSmallTuples tuples and their product is at most 2^16
+// (small_join_fits); when P exceeds kSmallPairs nothing but res[0] is
+// written and the general path runs.
+constexpr int kSmallTuples = 256;
+constexpr int kSmallPairs = 1024;
 bool small_join_fits(int64_t na, int64_t nb);
 void launch_small_join(ucl_ctx *ctx, const int32_t *keys_a, int ua, int64_t na, const int32_t *keys_b, int ub,
                        int64_t nb, const KeyPack &join_a, const KeyPack &join_b, const KeyPack &out_a,

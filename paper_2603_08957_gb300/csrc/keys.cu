@@ -587,7 +587,7 @@ __global__ void __launch_bounds__(kSmallThreads) small_join_kernel(
         cnt[i] = c;
     }
     __syncthreads();
-    // exclusive scan of cnt[0, na) (na <= 4096: four per thread)
+    // exclusive scan of cnt[0, na) (na <= 4 * kSmallThreads: four per thread)
     {
         int v[4], run = 0;
 #pragma unroll
@@ -723,7 +723,7 @@ __global__ void __launch_bounds__(kSmallThreads) small_join_kernel(
 }
 
 bool small_join_fits(int64_t na, int64_t nb) {
-    return na >= 1 && nb >= 1 && na <= kSmallTuples && nb <= kSmallTuples && na * nb <= (int64_t)1 << 22;
+    return na >= 1 && nb >= 1 && na <= kSmallTuples && nb <= kSmallTuples && na * nb <= (int64_t)1 << 16;
 }
 
 void launch_small_join(ucl_ctx *ctx, const int32_t *keys_a, int ua, int64_t na, const int32_t *keys_b, int ub,

@@ -285,11 +285,11 @@ def test_l2_hints_do_not_change_results(monkeypatch):
     assert torch.equal(outs[0][1], outs[1][1])
 
 
-@pytest.mark.parametrize("na,nb", [(64, 64), (65, 64), (100, 100), (2048, 2), (2049, 2)])
+@pytest.mark.parametrize("na,nb", [(32, 32), (33, 32), (100, 100), (256, 2), (257, 2)])
 def test_small_key_stage_and_fallback(ctx, na, nb):
     """Small binary EinSums run their whole key stage in one CTA (at most
-    2048 tuples per input, 4096 pairs); a cross product just past 4096 pairs,
-    or an input past 2048 tuples, takes the general path.  Both against the
+    256 tuples per input, 1024 pairs); a cross product just past 1024 pairs,
+    or an input past 256 tuples, takes the general path.  Both against the
     oracle; the small path launches far fewer kernels."""
     rng = np.random.default_rng(na * 7 + nb)
     a = (np.arange(na, dtype=np.int32)[:, None], (na,), torch.from_numpy(rng.standard_normal((na, 4))).float())
@@ -297,7 +297,7 @@ def test_small_key_stage_and_fallback(ctx, na, nb):
     out = ctx.einsum("Ii,Ki->IK", gpu_rel(ctx, a), gpu_rel(ctx, b))
     st = ctx.last_stats()
     assert_parity(out, oracle_ref("Ii,Ki->IK", [a, b]), torch.float32)
-    small = na * nb <= 4096 and na <= 2048 and nb <= 2048
+    small = na * nb <= 1024 and na <= 256 and nb <= 256
     assert (st["launches"] <= 4) == small, st
     # a join on a shared label, inputs shuffled
     pa, pb = rng.permutation(na), rng.permutation(nb)
