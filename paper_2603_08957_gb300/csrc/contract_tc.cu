@@ -940,7 +940,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if (pos < n) seg_end = (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb);
             fresh = true;
         };
-        uint32_t st = 0, ph = 0;
+        uint32_t st = 0, ph = 0, pmask = 0;   // pmask: stages whose release waits for a later fill
         int f = 0;
         for (; f * pps < n; ++f) {
             const int start = f * pps;
@@ -950,37 +950,74 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 break;
             }
             tc_fence_after();
-            for (int jj = 0; jj < np; ++jj) {
-                if (fresh && !open_seg()) {
-                    ok = false;
-                    break;
-                }
-                const uint32_t info = pinfo[st * 4 + jj];
-                const uint32_t d = dcol + (info & 0xFFu) * acc_cols;
-                const uint64_t ad = adesc0 + ((info >> 8) & 0xFFu) * stage16 + ((info >> 16) & 0xFFu) * apair16;
-                const uint64_t bd = bdesc0 + st * stage16 + (uint32_t)jj * bpair16;
-                if (elect_one()) {
+            uint32_t info[4];
 #pragma unroll
-                    for (int kk = 0; kk < KSTEPS; ++kk) {
-                        mma_bf16(d, ad + aoff[kk], bd + boff[kk], idesc, 1u);
-                        if (two_m) mma_bf16(d + ncol, ad + aoff[kk] + mb16, bd + boff[kk], idesc, 1u);
+            for (int jj = 0; jj < 4; ++jj) info[jj] = jj < np ? pinfo[st * 4 + jj] : 0u;
+            const int rel_st = prel[st];
+            const uint64_t bd0 = bdesc0 + st * stage16;
+            if (!fresh && start + np <= seg_end) {
+                // the whole fill accumulates into the open window: one
+                // elected region issues every pair and, unless a later pair
+                // still reads an A tile here, releases the stage
+                if (elect_one()) {
+                    for (int jj = 0; jj < np; ++jj) {
+                        const uint32_t d = dcol + (info[jj] & 0xFFu) * acc_cols;
+                        const uint64_t ad = adesc0 + ((info[jj] >> 8) & 0xFFu) * stage16 +
+                                            ((info[jj] >> 16) & 0xFFu) * apair16;
+                        const uint64_t bd = bd0 + (uint32_t)jj * bpair16;
+#pragma unroll
+                        for (int kk = 0; kk < KSTEPS; ++kk) {
+                            mma_bf16(d, ad + aoff[kk], bd + boff[kk], idesc, 1u);
+                            if (two_m) mma_bf16(d + ncol, ad + aoff[kk] + mb16, bd + boff[kk], idesc, 1u);
+                        }
                     }
+                    if (rel_st == f) mma_commit(empty0 + 8u * st);
                 }
                 __syncwarp();
-                if (start + jj + 1 == seg_end) close_seg(start + jj + 1);
-            }
-            if (!ok) break;
-            const int rel_st = prel[st];
+                if (start + np == seg_end) close_seg(seg_end);
+            } else {
+                // window boundaries inside the fill: pair by pair
+                for (int jj = 0; jj < np; ++jj) {
+                    if (fresh && !open_seg()) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t d = dcol + (info[jj] & 0xFFu) * acc_cols;
+                    const uint64_t ad = adesc0 + ((info[jj] >> 8) & 0xFFu) * stage16 +
+                                        ((info[jj] >> 16) & 0xFFu) * apair16;
+                    const uint64_t bd = bd0 + (uint32_t)jj * bpair16;
+                    if (elect_one()) {
 #pragma unroll
-            for (int i = 0; i < kMaxStages; ++i)   // constant indices: pend stays in registers
-                if (i == (int)st) pend[i] = rel_st;
-#pragma unroll
-            for (int i = 0; i < kMaxStages; ++i)
-                if (pend[i] == f) {
-                    if (elect_one()) mma_commit(empty0 + 8u * i);
+                        for (int kk = 0; kk < KSTEPS; ++kk) {
+                            mma_bf16(d, ad + aoff[kk], bd + boff[kk], idesc, 1u);
+                            if (two_m) mma_bf16(d + ncol, ad + aoff[kk] + mb16, bd + boff[kk], idesc, 1u);
+                        }
+                    }
                     __syncwarp();
-                    pend[i] = -1;
+                    if (start + jj + 1 == seg_end) close_seg(start + jj + 1);
                 }
+                if (!ok) break;
+                if (rel_st == f) {
+                    if (elect_one()) mma_commit(empty0 + 8u * st);
+                    __syncwarp();
+                }
+            }
+            if (rel_st != f) {
+                // a later pair reads an A tile loaded here: release after that fill
+#pragma unroll
+                for (int i = 0; i < kMaxStages; ++i)   // constant indices: pend stays in registers
+                    if (i == (int)st) pend[i] = rel_st;
+                pmask |= 1u << st;
+            }
+            if (pmask) {
+#pragma unroll
+                for (int i = 0; i < kMaxStages; ++i)
+                    if (((pmask >> i) & 1u) && pend[i] == f) {
+                        if (elect_one()) mma_commit(empty0 + 8u * i);
+                        __syncwarp();
+                        pmask &= ~(1u << i);
+                    }
+            }
             if (++st == (uint32_t)a.ns) {
                 st = 0;
                 ph ^= 1u;

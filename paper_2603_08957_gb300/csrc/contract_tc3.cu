@@ -32,7 +32,9 @@
 //               or end an output key; for each group opening there it waits
 //               until the epilogue has released the group's accumulator
 //               buffer and requests the group's E tile by TMA into that
-//               buffer's E slot; then it posts the stage's plan;
+//               buffer's E slot; for each group closing there it posts to the
+//               epilogue whether the group ends its output key; then it posts
+//               the stage's plan;
 //   warp 1      MMA issuer (owns TMEM): one thread issues two tcgen05.mma per
 //               triple into the group's accumulator buffer, following the
 //               plan, and commits a group's buffer after its last triple;
@@ -357,7 +359,7 @@ __global__ void __launch_bounds__(kThreads3, 1)
             return (f < nfills && lane < kPps3 && p < pe) ? a.idx_e[p] : 0u;
         };
         uint32_t ie = load_e(0);
-        uint32_t st = 0, ph = 0, e_last = 0, gb = 0, gph = 0, opened = 0;
+        uint32_t st = 0, ph = 0, e_last = 0, gb = 0, gph = 0, opened = 0, cb = 0;
         int64_t s = s_first;
         int seg_end = n > 0 ? (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) : 0;
         for (int f = 0; f < nfills; ++f) {
@@ -393,22 +395,30 @@ __global__ void __launch_bounds__(kThreads3, 1)
             if (lane == 0) {
                 okw = wait3f(empty0 + 8u * st, ph ^ 1u, abort_flag, a.status) ? 1u : 0u;
                 for (int j = 0; j < np && okw; ++j) {
-                    if (!((gmask >> j) & 1u)) continue;
-                    if (!wait3f(acce0 + 8u * gb, gph ^ 1u, abort_flag, a.status)) {
-                        okw = 0;
-                        break;
+                    if ((gmask >> j) & 1u) {
+                        if (!wait3f(acce0 + 8u * gb, gph ^ 1u, abort_flag, a.status)) {
+                            okw = 0;
+                            break;
+                        }
+                        uint32_t ei = e4[j];
+                        if ((int64_t)ei >= a.nE) {
+                            atomicOr(a.status, kStBadIndex);
+                            ei = 0;
+                        }
+                        arrive_tx(ef0 + 8u * gb, kEBytes);
+                        tma3d(eslot0 + gb * kEBytes, &tmE, (int)ei, ef0 + 8u * gb);
+                        ++opened;
+                        if (++gb == (uint32_t)kAcc3) {
+                            gb = 0;
+                            gph ^= 1u;
+                        }
                     }
-                    uint32_t ei = e4[j];
-                    if ((int64_t)ei >= a.nE) {
-                        atomicOr(a.status, kStBadIndex);
-                        ei = 0;
-                    }
-                    arrive_tx(ef0 + 8u * gb, kEBytes);
-                    tma3d(eslot0 + gb * kEBytes, &tmE, (int)ei, ef0 + 8u * gb);
-                    ++opened;
-                    if (++gb == (uint32_t)kAcc3) {
-                        gb = 0;
-                        gph ^= 1u;
+                    if ((cmask >> j) & 1u) {
+                        // the group ends after triple j: tell the epilogue
+                        // whether it also ends its output key
+                        info[2 * cb + 1] = (emask >> j) & 1u;
+                        arrive(infoc0 + 8u * cb);
+                        if (++cb == (uint32_t)kAcc3) cb = 0;
                     }
                 }
                 if (okw) {
@@ -428,8 +438,9 @@ __global__ void __launch_bounds__(kThreads3, 1)
         // ------------------------------------------------------------ MMA
         // One thread issues everything, following the group warp's plan: a
         // group accumulates into one TMEM buffer (its first MMA overwrites);
-        // after its last triple the thread posts whether the group ends its
-        // output key and commits the buffer to the epilogue.
+        // after its last triple the thread commits the buffer to the
+        // epilogue (the group warp has already posted whether the group ends
+        // its output key).
         if (lane == 0) {
             const uint64_t adesc = a.a_desc0, bdesc = a.b_desc0;
             const uint32_t idesc = a.idesc;
@@ -457,8 +468,6 @@ __global__ void __launch_bounds__(kThreads3, 1)
                     // x = 1: F^T in M rows 64-127 (zeros above), i in 8..15
                     mma(dcol, ad - (kFBytes >> 4), bd + ((kTBytes / 2) >> 4), idesc, 1u);
                     if ((flags >> (16 + jj)) & 1u) {
-                        info[2 * b + 1] = (flags >> (8 + jj)) & 1u;
-                        arrive(infoc0 + 8u * b);
                         commit(accf0 + 8u * b);
                         if (++b == (uint32_t)kAcc3) b = 0;
                     }
