@@ -743,6 +743,7 @@ ucl_status ucl_ctx_create(int device, void *stream, ucl_alloc_fn alloc, ucl_free
     if (const char *e = getenv("UCL_BANDS")) ctx->tune_bands = atoi(e);
     if (const char *e = getenv("UCL_L2_HINTS")) ctx->tune_hints = atoi(e);
     if (const char *e = getenv("UCL_TC_STAGES")) ctx->tune_tc_stages = atoi(e);
+    if (const char *e = getenv("UCL_TC_MMA")) ctx->tune_tc_mma = atoi(e);
     if (const char *e = getenv("UCL_TC_PREFETCH")) ctx->tune_tc_prefetch = atoi(e);
     if (const char *e = getenv("UCL_WINDOW")) ctx->tune_window = atoi(e);
     if (!st) st = cuda_check(ctx, cudaMalloc(&ctx->d_status, 256), "cudaMalloc status");

@@ -257,6 +257,30 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float *v) {
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// A role's position in the ring: fill number f, its stage and the parity of
+// its lap.  A role that owns the stages role, role + step, ... (< ns) moves
+// to its next own fill without a division.
+struct StageCursor {
+    int f;
+    uint32_t st, ph;
+    __device__ __forceinline__ void start(int role) {
+        f = role;
+        st = (uint32_t)role;
+        ph = 0;
+    }
+    __device__ __forceinline__ void next(int role, int step, uint32_t ns) {
+        const uint32_t nx = st + (uint32_t)step;
+        if (nx < ns) {
+            f += step;
+            st = nx;
+        } else {
+            f += (int)(ns - st) + role;
+            st = (uint32_t)role;
+            ph ^= 1u;
+        }
+    }
+};
+
 __device__ __forceinline__ int64_t find_seg(const int64_t *seg_start, int64_t S, int64_t p) {
     int64_t a = 0, b = S;
     while (a < b) {
@@ -776,14 +800,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
     if (warp < kProducers) {
         // ------------------------------------------------------ producers
-        // Producer w fills stages w, w + 2, ...; lane j takes pair j of the
-        // fill.  Each pair's A source comes from arun: its loader is the pair
-        // arun's low nibble back, or the unit's first pair if that is later.
+        // Producer w fills the stages s with s mod kProducers == w, in fill
+        // order (so each empty-barrier wait is for the release of that
+        // stage's previous fill, although held stages are released out of
+        // fill order); lane j takes pair j of the fill.  Each pair's A source
+        // comes from arun: its loader is the pair arun's low nibble back, or
+        // the unit's first pair if that is later.
         const int n = (int)(pe - pb), pps = a.pps;
         const int nfills = (n + pps - 1) / pps;
         const uint64_t pol_a = a.hint_a ? policy_of(a.hint_a) : 0ull, pol_b = a.hint_b ? policy_of(a.hint_b) : 0ull;
         uint32_t mine = 0;
-        uint32_t st = (uint32_t)(warp % a.ns), ph = (uint32_t)((warp / a.ns) & 1);
+        const uint32_t ns_u = (uint32_t)a.ns;
         // per-pair words loaded two own fills ahead (as in the plain kernel),
         // so that a fill never waits on the latency of its own index loads
         struct PairWords {
@@ -801,20 +828,23 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             return w;
         };
-        PairWords w0 = load_words(warp), w1 = load_words(warp + kProducers);
-        for (int f = warp; f < nfills; f += kProducers) {
-            const PairWords w2 = load_words(f + 2 * kProducers);
+        StageCursor c0, c1, c2;   // this fill and the next two own fills
+        c0.start(warp);
+        c1 = c0;
+        c1.next(warp, kProducers, ns_u);
+        c2 = c1;
+        c2.next(warp, kProducers, ns_u);
+        PairWords w0 = load_words(c0.f), w1 = load_words(c1.f);
+        for (; c0.f < nfills; c0 = c1, c1 = c2, c2.next(warp, kProducers, ns_u)) {
+            const int f = c0.f;
+            const uint32_t st = c0.st, ph = c0.ph;
+            const PairWords w2 = load_words(c2.f);
             const PairWords cur = w0;
             w0 = w1;
             w1 = w2;
             if (f == a.withhold_fill) {
                 // failure-detection test: this fill is neither posted nor copied
                 ++mine;
-                st += kProducers;
-                if (st >= (uint32_t)a.ns) {
-                    st -= (uint32_t)a.ns;
-                    ph ^= 1u;
-                }
                 continue;
             }
             const int np = n - f * pps < pps ? n - f * pps : pps;
@@ -890,11 +920,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             __syncwarp();
             ++mine;
-            st += kProducers;
-            if (st >= (uint32_t)a.ns) {
-                st -= (uint32_t)a.ns;
-                ph ^= 1u;
-            }
         }
         if (lane == 0) misc[4 + warp] = mine;
     } else if (warp == kProducers) {
@@ -1107,8 +1132,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     __syncthreads();
     if (*abort_flag) {
         if (warp < kProducers && lane == 0) {
-            for (uint32_t k = 0; k < misc[4 + warp]; ++k) {
-                const uint32_t it = (uint32_t)warp + k * kProducers;
+            // (the fills of this producer's stages, in fill order)
+            for (uint32_t it = 0, k = 0; k < misc[4 + warp]; ++it) {
+                if ((int)((it % (uint32_t)a.ns) % (uint32_t)kProducers) != warp) continue;
+                ++k;
                 if ((int)it == a.withhold_fill) continue;   // never copied: nothing in flight
                 if (it >= misc[2]) mbar_drain(full0 + 8u * (it % a.ns), (it / a.ns) & 1u);
             }
@@ -1187,8 +1214,9 @@ struct TcGeometry {
 // Ring of stages: whole pairs (kc = 1) when at least four stages of one pair
 // fit, else the fewest K chunks per pair that leave four.  With whole pairs, a
 // stage holds pps pairs (1..4): the largest pps that keeps a stage within
-// 72 KB and leaves an even number (>= 4) of stages.
-bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_override = 0, int ns_force = 0) {
+// 72 KB and leaves at least four stages.
+bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_override = 0, int ns_force = 0,
+              int mma_force = 0) {
     const uint32_t bar_bytes = kBarBytes;
     const uint32_t avail = kSmemLimit - 1024 - bar_bytes;
     bool found = false;
@@ -1239,7 +1267,15 @@ bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_overrid
     // the same warp, or a warp could wait on a stage's full barrier while the
     // other warp's older fill of that stage is still pending and the parity
     // test would pass a phase early.  An even ring guarantees it.  One MMA
-    // warp consumes in order and is safe with any ring size.
+    // warp consumes in order and is safe with any ring size.  The producers
+    // take alternate fills too, and the same two cases keep their
+    // empty-barrier waits exact: with an even ring every fill of a stage
+    // comes from one producer, and one MMA warp releases stages in fill
+    // order.  (Two MMA warps on an odd ring would release stages out of
+    // order while consecutive fills of a stage come from different
+    // producers, so a producer could pass a stage's empty barrier two phases
+    // early.  Stage-owned producers fix that, but split an odd ring unevenly
+    // between them and measured slower.)
     const bool two_fit = 512 / (2 * acc_cols) >= 2;
     if (ns_force > 0) {
         // a stage count chosen by the caller: two MMA warps only on an even ring
@@ -1259,6 +1295,7 @@ bool geometry(const TcPlan &tp, TcGeometry *g, std::string *why, int pps_overrid
     } else {
         g->nmma = 1;
     }
+    if (mma_force == 1) g->nmma = 1;   // caller's choice: one MMA warp (any ring)
     g->ns = ns;
     const int buf = acc_cols * g->nmma;
     g->nacc = 512 / buf < kMaxAcc ? 512 / buf : kMaxAcc;
@@ -1393,7 +1430,7 @@ ucl_status launch_contract_tc(ucl_ctx *ctx, const ContractArgs &a, const TcPlan 
     if (a.win_bits > 0) {
         if (!window_geometry(tp, a.win_bits, &g, &cap, &why)) return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why);
         if (cap != a.share_cap) return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: run cap disagrees with the key stage");
-    } else if (!geometry(tp, &g, &why, 0, ctx->tune_tc_stages)) {
+    } else if (!geometry(tp, &g, &why, 0, ctx->tune_tc_stages, ctx->tune_tc_mma)) {
         return fail(ctx, UCL_ERR_UNSUPPORTED, "tcgen05 path: " + why);
     }
     CUtensorMap mA, mB;

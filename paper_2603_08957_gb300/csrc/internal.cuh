@@ -163,9 +163,11 @@ struct ucl_ctx {
     int tune_bands = -1;
     int tune_hints = 1;
     // UCL_TC_STAGES (pipeline stages of the binary tcgen05 kernel, 0: its own
-    // choice) and UCL_TC_PREFETCH (-1: its own rule; 0: no L2 prefetch; 1:
-    // prefetch the streamed operand)
+    // choice), UCL_TC_MMA (1: one MMA warp; 0: its own choice) and
+    // UCL_TC_PREFETCH (-1: its own rule; 0: no L2 prefetch; 1: prefetch the
+    // streamed operand)
     int tune_tc_stages = 0;
+    int tune_tc_mma = 0;
     int tune_tc_prefetch = -1;
     // UCL_WINDOW (-1 or unset: automatic; 0: no windows; n: windows of 2^n
     // output keys where the windowed tcgen05 kernel applies)
