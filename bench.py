@@ -331,26 +331,32 @@ WORKLOADS = {"gnn": GnnChain, "repart": Repart, "blocksparse": Blocksparse, "mtt
 
 
 def contract_traffic(kernel_file, workload, units):
-    """DRAM bytes of one contraction launch, scaled by `units` (joined tuples)
-    from an ncu capture summarised in profiles/<kernel>_traffic.txt; None if
-    there is no capture for this workload or the kernel source changed since."""
+    """DRAM bytes of one contraction, scaled by `units` (joined tuples) from an
+    ncu capture summarised in profiles/<kernel>_traffic.txt; None if there is
+    no capture for this workload or the kernel source changed since.  The file
+    holds one block per workload, each opened by its `workload:` line."""
     import hashlib
     p = os.path.join(ROOT, "profiles", f"{kernel_file}_traffic.txt")
     src = os.path.join(ROOT, "paper_2603_08957_gb300", "csrc", f"{kernel_file}.cu")
     if not os.path.exists(p) or not os.path.exists(src):
         return None
-    kv = {}
+    blocks, kv = [], None
     for line in open(p):
         line = line.split("#", 1)[0].strip()
-        if ":" in line:
-            k, v = line.split(":", 1)
-            kv[k.strip()] = v.strip()
-    if hashlib.sha256(open(src, "rb").read()).hexdigest() != kv.get("source_sha256"):
-        return None
-    if kv.get("workload", "gnn") != workload:
-        return None
-    per = (int(kv["dram_read_bytes"]) + int(kv["dram_write_bytes"])) / int(kv["pairs"])
-    return per * units
+        if ":" not in line:
+            continue
+        k, v = (x.strip() for x in line.split(":", 1))
+        if k == "workload":
+            kv = {}
+            blocks.append(kv)
+        if kv is not None:
+            kv[k] = v
+    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
+    for kv in blocks:
+        if kv.get("workload") == workload and kv.get("source_sha256") == sha:
+            per = (int(kv["dram_read_bytes"]) + int(kv["dram_write_bytes"])) / int(kv["pairs"])
+            return per * units
+    return None
 
 
 def peaks():
