@@ -41,23 +41,35 @@ def oracle_ref(spec, rels, *, epi="none", scale=1.0, sample_keys=None, **ext):
     return oracle.einsum(spec, ins, epi=epi, scale=scale, out_dtype="f64", sample_keys=sample_keys, **ext)
 
 
+def _widen(t):
+    """Tile array as sent to a worker: bf16 travels as its raw 16-bit
+    patterns (half the bytes) and is widened exactly here."""
+    if isinstance(t, tuple) and t[0] == "bf16":
+        return (t[1].astype(np.uint16).astype(np.uint32) << 16).view(np.float32)
+    return t
+
+
 def _oracle_task(task):
     spec, rels, kw = task
-    return oracle.einsum(spec, rels, out_dtype="f64", **kw)
+    return oracle.einsum(spec, [(k, b, _widen(t)) for k, b, t in rels], out_dtype="f64", **kw)
+
+
+def _to_worker(t):
+    if torch.is_tensor(t) and t.dtype == torch.bfloat16:
+        return ("bf16", t.detach().contiguous().view(torch.int16).cpu().numpy())
+    return t.detach().to("cpu", torch.float32).numpy() if torch.is_tensor(t) else np.asarray(t, np.float32)
 
 
 def oracle_parallel(tasks):
     """oracle_ref for several independent (spec, rels, kwargs) tasks at once,
     one spawned process each (never a fork of a process holding a CUDA
-    context).  Tiles are passed as float32 arrays (bf16 and fp32 inputs are
+    context).  Tiles reach the oracle as float32 (bf16 and fp32 inputs are
     exact in float32); results come back in task order."""
     import multiprocessing as mpc
     import os
     conv = []
     for spec, rels, kw in tasks:
-        ins = [(np.asarray(k), tuple(int(x) for x in b),
-                t.detach().to("cpu", torch.float32).numpy() if torch.is_tensor(t) else np.asarray(t, np.float32))
-               for k, b, t in rels]
+        ins = [(np.asarray(k), tuple(int(x) for x in b), _to_worker(t)) for k, b, t in rels]
         conv.append((spec, ins, kw))
     n = max(1, min(len(conv), os.cpu_count() or 1))
     with mpc.get_context("spawn").Pool(n) as pool:

@@ -1,0 +1,130 @@
+"""Full-size value parity on 512 seeded output keys for the two largest
+workloads: the three-input MTTKRP (a 100000^3 tensor with 1e7 Zipf(1.1)
+nonzeros) and both message-passing EinSums of the two-layer GNN (2M
+vertices / 40M drawn edges).  The tests in test_gpu_parity.py check the whole
+key sets and the keys whose sums cross work units and bands; these check
+values on many keys.
+
+Keys are drawn uniformly, with a fixed seed, from the keys whose segment
+holds at most a cap of joined tuples (5000 triples, 1000 pairs: 98.6 % and
+88 % of the keys).  The rest is a long tail whose oracle time per key runs to
+minutes.  The keys are split into 16 groups, and each group is one spawned
+oracle process that gets exactly the tuples its keys join with."""
+import numpy as np
+import pytest
+import torch
+
+import workloads
+from paper_2603_08957_gb300 import Context
+from tests.parity import check_values, gpu_rel, oracle_parallel
+
+pytestmark = pytest.mark.gpu
+
+N_KEYS = 512
+GROUPS = 16
+
+
+@pytest.fixture(scope="module")
+def ctx():
+    c = Context(0)
+    yield c
+    c.close()
+
+
+def _pick(seed, cnt, cap):
+    """N_KEYS distinct keys among those with 1..cap tuples, ascending."""
+    pool = np.nonzero((cnt > 0) & (cnt <= cap))[0]
+    assert len(pool) >= N_KEYS
+    return np.sort(np.random.default_rng(seed).choice(pool, size=N_KEYS, replace=False))
+
+
+def _check_groups(out, groups, refs):
+    """Download the output once; each group's oracle result holds exactly
+    its keys, ascending."""
+    keys, tiles = out.download()
+    k0 = keys[:, 0]
+    checked = 0
+    for g, ref in zip(groups, refs):
+        idx = np.searchsorted(k0, g)
+        assert np.array_equal(keys[idx], ref["keys"]), "sampled keys differ"
+        gv = tiles[torch.as_tensor(idx)].to(torch.float64).numpy()
+        check_values(gv, ref["out"], ref["abs"], torch.bfloat16, out.dtype == torch.bfloat16)
+        checked += len(g)
+    return checked
+
+
+def test_mttkrp_full_size_512_keys(ctx):
+    w = workloads.mttkrp(seed=0, device="cuda")
+    dev = torch.device("cuda", 0)
+    rels = [gpu_rel(ctx, w[k]) for k in ("T", "B", "C")]
+    out = ctx.einsum(w["spec"], *rels)
+    kt = w["T"][0]
+    assert np.all(np.diff(kt[:, 0]) >= 0)   # T tuples ascend by I: key i holds rows [pre[i], pre[i + 1])
+    cnt = np.bincount(kt[:, 0])
+    pre = np.concatenate([[0], np.cumsum(cnt)])
+    keys = _pick(512, cnt, 5000)
+    groups = np.array_split(keys, GROUPS)
+
+    def factor_rows(f, rows):
+        rows = np.unique(rows)
+        return (rows[:, None].astype(np.int32), f[1], f[2][torch.as_tensor(rows, device=dev)])
+
+    tasks = []
+    for g in groups:
+        rows = np.concatenate([np.arange(pre[k], pre[k + 1]) for k in g])
+        tsub = (kt[rows], w["T"][1], w["T"][2][torch.as_tensor(rows, device=dev)])
+        tasks.append((w["spec"], [tsub, factor_rows(w["B"], kt[rows, 1]), factor_rows(w["C"], kt[rows, 2])],
+                      {"sample_keys": g[:, None].astype(np.int32)}))
+    assert _check_groups(out, groups, oracle_parallel(tasks)) == N_KEYS
+    for r in rels + [out]:
+        r.destroy()
+    del w, tasks
+    torch.cuda.empty_cache()
+
+
+def test_two_layer_gnn_full_size_512_keys(ctx):
+    """T1 = (X Y)^T on 512 keys; then, stage-locally from the computed H1 =
+    relu(T1 W1), T2 = (H1 Y)^T on those of the 512 keys it produces."""
+    w = workloads.gnn_two_layer(seed=0)
+    dev = torch.device("cuda", 0)
+    X, Y, W1 = (gpu_rel(ctx, w[k]) for k in ("X", "Y", "W1"))
+    ky = w["Y"][0]
+    cnt = np.bincount(ky[:, 1])
+    keys = _pick(513, cnt, 1000)
+    groups = np.array_split(keys, GROUPS)
+    yrows = [np.nonzero(np.isin(ky[:, 1], g))[0] for g in groups]
+
+    T1 = ctx.einsum(w["spec1"], X, Y, out_dtype="bf16")
+    assert ctx.last_stats()["n_bands"] > 1   # the banded path at full size
+    tasks = []
+    for g, rows in zip(groups, yrows):
+        jn = np.unique(ky[rows, 0])
+        xrel = (jn[:, None].astype(np.int32), w["X"][1], w["X"][2][torch.as_tensor(jn, device=dev)])
+        yrel = (ky[rows], w["Y"][1], w["Y"][2][torch.as_tensor(rows, device=dev)])
+        tasks.append((w["spec1"], [xrel, yrel], {"sample_keys": g[:, None].astype(np.int32)}))
+    assert _check_groups(T1, groups, oracle_parallel(tasks)) == N_KEYS
+    del tasks
+
+    H1 = ctx.einsum(w["spec2"], T1, W1, out_dtype="bf16", epi="relu")
+    T2 = ctx.einsum(w["spec3"], H1, Y, out_dtype="bf16")
+    hk, ht = H1.device_tensors()
+    hk0 = hk[:, 0].cpu().numpy()
+    k2 = T2.device_tensors()[0][:, 0].cpu().numpy()
+    groups2, tasks = [], []
+    for g, rows in zip(groups, yrows):
+        keep = rows[np.isin(ky[rows, 0], hk0)]   # only sources that H1 holds
+        g2 = g[np.isin(g, k2)]
+        assert np.array_equal(g2, np.unique(ky[keep, 1]))
+        if len(g2) == 0:
+            continue
+        jn = np.unique(ky[keep, 0])
+        hrel = (jn[:, None].astype(np.int32), H1.bounds, ht[torch.as_tensor(np.searchsorted(hk0, jn), device=dev)])
+        yrel = (ky[keep], w["Y"][1], w["Y"][2][torch.as_tensor(keep, device=dev)])
+        tasks.append((w["spec3"], [hrel, yrel], {"sample_keys": g2[:, None].astype(np.int32)}))
+        groups2.append(g2)
+    n2 = _check_groups(T2, groups2, oracle_parallel(tasks))
+    assert n2 >= 0.9 * N_KEYS, n2
+    for r in (X, Y, W1, T1, H1, T2):
+        r.destroy()
+    del w, tasks
+    torch.cuda.empty_cache()

@@ -87,3 +87,33 @@ def test_bf16_cast_term_is_the_unit_roundoff():
         check_values(np.array([cast - 2.0**-14]), want, mag, torch.float32, True)
     with pytest.raises(AssertionError):   # no cast term for an fp32 output
         check_values(np.array([cast]), want, mag, torch.float32, False)
+
+
+def test_bf16_reaches_oracle_workers_exactly():
+    """bf16 tiles travel to the oracle workers as raw 16-bit patterns and are
+    widened there: every pattern (signed zeros, infinities, NaN, subnormals)
+    must come out equal to torch's own bf16 -> float32 conversion."""
+    from tests.parity import _to_worker, _widen
+    bits = torch.arange(-32768, 32768, dtype=torch.int32).to(torch.int16)
+    t = bits.view(torch.bfloat16)
+    got = _widen(_to_worker(t))
+    want = t.float().numpy()
+    assert got.dtype == np.float32
+    assert np.array_equal(got.view(np.uint32), want.view(np.uint32))
+
+
+def test_oracle_parallel_matches_oracle_ref():
+    """The spawned-pool path gives the same oracle result as a direct call,
+    for bf16 and fp32 tiles, with sampled keys."""
+    from tests.parity import oracle_parallel, oracle_ref
+    g = torch.Generator().manual_seed(2)
+    ka = np.array([[0, 0], [0, 1], [1, 1], [2, 0]], np.int32)
+    kb = np.array([[0, 0], [1, 0], [1, 2]], np.int32)
+    ta = torch.randn((4, 4, 3), generator=g).to(torch.bfloat16)
+    tb = torch.randn((3, 3, 5), generator=g)
+    rels = [(ka, (3, 2), ta), (kb, (2, 3), tb)]
+    spec = "IiJj,JjKk->IiKk"
+    direct = oracle_ref(spec, rels, sample_keys=np.array([[0, 0], [2, 2]], np.int32))
+    (pooled,) = oracle_parallel([(spec, rels, {"sample_keys": np.array([[0, 0], [2, 2]], np.int32)})])
+    assert np.array_equal(direct["keys"], pooled["keys"])
+    assert np.array_equal(direct["out"], pooled["out"]) and np.array_equal(direct["abs"], pooled["abs"])
