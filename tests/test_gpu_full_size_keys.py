@@ -1,15 +1,19 @@
-"""Full-size value parity on 512 seeded output keys for the two largest
-workloads: the three-input MTTKRP (a 100000^3 tensor with 1e7 Zipf(1.1)
-nonzeros) and both message-passing EinSums of the two-layer GNN (2M
-vertices / 40M drawn edges).  The tests in test_gpu_parity.py check the whole
-key sets and the keys whose sums cross work units and bands; these check
-values on many keys.
+"""Full-size value parity on many output keys.
 
-Keys are drawn uniformly, with a fixed seed, from the keys whose segment
-holds at most a cap of joined tuples (5000 triples, 1000 pairs: 98.6 % and
-88 % of the keys).  The rest is a long tail whose oracle time per key runs to
-minutes.  The keys are split into 16 groups, and each group is one spawned
-oracle process that gets exactly the tuples its keys join with."""
+* Config 2 (GNN message passing, 100000 vertices, 358k Y tiles) and config 4
+  (SpGEMM, 65536^2 at 0.5 %): values on every output key, both EinSums of
+  the chain.
+* The three-input MTTKRP (a 100000^3 tensor with 1e7 Zipf(1.1) nonzeros) and
+  both message-passing EinSums of the two-layer GNN (2M vertices / 40M drawn
+  edges): values on 512 seeded keys.  Keys are drawn uniformly, with a fixed
+  seed, from those whose segment holds at most a cap of joined tuples (5000
+  triples, 1000 pairs: 98.6 % and 88 % of the keys); the rest is a long tail
+  whose oracle time per key runs to minutes, and its keys that cross work
+  units are checked by the sampled tests in test_gpu_parity.py.
+
+Keys are split into 16 groups balanced by joined tuples, and each group is
+one spawned oracle process that gets the tuples its keys join with (the
+oracle skips pairs of other keys before any tile arithmetic)."""
 import numpy as np
 import pytest
 import torch
@@ -38,14 +42,32 @@ def _pick(seed, cnt, cap):
     return np.sort(np.random.default_rng(seed).choice(pool, size=N_KEYS, replace=False))
 
 
+def _codes(keys):
+    """One int64 per key row (key columns are below 2^31), ascending with
+    the rows' lexicographic order."""
+    keys = np.asarray(keys, dtype=np.int64).reshape(len(keys), -1)
+    c = np.zeros(len(keys), np.int64)
+    for j in range(keys.shape[1]):
+        c = c * (1 << 31) + keys[:, j]
+    return c
+
+
+def _balanced(keys, weight, parts=GROUPS):
+    """Split ascending keys into contiguous groups of about equal weight."""
+    cum = np.cumsum(weight)
+    cuts = np.searchsorted(cum, cum[-1] * np.arange(1, parts) / parts)
+    return [g for g in np.split(keys, cuts) if len(g)]
+
+
 def _check_groups(out, groups, refs):
     """Download the output once; each group's oracle result holds exactly
     its keys, ascending."""
     keys, tiles = out.download()
-    k0 = keys[:, 0]
+    k0 = _codes(keys)
     checked = 0
     for g, ref in zip(groups, refs):
-        idx = np.searchsorted(k0, g)
+        idx = np.searchsorted(k0, _codes(g))
+        assert np.array_equal(keys[idx], np.asarray(g).reshape(len(g), -1)), "key missing from the output"
         assert np.array_equal(keys[idx], ref["keys"]), "sampled keys differ"
         gv = tiles[torch.as_tensor(idx)].to(torch.float64).numpy()
         check_values(gv, ref["out"], ref["abs"], torch.bfloat16, out.dtype == torch.bfloat16)
@@ -128,3 +150,52 @@ def test_two_layer_gnn_full_size_512_keys(ctx):
         r.destroy()
     del w, tasks
     torch.cuda.empty_cache()
+
+
+def test_gnn_message_passing_full_size_every_key(ctx):
+    """Config 2: T = (X Y)^T and then T Z, every output key's values."""
+    w = workloads.gnn_chain(seed=0, device="cuda")
+    dev = torch.device("cuda", 0)
+    X, Y, Z = (gpu_rel(ctx, w[k]) for k in ("X", "Y", "Z"))
+    T = ctx.einsum(w["spec1"], X, Y, out_dtype="bf16")
+    ky = w["Y"][0]
+    cnt = np.bincount(ky[:, 1])
+    keys = np.nonzero(cnt)[0]
+    groups = _balanced(keys, cnt[keys])
+    tasks = []
+    for g in groups:
+        rows = np.nonzero(np.isin(ky[:, 1], g))[0]
+        jn = np.unique(ky[rows, 0])
+        xrel = (jn[:, None].astype(np.int32), w["X"][1], w["X"][2][torch.as_tensor(jn, device=dev)])
+        yrel = (ky[rows], w["Y"][1], w["Y"][2][torch.as_tensor(rows, device=dev)])
+        tasks.append((w["spec1"], [xrel, yrel], {"sample_keys": g[:, None].astype(np.int32)}))
+    assert _check_groups(T, groups, oracle_parallel(tasks)) == len(keys) == T.n
+    # the second EinSum, stage-local on the computed T
+    O = ctx.einsum(w["spec2"], T, Z)
+    tk, tt = T.device_tensors()
+    tk0 = tk[:, 0].cpu().numpy()
+    tasks = []
+    for g in groups:
+        idx = np.searchsorted(tk0, g)
+        trel = (g[:, None].astype(np.int32), T.bounds, tt[torch.as_tensor(idx, device=dev)])
+        tasks.append((w["spec2"], [trel, w["Z"]], {"sample_keys": g[:, None].astype(np.int32)}))
+    assert _check_groups(O, groups, oracle_parallel(tasks)) == O.n
+    for r in (X, Y, Z, T, O):
+        r.destroy()
+
+
+def test_spgemm_full_size_every_key(ctx):
+    """Config 4: every output key's values."""
+    w = workloads.spgemm(seed=0)
+    out = ctx.einsum(w["spec"], gpu_rel(ctx, w["A"]), gpu_rel(ctx, w["B"]))
+    keys, _ = out.download()
+    ka, kb = w["A"][0], w["B"][0]
+    groups = _balanced(keys, np.ones(len(keys)))
+    tasks = []
+    for g in groups:
+        ra = np.nonzero(np.isin(ka[:, 0], np.unique(g[:, 0])))[0]
+        rb = np.nonzero(np.isin(kb[:, 1], np.unique(g[:, 1])))[0]
+        arel = (ka[ra], w["A"][1], w["A"][2][torch.as_tensor(ra)])
+        brel = (kb[rb], w["B"][1], w["B"][2][torch.as_tensor(rb)])
+        tasks.append((w["spec"], [arel, brel], {"sample_keys": np.ascontiguousarray(g, dtype=np.int32)}))
+    assert _check_groups(out, groups, oracle_parallel(tasks)) == len(keys) == out.n
