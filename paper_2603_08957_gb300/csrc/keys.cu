@@ -163,6 +163,7 @@ constexpr int kBuckets = 1 << kRadixBits;
 constexpr int kSortThreads = 256;
 constexpr int kSortItems = 16;
 constexpr int kSortTile = kSortThreads * kSortItems;
+static_assert(kSortThreads == kBuckets, "the scatter kernels keep one bucket per thread");
 
 __global__ void __launch_bounds__(kSortThreads) radix_hist_kernel(const uint64_t *__restrict__ k, int64_t n,
                                                                   int shift, uint32_t *hist, int nblocks) {
@@ -222,6 +223,89 @@ __global__ void __launch_bounds__(kSortThreads) radix_scatter_kernel(const uint6
             if (vin) vout[dst] = val;
         }
         __syncthreads();
+    }
+}
+
+// A whole LSD radix sort of at most kSortTile items in one CTA, for the short
+// arrays of small EinSums: per 8-bit pass each thread loads its kSortItems
+// items once, then a shared-memory histogram, its exclusive scan and the
+// stable scatter of radix_scatter_kernel (ranks in index order, 256 items a
+// round); passes alternate between the two buffers, with a block barrier
+// between them.  The buffers are read and written in the same launch, so they
+// are plain (coherent) pointers.
+__global__ void __launch_bounds__(kSortThreads) radix_sort_small_kernel(uint64_t *k0, uint64_t *v0, uint64_t *k1,
+                                                                        uint64_t *v1, int n, int lo, int bits) {
+    constexpr int kWarps = kSortThreads / 32;
+    __shared__ uint32_t base[kBuckets];
+    __shared__ uint32_t wcnt[kWarps][kBuckets];
+    __shared__ uint32_t wsum[kWarps];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const bool has_v = v0 != nullptr;
+    uint64_t *ks = k0, *vs = v0, *kd = k1, *vd = v1;
+    for (int shift = lo; shift < lo + bits; shift += kRadixBits) {
+        // this thread's items (round j holds item j * 256 + tid), loaded once per pass
+        uint64_t kk[kSortItems], vv[kSortItems];
+#pragma unroll
+        for (int j = 0; j < kSortItems; ++j) {
+            const int i = j * kSortThreads + tid;
+            kk[j] = i < n ? ks[i] : 0;
+            vv[j] = (i < n && has_v) ? vs[i] : 0;
+        }
+        base[tid] = 0;
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < kSortItems; ++j)
+            if (j * kSortThreads + tid < n) atomicAdd(&base[(uint32_t)(kk[j] >> shift) & (kBuckets - 1)], 1u);
+        __syncthreads();
+        // exclusive scan of the 256 bucket counts: within warps, then over the warps' totals
+        const uint32_t c = base[tid];
+        uint32_t x = c;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        if (lane == 31) wsum[warp] = x;
+        __syncthreads();
+        uint32_t before = 0;
+        for (int w = 0; w < warp; ++w) before += wsum[w];
+        base[tid] = before + x - c;
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < kSortItems; ++j) {
+            if (j * kSortThreads >= n) break;   // uniform
+            for (int q = tid; q < kWarps * kBuckets; q += kSortThreads) (&wcnt[0][0])[q] = 0;
+            __syncthreads();
+            const bool valid = j * kSortThreads + tid < n;
+            const uint32_t d = valid ? (uint32_t)(kk[j] >> shift) & (kBuckets - 1) : (uint32_t)kBuckets;
+            const uint32_t peers = __match_any_sync(0xffffffffu, d);
+            const uint32_t below = peers & ((1u << lane) - 1u);
+            if (valid && below == 0) wcnt[warp][d] = __popc(peers);
+            __syncthreads();
+            {
+                uint32_t run = base[tid];
+#pragma unroll
+                for (int w = 0; w < kWarps; ++w) {
+                    const uint32_t cw = wcnt[w][tid];
+                    wcnt[w][tid] = run;
+                    run += cw;
+                }
+                base[tid] = run;
+            }
+            __syncthreads();
+            if (valid) {
+                const uint32_t dst = wcnt[warp][d] + __popc(below);
+                kd[dst] = kk[j];
+                if (has_v) vd[dst] = vv[j];
+            }
+            __syncthreads();
+        }
+        uint64_t *t = ks;
+        ks = kd;
+        kd = t;
+        t = vs;
+        vs = vd;
+        vd = t;
     }
 }
 
@@ -454,6 +538,12 @@ void scan_i64(ucl_ctx *ctx, const int64_t *in, int64_t *out, int64_t n, int64_t 
 int radix_sort(ucl_ctx *ctx, uint64_t *kin, uint64_t *vin, uint64_t *kalt, uint64_t *valt, int64_t n, int bits,
                int lo) {
     if (bits <= 0 || n <= 1) return 0;
+    if (n <= kSortTile) {
+        // one launch for every pass
+        radix_sort_small_kernel<<<1, kSortThreads, 0, ctx->stream>>>(kin, vin, kalt, valt, (int)n, lo, bits);
+        ctx->launches++;
+        return ((bits + kRadixBits - 1) / kRadixBits) & 1;
+    }
     int nblocks = (int)((n + kSortTile - 1) / kSortTile);
     uint32_t *hist = (uint32_t *)ws_get(ctx, sizeof(uint32_t) * (size_t)kBuckets * nblocks);
     uint64_t *ks = kin, *vs = vin, *kd = kalt, *vd = valt;
