@@ -424,6 +424,7 @@ struct BandPlan {
 };
 
 constexpr int kMaxBands = 16;   // 2 (B + 1) band ranges are read in one sizing sync
+constexpr int64_t kSegUnitPairs = 16384;   // pair lists up to this size are cut at segment boundaries
 
 BandPlan plan_bands(ucl_ctx *ctx, const Spec &s, ucl_rel *const *in, KeyPlan &kp, bool tc_ok) {
     BandPlan bp;
@@ -743,6 +744,7 @@ ucl_status ucl_ctx_create(int device, void *stream, ucl_alloc_fn alloc, ucl_free
     if (const char *e = getenv("UCL_BANDS")) ctx->tune_bands = atoi(e);
     if (const char *e = getenv("UCL_L2_HINTS")) ctx->tune_hints = atoi(e);
     if (const char *e = getenv("UCL_TC_STAGES")) ctx->tune_tc_stages = atoi(e);
+    if (const char *e = getenv("UCL_SEG_UNITS")) ctx->tune_seg_units = atoi(e);
     if (const char *e = getenv("UCL_TC_MMA")) ctx->tune_tc_mma = atoi(e);
     if (const char *e = getenv("UCL_TC_PREFETCH")) ctx->tune_tc_prefetch = atoi(e);
     if (const char *e = getenv("UCL_WINDOW")) ctx->tune_window = atoi(e);
@@ -1389,9 +1391,21 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             if (wb > 0 && !use_tc) check(fail(ctx, UCL_ERR_UNSUPPORTED, "windowed pair list without the tcgen05 path"));
             int G = use_tc ? (n_in == 3 ? tc3_units(ctx, P) : tc_units(ctx, tp, P))
                            : (int)std::min<int64_t>(P, (int64_t)ctx->sm_count * 4);
+            // On the tcgen05 path, small pair lists and lists of one pair per
+            // segment are cut at segment boundaries (at most one unit per
+            // segment): no segment needs a partial or the fixup launch, and a
+            // unit's pairs stream through its pipeline either way.  The FFMA
+            // kernels walk a unit's pairs one after another, so they keep the
+            // even split (more, shorter units), as do banded and windowed
+            // launches.
+            const bool seg_units = use_tc && ctx->tune_seg_units != 0 && !banded && wb == 0 && Sseg > 0 &&
+                                   (P <= kSegUnitPairs || P == Sseg);
+            if (seg_units && G > Sseg) G = (int)Sseg;
             a.units.P = P;
             a.units.G = G;
             a.units.base = 0;
+            a.units.seg = seg_units ? seg_start : nullptr;
+            a.units.S = Sseg;
             a.bands = bp.B;
             a.l2_hints = ctx->tune_hints;
             stats.n_units = G;
@@ -1417,7 +1431,10 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
             if (!banded) {
                 contract(a);
                 record(ctx, 4);
-                if (wb > 0) launch_fixup_window(ctx, a); else launch_fixup(ctx, a);
+                if (wb > 0)
+                    launch_fixup_window(ctx, a);
+                else if (!seg_units)
+                    launch_fixup(ctx, a);
                 record(ctx, 5);
             } else {
                 // band after band into fp32 partials keyed (band, output
@@ -1432,6 +1449,7 @@ ucl_status ucl_einsum(ucl_ctx *ctx, const char *spec_text, int n_in, ucl_rel *co
                     c.seg_start = seg_start + band_seg[b];
                     c.S = band_seg[b + 1] - band_seg[b];
                     c.units.P = Pb;
+                    c.units.seg = nullptr;
                     c.units.G = use_tc ? tc_units(ctx, tp, Pb) : (int)std::min<int64_t>(Pb, (int64_t)ctx->sm_count * 4);
                     c.units.base = band_start[b];
                     c.out = wb > 0 ? part : part + (size_t)band_seg[b] * lp.tile_w;

@@ -91,7 +91,12 @@ struct Units {
     int64_t P;
     int G;
     int64_t base;
-    __host__ __device__ int64_t begin(int u) const { return base + P * u / G; }
+    // Optional cut at segment boundaries: unit u starts at segment S * u / G
+    // (seg: the S + 1 segment starts, device memory, seg[S] = the end), so no
+    // segment spans two units and no partial or fixup is needed (G <= S).
+    const int64_t *seg = nullptr;
+    int64_t S = 0;
+    __host__ __device__ int64_t begin(int u) const { return seg ? seg[S * u / G] : base + P * u / G; }
 };
 
 // Stream-ordered bump allocator over blocks obtained from the context hooks.
@@ -168,6 +173,10 @@ struct ucl_ctx {
     // streamed operand)
     int tune_tc_stages = 0;
     int tune_tc_mma = 0;
+    // UCL_SEG_UNITS (0: always split pair lists evenly into work units, so
+    // that segments may span units; else small lists are cut at segment
+    // boundaries)
+    int tune_seg_units = 1;
     int tune_tc_prefetch = -1;
     // UCL_WINDOW (-1 or unset: automatic; 0: no windows; n: windows of 2^n
     // output keys where the windowed tcgen05 kernel applies)

@@ -25,6 +25,23 @@ def ctx():
     c.close()
 
 
+@pytest.fixture(scope="module")
+def ctx_even():
+    """A context that always splits pair lists evenly into work units, so
+    that even small lists have segments spanning units (partials + fixup)."""
+    old = os.environ.get("UCL_SEG_UNITS")
+    os.environ["UCL_SEG_UNITS"] = "0"
+    try:
+        c = Context(0)
+    finally:
+        if old is None:
+            del os.environ["UCL_SEG_UNITS"]
+        else:
+            os.environ["UCL_SEG_UNITS"] = old
+    yield c
+    c.close()
+
+
 def _bf16_exact(a):
     """Round a float64 array to bf16 values (both sides then see the same inputs)."""
     return torch.from_numpy(np.asarray(a)).to(torch.bfloat16).to(torch.float64).numpy()
@@ -77,10 +94,11 @@ TC_CASES = [
 
 
 @pytest.mark.parametrize("ou,ov,ow,ext", TC_CASES)
-def test_tc_gemm_layouts(ctx, ou, ov, ow, ext):
+def test_tc_gemm_layouts(ctx_even, ou, ov, ow, ext):
     """Block-sparse tiled matmul whose tile kernel is a bf16 GEMM in every
     operand major order, output transpose and swizzle width: 3 x 40 x 2 key
     grid, 240 pairs over 6 output keys (segments split across work units)."""
+    ctx = ctx_even
     rng = np.random.default_rng(hash((ou, ov, ow)) % 2**31)
     nI, nJ, nK = 3, 40, 2
 
@@ -376,9 +394,10 @@ def test_empty_relation_and_empty_join(ctx):
     assert out.n == 0 and ctx.last_stats()["n_pairs"] == 0
 
 
-def test_one_segment_across_all_units(ctx):
+def test_one_segment_across_all_units(ctx_even):
     """All pairs share one output key (a key-less output summed over J): the
     segment is split across every work unit and reassembled by the fixup."""
+    ctx = ctx_even
     rng = np.random.default_rng(4)
     nJ = 3000
     ka = np.arange(nJ, dtype=np.int32)[:, None]
@@ -386,7 +405,36 @@ def test_one_segment_across_all_units(ctx):
     B = (ka.copy(), (nJ,), torch.from_numpy(rng.standard_normal((nJ, 5, 6)).astype(np.float32)))
     ref = oracle_ref("Jij,Jjk->ik", [A, B])
     out = ctx.einsum("Jij,Jjk->ik", gpu_rel(ctx, A), gpu_rel(ctx, B))
+    assert ctx.last_stats()["n_units"] > 1
     assert_parity(out, ref, torch.float32)
+
+
+@pytest.mark.parametrize("path", ["tc", "simt"])
+def test_small_lists_cut_at_segments(ctx, ctx_even, path):
+    """On the tcgen05 path small pair lists are cut into work units at
+    segment boundaries: no segment spans two units and the fixup moves
+    nothing.  The FFMA path keeps the even split.  Both cuts match the
+    oracle."""
+    rng = np.random.default_rng(21)
+    nI, nJ, nK = 12, 30, 5
+    keys_u = [(i, j) for i in range(nI) for j in range(nJ) if rng.random() < 0.6]
+    keys_v = [(j, k) for j in range(nJ) for k in range(nK) if rng.random() < 0.6]
+    U = (np.array(keys_u, np.int32), (nI, nJ), torch.randn((len(keys_u), 128, 64)).to(torch.bfloat16))
+    V = (np.array(keys_v, np.int32), (nJ, nK), torch.randn((len(keys_v), 64, 64)).to(torch.bfloat16))
+    spec = "IiJj,JjKk->IiKk"
+    ref = oracle_ref(spec, [U, V])
+    for c, cut in ((ctx, True), (ctx_even, False)):
+        c.fixup_bytes(reset=True)
+        out = c.einsum(spec, gpu_rel(c, U), gpu_rel(c, V), path=path)
+        st = c.last_stats()
+        assert st["n_pairs"] == ref["n_pairs"] and st["path"] == path
+        assert_parity(out, ref, torch.bfloat16)
+        c.synchronize()
+        moved = c.fixup_bytes(reset=True)
+        if cut and path == "tc":
+            assert moved == 0 and st["n_units"] <= st["n_segments"]
+        else:
+            assert moved > 0
 
 
 def test_unary_relu_scale_bf16_out(ctx):
