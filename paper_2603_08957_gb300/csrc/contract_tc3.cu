@@ -288,7 +288,8 @@ __global__ void __launch_bounds__(kThreads3, 1)
     if (warp == 0) {
         // ------------------------------------------------------- producer
         // Copies only: lane j < pps handles triple j of each stage (indices
-        // loaded one stage ahead) and issues its T and F copies.  The group
+        // loaded one stage ahead, checked when used) and issues its T and F
+        // copies.  The group
         // plan of a stage is posted separately by the group warp.
         const int nfills = (n + kPps3 - 1) / kPps3;
         auto load_idx = [&](int f, uint32_t &it, uint32_t &iff) {
@@ -298,11 +299,6 @@ __global__ void __launch_bounds__(kThreads3, 1)
             if (f < nfills && lane < kPps3 && p < pe) {
                 it = a.idx_t[p];
                 iff = a.idx_f[p];
-                if ((int64_t)it >= a.nT || (int64_t)iff >= a.nF) {
-                    atomicOr(a.status, kStBadIndex);
-                    it = 0;
-                    iff = 0;
-                }
             }
         };
         uint32_t it, iff;
@@ -311,6 +307,13 @@ __global__ void __launch_bounds__(kThreads3, 1)
         for (int f = 0; f < nfills; ++f) {
             uint32_t nit, niff;
             load_idx(f + 1, nit, niff);
+            // indices are checked when used, a stage after their load, so the
+            // next stage's loads stay in flight meanwhile
+            if ((int64_t)it >= a.nT || (int64_t)iff >= a.nF) {
+                atomicOr(a.status, kStBadIndex);
+                it = 0;
+                iff = 0;
+            }
             const int start = f * kPps3;
             const int np = n - start < kPps3 ? n - start : kPps3;
             uint32_t okw = 1;
@@ -358,12 +361,14 @@ __global__ void __launch_bounds__(kThreads3, 1)
             const int64_t p = pb + (int64_t)f * kPps3 + lane;
             return (f < nfills && lane < kPps3 && p < pe) ? a.idx_e[p] : 0u;
         };
-        uint32_t ie = load_e(0);
+        // E tuples of this stage and the next (loaded a stage earlier, so that
+        // the next stage's first one is read without waiting on a load)
+        uint32_t ie = load_e(0), nie = load_e(1);
         uint32_t st = 0, ph = 0, e_last = 0, gb = 0, gph = 0, opened = 0, cb = 0;
         int64_t s = s_first;
         int seg_end = n > 0 ? (int)((a.seg_start[s + 1] < pe ? a.seg_start[s + 1] : pe) - pb) : 0;
         for (int f = 0; f < nfills; ++f) {
-            const uint32_t nie = load_e(f + 1);
+            const uint32_t nnie = load_e(f + 2);
             const int start = f * kPps3;
             const int np = n - start < kPps3 ? n - start : kPps3;
             // segment starts inside this stage (uniform; rare)
@@ -428,6 +433,7 @@ __global__ void __launch_bounds__(kThreads3, 1)
             }
             if (!__shfl_sync(0xffffffffu, okw, 0)) break;
             ie = nie;
+            nie = nnie;
             if (++st == (uint32_t)kStages3) {
                 st = 0;
                 ph ^= 1u;
